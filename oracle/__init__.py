@@ -1,0 +1,163 @@
+"""Oracle for ROI-aware multi-sweep LiDAR voxelization (MM-BEV, Sec. IV-D, IV-F).
+
+TEST INFRASTRUCTURE. This package is the plain, slow, single-threaded CPU
+statement of the path (motion compensation, Eq. 6-7; inside-ROI test of
+Alg. 1 with the boxes of Eq. 1; hard voxelization with a per-voxel and a
+per-frame cap; mean voxel features). Only ``tests/``, ``__graft_entry__.smoke``
+and the CPU-baseline leg of ``bench.py`` may import it. It shares no code with
+the CUDA library and never imports it.
+
+The arithmetic lives in ``mmbev_oracle.c`` (plain C, built with
+``-O2 -ffp-contract=off``); this module only loads it with ctypes and moves
+numpy arrays in and out.
+
+Every function here is pinned by ``tests/test_oracle_pins.py`` against facts
+the paper and the mathematics fix (identity and translation transforms, the
+ghost-collapse property of compensation, a brute-force polygon test,
+hand-built voxels with known means, exhaustive bucketing on tiny grids and the
+invariants of the cap rule).
+"""
+from __future__ import annotations
+
+import ctypes
+import os
+import subprocess
+import sysconfig
+
+import numpy as np
+
+_HERE = os.path.dirname(os.path.abspath(__file__))
+_SRC = os.path.join(_HERE, "mmbev_oracle.c")
+_LIB = os.path.join(_HERE, "liboracle.so")
+
+_lib = None
+
+
+def build(force: bool = False) -> str:
+    """Compile the oracle into ``oracle/liboracle.so`` (gcc, no contraction)."""
+    if not force and os.path.exists(_LIB) and os.path.getmtime(_LIB) >= os.path.getmtime(_SRC):
+        return _LIB
+    cc = os.environ.get("CC", "gcc")
+    tmp = _LIB + f".tmp{os.getpid()}"
+    cmd = [cc, "-O2", "-ffp-contract=off", "-fno-fast-math", "-fPIC", "-shared",
+           "-std=c11", "-o", tmp, _SRC, "-lm"]
+    subprocess.run(cmd, check=True)
+    os.replace(tmp, _LIB)
+    return _LIB
+
+
+def _load():
+    global _lib
+    if _lib is None:
+        build()
+        lib = ctypes.CDLL(_LIB)
+        P = ctypes.c_void_p
+        i32, i64, f32 = ctypes.c_int32, ctypes.c_int64, ctypes.c_float
+        lib.oracle_classify.argtypes = [P, P, i32, P, P, i32, f32, P, P, P, P, P]
+        lib.oracle_classify.restype = ctypes.c_int
+        lib.oracle_voxelize_roi.argtypes = [P, P, i32, P, P, i32, f32, P, P,
+                                            i32, i32, P, P, P, P]
+        lib.oracle_voxelize_roi.restype = ctypes.c_int
+        lib.oracle_voxelize_roi_batched.argtypes = [P, P, i32, P, P, i32, f32, P, P,
+                                                    i32, i32, i32, P, P, P, P, P, P]
+        lib.oracle_voxelize_roi_batched.restype = ctypes.c_int
+        _lib = lib
+    return _lib
+
+
+def _ptr(a: np.ndarray):
+    return a.ctypes.data_as(ctypes.c_void_p)
+
+
+def _c(a, dtype):
+    return np.ascontiguousarray(np.asarray(a, dtype=dtype))
+
+
+def classify(points, sweep_offsets, sweep_tf, rois, roi_margin, voxel_size, pc_range):
+    """Per point: compensated xyz (float32 [N,3]), voxel linear index (int64,
+    -1 when dropped) and ROI rank (int32, -1 when dropped)."""
+    lib = _load()
+    points = _c(points, np.float32).reshape(-1, 5)
+    so = _c(sweep_offsets, np.int64)
+    tf = _c(sweep_tf, np.float32).reshape(-1, 16)
+    rois = _c(rois, np.float32).reshape(-1, 5)
+    vs = _c(voxel_size, np.float32)
+    rg = _c(pc_range, np.float32)
+    n = points.shape[0]
+    xyz = np.zeros((n, 3), np.float32)
+    lin = np.full(n, -1, np.int64)
+    rank = np.full(n, -1, np.int32)
+    rc = lib.oracle_classify(_ptr(points), _ptr(so), len(so) - 1, _ptr(tf), _ptr(rois),
+                             rois.shape[0], float(roi_margin), _ptr(vs), _ptr(rg),
+                             _ptr(xyz), _ptr(lin), _ptr(rank))
+    if rc != 0:
+        raise ValueError(f"oracle_classify failed with status {rc}")
+    return xyz, lin, rank
+
+
+def voxelize_roi(points, sweep_offsets, sweep_tf, rois, roi_margin, voxel_size,
+                 pc_range, max_pts_per_voxel, max_voxels):
+    """One frame. Returns (feats [nvox,5], coords [nvox,3] (z,y,x), counts [nvox])."""
+    lib = _load()
+    points = _c(points, np.float32).reshape(-1, 5)
+    so = _c(sweep_offsets, np.int64)
+    tf = _c(sweep_tf, np.float32).reshape(-1, 16)
+    rois = _c(rois, np.float32).reshape(-1, 5)
+    vs = _c(voxel_size, np.float32)
+    rg = _c(pc_range, np.float32)
+    mv = int(max_voxels)
+    feats = np.zeros((max(mv, 1), 5), np.float32)
+    coords = np.zeros((max(mv, 1), 3), np.int32)
+    counts = np.zeros(max(mv, 1), np.int32)
+    nvox = np.zeros(1, np.int32)
+    rc = lib.oracle_voxelize_roi(_ptr(points), _ptr(so), len(so) - 1, _ptr(tf), _ptr(rois),
+                                 rois.shape[0], float(roi_margin), _ptr(vs), _ptr(rg),
+                                 int(max_pts_per_voxel), mv, _ptr(feats), _ptr(coords),
+                                 _ptr(counts), _ptr(nvox))
+    if rc != 0:
+        raise ValueError(f"oracle_voxelize_roi failed with status {rc}")
+    k = int(nvox[0])
+    return feats[:k].copy(), coords[:k].copy(), counts[:k].copy()
+
+
+def voxelize_roi_batched(points, sweep_offsets, sweep_tf, rois, roi_margin, voxel_size,
+                         pc_range, max_pts_per_voxel, max_voxels, frame_sweep_offsets,
+                         frame_roi_offsets):
+    """Independent frames in one call. Returns a list of per-frame
+    (feats, coords, counts) tuples."""
+    lib = _load()
+    points = _c(points, np.float32).reshape(-1, 5)
+    so = _c(sweep_offsets, np.int64)
+    tf = _c(sweep_tf, np.float32).reshape(-1, 16)
+    rois = _c(rois, np.float32).reshape(-1, 5)
+    vs = _c(voxel_size, np.float32)
+    rg = _c(pc_range, np.float32)
+    fso = _c(frame_sweep_offsets, np.int32)
+    fro = _c(frame_roi_offsets, np.int32)
+    nf = len(fso) - 1
+    mv = int(max_voxels)
+    rows = max(nf * mv, 1)
+    feats = np.zeros((rows, 5), np.float32)
+    coords = np.zeros((rows, 3), np.int32)
+    counts = np.zeros(rows, np.int32)
+    nvox = np.zeros(max(nf, 1), np.int32)
+    rc = lib.oracle_voxelize_roi_batched(
+        _ptr(points), _ptr(so), len(so) - 1, _ptr(tf), _ptr(rois), rois.shape[0],
+        float(roi_margin), _ptr(vs), _ptr(rg), int(max_pts_per_voxel), mv, nf,
+        _ptr(fso), _ptr(fro), _ptr(feats), _ptr(coords), _ptr(counts), _ptr(nvox))
+    if rc != 0:
+        raise ValueError(f"oracle_voxelize_roi_batched failed with status {rc}")
+    out = []
+    for f in range(nf):
+        k = int(nvox[f])
+        r0 = f * mv
+        out.append((feats[r0:r0 + k].copy(), coords[r0:r0 + k].copy(), counts[r0:r0 + k].copy()))
+    return out
+
+
+def grid_dims(voxel_size, pc_range):
+    """(nx, ny, nz) = round-half-away((max - min) / size) in double, as the
+    oracle's llround does for these positive extents."""
+    vs = np.asarray(voxel_size, np.float32).astype(np.float64)
+    rg = np.asarray(pc_range, np.float32).astype(np.float64)
+    return tuple(int(np.floor((rg[a + 3] - rg[a]) / vs[a] + 0.5)) for a in range(3))

@@ -1,0 +1,313 @@
+/*
+ * Oracle for ROI-aware multi-sweep LiDAR voxelization (MM-BEV, Sec. IV-D and
+ * Sec. IV-F).
+ *
+ * TEST INFRASTRUCTURE. This file is the plain, slow, single-threaded CPU
+ * statement of what the GPU path computes. Only the test suite, the smoke
+ * check and the benchmark's CPU-baseline leg may load it. It shares no code,
+ * header, table or helper with the CUDA library; the two meet only through
+ * the seeded input generator.
+ *
+ * Build: gcc -O2 -ffp-contract=off -fPIC -shared (contraction off so that
+ * every fp32 multiply and add is rounded on its own, as the GPU path does).
+ *
+ * What is computed, step by step, in the order the paper gives it:
+ *   1. Eq. 6 / Eq. 7: each point of sweep s is mapped into the current frame
+ *      by that sweep's rotation and translation, p' = R p + T, taken from a
+ *      row-major 4x4 whose last row is ignored. fp32, each product and sum
+ *      rounded, summed left to right: ((r0*x + r1*y) + r2*z) + t.
+ *   2. Range crop: xmin <= x' < xmax (same for y, z). NaN fails.
+ *   3. Alg. 1 (inside-any-box test) with the boxes of Eq. 1: a point is kept
+ *      when it lies inside some ROI box, the box grown by the margin r on each
+ *      half-extent. The ROIs arrive in criticality order (Sec. IV-C); the
+ *      point's rank is the index of the first box that contains it. The
+ *      out-of-ROI keep probability of Alg. 1 is taken as zero.
+ *   4. Hard voxelization (Sec. IV-F): voxel c = floor((p' - min) / size) per
+ *      axis, dropped when c >= n; linear index lin = (cz*ny + cy)*nx + cx.
+ *      Each voxel keeps the K points with the smallest input index. When more
+ *      voxels than max_voxels exist, the max_voxels smallest by
+ *      (minimum rank, lin) are kept, so mandatory ROIs keep full fidelity
+ *      (Sec. IV-C). Output voxels are in ascending lin.
+ *   5. Voxel feature encoder (Alg. 1): mean of (x', y', z', intensity, dt)
+ *      over the kept points, an fp32 sum in index order and one fp32 divide.
+ *
+ * Batched form: every frame is an independent problem; frame f owns sweeps
+ * [fso[f], fso[f+1]) and ROIs [fro[f], fro[f+1]); its outputs start at row
+ * f*max_voxels.
+ */
+#include <math.h>
+#include <stdint.h>
+#include <stdlib.h>
+#include <string.h>
+
+typedef struct { float cx, cy, w, l, yaw; } oracle_roi_t;
+
+enum { ORACLE_OK = 0, ORACLE_EINVAL = -1, ORACLE_ENOMEM = -5 };
+
+/* One kept point: voxel linear index, input index, ROI rank, features. */
+typedef struct {
+    int64_t lin;
+    int64_t idx;
+    int32_t rank;
+    float f[5];
+} kept_point_t;
+
+/* One voxel: its linear index, first member in the sorted list, size, and
+ * the smallest ROI rank among its points. */
+typedef struct {
+    int64_t lin;
+    int64_t start;
+    int64_t n;
+    int32_t minrank;
+} voxel_t;
+
+/* Grid extent along one axis: round((max - min) / size) in double. */
+static int64_t grid_dim(float lo, float hi, float size)
+{
+    return (int64_t)llround(((double)hi - (double)lo) / (double)size);
+}
+
+/* Eq. 6: rotate and translate one point with the 4x4 T (row-major). */
+static void compensate(const float *T, float x, float y, float z,
+                       float *xo, float *yo, float *zo)
+{
+    float a, b, c;
+    a = T[0] * x; b = T[1] * y; a = a + b; c = T[2] * z; a = a + c; *xo = a + T[3];
+    a = T[4] * x; b = T[5] * y; a = a + b; c = T[6] * z; a = a + c; *yo = a + T[7];
+    a = T[8] * x; b = T[9] * y; a = a + b; c = T[10] * z; a = a + c; *zo = a + T[11];
+}
+
+/* Eq. 1 box, rotated by yaw, half-extents grown by the margin. The point is
+ * inside when its coordinates in the box frame lie within the half-extents
+ * (boundary included). l runs along the heading, w across it. */
+static int inside_roi(const oracle_roi_t *r, float margin, float x, float y)
+{
+    float c = (float)cos((double)r->yaw);
+    float s = (float)sin((double)r->yaw);
+    float hl = 0.5f * r->l + margin;
+    float hw = 0.5f * r->w + margin;
+    float dx = x - r->cx;
+    float dy = y - r->cy;
+    float p, q, u, v;
+    p = dx * c; q = dy * s; u = p + q;
+    p = dy * c; q = dx * s; v = p - q;
+    return fabsf(u) <= hl && fabsf(v) <= hw;
+}
+
+static int validate_grid(const float vs[3], const float range[6], int64_t dims[3])
+{
+    for (int a = 0; a < 3; ++a) {
+        if (!(vs[a] > 0.0f) || !isfinite(vs[a])) return ORACLE_EINVAL;
+        if (!isfinite(range[a]) || !isfinite(range[a + 3])) return ORACLE_EINVAL;
+        if (!(range[a + 3] > range[a])) return ORACLE_EINVAL;
+        dims[a] = grid_dim(range[a], range[a + 3], vs[a]);
+        if (dims[a] < 1) return ORACLE_EINVAL;
+    }
+    return ORACLE_OK;
+}
+
+/*
+ * Steps 1-4 for every point, in input order: writes the compensated
+ * coordinates, the voxel linear index (-1 when dropped) and the ROI rank
+ * (-1 when dropped). The per-point view of the path, used to test the first
+ * two steps on their own.
+ */
+int oracle_classify(const float *points, const int64_t *sweep_offsets,
+                    int32_t num_sweeps, const float *sweep_tf,
+                    const oracle_roi_t *rois, int32_t num_rois, float margin,
+                    const float voxel_size[3], const float range[6],
+                    float *out_xyz, int64_t *out_lin, int32_t *out_rank)
+{
+    int64_t dims[3];
+    if (num_sweeps < 0 || num_rois < 0) return ORACLE_EINVAL;
+    if (validate_grid(voxel_size, range, dims) != ORACLE_OK) return ORACLE_EINVAL;
+    for (int32_t s = 0; s < num_sweeps; ++s) {
+        const float *T = sweep_tf + 16 * (int64_t)s;
+        for (int64_t i = sweep_offsets[s]; i < sweep_offsets[s + 1]; ++i) {
+            const float *p = points + 5 * i;
+            float x, y, z;
+            compensate(T, p[0], p[1], p[2], &x, &y, &z);
+            out_xyz[3 * i + 0] = x;
+            out_xyz[3 * i + 1] = y;
+            out_xyz[3 * i + 2] = z;
+            out_lin[i] = -1;
+            out_rank[i] = -1;
+            if (!(range[0] <= x && x < range[3])) continue;
+            if (!(range[1] <= y && y < range[4])) continue;
+            if (!(range[2] <= z && z < range[5])) continue;
+            int32_t rank = -1;
+            for (int32_t r = 0; r < num_rois; ++r) {
+                if (inside_roi(&rois[r], margin, x, y)) { rank = r; break; }
+            }
+            if (rank < 0) continue;
+            int64_t cx = (int64_t)floorf((x - range[0]) / voxel_size[0]);
+            int64_t cy = (int64_t)floorf((y - range[1]) / voxel_size[1]);
+            int64_t cz = (int64_t)floorf((z - range[2]) / voxel_size[2]);
+            if (cx >= dims[0] || cy >= dims[1] || cz >= dims[2]) continue;
+            out_lin[i] = (cz * dims[1] + cy) * dims[0] + cx;
+            out_rank[i] = rank;
+        }
+    }
+    return ORACLE_OK;
+}
+
+static int cmp_point(const void *a, const void *b)
+{
+    const kept_point_t *p = (const kept_point_t *)a, *q = (const kept_point_t *)b;
+    if (p->lin != q->lin) return p->lin < q->lin ? -1 : 1;
+    if (p->idx != q->idx) return p->idx < q->idx ? -1 : 1;
+    return 0;
+}
+
+static int cmp_voxel_rank_lin(const void *a, const void *b)
+{
+    const voxel_t *u = (const voxel_t *)a, *v = (const voxel_t *)b;
+    if (u->minrank != v->minrank) return u->minrank < v->minrank ? -1 : 1;
+    if (u->lin != v->lin) return u->lin < v->lin ? -1 : 1;
+    return 0;
+}
+
+static int cmp_voxel_lin(const void *a, const void *b)
+{
+    const voxel_t *u = (const voxel_t *)a, *v = (const voxel_t *)b;
+    if (u->lin != v->lin) return u->lin < v->lin ? -1 : 1;
+    return 0;
+}
+
+/* One frame, host pointers. Sweep s of the frame covers points
+ * [sweep_offsets[s], sweep_offsets[s+1]); indices are global, so "first K by
+ * input index" compares global indices. Rows >= *out_nvox are not written. */
+int oracle_voxelize_roi(const float *points, const int64_t *sweep_offsets,
+                        int32_t num_sweeps, const float *sweep_tf,
+                        const oracle_roi_t *rois, int32_t num_rois, float margin,
+                        const float voxel_size[3], const float range[6],
+                        int32_t max_pts_per_voxel, int32_t max_voxels,
+                        float *out_feats, int32_t *out_coords,
+                        int32_t *out_counts, int32_t *out_nvox)
+{
+    int64_t dims[3];
+    if (num_sweeps < 0 || num_rois < 0 || max_pts_per_voxel < 1 || max_voxels < 0)
+        return ORACLE_EINVAL;
+    if (validate_grid(voxel_size, range, dims) != ORACLE_OK) return ORACLE_EINVAL;
+    if (!(margin >= 0.0f)) return ORACLE_EINVAL;
+
+    int64_t first = num_sweeps > 0 ? sweep_offsets[0] : 0;
+    int64_t last = num_sweeps > 0 ? sweep_offsets[num_sweeps] : 0;
+    int64_t npts = last - first;
+    kept_point_t *kept = (kept_point_t *)malloc(sizeof(kept_point_t) * (size_t)(npts > 0 ? npts : 1));
+    if (!kept) return ORACLE_ENOMEM;
+    int64_t m = 0;
+
+    /* Steps 1-4 (per point). */
+    for (int32_t s = 0; s < num_sweeps; ++s) {
+        const float *T = sweep_tf + 16 * (int64_t)s;
+        for (int64_t i = sweep_offsets[s]; i < sweep_offsets[s + 1]; ++i) {
+            const float *p = points + 5 * i;
+            float x, y, z;
+            compensate(T, p[0], p[1], p[2], &x, &y, &z);
+            if (!(range[0] <= x && x < range[3])) continue;
+            if (!(range[1] <= y && y < range[4])) continue;
+            if (!(range[2] <= z && z < range[5])) continue;
+            int32_t rank = -1;
+            for (int32_t r = 0; r < num_rois; ++r) {
+                if (inside_roi(&rois[r], margin, x, y)) { rank = r; break; }
+            }
+            if (rank < 0) continue;
+            int64_t cx = (int64_t)floorf((x - range[0]) / voxel_size[0]);
+            int64_t cy = (int64_t)floorf((y - range[1]) / voxel_size[1]);
+            int64_t cz = (int64_t)floorf((z - range[2]) / voxel_size[2]);
+            if (cx >= dims[0] || cy >= dims[1] || cz >= dims[2]) continue;
+            kept[m].lin = (cz * dims[1] + cy) * dims[0] + cx;
+            kept[m].idx = i;
+            kept[m].rank = rank;
+            kept[m].f[0] = x;
+            kept[m].f[1] = y;
+            kept[m].f[2] = z;
+            kept[m].f[3] = p[3];
+            kept[m].f[4] = p[4];
+            ++m;
+        }
+    }
+
+    /* Group by voxel; inside a voxel, points in input order. */
+    qsort(kept, (size_t)m, sizeof(kept_point_t), cmp_point);
+    voxel_t *vox = (voxel_t *)malloc(sizeof(voxel_t) * (size_t)(m > 0 ? m : 1));
+    if (!vox) { free(kept); return ORACLE_ENOMEM; }
+    int64_t u = 0;
+    for (int64_t j = 0; j < m; ++j) {
+        if (j == 0 || kept[j].lin != kept[j - 1].lin) {
+            vox[u].lin = kept[j].lin;
+            vox[u].start = j;
+            vox[u].n = 0;
+            vox[u].minrank = kept[j].rank;
+            ++u;
+        }
+        voxel_t *v = &vox[u - 1];
+        v->n += 1;
+        if (kept[j].rank < v->minrank) v->minrank = kept[j].rank;
+    }
+
+    /* Voxel cap: keep the max_voxels smallest by (minrank, lin), then
+     * restore ascending lin. */
+    if (u > max_voxels) {
+        qsort(vox, (size_t)u, sizeof(voxel_t), cmp_voxel_rank_lin);
+        u = max_voxels;
+        qsort(vox, (size_t)u, sizeof(voxel_t), cmp_voxel_lin);
+    }
+
+    /* Step 5: mean over the first K points of each kept voxel. */
+    for (int64_t v = 0; v < u; ++v) {
+        int64_t lin = vox[v].lin;
+        int64_t cx = lin % dims[0];
+        int64_t cy = (lin / dims[0]) % dims[1];
+        int64_t cz = lin / (dims[0] * dims[1]);
+        int64_t cnt = vox[v].n < max_pts_per_voxel ? vox[v].n : max_pts_per_voxel;
+        out_coords[3 * v + 0] = (int32_t)cz;
+        out_coords[3 * v + 1] = (int32_t)cy;
+        out_coords[3 * v + 2] = (int32_t)cx;
+        out_counts[v] = (int32_t)cnt;
+        for (int c = 0; c < 5; ++c) {
+            float acc = 0.0f;
+            for (int64_t j = 0; j < cnt; ++j) acc = acc + kept[vox[v].start + j].f[c];
+            out_feats[5 * v + c] = acc / (float)cnt;
+        }
+    }
+    *out_nvox = (int32_t)u;
+    free(vox);
+    free(kept);
+    return ORACLE_OK;
+}
+
+/* Batched form: num_frames independent frames, each an oracle_voxelize_roi
+ * call on its own sweeps and ROIs; frame f writes rows starting at
+ * f*max_voxels and out_nvox[f]. */
+int oracle_voxelize_roi_batched(const float *points, const int64_t *sweep_offsets,
+                                int32_t num_sweeps, const float *sweep_tf,
+                                const oracle_roi_t *rois, int32_t num_rois,
+                                float margin, const float voxel_size[3],
+                                const float range[6], int32_t max_pts_per_voxel,
+                                int32_t max_voxels, int32_t num_frames,
+                                const int32_t *frame_sweep_offsets,
+                                const int32_t *frame_roi_offsets,
+                                float *out_feats, int32_t *out_coords,
+                                int32_t *out_counts, int32_t *out_nvox)
+{
+    if (num_frames < 0) return ORACLE_EINVAL;
+    if (num_frames > 0 && (frame_sweep_offsets[num_frames] != num_sweeps ||
+                           frame_roi_offsets[num_frames] != num_rois))
+        return ORACLE_EINVAL;
+    for (int32_t f = 0; f < num_frames; ++f) {
+        int32_t s0 = frame_sweep_offsets[f], s1 = frame_sweep_offsets[f + 1];
+        int32_t r0 = frame_roi_offsets[f], r1 = frame_roi_offsets[f + 1];
+        if (s1 < s0 || r1 < r0) return ORACLE_EINVAL;
+        int64_t row = (int64_t)f * max_voxels;
+        int rc = oracle_voxelize_roi(points, sweep_offsets + s0, s1 - s0,
+                                     sweep_tf + 16 * (int64_t)s0, rois + r0, r1 - r0,
+                                     margin, voxel_size, range, max_pts_per_voxel,
+                                     max_voxels, out_feats + 5 * row,
+                                     out_coords + 3 * row, out_counts + row,
+                                     out_nvox + f);
+        if (rc != ORACLE_OK) return rc;
+    }
+    return ORACLE_OK;
+}
