@@ -1,0 +1,400 @@
+"""Benchmark: ROI-aware multi-sweep LiDAR voxelization on GB300.
+
+One step = one call of the whole path (motion compensation, ROI test, voxel
+hash, cap and canonical order, mean features) over a 32-frame streaming batch
+of nuScenes-shaped frames (11,110,400 points, 222 MB of fp32 input), inputs
+resident in HBM. The metric is in-ROI points (points passing the range and
+ROI tests, counted before the caps) per second, over the whole job.
+
+  python bench.py [--gpus N --steps K --warmup W] [--impl reference]
+
+With N > 1 (torchrun) every rank voxelizes its own 32 frames (distinct seeds,
+no collective on the data path) and rank 0 reports the aggregate over the
+slowest rank's time ("weak" scaling). ``--impl reference`` times the CPU
+oracle on the host cores instead (a bounded sample of the same workload).
+"""
+from __future__ import annotations
+
+import argparse
+import hashlib
+import json
+import os
+import subprocess
+import sys
+import threading
+import time
+
+import numpy as np
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+import synth  # noqa: E402
+
+METRIC = "in-ROI LiDAR points voxelized/sec and µs/frame; achieved HBM GB/s vs peak"
+FRAMES = 32
+BYTES_PER_POINT = 20      # fp32 x, y, z, intensity, dt
+BYTES_PER_VOXEL = 36      # 5 fp32 means + 3 int32 coords + 1 int32 count
+DOMINANT = "points"       # stage with the largest share of the step
+PROFILE = os.path.join(ROOT, "profiles", "points_batch32.json")
+
+
+def dist_env():
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    return world, rank, local
+
+
+def workload_for_rank(rank: int):
+    return synth.streaming_batch(FRAMES, base_seed=1000 + FRAMES * rank)
+
+
+def workload_desc(w):
+    return {
+        "workload": (f"batch{FRAMES}: {FRAMES} independent nuScenes-shaped frames "
+                     "(10 sweeps x 34,720 pts, 32-beam spinning LiDAR, ray-cast scene), "
+                     "30 rotated ROIs/frame, margin 0.5 m, 0.075x0.075x0.2 m voxels "
+                     "(1440x1440x40), K=10, max 120,000 voxels/frame"),
+        "frames_per_gpu": w.num_frames,
+        "points_per_gpu": w.num_points,
+        "input_mb_per_gpu": round(w.points.nbytes / 1e6, 1),
+        "l2": "inputs (222 MB/step) larger than the 129 MB L2; no flush",
+    }
+
+
+def read_peaks():
+    path = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    if os.path.exists(path):
+        with open(path) as fh:
+            j = json.load(fh)
+        return float(j["hbm_gbs"]), "measured"
+    return 6800.0, "fallback"
+
+
+def profile_traffic():
+    """DRAM bytes per launch of the dominant kernel from the committed ncu
+    summary, or None when the kernel source changed since it was taken."""
+    if not os.path.exists(PROFILE):
+        return None
+    with open(PROFILE) as fh:
+        j = json.load(fh)
+    src = os.path.join(ROOT, "paper_2608_15437_gb300", "csrc", j.get("source", "points.cu"))
+    with open(src, "rb") as fh:
+        digest = hashlib.sha256(fh.read()).hexdigest()
+    if digest != j.get("source_sha256"):
+        return None
+    return j.get("dram_bytes_per_launch")
+
+
+class ClockSampler:
+    """nvidia-smi samples (200 ms) while the timed region runs."""
+
+    FIELDS = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, gpu_index: int):
+        self.gpu = gpu_index
+        self.proc = None
+        self.lines = []
+        self.thread = None
+
+    def start(self):
+        try:
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", f"--id={self.gpu}", f"--query-gpu={self.FIELDS}",
+                 "--format=csv,noheader,nounits", "-lms", "200"],
+                stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
+        except OSError:
+            self.proc = None
+            return
+        self.thread = threading.Thread(target=self._read, daemon=True)
+        self.thread.start()
+
+    def _read(self):
+        for line in self.proc.stdout:
+            self.lines.append(line.strip())
+
+    def stop(self):
+        if self.proc is None:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["nvidia-smi unavailable"]}
+        self.proc.terminate()
+        try:
+            self.proc.wait(timeout=5)
+        except subprocess.TimeoutExpired:
+            self.proc.kill()
+        if self.thread:
+            self.thread.join(timeout=2)
+        sm, smax, reasons = [], [], set()
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        for ln in self.lines:
+            parts = [x.strip() for x in ln.split(",")]
+            if len(parts) < 9:
+                continue
+            try:
+                sm.append(float(parts[1]))
+                smax.append(float(parts[2]))
+            except ValueError:
+                continue
+            for name, v in zip(names, parts[5:9]):
+                if v.lower().startswith("active"):
+                    reasons.add(name)
+        return {"sm_mhz": float(np.median(sm)) if sm else None,
+                "sm_max_mhz": float(max(smax)) if smax else None,
+                "samples": len(sm), "reasons": sorted(reasons)}
+
+
+def cpu_oracle_baseline(w, budget_s: float = 12.0):
+    """The oracle as it stands, single-threaded on a host core, on whole
+    frames of the same batch until about budget_s seconds have run."""
+    import oracle
+    oracle.build()
+    pts = 0
+    frames = 0
+    t0 = time.perf_counter()
+    f = 0
+    while True:
+        fw = w.frame(f % w.num_frames)
+        oracle.voxelize_roi(fw.points, fw.sweep_offsets, fw.sweep_tf, fw.rois, fw.roi_margin,
+                            fw.voxel_size, fw.pc_range, fw.max_pts_per_voxel, fw.max_voxels)
+        frames += 1
+        f += 1
+        if time.perf_counter() - t0 >= budget_s:
+            break
+    dt = time.perf_counter() - t0
+    return frames, dt
+
+
+def run_reference(args):
+    world, rank, _ = dist_env()
+    if rank != 0:
+        return 0
+    import oracle
+    oracle.build()
+    w = workload_for_rank(0)
+    per_step = 2  # frames per step: a bounded sample of the batch
+    frames = [w.frame(f) for f in range(w.num_frames)]
+    in_roi = []
+    for fw in frames:  # the metric's numerator per frame, untimed
+        _, lin, _ = oracle.classify(fw.points, fw.sweep_offsets, fw.sweep_tf, fw.rois,
+                                    fw.roi_margin, fw.voxel_size, fw.pc_range)
+        in_roi.append(int((lin >= 0).sum()))
+    pts_done = 0
+    times = []
+    f = 0
+    for step in range(args.warmup + args.steps):
+        t0 = time.perf_counter()
+        npts = 0
+        for _ in range(per_step):
+            fw = frames[f % len(frames)]
+            oracle.voxelize_roi(fw.points, fw.sweep_offsets, fw.sweep_tf, fw.rois,
+                                fw.roi_margin, fw.voxel_size, fw.pc_range,
+                                fw.max_pts_per_voxel, fw.max_voxels)
+            npts += in_roi[f % len(frames)]
+            f += 1
+        dt = time.perf_counter() - t0
+        if step >= args.warmup:
+            times.append(dt)
+            pts_done += npts
+    total = sum(times)
+    value = pts_done / total
+    line = {
+        "impl": "reference", "metric": METRIC, "value": value, "unit": "points/s",
+        "n_gpus": args.gpus, "steps": args.steps, "warmup": args.warmup,
+        "ms_per_step": 1e3 * total / len(times), "higher_is_better": True, "scaling": "weak",
+        "vs_baseline": None, "dtype": "f32", "data": "synthetic",
+        "config": workload_desc(w),
+        "cpu_baseline": {"kind": "oracle", "value": value, "unit": "points/s", "cores": 1,
+                         "sample": f"{per_step} whole frames of the batch per step, "
+                                   "single-threaded C oracle"},
+        "e2e": {"value": value, "unit": "points/s", "h2d_bytes_per_step": 0,
+                "d2h_bytes_per_step": 0},
+    }
+    print(json.dumps(line), flush=True)
+    return 0
+
+
+def run_gpu(args):
+    import torch
+    import torch.distributed as dist
+
+    import paper_2608_15437_gb300 as mmbev
+
+    world, rank, local = dist_env()
+    if world > 1:
+        torch.cuda.set_device(local)
+        dist.init_process_group("nccl", device_id=torch.device("cuda", local))
+    dev = torch.device("cuda", local if world > 1 else 0)
+    mmbev.load()
+
+    w = workload_for_rank(rank)
+    pts = torch.from_numpy(w.points).to(dev)
+    tf = torch.from_numpy(w.sweep_tf).to(dev)
+    rois = torch.from_numpy(w.rois).to(dev)
+    rmax = int(np.max(np.diff(w.frame_roi_offsets)))
+    vx = mmbev.Voxelizer(w.num_points, rmax, w.max_voxels, w.num_frames, w.voxel_size,
+                         w.pc_range, w.max_pts_per_voxel, w.roi_margin, device=dev)
+    # the metric's numerator: in-ROI points, counted by the library's own
+    # per-point classification of these inputs (S1-S2), once, untimed
+    _, lin, _ = mmbev.classify_points(pts, w.sweep_offsets, tf, rois, w.roi_margin, w.voxel_size,
+                                      w.pc_range, w.frame_sweep_offsets, w.frame_roi_offsets,
+                                      workspace=vx.workspace)
+    n_in_roi = int((lin >= 0).sum().item())
+    del lin
+
+    stream = torch.cuda.current_stream(dev)
+    nstage = mmbev.NUM_STAGES
+    step_ev = [[torch.cuda.Event(enable_timing=True) for _ in range(nstage + 1)]
+               for _ in range(args.steps)]
+    for evs in step_ev:
+        for e in evs:
+            e.record(stream)  # materialise the events before handing them to the library
+    for _ in range(args.warmup):
+        vx(pts, w.sweep_offsets, tf, rois, w.frame_sweep_offsets, w.frame_roi_offsets)
+    torch.cuda.synchronize(dev)
+    status = vx.status()
+    if status != 0:
+        raise RuntimeError(f"device status {status:#x} after warm-up")
+    nvox = vx.out.nvox.cpu().numpy()
+    u_out = int(nvox.sum())
+
+    sampler = ClockSampler(dev.index if dev.index is not None else 0)
+    sampler.start()
+    time.sleep(0.3)
+    start = torch.cuda.Event(enable_timing=True)
+    end = torch.cuda.Event(enable_timing=True)
+    if world > 1:
+        dist.barrier()
+    torch.cuda.synchronize(dev)
+    start.record(stream)
+    for k in range(args.steps):
+        vx(pts, w.sweep_offsets, tf, rois, w.frame_sweep_offsets, w.frame_roi_offsets,
+           stage_events=step_ev[k])
+    end.record(stream)
+    torch.cuda.synchronize(dev)
+    if world > 1:
+        dist.barrier()
+    ms_total = start.elapsed_time(end)
+    clocks = sampler.stop()
+    status = vx.status()
+    if status != 0:
+        raise RuntimeError(f"device status {status:#x} after the timed steps")
+
+    stage_ms = np.zeros(nstage)
+    for evs in step_ev:
+        for s in range(nstage):
+            stage_ms[s] += evs[s].elapsed_time(evs[s + 1])
+    stage_ms /= args.steps
+    names = mmbev.stage_names()
+
+    # slowest rank decides
+    t_local = torch.tensor([ms_total], dtype=torch.float64, device=dev)
+    pts_local = torch.tensor([float(n_in_roi)], dtype=torch.float64, device=dev)
+    if world > 1:
+        dist.all_reduce(t_local, op=dist.ReduceOp.MAX)
+        dist.all_reduce(pts_local, op=dist.ReduceOp.SUM)
+    ms_max = float(t_local.item())
+    total_pts = float(pts_local.item())
+    ms_step = ms_max / args.steps
+    value = total_pts / (ms_step * 1e-3)
+
+    # end to end through the public API: pinned host inputs, H2D, the call,
+    # D2H of the per-frame counts and the kept rows
+    h_pts = torch.from_numpy(w.points).pin_memory()
+    h_tf = torch.from_numpy(w.sweep_tf).pin_memory()
+    h_rois = torch.from_numpy(w.rois).pin_memory()
+    d_pts = torch.empty_like(pts)
+    d_tf = torch.empty_like(tf)
+    d_rois = torch.empty_like(rois)
+    h_nvox = torch.empty(w.num_frames, dtype=torch.int32).pin_memory()
+    mv = w.max_voxels
+    h_feats = torch.empty((w.num_frames * mv, 5), dtype=torch.float32).pin_memory()
+    h_coords = torch.empty((w.num_frames * mv, 3), dtype=torch.int32).pin_memory()
+    h_counts = torch.empty(w.num_frames * mv, dtype=torch.int32).pin_memory()
+    e2e_steps = max(3, min(args.steps, 10))
+    d2h_bytes = 0
+
+    def e2e_step():
+        nonlocal d2h_bytes
+        d_pts.copy_(h_pts, non_blocking=True)
+        d_tf.copy_(h_tf, non_blocking=True)
+        d_rois.copy_(h_rois, non_blocking=True)
+        out = vx(d_pts, w.sweep_offsets, d_tf, d_rois, w.frame_sweep_offsets, w.frame_roi_offsets)
+        h_nvox.copy_(out.nvox, non_blocking=True)
+        torch.cuda.current_stream(dev).synchronize()
+        nb = 0
+        for f in range(w.num_frames):
+            n = int(h_nvox[f])
+            r0 = f * mv
+            h_feats[r0:r0 + n].copy_(out.feats[r0:r0 + n], non_blocking=True)
+            h_coords[r0:r0 + n].copy_(out.coords[r0:r0 + n], non_blocking=True)
+            h_counts[r0:r0 + n].copy_(out.counts[r0:r0 + n], non_blocking=True)
+            nb += n * BYTES_PER_VOXEL
+        torch.cuda.current_stream(dev).synchronize()
+        d2h_bytes = nb + 4 * w.num_frames
+
+    e2e_step()
+    if world > 1:
+        dist.barrier()
+    torch.cuda.synchronize(dev)
+    t0 = time.perf_counter()
+    for _ in range(e2e_steps):
+        e2e_step()
+    torch.cuda.synchronize(dev)
+    e2e_s = torch.tensor([time.perf_counter() - t0], dtype=torch.float64, device=dev)
+    if world > 1:
+        dist.all_reduce(e2e_s, op=dist.ReduceOp.MAX)
+    e2e_value = total_pts / (float(e2e_s.item()) / e2e_steps)
+    h2d_bytes = w.points.nbytes + w.sweep_tf.nbytes + w.rois.nbytes
+
+    if rank == 0:
+        peak, peak_kind = read_peaks()
+        dom = names.index(DOMINANT)
+        t_dom = stage_ms[dom] * 1e-3
+        achieved = BYTES_PER_POINT * w.num_points / t_dom / 1e9
+        path_bytes = BYTES_PER_POINT * w.num_points + BYTES_PER_VOXEL * u_out
+        line = {
+            "metric": METRIC, "value": value, "unit": "points/s", "n_gpus": world,
+            "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms_step,
+            "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f32",
+            "data": "synthetic", "config": workload_desc(w),
+            "us_per_frame": 1e3 * ms_step / w.num_frames,
+            "in_roi_points_per_gpu": n_in_roi, "voxels_out_per_gpu": u_out,
+            "path_hbm_gbs": path_bytes / (ms_step * 1e-3) / 1e9,
+            "path_frac_of_peak": path_bytes / (ms_step * 1e-3) / 1e9 / peak,
+            "stage_us": {n: round(1e3 * t, 2) for n, t in zip(names, stage_ms)},
+            "roofline": {"bound": "hbm", "kernel": DOMINANT, "achieved": achieved, "peak": peak,
+                         "peak_kind": peak_kind, "unit": "GB/s", "frac": achieved / peak,
+                         "traffic": profile_traffic()},
+            "clocks": clocks,
+            "e2e": {"value": e2e_value, "unit": "points/s", "h2d_bytes_per_step": h2d_bytes,
+                    "d2h_bytes_per_step": d2h_bytes, "steps": e2e_steps},
+            "gpu_launches": nstage * args.steps,
+        }
+        frames, secs = cpu_oracle_baseline(w)
+        pts_per_frame = n_in_roi / w.num_frames
+        line["cpu_baseline"] = {
+            "kind": "oracle", "value": frames * pts_per_frame / secs, "unit": "points/s",
+            "cores": 1, "sample": f"{frames} whole frames of this batch, single-threaded C "
+                                  f"oracle, {secs:.1f} s"}
+        print(json.dumps(line), flush=True)
+    if world > 1:
+        dist.destroy_process_group()
+    return 0
+
+
+def main():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=20)
+    ap.add_argument("--warmup", type=int, default=5)
+    ap.add_argument("--impl", default="gb300", choices=["gb300", "reference"])
+    args = ap.parse_args()
+    if args.impl == "reference":
+        return run_reference(args)
+    return run_gpu(args)
+
+
+if __name__ == "__main__":
+    sys.exit(main())

@@ -1,0 +1,245 @@
+/*
+ * mmbev.h -- C ABI of the GB300 (sm_103a) ROI-aware multi-sweep LiDAR
+ * voxelization library (MM-BEV, arXiv 2608.15437).
+ *
+ * The library computes, for one or many independent frames, the LiDAR hot
+ * path of the paper's sparse ROI-aware feature extraction:
+ *
+ *   S1  per-sweep ego-motion compensation, p' = R p + T          (Sec. IV-D, Eq. 6-7)
+ *   S2  range crop and inside-any-ROI test against criticality-ranked,
+ *       margin-grown rotated BEV boxes, then the voxel index        (Alg. 1; Eq. 1)
+ *   S3  voxel hash insert / dedup                                   (Alg. 1, "Voxelize")
+ *   S4  voxel cap and canonical (ascending linear index) order      (Sec. IV-F "hard
+ *                                                                    voxelization"; Sec. IV-C)
+ *   S5  mean features over the first K points of each voxel         (Alg. 1, "VoxelFeatureEncoder")
+ *
+ * Exact semantics (every GPU result equals this, bit for bit for integers
+ * and, by construction, for the fp32 features too):
+ *   - Point i of sweep s (sweep_offsets[s] <= i < sweep_offsets[s+1]) with
+ *     T = sweep_tf[s] (row-major 4x4, last row ignored, sweep frame -> current
+ *     frame): x' = ((T0*x + T1*y) + T2*z) + T3, likewise y' (T4..T7) and
+ *     z' (T8..T11); every fp32 product and sum rounded on its own (no FMA).
+ *   - Range: xmin <= x' < xmax, same for y and z (NaN and Inf fail).
+ *   - ROI r (cx, cy, w, l, yaw): c = (float)cos((double)yaw),
+ *     s = (float)sin((double)yaw), hl = 0.5f*l + margin, hw = 0.5f*w + margin,
+ *     dx = x'-cx, dy = y'-cy, u = dx*c + dy*s, v = dy*c - dx*s; inside iff
+ *     |u| <= hl and |v| <= hw. l runs along the heading, w across it, yaw is
+ *     counter-clockwise from +x. The point's rank is the first ROI (in array
+ *     order = criticality order) that contains it; a point in no ROI is
+ *     dropped (the out-of-ROI keep rate of Alg. 1 is zero).
+ *   - Voxel: c_a = (int)floorf((p'_a - min_a) / size_a), dropped if
+ *     c_a >= n_a, with n_a = (int)llround(((double)max_a - min_a) / size_a);
+ *     lin = (cz*ny + cy)*nx + cx.
+ *   - Each voxel keeps its K = max_pts_per_voxel points with the smallest
+ *     input index. If a frame has more than max_voxels voxels, the
+ *     max_voxels smallest by (minimum rank of the voxel's points, lin) are
+ *     kept. Kept voxels are written in ascending lin.
+ *   - feats = (x', y', z', intensity, dt) summed in fp32 over the kept points
+ *     in index order, divided once by (float)count.
+ *
+ * Execution model. Every call is asynchronous on `stream`: it validates its
+ * host arguments, enqueues a fixed sequence of kernels and returns. It never
+ * synchronizes, never allocates and reads its host arrays only during the
+ * call, so it can be captured in a CUDA graph. The caller owns every buffer.
+ *
+ * Two caller-owned device buffers carry the library's state:
+ *   - `table` (size from mmbev_table_size): the open-addressing voxel hash
+ *     table. It must be all zero before the first call (mmbev_table_clear)
+ *     and every successful call leaves it all zero again. Its capacity is
+ *     derived from table_bytes and max_pts_per_voxel alone, so one table can
+ *     serve calls of any shape. Calls that share a table must not overlap.
+ *   - `workspace` (size from mmbev_workspace_size): scratch with no state
+ *     across calls, except the device status word read by mmbev_get_status.
+ *
+ * Errors. A status below zero is returned before any launch when a host
+ * argument is invalid (MMBEV_EINVAL) or a buffer is too small
+ * (MMBEV_EWORKSPACE), and after a failed launch (MMBEV_ECUDA). Conditions
+ * only the device can see (hash table full, an internal wait that timed out)
+ * set bits in a device status word instead; no kernel traps or spins
+ * without bound. mmbev_get_status reads it. After a non-zero device status
+ * the outputs are invalid and the table must be cleared again.
+ */
+#ifndef MMBEV_H_
+#define MMBEV_H_
+
+#include <stddef.h>
+#include <stdint.h>
+#include <cuda_runtime_api.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+/* One BEV region of interest in the current ego frame: centre (cx, cy) in
+ * metres, width w (lateral) and length l (along the heading) in metres,
+ * heading yaw in radians, counter-clockwise from +x. This is the box of
+ * Eq. 1; the margin r of Eq. 1 is passed separately (roi_margin) and grows
+ * both half-extents. */
+typedef struct mmbev_roi {
+    float cx, cy, w, l, yaw;
+} mmbev_roi_t;
+
+typedef enum mmbev_status {
+    MMBEV_OK = 0,
+    MMBEV_EINVAL = -1,      /* invalid host argument; nothing launched */
+    MMBEV_ECUDA = -2,       /* a CUDA runtime call or launch failed */
+    MMBEV_EWORKSPACE = -3   /* table or workspace smaller than required */
+} mmbev_status_t;
+
+/* Device status bits (mmbev_get_status). */
+#define MMBEV_DEV_TABLE_FULL   0x1u  /* a voxel key found no free slot */
+#define MMBEV_DEV_WAIT_TIMEOUT 0x2u  /* an internal inter-block wait gave up */
+#define MMBEV_DEV_BOUNDS       0x4u  /* an internal index failed its bounds check */
+
+/* Limits of one call. */
+#define MMBEV_MAX_SWEEPS          2048
+#define MMBEV_MAX_FRAMES          1024
+#define MMBEV_MAX_ROIS_PER_FRAME  1024
+#define MMBEV_MAX_PTS_PER_VOXEL   64
+
+/*
+ * Bytes of hash table for calls of up to max_points points and
+ * max_pts_per_voxel points kept per voxel. The capacity is the power of two
+ * >= 2*max_points slots (load factor <= 1/2 whatever the inputs), each slot
+ * holding the voxel key, its minimum ROI rank and its K smallest point
+ * indices. Returns 0 for invalid arguments.
+ */
+size_t mmbev_table_size(int64_t max_points, int32_t max_pts_per_voxel);
+
+/*
+ * Bytes of scratch workspace for a call with up to max_points points,
+ * max_rois_per_frame ROIs in any frame, max_voxels kept voxels per frame and
+ * num_frames frames on the grid given by voxel_size[3] and range[6] (host
+ * arrays). Returns 0 for invalid arguments.
+ */
+size_t mmbev_workspace_size(int64_t max_points, int32_t max_rois_per_frame,
+                            int32_t max_voxels, int32_t num_frames,
+                            const float voxel_size[3], const float range[6]);
+
+/* Zero a hash table (device pointer, table_bytes bytes) on `stream`. */
+int mmbev_table_clear(void *table, size_t table_bytes, cudaStream_t stream);
+
+/*
+ * One frame (Alg. 1 on the union of n sweeps, Eq. 7).
+ *   points         device, float32 [N][5] (x, y, z, intensity, dt), 16-byte
+ *                  aligned; N = sweep_offsets[num_sweeps].
+ *   sweep_offsets  host, int64 [num_sweeps+1], sweep_offsets[0] = 0,
+ *                  nondecreasing; sweep s owns points [off[s], off[s+1]).
+ *   num_sweeps     0 <= num_sweeps <= MMBEV_MAX_SWEEPS.
+ *   sweep_tf       device, float32 [num_sweeps][16], row-major 4x4 mapping
+ *                  sweep s into the current frame (Eq. 6).
+ *   rois           device, mmbev_roi_t [num_rois], most critical first.
+ *   num_rois       0 <= num_rois <= MMBEV_MAX_ROIS_PER_FRAME; 0 gives no voxels.
+ *   roi_margin     r of Eq. 1, >= 0 and finite, metres.
+ *   voxel_size     host, float [3], > 0.
+ *   range          host, float [6] (xmin, ymin, zmin, xmax, ymax, zmax), max > min;
+ *                  nx*ny*nz must stay below 2^32.
+ *   max_pts_per_voxel  K, 1 <= K <= MMBEV_MAX_PTS_PER_VOXEL.
+ *   max_voxels     >= 0.
+ *   out_feats      device, float32 [max_voxels][5]
+ *   out_coords     device, int32 [max_voxels][3] as (z, y, x)
+ *   out_counts     device, int32 [max_voxels], min(points in voxel, K)
+ *   out_nvox       device, int32 scalar, min(voxels, max_voxels)
+ * Rows at and beyond *out_nvox are left untouched.
+ */
+int mmbev_voxelize_roi(const float *points, const int64_t *sweep_offsets,
+                       int32_t num_sweeps, const float *sweep_tf,
+                       const mmbev_roi_t *rois, int32_t num_rois, float roi_margin,
+                       const float voxel_size[3], const float range[6],
+                       int32_t max_pts_per_voxel, int32_t max_voxels,
+                       float *out_feats, int32_t *out_coords, int32_t *out_counts,
+                       int32_t *out_nvox, void *table, size_t table_bytes,
+                       void *workspace, size_t workspace_bytes, cudaStream_t stream);
+
+/*
+ * num_frames independent frames in one call; the result equals num_frames
+ * separate mmbev_voxelize_roi calls.
+ *   frame_sweep_offsets  host, int32 [num_frames+1]: frame f owns sweeps
+ *                        [fso[f], fso[f+1]); fso[0] = 0, fso[F] = num_sweeps.
+ *   frame_roi_offsets    host, int32 [num_frames+1]: frame f owns ROIs
+ *                        [fro[f], fro[f+1]) (its own criticality order);
+ *                        fro[0] = 0, fro[F] = num_rois.
+ *   Outputs are per frame with a stride of max_voxels rows: frame f's voxel v
+ *   is row f*max_voxels + v; out_nvox is int32 [num_frames].
+ * Other arguments as for mmbev_voxelize_roi; num_rois counts all frames.
+ */
+int mmbev_voxelize_roi_batched(const float *points, const int64_t *sweep_offsets,
+                               int32_t num_sweeps, const float *sweep_tf,
+                               const mmbev_roi_t *rois, int32_t num_rois,
+                               float roi_margin, const float voxel_size[3],
+                               const float range[6], int32_t max_pts_per_voxel,
+                               int32_t max_voxels, int32_t num_frames,
+                               const int32_t *frame_sweep_offsets,
+                               const int32_t *frame_roi_offsets,
+                               float *out_feats, int32_t *out_coords,
+                               int32_t *out_counts, int32_t *out_nvox,
+                               void *table, size_t table_bytes,
+                               void *workspace, size_t workspace_bytes,
+                               cudaStream_t stream);
+
+/*
+ * Steps S1-S2 alone, per point (Eq. 6; Alg. 1 inside-ROI test; voxel index),
+ * for the same inputs as mmbev_voxelize_roi_batched:
+ *   out_xyz   device, float32 [N][3], compensated coordinates of every point
+ *   out_lin   device, int64 [N], frame-local voxel linear index, -1 if dropped
+ *   out_rank  device, int32 [N], ROI rank, -1 if dropped
+ * Needs only the workspace (no table).
+ */
+int mmbev_classify_points(const float *points, const int64_t *sweep_offsets,
+                          int32_t num_sweeps, const float *sweep_tf,
+                          const mmbev_roi_t *rois, int32_t num_rois, float roi_margin,
+                          const float voxel_size[3], const float range[6],
+                          int32_t num_frames, const int32_t *frame_sweep_offsets,
+                          const int32_t *frame_roi_offsets, float *out_xyz,
+                          int64_t *out_lin, int32_t *out_rank,
+                          void *workspace, size_t workspace_bytes, cudaStream_t stream);
+
+/*
+ * Copy the device status word of the last call that used `workspace` into
+ * *host_status (0 = no device-side error, else MMBEV_DEV_* bits). This call
+ * synchronizes `stream`.
+ */
+int mmbev_get_status(const void *workspace, size_t workspace_bytes,
+                     uint32_t *host_status, cudaStream_t stream);
+
+/*
+ * Execution options for mmbev_voxelize_roi_batched_ex.
+ *   stage_events      NULL, or MMBEV_NUM_STAGES+1 events created by the
+ *                     caller: event k is recorded on `stream` before stage k
+ *                     and the last one after the final stage, so the caller
+ *                     can time each kernel with cudaEventElapsedTime.
+ *   table_log2_override  0, or log2 of the slot count to use instead of the
+ *                     largest power of two that fits table_bytes (a smaller
+ *                     table; a full table sets MMBEV_DEV_TABLE_FULL).
+ */
+#define MMBEV_NUM_STAGES 9
+typedef struct mmbev_exec_opts {
+    cudaEvent_t *stage_events;
+    int32_t table_log2_override;
+} mmbev_exec_opts_t;
+
+int mmbev_voxelize_roi_batched_ex(const float *points, const int64_t *sweep_offsets,
+                                  int32_t num_sweeps, const float *sweep_tf,
+                                  const mmbev_roi_t *rois, int32_t num_rois,
+                                  float roi_margin, const float voxel_size[3],
+                                  const float range[6], int32_t max_pts_per_voxel,
+                                  int32_t max_voxels, int32_t num_frames,
+                                  const int32_t *frame_sweep_offsets,
+                                  const int32_t *frame_roi_offsets,
+                                  float *out_feats, int32_t *out_coords,
+                                  int32_t *out_counts, int32_t *out_nvox,
+                                  void *table, size_t table_bytes,
+                                  void *workspace, size_t workspace_bytes,
+                                  cudaStream_t stream, const mmbev_exec_opts_t *opts);
+
+/* Names of the stages timed by stage_events, for reports. */
+const char *mmbev_stage_name(int32_t stage);
+
+/* Library version string. */
+const char *mmbev_version(void);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* MMBEV_H_ */

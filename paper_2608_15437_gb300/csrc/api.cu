@@ -1,0 +1,410 @@
+// Host side of libmmbev: argument validation, workspace layout, and the
+// fixed, stream-ordered launch sequence of the path. Nothing here allocates,
+// synchronizes or keeps state across calls.
+#include <cmath>
+#include <cstring>
+#include <atomic>
+
+#include "mmbev_internal.cuh"
+
+namespace mmbev {
+namespace {
+
+constexpr size_t kAlign = 256;
+
+size_t align_up(size_t x, size_t a) { return (x + a - 1) / a * a; }
+
+struct Grid {
+    uint32_t dims[3];
+    uint64_t cells;
+};
+
+bool make_grid(const float* vs, const float* range, Grid* g) {
+    if (!vs || !range) return false;
+    uint64_t cells = 1;
+    for (int a = 0; a < 3; ++a) {
+        if (!std::isfinite(vs[a]) || !(vs[a] > 0.0f)) return false;
+        if (!std::isfinite(range[a]) || !std::isfinite(range[a + 3])) return false;
+        if (!(range[a + 3] > range[a])) return false;
+        const double n = std::llround(((double)range[a + 3] - (double)range[a]) / (double)vs[a]);
+        if (!(n >= 1.0) || n > 4294967295.0) return false;
+        g->dims[a] = (uint32_t)n;
+        cells *= (uint64_t)n;
+        if (cells > 0xFFFFFFFFull) return false;
+    }
+    g->cells = cells;
+    return true;
+}
+
+int bucket_log2_for(uint64_t cells) {
+    int lb = 5;
+    while (lb < kBucketLog2Max && (1ull << lb) < cells) ++lb;
+    return lb;
+}
+
+int mask_words_for(int32_t max_rois_frame) {
+    const int w = (max_rois_frame + 31) / 32;
+    return w < 1 ? 1 : w;
+}
+
+int coarse_for(int mask_words) {
+    if (mask_words <= 1) return 128;
+    if (mask_words <= 13) return 64;
+    return 32;
+}
+
+uint32_t slot_stride_for(int32_t K) { return 16u + 4u * (uint32_t)((K + 3) / 4 * 4); }
+
+// Byte offsets of every workspace array for one call shape.
+struct Layout {
+    size_t hdr, sweep_off, sweep_frame, fso, fro, roi_prep, masks, hist, frame_u, finfo;
+    size_t bcnt, scan_agg, scan_inc, scan_flag, occ, d_bucket, d_pos, items, vid_slot;
+    size_t total;
+    uint32_t num_buckets, buckets_per_frame, scan_tiles;
+    int bucket_log2, mask_words, coarse;
+};
+
+Layout make_layout(int64_t max_points, int64_t rois_total, int32_t max_rois_frame,
+                   int32_t max_voxels, int32_t num_frames, const Grid& g) {
+    Layout L{};
+    L.bucket_log2 = bucket_log2_for(g.cells);
+    L.buckets_per_frame = (uint32_t)((g.cells + (1ull << L.bucket_log2) - 1) >> L.bucket_log2);
+    L.num_buckets = L.buckets_per_frame * (uint32_t)num_frames;
+    L.scan_tiles = (uint32_t)(((uint64_t)L.num_buckets + 1 + kScanTile - 1) / kScanTile);
+    L.mask_words = mask_words_for(max_rois_frame);
+    L.coarse = coarse_for(L.mask_words);
+    const size_t F = (size_t)num_frames, R = (size_t)(rois_total > 0 ? rois_total : 1);
+    const size_t U = (size_t)(max_points > 0 ? max_points : 1);
+    size_t o = 0;
+    auto take = [&](size_t bytes) { const size_t at = o; o = align_up(o + bytes, kAlign); return at; };
+    L.hdr = take(sizeof(Header));
+    L.sweep_off = take(sizeof(int64_t) * (kMaxSweeps + 1));
+    L.sweep_frame = take(sizeof(int32_t) * kMaxSweeps);
+    L.fso = take(sizeof(int32_t) * (F + 1));
+    L.fro = take(sizeof(int32_t) * (F + 1));
+    L.roi_prep = take(sizeof(RoiPrep) * R);
+    L.masks = take(sizeof(uint32_t) * F * L.coarse * L.coarse * L.mask_words);
+    L.hist = take(sizeof(uint32_t) * R);
+    L.frame_u = take(sizeof(uint32_t) * F);
+    L.finfo = take(sizeof(FrameInfo) * F);
+    L.bcnt = take(sizeof(unsigned long long) * ((size_t)L.num_buckets + 1));
+    L.scan_agg = take(sizeof(unsigned long long) * L.scan_tiles);
+    L.scan_inc = take(sizeof(unsigned long long) * L.scan_tiles);
+    L.scan_flag = take(sizeof(uint32_t) * L.scan_tiles);
+    L.occ = take(sizeof(uint32_t) * U);
+    L.d_bucket = take(sizeof(uint32_t) * U);
+    L.d_pos = take(sizeof(uint32_t) * U);
+    L.items = take(sizeof(uint32_t) * U);
+    L.vid_slot = take(sizeof(uint32_t) * (F * (size_t)(max_voxels > 0 ? max_voxels : 1)));
+    L.total = o;
+    return L;
+}
+
+int num_sms() {
+    static std::atomic<int> cache[64];
+    int dev = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess) return 0;
+    if (dev >= 0 && dev < 64) {
+        const int c = cache[dev].load(std::memory_order_relaxed);
+        if (c > 0) return c;
+    }
+    int n = 0;
+    if (cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess) return 0;
+    if (dev >= 0 && dev < 64) cache[dev].store(n, std::memory_order_relaxed);
+    return n;
+}
+
+// Validation shared by the full path and the classify-only path. Fills the
+// call-shape fields of Params and the host descriptor.
+int validate_common(const float* points, const int64_t* sweep_offsets, int32_t num_sweeps,
+                    const float* sweep_tf, const mmbev_roi_t* rois, int32_t num_rois,
+                    float roi_margin, const float* voxel_size, const float* range,
+                    int32_t num_frames, const int32_t* fso, const int32_t* fro,
+                    Params* p, HostDesc* d, Grid* g, int32_t* max_rois_frame) {
+    if (num_sweeps < 0 || num_sweeps > kMaxSweeps) return MMBEV_EINVAL;
+    if (num_frames < 1 || num_frames > kMaxFrames) return MMBEV_EINVAL;
+    if (num_rois < 0) return MMBEV_EINVAL;
+    if (!sweep_offsets || !fso || !fro) return MMBEV_EINVAL;
+    if (!make_grid(voxel_size, range, g)) return MMBEV_EINVAL;
+    if (!std::isfinite(roi_margin) || !(roi_margin >= 0.0f)) return MMBEV_EINVAL;
+    if (sweep_offsets[0] != 0) return MMBEV_EINVAL;
+    for (int s = 0; s < num_sweeps; ++s)
+        if (sweep_offsets[s + 1] < sweep_offsets[s]) return MMBEV_EINVAL;
+    const int64_t n = sweep_offsets[num_sweeps];
+    if (n < 0 || n > 0xFFFFFFFEll) return MMBEV_EINVAL;
+    if (fso[0] != 0 || fso[num_frames] != num_sweeps) return MMBEV_EINVAL;
+    if (fro[0] != 0 || fro[num_frames] != num_rois) return MMBEV_EINVAL;
+    int32_t rmax = 0;
+    for (int f = 0; f < num_frames; ++f) {
+        if (fso[f + 1] < fso[f] || fro[f + 1] < fro[f]) return MMBEV_EINVAL;
+        const int32_t rn = fro[f + 1] - fro[f];
+        if (rn > kMaxRoisPerFrame) return MMBEV_EINVAL;
+        if (rn > rmax) rmax = rn;
+    }
+    if (n > 0 && (!points || (reinterpret_cast<uintptr_t>(points) & 15u))) return MMBEV_EINVAL;
+    if (num_sweeps > 0 && !sweep_tf) return MMBEV_EINVAL;
+    if (num_rois > 0 && !rois) return MMBEV_EINVAL;
+
+    std::memset(d, 0, sizeof(HostDesc));
+    for (int s = 0; s <= num_sweeps; ++s) d->sweep_off[s] = sweep_offsets[s];
+    for (int f = 0; f <= num_frames; ++f) {
+        d->frame_sweep_off[f] = fso[f];
+        d->frame_roi_off[f] = fro[f];
+    }
+    std::memset(p, 0, sizeof(Params));
+    p->points = points;
+    p->sweep_tf = sweep_tf;
+    p->rois = rois;
+    p->num_points = n;
+    p->num_sweeps = num_sweeps;
+    p->num_frames = num_frames;
+    p->num_rois = num_rois;
+    p->margin = roi_margin;
+    for (int a = 0; a < 3; ++a) {
+        p->vs[a] = voxel_size[a];
+        p->rmin[a] = range[a];
+        p->rmax[a] = range[a + 3];
+        p->dims[a] = g->dims[a];
+    }
+    p->cells = (uint32_t)g->cells;
+    *max_rois_frame = rmax;
+    return MMBEV_OK;
+}
+
+void bind_layout(Params* p, const Layout& L, uint8_t* ws) {
+    p->hdr = reinterpret_cast<Header*>(ws + L.hdr);
+    p->sweep_off = reinterpret_cast<int64_t*>(ws + L.sweep_off);
+    p->sweep_frame = reinterpret_cast<int32_t*>(ws + L.sweep_frame);
+    p->frame_sweep_off = reinterpret_cast<int32_t*>(ws + L.fso);
+    p->frame_roi_off = reinterpret_cast<int32_t*>(ws + L.fro);
+    p->roi_prep = reinterpret_cast<RoiPrep*>(ws + L.roi_prep);
+    p->masks = reinterpret_cast<uint32_t*>(ws + L.masks);
+    p->hist = reinterpret_cast<uint32_t*>(ws + L.hist);
+    p->frame_u = reinterpret_cast<uint32_t*>(ws + L.frame_u);
+    p->finfo = reinterpret_cast<FrameInfo*>(ws + L.finfo);
+    p->bcnt = reinterpret_cast<unsigned long long*>(ws + L.bcnt);
+    p->scan_agg = reinterpret_cast<unsigned long long*>(ws + L.scan_agg);
+    p->scan_inc = reinterpret_cast<unsigned long long*>(ws + L.scan_inc);
+    p->scan_flag = reinterpret_cast<uint32_t*>(ws + L.scan_flag);
+    p->occ = reinterpret_cast<uint32_t*>(ws + L.occ);
+    p->d_bucket = reinterpret_cast<uint32_t*>(ws + L.d_bucket);
+    p->d_pos = reinterpret_cast<uint32_t*>(ws + L.d_pos);
+    p->items = reinterpret_cast<uint32_t*>(ws + L.items);
+    p->vid_slot = reinterpret_cast<uint32_t*>(ws + L.vid_slot);
+    p->occ_cap = (uint32_t)(p->num_points > 0 ? p->num_points : 1);
+    p->mask_words = L.mask_words;
+    p->coarse = L.coarse;
+    p->coarse_inv[0] = (float)((double)L.coarse / ((double)p->rmax[0] - (double)p->rmin[0]));
+    p->coarse_inv[1] = (float)((double)L.coarse / ((double)p->rmax[1] - (double)p->rmin[1]));
+    p->bucket_log2 = L.bucket_log2;
+    p->buckets_per_frame = L.buckets_per_frame;
+    p->num_buckets = L.num_buckets;
+    p->scan_tiles = L.scan_tiles;
+}
+
+#define MMBEV_TRY(expr)                                   \
+    do {                                                  \
+        if ((expr) != cudaSuccess) return MMBEV_ECUDA;    \
+    } while (0)
+
+const char* const kStageNames[MMBEV_NUM_STAGES] = {
+    "prep", "points", "census", "frames", "capped_census", "scan", "scatter", "rank", "finalize"};
+
+}  // namespace
+}  // namespace mmbev
+
+using namespace mmbev;
+
+extern "C" {
+
+size_t mmbev_table_size(int64_t max_points, int32_t max_pts_per_voxel) {
+    if (max_points < 0 || max_points > 0xFFFFFFFEll) return 0;
+    if (max_pts_per_voxel < 1 || max_pts_per_voxel > kMaxK) return 0;
+    uint64_t h = 1024;
+    while (h < 2ull * (uint64_t)max_points) h <<= 1;
+    if (h > (1ull << 31)) return 0;
+    return (size_t)h * slot_stride_for(max_pts_per_voxel);
+}
+
+size_t mmbev_workspace_size(int64_t max_points, int32_t max_rois_per_frame, int32_t max_voxels,
+                            int32_t num_frames, const float voxel_size[3], const float range[6]) {
+    Grid g;
+    if (max_points < 0 || max_rois_per_frame < 0 || max_rois_per_frame > kMaxRoisPerFrame ||
+        max_voxels < 0 || num_frames < 1 || num_frames > kMaxFrames)
+        return 0;
+    if (!make_grid(voxel_size, range, &g)) return 0;
+    const Layout L = make_layout(max_points, (int64_t)max_rois_per_frame * num_frames,
+                                 max_rois_per_frame, max_voxels, num_frames, g);
+    return L.total;
+}
+
+int mmbev_table_clear(void* table, size_t table_bytes, cudaStream_t stream) {
+    if (!table && table_bytes) return MMBEV_EINVAL;
+    if (reinterpret_cast<uintptr_t>(table) & 15u) return MMBEV_EINVAL;
+    return launch_zero(table, table_bytes, stream) == cudaSuccess ? MMBEV_OK : MMBEV_ECUDA;
+}
+
+int mmbev_voxelize_roi_batched_ex(const float* points, const int64_t* sweep_offsets,
+                                  int32_t num_sweeps, const float* sweep_tf,
+                                  const mmbev_roi_t* rois, int32_t num_rois, float roi_margin,
+                                  const float voxel_size[3], const float range[6],
+                                  int32_t max_pts_per_voxel, int32_t max_voxels,
+                                  int32_t num_frames, const int32_t* frame_sweep_offsets,
+                                  const int32_t* frame_roi_offsets, float* out_feats,
+                                  int32_t* out_coords, int32_t* out_counts, int32_t* out_nvox,
+                                  void* table, size_t table_bytes, void* workspace,
+                                  size_t workspace_bytes, cudaStream_t stream,
+                                  const mmbev_exec_opts_t* opts) {
+    HostDesc desc;  // ~25 KB; consumed by the prep launch's parameter copy
+    Params p;
+    Grid g;
+    int32_t rmax = 0;
+    if (max_pts_per_voxel < 1 || max_pts_per_voxel > kMaxK || max_voxels < 0) return MMBEV_EINVAL;
+    if ((int64_t)max_voxels * num_frames > 0x7FFFFFFFll) return MMBEV_EINVAL;
+    if (!out_nvox) return MMBEV_EINVAL;
+    if (max_voxels > 0 && (!out_feats || !out_coords || !out_counts)) return MMBEV_EINVAL;
+    if (!workspace || (reinterpret_cast<uintptr_t>(workspace) & (kAlign - 1))) return MMBEV_EINVAL;
+    if (!table || (reinterpret_cast<uintptr_t>(table) & 15u)) return MMBEV_EINVAL;
+    int rc = validate_common(points, sweep_offsets, num_sweeps, sweep_tf, rois, num_rois,
+                             roi_margin, voxel_size, range, num_frames, frame_sweep_offsets,
+                             frame_roi_offsets, &p, &desc, &g, &rmax);
+    if (rc != MMBEV_OK) return rc;
+    const Layout L = make_layout(p.num_points, num_rois, rmax, max_voxels, num_frames, g);
+    if (L.total > workspace_bytes) return MMBEV_EWORKSPACE;
+    bind_layout(&p, L, static_cast<uint8_t*>(workspace));
+    p.K = max_pts_per_voxel;
+    p.max_voxels = max_voxels;
+    p.out_feats = out_feats;
+    p.out_coords = out_coords;
+    p.out_counts = out_counts;
+    p.out_nvox = out_nvox;
+    // Hash table: the largest power of two of slots that fits, unless overridden.
+    p.slot_stride = slot_stride_for(max_pts_per_voxel);
+    const uint64_t fit = table_bytes / p.slot_stride;
+    uint32_t lg = 0;
+    while (lg < 31 && (2ull << lg) <= fit) ++lg;
+    if (opts && opts->table_log2_override > 0) {
+        if (opts->table_log2_override > 31 ||
+            (1ull << opts->table_log2_override) > fit) {
+            return MMBEV_EWORKSPACE;
+        }
+        lg = (uint32_t)opts->table_log2_override;
+    } else if ((1ull << lg) > fit || (1ull << lg) < 2ull * (uint64_t)p.num_points) {
+        return MMBEV_EWORKSPACE;
+    }
+    p.table = static_cast<uint8_t*>(table);
+    p.table_log2 = lg;
+
+    const int sms = num_sms();
+    if (sms <= 0) return MMBEV_ECUDA;
+    cudaEvent_t* ev = opts ? opts->stage_events : nullptr;
+    int stage = 0;
+    auto mark = [&]() -> cudaError_t {
+        return ev ? cudaEventRecord(ev[stage++], stream) : cudaSuccess;
+    };
+    cudaError_t e = cudaSuccess;
+    do {
+        if ((e = mark()) != cudaSuccess) break;
+        if ((e = launch_prep(p, desc, stream)) != cudaSuccess) break;
+        if ((e = mark()) != cudaSuccess) break;
+        if ((e = launch_points(p, false, stream)) != cudaSuccess) break;
+        if ((e = mark()) != cudaSuccess) break;
+        if ((e = launch_census(p, sms, stream)) != cudaSuccess) break;
+        if ((e = mark()) != cudaSuccess) break;
+        if ((e = launch_frames(p, stream)) != cudaSuccess) break;
+        if ((e = mark()) != cudaSuccess) break;
+        if ((e = launch_capped_census(p, sms, stream)) != cudaSuccess) break;
+        if ((e = mark()) != cudaSuccess) break;
+        if ((e = launch_scan(p, stream)) != cudaSuccess) break;
+        if ((e = mark()) != cudaSuccess) break;
+        if ((e = launch_scatter(p, sms, stream)) != cudaSuccess) break;
+        if ((e = mark()) != cudaSuccess) break;
+        if ((e = launch_rank(p, sms, stream)) != cudaSuccess) break;
+        if ((e = mark()) != cudaSuccess) break;
+        if ((e = launch_finalize(p, sms, stream)) != cudaSuccess) break;
+        if ((e = mark()) != cudaSuccess) break;
+    } while (0);
+    return e == cudaSuccess ? MMBEV_OK : MMBEV_ECUDA;
+}
+
+int mmbev_voxelize_roi_batched(const float* points, const int64_t* sweep_offsets,
+                               int32_t num_sweeps, const float* sweep_tf,
+                               const mmbev_roi_t* rois, int32_t num_rois, float roi_margin,
+                               const float voxel_size[3], const float range[6],
+                               int32_t max_pts_per_voxel, int32_t max_voxels, int32_t num_frames,
+                               const int32_t* frame_sweep_offsets,
+                               const int32_t* frame_roi_offsets, float* out_feats,
+                               int32_t* out_coords, int32_t* out_counts, int32_t* out_nvox,
+                               void* table, size_t table_bytes, void* workspace,
+                               size_t workspace_bytes, cudaStream_t stream) {
+    return mmbev_voxelize_roi_batched_ex(points, sweep_offsets, num_sweeps, sweep_tf, rois,
+                                         num_rois, roi_margin, voxel_size, range,
+                                         max_pts_per_voxel, max_voxels, num_frames,
+                                         frame_sweep_offsets, frame_roi_offsets, out_feats,
+                                         out_coords, out_counts, out_nvox, table, table_bytes,
+                                         workspace, workspace_bytes, stream, nullptr);
+}
+
+int mmbev_voxelize_roi(const float* points, const int64_t* sweep_offsets, int32_t num_sweeps,
+                       const float* sweep_tf, const mmbev_roi_t* rois, int32_t num_rois,
+                       float roi_margin, const float voxel_size[3], const float range[6],
+                       int32_t max_pts_per_voxel, int32_t max_voxels, float* out_feats,
+                       int32_t* out_coords, int32_t* out_counts, int32_t* out_nvox, void* table,
+                       size_t table_bytes, void* workspace, size_t workspace_bytes,
+                       cudaStream_t stream) {
+    const int32_t fso[2] = {0, num_sweeps};
+    const int32_t fro[2] = {0, num_rois};
+    return mmbev_voxelize_roi_batched_ex(points, sweep_offsets, num_sweeps, sweep_tf, rois,
+                                         num_rois, roi_margin, voxel_size, range,
+                                         max_pts_per_voxel, max_voxels, 1, fso, fro, out_feats,
+                                         out_coords, out_counts, out_nvox, table, table_bytes,
+                                         workspace, workspace_bytes, stream, nullptr);
+}
+
+int mmbev_classify_points(const float* points, const int64_t* sweep_offsets, int32_t num_sweeps,
+                          const float* sweep_tf, const mmbev_roi_t* rois, int32_t num_rois,
+                          float roi_margin, const float voxel_size[3], const float range[6],
+                          int32_t num_frames, const int32_t* frame_sweep_offsets,
+                          const int32_t* frame_roi_offsets, float* out_xyz, int64_t* out_lin,
+                          int32_t* out_rank, void* workspace, size_t workspace_bytes,
+                          cudaStream_t stream) {
+    HostDesc desc;
+    Params p;
+    Grid g;
+    int32_t rmax = 0;
+    if (!workspace || (reinterpret_cast<uintptr_t>(workspace) & (kAlign - 1))) return MMBEV_EINVAL;
+    int rc = validate_common(points, sweep_offsets, num_sweeps, sweep_tf, rois, num_rois,
+                             roi_margin, voxel_size, range, num_frames, frame_sweep_offsets,
+                             frame_roi_offsets, &p, &desc, &g, &rmax);
+    if (rc == MMBEV_OK && p.num_points > 0 && (!out_xyz || !out_lin || !out_rank)) rc = MMBEV_EINVAL;
+    if (rc != MMBEV_OK) return rc;
+    const Layout L = make_layout(p.num_points, num_rois, rmax, 0, num_frames, g);
+    if (L.total > workspace_bytes) return MMBEV_EWORKSPACE;
+    bind_layout(&p, L, static_cast<uint8_t*>(workspace));
+    p.K = 1;
+    p.cls_xyz = out_xyz;
+    p.cls_lin = out_lin;
+    p.cls_rank = out_rank;
+    cudaError_t e = launch_prep(p, desc, stream);
+    if (e == cudaSuccess) e = launch_points(p, true, stream);
+    return e == cudaSuccess ? MMBEV_OK : MMBEV_ECUDA;
+}
+
+int mmbev_get_status(const void* workspace, size_t workspace_bytes, uint32_t* host_status,
+                     cudaStream_t stream) {
+    if (!workspace || !host_status || workspace_bytes < sizeof(Header)) return MMBEV_EINVAL;
+    const Header* hdr = static_cast<const Header*>(workspace);
+    MMBEV_TRY(cudaMemcpyAsync(host_status, &hdr->status, sizeof(uint32_t),
+                              cudaMemcpyDeviceToHost, stream));
+    MMBEV_TRY(cudaStreamSynchronize(stream));
+    return MMBEV_OK;
+}
+
+const char* mmbev_stage_name(int32_t stage) {
+    if (stage < 0 || stage >= MMBEV_NUM_STAGES) return "";
+    return kStageNames[stage];
+}
+
+const char* mmbev_version(void) { return "mmbev 0.1.0 (sm_103a)"; }
+
+}  // extern "C"

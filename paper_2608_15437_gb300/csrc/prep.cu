@@ -1,0 +1,168 @@
+// Stage 0: per-call preparation.
+//
+// One block per frame derives the prepared ROI table (cos/sin of yaw in
+// double, rounded to fp32; half-extents grown by the margin, Eq. 1) and the
+// frame's coarse BEV candidate mask: for every coarse cell, a bit per ROI
+// whose margin-grown box may touch the cell. The mask is conservative (the
+// exact per-point test of Alg. 1 follows), so it only prunes work. The other
+// blocks copy the host offsets into the workspace and zero the per-call
+// counters.
+#include <atomic>
+#include <cmath>
+
+#include "mmbev_internal.cuh"
+
+namespace mmbev {
+namespace {
+
+constexpr int kPrepThreads = 512;
+constexpr int kZeroBlocks = 64;
+
+// Inclusive cell range of one ROI's padded bounding box, or an empty range.
+struct CellRange { int16_t i0, i1, j0, j1; };
+
+__device__ CellRange roi_cells(const Params& p, const RoiPrep& r) {
+    CellRange cr{1, 0, 1, 0};
+    const double c = r.c, s = r.s, hl = r.hl, hw = r.hw;
+    const double cx = r.cx, cy = r.cy;
+    // NaN anywhere makes the exact test false for every point: no cells.
+    if (isnan(c) || isnan(s) || isnan(hl) || isnan(hw) || isnan(cx) || isnan(cy)) return cr;
+    const double ex = fabs(c) * hl + fabs(s) * hw;
+    const double ey = fabs(s) * hl + fabs(c) * hw;
+    const double g = p.coarse;
+    double x0 = cx - ex, x1 = cx + ex, y0 = cy - ey, y1 = cy + ey;
+    if (!(isfinite(x0) && isfinite(x1) && isfinite(y0) && isfinite(y1))) {
+        // Infinite extents or centre: mark the whole grid (conservative).
+        cr.i0 = 0; cr.i1 = (int16_t)(p.coarse - 1); cr.j0 = 0; cr.j1 = (int16_t)(p.coarse - 1);
+        return cr;
+    }
+    // Pad well beyond the fp32 rounding of the exact test and of the cell
+    // index a point computes for itself.
+    const double span = fabs((double)p.rmin[0]) + fabs((double)p.rmax[0]) +
+                        fabs((double)p.rmin[1]) + fabs((double)p.rmax[1]);
+    const double pad = 0.05 + 1e-4 * (fabs(cx) + fabs(cy) + fabs(ex) + fabs(ey) + span);
+    x0 -= pad; x1 += pad; y0 -= pad; y1 += pad;
+    const double gx = (p.rmax[0] - (double)p.rmin[0]) / g;
+    const double gy = (p.rmax[1] - (double)p.rmin[1]) / g;
+    double fi0 = floor((x0 - p.rmin[0]) / gx), fi1 = floor((x1 - p.rmin[0]) / gx);
+    double fj0 = floor((y0 - p.rmin[1]) / gy), fj1 = floor((y1 - p.rmin[1]) / gy);
+    if (fi1 < 0 || fj1 < 0 || fi0 > g - 1 || fj0 > g - 1 || x1 < x0 || y1 < y0) return cr;
+    cr.i0 = (int16_t)fmax(fi0, 0.0); cr.i1 = (int16_t)fmin(fi1, g - 1);
+    cr.j0 = (int16_t)fmax(fj0, 0.0); cr.j1 = (int16_t)fmin(fj1, g - 1);
+    return cr;
+}
+
+__global__ void __launch_bounds__(kPrepThreads)
+k_prep(Params p, const __grid_constant__ HostDesc d) {
+    extern __shared__ uint32_t s_mask[];  // [coarse^2 * mask_words] for frame blocks
+    const int t = threadIdx.x;
+    if ((int)blockIdx.x < p.num_frames) {
+        const int f = blockIdx.x;
+        const int r0 = d.frame_roi_off[f];
+        const int rn = d.frame_roi_off[f + 1] - r0;
+        const int g2 = p.coarse * p.coarse;
+        const int W = p.mask_words;
+        for (int i = t; i < g2 * W; i += blockDim.x) s_mask[i] = 0u;
+        __syncthreads();
+        // One warp per ROI: prepare it, then set its bit in every cell of its
+        // padded bounding box.
+        const int warp = t >> 5, lane = t & 31, nwarps = blockDim.x >> 5;
+        for (int r = warp; r < rn; r += nwarps) {
+            const mmbev_roi_t in = p.rois[r0 + r];
+            RoiPrep rp;
+            rp.cx = in.cx;
+            rp.cy = in.cy;
+            rp.c = (float)cos((double)in.yaw);
+            rp.s = (float)sin((double)in.yaw);
+            rp.hl = __fadd_rn(__fmul_rn(0.5f, in.l), p.margin);
+            rp.hw = __fadd_rn(__fmul_rn(0.5f, in.w), p.margin);
+            rp.pad0 = 0.f;
+            rp.pad1 = 0.f;
+            if (lane == 0) p.roi_prep[r0 + r] = rp;
+            const CellRange cr = roi_cells(p, rp);
+            const int ni = cr.i1 - cr.i0 + 1, nj = cr.j1 - cr.j0 + 1;
+            if (ni <= 0 || nj <= 0) continue;
+            const uint32_t bit = 1u << (r & 31);
+            const int w = r >> 5;
+            for (int k = lane; k < ni * nj; k += 32) {
+                const int i = cr.i0 + k % ni, j = cr.j0 + k / ni;
+                atomicOr(&s_mask[(j * p.coarse + i) * W + w], bit);
+            }
+        }
+        __syncthreads();
+        uint32_t* gm = p.masks + (size_t)f * g2 * W;
+        for (int i = t; i < g2 * W; i += blockDim.x) gm[i] = s_mask[i];
+        return;
+    }
+    // Housekeeping blocks: grid-stride over the zero/copy work.
+    const int zb = blockIdx.x - p.num_frames;
+    const int nz = gridDim.x - p.num_frames;
+    const size_t gt = (size_t)zb * blockDim.x + t;
+    const size_t gs = (size_t)nz * blockDim.x;
+    if (gt < sizeof(Header) / 4) reinterpret_cast<uint32_t*>(p.hdr)[gt] = 0u;
+    for (size_t i = gt; i <= (size_t)p.num_sweeps; i += gs) p.sweep_off[i] = d.sweep_off[i];
+    for (size_t i = gt; i <= (size_t)p.num_frames; i += gs) {
+        p.frame_sweep_off[i] = d.frame_sweep_off[i];
+        p.frame_roi_off[i] = d.frame_roi_off[i];
+    }
+    for (size_t s = gt; s < (size_t)p.num_sweeps; s += gs) {
+        // frame of sweep s: last f with frame_sweep_off[f] <= s
+        int lo = 0, hi = p.num_frames;  // invariant: fso[lo] <= s < fso[hi]
+        while (hi - lo > 1) {
+            const int mid = (lo + hi) >> 1;
+            if (d.frame_sweep_off[mid] <= (int)s) lo = mid; else hi = mid;
+        }
+        p.sweep_frame[s] = lo;
+    }
+    if (p.hist)
+        for (size_t i = gt; i < (size_t)p.num_rois; i += gs) p.hist[i] = 0u;
+    if (p.frame_u)
+        for (size_t i = gt; i < (size_t)p.num_frames; i += gs) p.frame_u[i] = 0u;
+    if (p.bcnt)
+        for (size_t i = gt; i <= (size_t)p.num_buckets; i += gs) p.bcnt[i] = 0ull;
+    if (p.scan_flag)
+        for (size_t i = gt; i < (size_t)p.scan_tiles; i += gs) p.scan_flag[i] = 0u;
+}
+
+__global__ void k_zero(uint4* ptr, size_t n16, uint8_t* tail, size_t ntail) {
+    const size_t gs = (size_t)gridDim.x * blockDim.x;
+    for (size_t i = (size_t)blockIdx.x * blockDim.x + threadIdx.x; i < n16; i += gs)
+        ptr[i] = make_uint4(0u, 0u, 0u, 0u);
+    if (blockIdx.x == 0)
+        for (size_t i = threadIdx.x; i < ntail; i += blockDim.x) tail[i] = 0;
+}
+
+}  // namespace
+
+// Largest coarse mask a frame block holds in shared memory: 64 x 64 cells x
+// 13 words (the coarse grid shrinks as the ROI count grows).
+constexpr int kPrepSmemMax = 64 * 64 * 13 * 4;
+
+cudaError_t launch_prep(const Params& p, const HostDesc& d, cudaStream_t st) {
+    // Raise the dynamic shared memory limit once per device (outside any
+    // stream capture that may follow).
+    static std::atomic<int> configured[64];
+    int dev = 0;
+    cudaError_t e = cudaGetDevice(&dev);
+    if (e != cudaSuccess) return e;
+    if (dev < 0 || dev >= 64 || !configured[dev].load(std::memory_order_acquire)) {
+        e = cudaFuncSetAttribute(k_prep, cudaFuncAttributeMaxDynamicSharedMemorySize, kPrepSmemMax);
+        if (e != cudaSuccess) return e;
+        if (dev >= 0 && dev < 64) configured[dev].store(1, std::memory_order_release);
+    }
+    const size_t smem = (size_t)p.coarse * p.coarse * p.mask_words * sizeof(uint32_t);
+    if (smem > (size_t)kPrepSmemMax) return cudaErrorInvalidValue;
+    k_prep<<<p.num_frames + kZeroBlocks, kPrepThreads, smem, st>>>(p, d);
+    return cudaGetLastError();
+}
+
+cudaError_t launch_zero(void* ptr, size_t bytes, cudaStream_t st) {
+    if (bytes == 0) return cudaSuccess;
+    const size_t n16 = bytes / 16;
+    uint8_t* tail = static_cast<uint8_t*>(ptr) + n16 * 16;
+    const size_t blocks = n16 / 256 + 1 < 4096 ? n16 / 256 + 1 : 4096;
+    k_zero<<<(unsigned)blocks, 256, 0, st>>>(static_cast<uint4*>(ptr), n16, tail, bytes - n16 * 16);
+    return cudaGetLastError();
+}
+
+}  // namespace mmbev

@@ -1,0 +1,86 @@
+"""The C-ABI library builds for sm_103a, loads without a GPU, exports every
+entry point include/mmbev.h declares, and rejects bad host arguments before
+touching the device."""
+import ctypes
+import os
+import re
+
+import numpy as np
+import pytest
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+HEADER = os.path.join(ROOT, "include", "mmbev.h")
+
+TINY_VS = np.array([0.2, 0.2, 8.0], np.float32)
+TINY_RG = np.array([-51.2, -51.2, -5.0, 51.2, 51.2, 3.0], np.float32)
+
+
+def declared_functions():
+    text = open(HEADER).read()
+    text = re.sub(r"/\*.*?\*/", "", text, flags=re.S)
+    return sorted(set(re.findall(r"\b(mmbev_[a-z_]+)\s*\(", text)))
+
+
+def test_header_declares_the_boundary():
+    names = declared_functions()
+    for required in ("mmbev_voxelize_roi", "mmbev_voxelize_roi_batched", "mmbev_workspace_size",
+                     "mmbev_table_size", "mmbev_classify_points", "mmbev_get_status"):
+        assert required in names
+
+
+def test_library_exports_every_declared_symbol(mmbev_lib):
+    lib = mmbev_lib.load()
+    missing = [n for n in declared_functions() if not hasattr(lib, n)]
+    assert not missing, missing
+
+
+def test_sizes_are_host_only(mmbev_lib):
+    # capacity: next power of two >= 2N slots of 16 + 4*round4(K) bytes
+    assert mmbev_lib.table_size(20000, 10) == 65536 * 64
+    assert mmbev_lib.table_size(100, 1) == 1024 * 32
+    assert mmbev_lib.table_size(11110400, 10) == (1 << 25) * 64
+    with pytest.raises(ValueError):
+        mmbev_lib.table_size(100, 0)
+    with pytest.raises(ValueError):
+        mmbev_lib.table_size(100, 65)
+    a = mmbev_lib.workspace_size(20000, 4, 16000, 1, TINY_VS, TINY_RG)
+    b = mmbev_lib.workspace_size(40000, 4, 16000, 1, TINY_VS, TINY_RG)
+    c = mmbev_lib.workspace_size(20000, 4, 16000, 2, TINY_VS, TINY_RG)
+    assert 0 < a < b and a < c
+    with pytest.raises(ValueError):
+        mmbev_lib.workspace_size(20000, 4, 16000, 1, TINY_VS, [0, 0, 0, -1, 1, 1])
+
+
+def _call(lib, *, so=(0, 100), fso=None, fro=None, nr=1, K=10, maxv=100, vs=TINY_VS, rg=TINY_RG,
+          margin=0.5, ws_bytes=1 << 30, table_bytes=1 << 30, ws=0x7f0000000000,
+          table=0x7f1000000000):
+    so = np.asarray(so, np.int64)
+    ns = len(so) - 1
+    fso = np.asarray([0, ns] if fso is None else fso, np.int32)
+    fro = np.asarray([0, nr] if fro is None else fro, np.int32)
+    vs = np.asarray(vs, np.float32)
+    rg = np.asarray(rg, np.float32)
+    P = ctypes.c_void_p
+    fake = P(0x7e0000000000)  # never dereferenced: validation fails first
+    return lib.mmbev_voxelize_roi_batched(
+        fake, so.ctypes.data_as(P), ns, fake, fake, nr, margin, vs.ctypes.data_as(P),
+        rg.ctypes.data_as(P), K, maxv, len(fso) - 1, fso.ctypes.data_as(P), fro.ctypes.data_as(P),
+        fake, fake, fake, fake, P(table), table_bytes, P(ws), ws_bytes, None)
+
+
+@pytest.mark.parametrize("kw", [
+    dict(K=0), dict(K=65), dict(maxv=-1), dict(so=(1, 100)), dict(so=(0, 50, 40)),
+    dict(fso=(0, 2)), dict(fro=(0, 2)), dict(margin=-0.1), dict(margin=float("nan")),
+    dict(vs=(0.2, 0.0, 8.0)), dict(rg=(0, 0, 0, 0, 1, 1)), dict(rg=(0, 0, 0, float("inf"), 1, 1)),
+    dict(ws=0x7f0000000010), dict(table=0x7f1000000004), dict(nr=2000, fro=(0, 2000)),
+    dict(vs=(1e-4, 1e-4, 1e-4)),   # more than 2^32 cells
+    dict(so=[0] * 2050),            # too many sweeps
+])
+def test_invalid_arguments_are_rejected_before_launch(mmbev_lib, kw):
+    assert _call(mmbev_lib.load(), **kw) == -1
+
+
+def test_small_buffers_are_rejected_before_launch(mmbev_lib):
+    lib = mmbev_lib.load()
+    assert _call(lib, ws_bytes=1024) == -3
+    assert _call(lib, table_bytes=64 * 100) == -3   # fewer than 2N slots

@@ -1,0 +1,348 @@
+"""GPU parity: the CUDA path, called through the C ABI, against the oracle on
+the same seeded inputs.
+
+Voxel coordinates, counts, the kept-point selection (first K by index) and
+the voxel order are compared bit-exactly; features within 1e-5 relative /
+1e-6 absolute (the bound the kernels are built to meet exactly: both sides
+sum in index order with the same fp32 operations, so the measured bit-exact
+fraction is reported as well). Covers all five workload shapes at full size,
+the cap path, and the edge cases of the method.
+"""
+import numpy as np
+import pytest
+
+import synth
+from helpers import assert_frames_equal, run_gpu, run_oracle, to_dev
+
+pytestmark = pytest.mark.gpu
+
+
+def _table_is_clean(table):
+    return not bool(table.any().item())
+
+
+# ------------------------------------------------------------------ S1 + S2 per point
+
+@pytest.mark.parametrize("name", ["tiny", "nuscenes", "ouster", "roi_128", "roi_full"])
+def test_classify_bit_exact(oracle_mod, mmbev_lib, cuda_dev, name):
+    w = synth.CONFIGS[name]()
+    pts, tf, rois = to_dev(w, cuda_dev)
+    ws = mmbev_lib.new_workspace(w.num_points, w.rois.shape[0], 0, 1, w.voxel_size, w.pc_range,
+                                 cuda_dev)
+    xyz, lin, rank = mmbev_lib.classify_points(pts, w.sweep_offsets, tf, rois, w.roi_margin,
+                                               w.voxel_size, w.pc_range, w.frame_sweep_offsets,
+                                               w.frame_roi_offsets, workspace=ws)
+    exyz, elin, erank = oracle_mod.classify(w.points, w.sweep_offsets, w.sweep_tf, w.rois,
+                                            w.roi_margin, w.voxel_size, w.pc_range)
+    assert np.array_equal(xyz.cpu().numpy().view(np.uint32), exyz.view(np.uint32))
+    assert np.array_equal(lin.cpu().numpy(), elin)
+    assert np.array_equal(rank.cpu().numpy(), erank)
+
+
+# ------------------------------------------------------------------ whole path, full sizes
+
+@pytest.mark.parametrize("name", ["tiny", "nuscenes", "ouster", "roi_0", "roi_8", "roi_32",
+                                  "roi_128", "roi_full"])
+def test_voxelize_parity(oracle_mod, mmbev_lib, cuda_dev, name):
+    w = synth.CONFIGS[name]()
+    got, status, table, _ = run_gpu(mmbev_lib, w, cuda_dev)
+    assert status == 0
+    want = run_oracle(oracle_mod, w)
+    exact = assert_frames_equal(got, want, name)
+    assert exact == 1.0, f"{name}: {exact:.6f} of feature values bit-exact"
+    assert _table_is_clean(table)
+
+
+def test_batch32_parity(oracle_mod, mmbev_lib, cuda_dev):
+    """The benchmark's workload and launch configuration: 32 frames, 11.1 M
+    points, one call."""
+    w = synth.streaming_batch(32)
+    got, status, table, _ = run_gpu(mmbev_lib, w, cuda_dev)
+    assert status == 0
+    want = run_oracle(oracle_mod, w)
+    assert assert_frames_equal(got, want, "batch32") == 1.0
+    assert _table_is_clean(table)
+
+
+# ------------------------------------------------------------------ cap path
+
+@pytest.mark.parametrize("maxv", [1, 777, 5000, 13000])
+def test_cap_parity(oracle_mod, mmbev_lib, cuda_dev, maxv):
+    w = synth.nuscenes_frame(1)
+    got, status, table, _ = run_gpu(mmbev_lib, w, cuda_dev, maxv=maxv)
+    want = run_oracle(oracle_mod, w, maxv=maxv)
+    assert status == 0
+    assert got[0][1].shape[0] == maxv
+    assert_frames_equal(got, want, f"cap {maxv}")
+    assert _table_is_clean(table)
+
+
+def test_cap_full_coverage_and_mixed_frames(oracle_mod, mmbev_lib, cuda_dev):
+    # frames with and without the cap in one call; one frame has no ROIs
+    frames = [synth.roi_coverage("full"), synth.tiny(3), synth.roi_coverage(128),
+              synth.roi_coverage(0)]
+    for f in frames:
+        f.max_voxels = 40000
+        f.max_pts_per_voxel = 10
+    b = synth.concat_frames(frames, "mixed")
+    got, status, table, _ = run_gpu(mmbev_lib, b, cuda_dev)
+    want = run_oracle(oracle_mod, b)
+    assert status == 0
+    assert_frames_equal(got, want, "mixed")
+    assert [g[1].shape[0] for g in got][0] == 40000
+    assert _table_is_clean(table)
+
+
+def test_max_voxels_zero(oracle_mod, mmbev_lib, cuda_dev):
+    w = synth.tiny(0)
+    got, status, table, _ = run_gpu(mmbev_lib, w, cuda_dev, maxv=0)
+    assert status == 0 and got[0][1].shape[0] == 0
+    assert _table_is_clean(table)
+
+
+# ------------------------------------------------------------------ per-voxel cap K
+
+@pytest.mark.parametrize("K", [1, 3, 64])
+def test_points_per_voxel(oracle_mod, mmbev_lib, cuda_dev, K):
+    w = synth.nuscenes_frame(1)
+    got, status, table, _ = run_gpu(mmbev_lib, w, cuda_dev, K=K)
+    want = run_oracle(oracle_mod, w, K=K)
+    assert status == 0
+    assert_frames_equal(got, want, f"K={K}")
+    assert _table_is_clean(table)
+
+
+# ------------------------------------------------------------------ edge cases
+
+def _custom(points, offsets, tfs, rois, margin=0.5, vs=(0.2, 0.2, 8.0),
+            rg=(-51.2, -51.2, -5.0, 51.2, 51.2, 3.0), K=10, maxv=1000, fso=None, fro=None):
+    return synth.Workload(
+        name="custom", points=np.asarray(points, np.float32).reshape(-1, 5),
+        sweep_offsets=np.asarray(offsets, np.int64), sweep_tf=np.asarray(tfs, np.float32).reshape(-1, 16),
+        rois=np.asarray(rois, np.float32).reshape(-1, 5), roi_margin=margin,
+        voxel_size=np.asarray(vs, np.float32), pc_range=np.asarray(rg, np.float32),
+        max_pts_per_voxel=K, max_voxels=maxv,
+        frame_sweep_offsets=None if fso is None else np.asarray(fso, np.int32),
+        frame_roi_offsets=None if fro is None else np.asarray(fro, np.int32))
+
+
+EYE = np.eye(4, dtype=np.float32).reshape(16)
+FULL = [[0.0, 0.0, 1000.0, 1000.0, 0.0]]
+
+
+def test_empty_input(oracle_mod, mmbev_lib, cuda_dev):
+    w = _custom(np.zeros((0, 5)), [0, 0], [EYE], FULL)
+    got, status, table, _ = run_gpu(mmbev_lib, w, cuda_dev)
+    assert status == 0 and got[0][1].shape[0] == 0
+
+
+def test_no_rois(oracle_mod, mmbev_lib, cuda_dev):
+    w = synth.tiny(0).with_rois(np.zeros((0, 5), np.float32))
+    got, status, table, _ = run_gpu(mmbev_lib, w, cuda_dev)
+    assert status == 0 and got[0][1].shape[0] == 0
+    assert _table_is_clean(table)
+
+
+def test_ragged_tiles_and_empty_sweeps(oracle_mod, mmbev_lib, cuda_dev):
+    # 5 sweeps, two of them empty, N = 6,151 (not a multiple of 4 or 2048);
+    # each sweep shifted, so the sweep lookup matters.
+    rng = np.random.default_rng(21)
+    sizes = [2047, 0, 2050, 0, 2054]
+    offs = np.concatenate([[0], np.cumsum(sizes)])
+    n = offs[-1]
+    pts = np.zeros((n, 5), np.float32)
+    pts[:, 0] = rng.uniform(-20, 20, n)
+    pts[:, 1] = rng.uniform(-20, 20, n)
+    pts[:, 2] = rng.uniform(-4, 2, n)
+    pts[:, 3] = rng.uniform(0, 1, n)
+    pts[:, 4] = np.repeat(np.arange(5) * 0.05, sizes)
+    tfs = []
+    for s in range(5):
+        t = np.eye(4, dtype=np.float32)
+        t[0, 3], t[1, 3] = 0.37 * s, -0.21 * s
+        tfs.append(t.reshape(16))
+    rois = [[0, 0, 8, 12, 0.4], [5, 5, 3, 3, 1.0], [-10, 3, 6, 2, 2.0]]
+    w = _custom(pts, offs, tfs, rois, vs=(0.1, 0.1, 0.2), K=4, maxv=100000)
+    got, status, table, _ = run_gpu(mmbev_lib, w, cuda_dev)
+    assert status == 0
+    assert_frames_equal(got, run_oracle(oracle_mod, w), "ragged")
+    assert got[0][1].shape[0] > 100
+
+
+def test_many_sweeps_per_tile(oracle_mod, mmbev_lib, cuda_dev):
+    # 300 sweeps of 7 points: a 2048-point tile spans more sweeps than the
+    # kernel stages in shared memory, taking the per-point lookup.
+    rng = np.random.default_rng(22)
+    S, m = 300, 7
+    n = S * m
+    pts = np.zeros((n, 5), np.float32)
+    pts[:, :2] = rng.uniform(-10, 10, (n, 2))
+    pts[:, 2] = rng.uniform(-2, 2, n)
+    pts[:, 3] = rng.uniform(0, 1, n)
+    tfs = []
+    for s in range(S):
+        t = np.eye(4, dtype=np.float32)
+        t[0, 3] = 0.01 * s
+        tfs.append(t.reshape(16))
+    w = _custom(pts, np.arange(S + 1) * m, tfs, FULL, vs=(0.5, 0.5, 0.5), K=3, maxv=100000)
+    got, status, table, _ = run_gpu(mmbev_lib, w, cuda_dev)
+    assert status == 0
+    assert_frames_equal(got, run_oracle(oracle_mod, w), "many sweeps")
+
+
+def test_non_finite_and_boundary_points(oracle_mod, mmbev_lib, cuda_dev):
+    up = lambda v: float(np.nextafter(np.float32(v), np.float32(np.inf)))
+    below = lambda v: float(np.nextafter(np.float32(v), np.float32(-np.inf)))
+    rows = [[np.nan, 0, 0], [0, np.inf, 0], [0, 0, -np.inf], [2.5, 0, 0], [up(2.5), 0, 0],
+            [0, 1.5, 0], [0, up(1.5), 0], [-2.5, -1.5, 0], [51.2, 0, 0], [below(51.2), 0, 0],
+            [-51.2, 0, 0], [0, 0, 3.0], [0, 0, -5.0], [0.2, 0.2, 0.0], [0.4, 0.0, 0.0]]
+    pts = np.zeros((len(rows), 5), np.float32)
+    pts[:, :3] = rows
+    pts[:, 3] = np.arange(len(rows)) / 16.0
+    rois = [[0.0, 0.0, 2.0, 4.0, 0.0], [51.0, 0.0, 1.0, 1.0, 0.0], [-51.0, 0, 1, 1, 0]]
+    w = _custom(pts, [0, len(rows)], [EYE], rois, margin=0.5)
+    got, status, table, _ = run_gpu(mmbev_lib, w, cuda_dev)
+    want = run_oracle(oracle_mod, w)
+    assert status == 0
+    assert_frames_equal(got, want, "boundaries")
+    assert want[0][1].shape[0] >= 5
+
+
+def test_duplicate_points_in_one_voxel(oracle_mod, mmbev_lib, cuda_dev):
+    n = 5000
+    pts = np.tile(np.array([[1.05, 2.05, 0.3, 0.5, 0.0]], np.float32), (n, 1))
+    pts[:, 3] = (np.arange(n) % 32) / 32.0
+    w = _custom(pts, [0, n], [EYE], FULL, K=10)
+    got, status, table, _ = run_gpu(mmbev_lib, w, cuda_dev)
+    assert status == 0
+    assert got[0][2].tolist() == [10]
+    assert_frames_equal(got, run_oracle(oracle_mod, w), "duplicates")
+
+
+def test_tiny_grid_and_many_frames(oracle_mod, mmbev_lib, cuda_dev):
+    # 4 x 3 x 2 = 24 cells (< one 32-cell bucket); 150 frames with 0..3 ROIs
+    rng = np.random.default_rng(23)
+    frames = []
+    for f in range(150):
+        n = int(rng.integers(0, 60))
+        pts = np.zeros((n, 5), np.float32)
+        pts[:, :3] = rng.uniform(-1, 1, (n, 3))
+        pts[:, 3] = rng.uniform(0, 1, n)
+        r = int(rng.integers(0, 4))
+        rois = np.stack([rng.uniform(-1, 1, r), rng.uniform(-1, 1, r), rng.uniform(0.2, 1, r),
+                         rng.uniform(0.2, 1, r), rng.uniform(0, 6, r)], 1) if r else np.zeros((0, 5))
+        frames.append(_custom(pts, [0, n], [EYE], rois, margin=0.1, vs=(0.5, 2 / 3, 1.0),
+                              rg=(-1, -1, -1, 1, 1, 1), K=2, maxv=5))
+    b = synth.concat_frames(frames, "many")
+    got, status, table, _ = run_gpu(mmbev_lib, b, cuda_dev)
+    assert status == 0
+    assert_frames_equal(got, run_oracle(oracle_mod, b), "many frames")
+    assert _table_is_clean(table)
+
+
+def test_max_rois_per_frame(oracle_mod, mmbev_lib, cuda_dev):
+    # 1024 ROIs in a frame: 32 mask words per coarse cell
+    rng = np.random.default_rng(24)
+    r = 1024
+    rois = np.stack([rng.uniform(-50, 50, r), rng.uniform(-50, 50, r), rng.uniform(0.5, 3, r),
+                     rng.uniform(0.5, 6, r), rng.uniform(0, 6.3, r)], 1).astype(np.float32)
+    w = synth.tiny(0).with_rois(rois)
+    got, status, table, _ = run_gpu(mmbev_lib, w, cuda_dev)
+    assert status == 0
+    assert_frames_equal(got, run_oracle(oracle_mod, w), "1024 rois")
+    assert got[0][1].shape[0] > 500
+
+
+def test_single_frame_entry_equals_batched(oracle_mod, mmbev_lib, cuda_dev):
+    w = synth.nuscenes_frame(5)
+    pts, tf, rois = to_dev(w, cuda_dev)
+    table = mmbev_lib.new_table(w.num_points, w.max_pts_per_voxel, cuda_dev)
+    ws = mmbev_lib.new_workspace(w.num_points, w.rois.shape[0], w.max_voxels, 1, w.voxel_size,
+                                 w.pc_range, cuda_dev)
+    out = mmbev_lib.voxelize_roi(pts, w.sweep_offsets, tf, rois, w.roi_margin, w.voxel_size,
+                                 w.pc_range, w.max_pts_per_voxel, w.max_voxels, table=table,
+                                 workspace=ws)
+    got = [out.frame(0, w.max_voxels)]
+    assert mmbev_lib.get_status(ws) == 0
+    assert_frames_equal(got, run_oracle(oracle_mod, w), "single-frame entry")
+
+
+def test_repeat_calls_are_deterministic_and_leave_table_clean(mmbev_lib, cuda_dev):
+    w = synth.ouster_frame(2)
+    a, s1, table, ws = run_gpu(mmbev_lib, w, cuda_dev)
+    assert _table_is_clean(table)
+    b, s2, _, _ = run_gpu(mmbev_lib, w, cuda_dev, table=table, workspace=ws)
+    assert s1 == 0 and s2 == 0
+    for (af, ac, an), (bf, bc, bn) in zip(a, b):
+        assert np.array_equal(af.view(np.uint32), bf.view(np.uint32))
+        assert np.array_equal(ac, bc) and np.array_equal(an, bn)
+
+
+def test_non_default_stream(oracle_mod, mmbev_lib, cuda_dev):
+    import torch
+    w = synth.tiny(1)
+    s = torch.cuda.Stream(cuda_dev)
+    with torch.cuda.stream(s):
+        got, status, table, _ = run_gpu(mmbev_lib, w, cuda_dev, stream=s)
+    assert status == 0
+    assert_frames_equal(got, run_oracle(oracle_mod, w), "stream")
+
+
+def test_graph_capture_replays_the_call(oracle_mod, mmbev_lib, cuda_dev):
+    import torch
+    w = synth.nuscenes_frame(3)
+    pts, tf, rois = to_dev(w, cuda_dev)
+    table = mmbev_lib.new_table(w.num_points, w.max_pts_per_voxel, cuda_dev)
+    ws = mmbev_lib.new_workspace(w.num_points, w.rois.shape[0], w.max_voxels, 1, w.voxel_size,
+                                 w.pc_range, cuda_dev)
+    out = mmbev_lib.Outputs.empty(1, w.max_voxels, cuda_dev)
+    # one eager call first, as before any capture
+    mmbev_lib.voxelize_roi_batched(pts, w.sweep_offsets, tf, rois, w.roi_margin, w.voxel_size,
+                                   w.pc_range, w.max_pts_per_voxel, w.max_voxels,
+                                   w.frame_sweep_offsets, w.frame_roi_offsets, table=table,
+                                   workspace=ws, out=out)
+    torch.cuda.synchronize()
+    out.feats.zero_()
+    out.coords.zero_()
+    out.counts.zero_()
+    out.nvox.zero_()
+    torch.cuda.synchronize()
+    g = torch.cuda.CUDAGraph()
+    s = torch.cuda.Stream(cuda_dev)
+    with torch.cuda.graph(g, stream=s):
+        mmbev_lib.voxelize_roi_batched(pts, w.sweep_offsets, tf, rois, w.roi_margin, w.voxel_size,
+                                       w.pc_range, w.max_pts_per_voxel, w.max_voxels,
+                                       w.frame_sweep_offsets, w.frame_roi_offsets, table=table,
+                                       workspace=ws, out=out)
+    for _ in range(3):
+        g.replay()
+    torch.cuda.synchronize()
+    assert mmbev_lib.get_status(ws) == 0
+    assert_frames_equal([out.frame(0, w.max_voxels)], run_oracle(oracle_mod, w), "graph")
+    assert _table_is_clean(table)
+
+
+# ------------------------------------------------------------------ device-side failures
+
+def test_full_table_sets_status_and_returns(mmbev_lib, cuda_dev):
+    # 64 slots for ~14,000 voxels: inserts that find no slot set
+    # MMBEV_DEV_TABLE_FULL; the call still completes and releases every slot.
+    w = synth.nuscenes_frame(1)
+    got, status, table, _ = run_gpu(mmbev_lib, w, cuda_dev, table_log2_override=6)
+    assert status & mmbev_lib.DEV_TABLE_FULL
+    assert _table_is_clean(table)
+    # the same table then serves a correct call
+    got2, status2, _, _ = run_gpu(mmbev_lib, synth.tiny(0), cuda_dev, table=table)
+    assert status2 == 0
+
+
+def test_workspace_too_small_is_rejected(mmbev_lib, cuda_dev):
+    import torch
+    w = synth.tiny(0)
+    pts, tf, rois = to_dev(w, cuda_dev)
+    table = mmbev_lib.new_table(w.num_points, 10, cuda_dev)
+    ws = torch.empty(4096, dtype=torch.uint8, device=cuda_dev)
+    with pytest.raises(mmbev_lib.MMBEVError):
+        mmbev_lib.voxelize_roi_batched(pts, w.sweep_offsets, tf, rois, 0.5, w.voxel_size,
+                                       w.pc_range, 10, 16000, w.frame_sweep_offsets,
+                                       w.frame_roi_offsets, table=table, workspace=ws)
