@@ -232,6 +232,41 @@ int mmbev_voxelize_roi_batched_ex(const float *points, const int64_t *sweep_offs
                                   void *workspace, size_t workspace_bytes,
                                   cudaStream_t stream, const mmbev_exec_opts_t *opts);
 
+/*
+ * Single-frame voxelization for callers that cannot allocate device memory.
+ * The paper has no counterpart: this is a deployment variant of
+ * mmbev_voxelize_roi. Some callers cannot call cudaMalloc at all, for
+ * example a real-time perception process that forbids allocation after
+ * start-up (allocation may synchronize the device and has unbounded
+ * latency), or a host that owns every device buffer and lends the library
+ * only its inputs and outputs. Here the hash table and the workspace come
+ * from one file-scope device array of MMBEV_NOALLOC_SCRATCH_BYTES, which
+ * every GPU that loads the library keeps until the process exits; the call
+ * allocates nothing.
+ *   Arguments are those of mmbev_voxelize_roi without the table and
+ *   workspace, plus
+ *   out_status  device, uint32 scalar or NULL: receives the call's device
+ *               status word (MMBEV_DEV_* bits, 0 = no device-side error).
+ *   Returns MMBEV_EWORKSPACE, before any launch, when the call needs more
+ *   than the array holds: mmbev_table_size(N, K) rounded up to 256 bytes
+ *   plus mmbev_workspace_size(N, num_rois, max_voxels, 1, voxel_size, range)
+ *   must not exceed MMBEV_NOALLOC_SCRATCH_BYTES (a 400,000-point frame with
+ *   K <= 12 fits).
+ * The first call on a device looks up the array's device address with that
+ * device current; make that first call before any stream capture. Every
+ * call zeroes the table part of the array first, since the array keeps the
+ * previous call's contents. All calls on a device share the one array:
+ * calls whose executions overlap on the GPU race and must be serialized.
+ */
+#define MMBEV_NOALLOC_SCRATCH_BYTES (80u << 20)
+int mmbev_voxelize_roi_noalloc(const float *points, const int64_t *sweep_offsets,
+                               int32_t num_sweeps, const float *sweep_tf,
+                               const mmbev_roi_t *rois, int32_t num_rois, float roi_margin,
+                               const float voxel_size[3], const float range[6],
+                               int32_t max_pts_per_voxel, int32_t max_voxels,
+                               float *out_feats, int32_t *out_coords, int32_t *out_counts,
+                               int32_t *out_nvox, uint32_t *out_status, cudaStream_t stream);
+
 /* Names of the stages timed by stage_events, for reports. */
 const char *mmbev_stage_name(int32_t stage);
 

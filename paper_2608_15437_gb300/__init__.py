@@ -65,6 +65,8 @@ def load():
     lib.mmbev_classify_points.argtypes = [P, P, i32, P, P, i32, f32, P, P, i32, P, P,
                                           P, P, P, P, sz, P]
     lib.mmbev_classify_points.restype = ctypes.c_int
+    lib.mmbev_voxelize_roi_noalloc.argtypes = vox + [P, P, P, P, P, P]
+    lib.mmbev_voxelize_roi_noalloc.restype = ctypes.c_int
     lib.mmbev_get_status.argtypes = [P, sz, ctypes.POINTER(ctypes.c_uint32), P]
     lib.mmbev_get_status.restype = ctypes.c_int
     lib.mmbev_stage_name.argtypes = [i32]
@@ -250,6 +252,29 @@ def voxelize_roi(points: torch.Tensor, sweep_offsets, sweep_tf: torch.Tensor, ro
         _dptr(table, torch.uint8, "table"), table.numel(),
         _dptr(workspace, torch.uint8, "workspace"), workspace.numel(), _stream(stream))
     _check(rc, "mmbev_voxelize_roi")
+    return out
+
+
+def voxelize_roi_noalloc(points: torch.Tensor, sweep_offsets, sweep_tf: torch.Tensor,
+                         rois: torch.Tensor, roi_margin: float, voxel_size, pc_range,
+                         max_pts_per_voxel: int, max_voxels: int, *, out: Outputs,
+                         status: torch.Tensor | None = None, stream=None) -> Outputs:
+    """One frame without table or workspace (``mmbev_voxelize_roi_noalloc``),
+    for callers that cannot allocate device memory: the library's own
+    file-scope device array serves as scratch. ``out`` (and ``status``, a
+    1-element uint32/int32 device tensor) must be allocated by the caller."""
+    lib = load()
+    so = _host(sweep_offsets, np.int64)
+    vs = _host(voxel_size, np.float32)
+    rg = _host(pc_range, np.float32)
+    nr = rois.shape[0] if rois.dim() > 1 else rois.numel() // 5
+    rc = lib.mmbev_voxelize_roi_noalloc(
+        _dptr(points, torch.float32, "points"), _hptr(so), len(so) - 1,
+        _dptr(sweep_tf, torch.float32, "sweep_tf"), _dptr(rois, torch.float32, "rois"), nr,
+        float(roi_margin), _hptr(vs), _hptr(rg), int(max_pts_per_voxel), int(max_voxels),
+        _dptr(out.feats), _dptr(out.coords), _dptr(out.counts), _dptr(out.nvox),
+        _dptr(status), _stream(stream))
+    _check(rc, "mmbev_voxelize_roi_noalloc")
     return out
 
 
