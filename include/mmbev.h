@@ -98,11 +98,13 @@ typedef enum mmbev_status {
 #define MMBEV_MAX_PTS_PER_VOXEL   64
 
 /*
- * Bytes of hash table for calls of up to max_points points and
- * max_pts_per_voxel points kept per voxel. The capacity is the power of two
- * >= 2*max_points slots (load factor <= 1/2 whatever the inputs), each slot
- * holding the voxel key, its minimum ROI rank and its K smallest point
- * indices. Returns 0 for invalid arguments.
+ * Bytes of hash table for calls of up to max_points points (and
+ * max_pts_per_voxel points kept per voxel, which must lie in
+ * [1, MMBEV_MAX_PTS_PER_VOXEL] but does not change the size). The capacity
+ * is the power of two >= 2*max_points slots of 32 bytes (load factor <= 1/2
+ * whatever the inputs), each slot holding a voxel key, its minimum ROI rank,
+ * its point count and the start of its point list. Returns 0 for invalid
+ * arguments.
  */
 size_t mmbev_table_size(int64_t max_points, int32_t max_pts_per_voxel);
 
@@ -208,11 +210,12 @@ int mmbev_get_status(const void *workspace, size_t workspace_bytes,
  *                     caller: event k is recorded on `stream` before stage k
  *                     and the last one after the final stage, so the caller
  *                     can time each kernel with cudaEventElapsedTime.
- *   table_log2_override  0, or log2 of the slot count to use instead of the
- *                     largest power of two that fits table_bytes (a smaller
- *                     table; a full table sets MMBEV_DEV_TABLE_FULL).
+ *   table_log2_override  0, or log2 of the slot count the insert stage uses
+ *                     instead of the power of two >= 1.25 x the call's kept
+ *                     points (at most table_bytes / 16; a full table sets
+ *                     MMBEV_DEV_TABLE_FULL).
  */
-#define MMBEV_NUM_STAGES 9
+#define MMBEV_NUM_STAGES 13
 typedef struct mmbev_exec_opts {
     cudaEvent_t *stage_events;
     int32_t table_log2_override;
@@ -258,7 +261,7 @@ int mmbev_voxelize_roi_batched_ex(const float *points, const int64_t *sweep_offs
  * previous call's contents. All calls on a device share the one array:
  * calls whose executions overlap on the GPU race and must be serialized.
  */
-#define MMBEV_NOALLOC_SCRATCH_BYTES (80u << 20)
+#define MMBEV_NOALLOC_SCRATCH_BYTES (96u << 20)
 int mmbev_voxelize_roi_noalloc(const float *points, const int64_t *sweep_offsets,
                                int32_t num_sweeps, const float *sweep_tf,
                                const mmbev_roi_t *rois, int32_t num_rois, float roi_margin,

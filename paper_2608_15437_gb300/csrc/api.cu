@@ -47,20 +47,26 @@ int mask_words_for(int32_t max_rois_frame) {
     return w < 1 ? 1 : w;
 }
 
+// Coarse candidate grid: at most 4,096 mask words per frame, so a frame's
+// mask fits the classify kernel's 16 KB shared-memory slot.
 int coarse_for(int mask_words) {
-    if (mask_words <= 1) return 128;
-    if (mask_words <= 13) return 64;
-    return 32;
+    if (mask_words <= 1) return 64;
+    if (mask_words <= 4) return 32;
+    if (mask_words <= 16) return 16;
+    return 8;
 }
 
-uint32_t slot_stride_for(int32_t K) { return 16u + 4u * (uint32_t)((K + 3) / 4 * 4); }
+constexpr uint32_t kMaxInsertBlocks = 4096;
+
+constexpr uint32_t kSlotStride = 16;
 
 // Byte offsets of every workspace array for one call shape.
 struct Layout {
     size_t hdr, sweep_off, sweep_frame, fso, fro, roi_prep, masks, hist, frame_u, finfo;
-    size_t bcnt, scan_agg, scan_inc, scan_flag, occ, d_bucket, d_pos, items, vid_slot;
+    size_t records, reg_cnt, rec_slot, seg, newlist, blockcount, bcnt, bcnt2, boff, nonempty, occ, d_bucket,
+        d_pos, d_lin, items, vid_slot, heavy;
     size_t total;
-    uint32_t num_buckets, buckets_per_frame, scan_tiles;
+    uint32_t num_buckets, buckets_per_frame, num_tiles;
     int bucket_log2, mask_words, coarse;
 };
 
@@ -70,11 +76,13 @@ Layout make_layout(int64_t max_points, int64_t rois_total, int32_t max_rois_fram
     L.bucket_log2 = bucket_log2_for(g.cells);
     L.buckets_per_frame = (uint32_t)((g.cells + (1ull << L.bucket_log2) - 1) >> L.bucket_log2);
     L.num_buckets = L.buckets_per_frame * (uint32_t)num_frames;
-    L.scan_tiles = (uint32_t)(((uint64_t)L.num_buckets + 1 + kScanTile - 1) / kScanTile);
     L.mask_words = mask_words_for(max_rois_frame);
     L.coarse = coarse_for(L.mask_words);
     const size_t F = (size_t)num_frames, R = (size_t)(rois_total > 0 ? rois_total : 1);
     const size_t U = (size_t)(max_points > 0 ? max_points : 1);
+    const size_t B2 = ((size_t)L.num_buckets + 1) / 2 * 2;  // zeroed as 16-byte pairs
+    L.num_tiles = (uint32_t)((U + kTile - 1) / kTile);
+    const size_t TS = (size_t)L.num_tiles * kTile;        // record slots, tile-aligned
     size_t o = 0;
     auto take = [&](size_t bytes) { const size_t at = o; o = align_up(o + bytes, kAlign); return at; };
     L.hdr = take(sizeof(Header));
@@ -87,15 +95,23 @@ Layout make_layout(int64_t max_points, int64_t rois_total, int32_t max_rois_fram
     L.hist = take(sizeof(uint32_t) * R);
     L.frame_u = take(sizeof(uint32_t) * F);
     L.finfo = take(sizeof(FrameInfo) * F);
-    L.bcnt = take(sizeof(unsigned long long) * ((size_t)L.num_buckets + 1));
-    L.scan_agg = take(sizeof(unsigned long long) * L.scan_tiles);
-    L.scan_inc = take(sizeof(unsigned long long) * L.scan_tiles);
-    L.scan_flag = take(sizeof(uint32_t) * L.scan_tiles);
+    L.records = take(32 * TS);
+    L.reg_cnt = take(sizeof(uint32_t) * L.num_tiles * (kTile / kRegion));
+    L.rec_slot = take(sizeof(uint2) * TS);
+    L.seg = take(sizeof(uint32_t) * U);
+    L.newlist = take(16 * TS);
+    L.blockcount = take(sizeof(uint32_t) * kMaxInsertBlocks);
+    L.bcnt = take(sizeof(unsigned long long) * B2);
+    L.bcnt2 = take(sizeof(unsigned long long) * B2);
+    L.boff = take(sizeof(unsigned long long) * B2);
+    L.nonempty = take(sizeof(uint32_t) * B2);
     L.occ = take(sizeof(uint32_t) * U);
     L.d_bucket = take(sizeof(uint32_t) * U);
     L.d_pos = take(sizeof(uint32_t) * U);
-    L.items = take(sizeof(uint32_t) * U);
+    L.d_lin = take(sizeof(uint32_t) * U);
+    L.items = take(sizeof(uint2) * U);
     L.vid_slot = take(sizeof(uint32_t) * (F * (size_t)(max_voxels > 0 ? max_voxels : 1)));
+    L.heavy = take(sizeof(uint32_t) * (F * (size_t)(max_voxels > 0 ? max_voxels : 1)));
     L.total = o;
     return L;
 }
@@ -182,16 +198,26 @@ void bind_layout(Params* p, const Layout& L, uint8_t* ws) {
     p->hist = reinterpret_cast<uint32_t*>(ws + L.hist);
     p->frame_u = reinterpret_cast<uint32_t*>(ws + L.frame_u);
     p->finfo = reinterpret_cast<FrameInfo*>(ws + L.finfo);
+    p->records = reinterpret_cast<uint4*>(ws + L.records);
+    p->reg_cnt = reinterpret_cast<uint32_t*>(ws + L.reg_cnt);
+    p->rec_slot = reinterpret_cast<uint2*>(ws + L.rec_slot);
+    p->seg = reinterpret_cast<uint32_t*>(ws + L.seg);
+    p->num_regions = (uint32_t)((p->num_points + kTile - 1) / kTile) * (kTile / kRegion);
+    p->newlist = reinterpret_cast<uint4*>(ws + L.newlist);
+    p->blockcount = reinterpret_cast<uint32_t*>(ws + L.blockcount);
     p->bcnt = reinterpret_cast<unsigned long long*>(ws + L.bcnt);
-    p->scan_agg = reinterpret_cast<unsigned long long*>(ws + L.scan_agg);
-    p->scan_inc = reinterpret_cast<unsigned long long*>(ws + L.scan_inc);
-    p->scan_flag = reinterpret_cast<uint32_t*>(ws + L.scan_flag);
+    p->bcnt2 = reinterpret_cast<unsigned long long*>(ws + L.bcnt2);
+    p->boff = reinterpret_cast<unsigned long long*>(ws + L.boff);
+    p->nonempty = reinterpret_cast<uint32_t*>(ws + L.nonempty);
     p->occ = reinterpret_cast<uint32_t*>(ws + L.occ);
     p->d_bucket = reinterpret_cast<uint32_t*>(ws + L.d_bucket);
     p->d_pos = reinterpret_cast<uint32_t*>(ws + L.d_pos);
-    p->items = reinterpret_cast<uint32_t*>(ws + L.items);
+    p->d_lin = reinterpret_cast<uint32_t*>(ws + L.d_lin);
+    p->items = reinterpret_cast<uint2*>(ws + L.items);
     p->vid_slot = reinterpret_cast<uint32_t*>(ws + L.vid_slot);
+    p->heavy = reinterpret_cast<uint32_t*>(ws + L.heavy);
     p->occ_cap = (uint32_t)(p->num_points > 0 ? p->num_points : 1);
+    p->rec_cap = p->occ_cap;
     p->mask_words = L.mask_words;
     p->coarse = L.coarse;
     p->coarse_inv[0] = (float)((double)L.coarse / ((double)p->rmax[0] - (double)p->rmin[0]));
@@ -199,7 +225,6 @@ void bind_layout(Params* p, const Layout& L, uint8_t* ws) {
     p->bucket_log2 = L.bucket_log2;
     p->buckets_per_frame = L.buckets_per_frame;
     p->num_buckets = L.num_buckets;
-    p->scan_tiles = L.scan_tiles;
 }
 
 #define MMBEV_TRY(expr)                                   \
@@ -208,7 +233,8 @@ void bind_layout(Params* p, const Layout& L, uint8_t* ws) {
     } while (0)
 
 const char* const kStageNames[MMBEV_NUM_STAGES] = {
-    "prep", "points", "census", "frames", "capped_census", "scan", "scatter", "rank", "finalize"};
+    "prep", "classify", "insert", "compact", "scatter_points", "capped_hist", "frames",
+    "capped_census", "scan", "scatter", "rank", "finalize", "finalize_heavy"};
 
 }  // namespace
 }  // namespace mmbev
@@ -223,7 +249,7 @@ size_t mmbev_table_size(int64_t max_points, int32_t max_pts_per_voxel) {
     uint64_t h = 1024;
     while (h < 2ull * (uint64_t)max_points) h <<= 1;
     if (h > (1ull << 31)) return 0;
-    return (size_t)h * slot_stride_for(max_pts_per_voxel);
+    return (size_t)h * kSlotStride;
 }
 
 size_t mmbev_workspace_size(int64_t max_points, int32_t max_rois_per_frame, int32_t max_voxels,
@@ -278,18 +304,18 @@ int mmbev_voxelize_roi_batched_ex(const float* points, const int64_t* sweep_offs
     p.out_coords = out_coords;
     p.out_counts = out_counts;
     p.out_nvox = out_nvox;
-    // Hash table: the largest power of two of slots that fits, unless overridden.
-    p.slot_stride = slot_stride_for(max_pts_per_voxel);
-    const uint64_t fit = table_bytes / p.slot_stride;
+    // Hash table: its capacity is the largest power of two of slots that
+    // fits and must reach 2N; the insert stage then uses the first
+    // pow2(1.25 x kept points) of them, or the override.
+    const uint64_t fit = table_bytes / kSlotStride;
     uint32_t lg = 0;
     while (lg < 31 && (2ull << lg) <= fit) ++lg;
+    if ((1ull << lg) > fit) return MMBEV_EWORKSPACE;
+    p.table_log2_fixed = 0;
     if (opts && opts->table_log2_override > 0) {
-        if (opts->table_log2_override > 31 ||
-            (1ull << opts->table_log2_override) > fit) {
-            return MMBEV_EWORKSPACE;
-        }
-        lg = (uint32_t)opts->table_log2_override;
-    } else if ((1ull << lg) > fit || (1ull << lg) < 2ull * (uint64_t)p.num_points) {
+        if (opts->table_log2_override > (int32_t)lg) return MMBEV_EWORKSPACE;
+        p.table_log2_fixed = opts->table_log2_override;
+    } else if ((1ull << lg) < 2ull * (uint64_t)p.num_points) {
         return MMBEV_EWORKSPACE;
     }
     p.table = static_cast<uint8_t*>(table);
@@ -297,31 +323,45 @@ int mmbev_voxelize_roi_batched_ex(const float* points, const int64_t* sweep_offs
 
     const int sms = num_sms();
     if (sms <= 0) return MMBEV_ECUDA;
+    p.ins_blocks = insert_blocks(sms);
+    if (p.ins_blocks > kMaxInsertBlocks) p.ins_blocks = kMaxInsertBlocks;
     cudaEvent_t* ev = opts ? opts->stage_events : nullptr;
     int stage = 0;
     auto mark = [&]() -> cudaError_t {
         return ev ? cudaEventRecord(ev[stage++], stream) : cudaSuccess;
     };
     cudaError_t e = cudaSuccess;
+    // The first kernel follows the stream's earlier work in full; the rest
+    // are programmatic dependents of their predecessor (each waits for it
+    // with griddepcontrol.wait before touching its results).
+    const bool pdl = ev == nullptr;  // events between kernels break the chain anyway
     do {
         if ((e = mark()) != cudaSuccess) break;
         if ((e = launch_prep(p, desc, stream)) != cudaSuccess) break;
         if ((e = mark()) != cudaSuccess) break;
-        if ((e = launch_points(p, false, stream)) != cudaSuccess) break;
+        if ((e = launch_classify(p, rmax, sms, pdl, stream)) != cudaSuccess) break;
         if ((e = mark()) != cudaSuccess) break;
-        if ((e = launch_census(p, sms, stream)) != cudaSuccess) break;
+        if ((e = launch_insert(p, pdl, stream)) != cudaSuccess) break;
         if ((e = mark()) != cudaSuccess) break;
-        if ((e = launch_frames(p, stream)) != cudaSuccess) break;
+        if ((e = launch_compact(p, pdl, stream)) != cudaSuccess) break;
         if ((e = mark()) != cudaSuccess) break;
-        if ((e = launch_capped_census(p, sms, stream)) != cudaSuccess) break;
+        if ((e = launch_scatter_points(p, pdl, stream)) != cudaSuccess) break;
         if ((e = mark()) != cudaSuccess) break;
-        if ((e = launch_scan(p, stream)) != cudaSuccess) break;
+        if ((e = launch_capped_hist(p, sms, pdl, stream)) != cudaSuccess) break;
         if ((e = mark()) != cudaSuccess) break;
-        if ((e = launch_scatter(p, sms, stream)) != cudaSuccess) break;
+        if ((e = launch_frames(p, pdl, stream)) != cudaSuccess) break;
         if ((e = mark()) != cudaSuccess) break;
-        if ((e = launch_rank(p, sms, stream)) != cudaSuccess) break;
+        if ((e = launch_capped_census(p, sms, pdl, stream)) != cudaSuccess) break;
         if ((e = mark()) != cudaSuccess) break;
-        if ((e = launch_finalize(p, sms, stream)) != cudaSuccess) break;
+        if ((e = launch_scan(p, pdl, stream)) != cudaSuccess) break;
+        if ((e = mark()) != cudaSuccess) break;
+        if ((e = launch_scatter(p, sms, pdl, stream)) != cudaSuccess) break;
+        if ((e = mark()) != cudaSuccess) break;
+        if ((e = launch_rank(p, sms, pdl, stream)) != cudaSuccess) break;
+        if ((e = mark()) != cudaSuccess) break;
+        if ((e = launch_finalize(p, sms, pdl, stream)) != cudaSuccess) break;
+        if ((e = mark()) != cudaSuccess) break;
+        if ((e = launch_finalize_heavy(p, sms, pdl, stream)) != cudaSuccess) break;
         if ((e = mark()) != cudaSuccess) break;
     } while (0);
     return e == cudaSuccess ? MMBEV_OK : MMBEV_ECUDA;
@@ -386,7 +426,7 @@ int mmbev_classify_points(const float* points, const int64_t* sweep_offsets, int
     p.cls_lin = out_lin;
     p.cls_rank = out_rank;
     cudaError_t e = launch_prep(p, desc, stream);
-    if (e == cudaSuccess) e = launch_points(p, true, stream);
+    if (e == cudaSuccess) e = launch_classify_points(p, stream);
     return e == cudaSuccess ? MMBEV_OK : MMBEV_ECUDA;
 }
 

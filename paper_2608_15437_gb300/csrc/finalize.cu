@@ -1,96 +1,213 @@
-// Stage 8: voxel feature encoder (S5 of the path; Alg. 1 "VoxelFeatureEncoder").
+// Stages: voxel feature encoder (S5 of the path; Alg. 1 "VoxelFeatureEncoder").
 //
-// One thread per kept voxel, in output order. The voxel's slot holds the
-// bitwise-NOT of its K smallest point indices, largest first, i.e. in
-// ascending point index. The thread gathers those points, recomputes their
-// motion-compensated coordinates with the same fp32 operation order as the
-// point pass (Eq. 6), sums (x', y', z', intensity, dt) in index order, divides
-// once by the count, writes the feature row and the count, and returns the
-// slot to the all-zero state.
+// Each kept voxel's slot gives its point count n and the start of its
+// segment in `seg`, which lists the record positions of all n points (in
+// arrival order). Record positions grow with the point index, so the voxel's
+// first K points by index are its K smallest positions. The records (32
+// bytes each, one sector) hold the compensated x', y', z' computed once by
+// the classify pass with the Eq. 6 operation order, the intensity and dt.
+// The five features are summed over the kept points in index order in fp32
+// and divided once by the count; the feature row and the count are written
+// and the slot is returned to the all-zero state.
+//
+// Light kernel: one thread per kept voxel with at most 32 points keeps the K
+// smallest positions in a sorted register array (each position bubbles in
+// with compare-and-swap steps). Voxels with more points go to a list.
+// Heavy kernel: one warp per listed voxel; each lane keeps the smallest
+// positions of its share of the segment, then K rounds of a warp minimum
+// pick the voxel's K smallest in ascending order, the lanes fetch those
+// records in parallel and lane 0 adds them up in order.
 #include "mmbev_internal.cuh"
 
 namespace mmbev {
 namespace {
 
 constexpr int kThreads = 256;
+constexpr uint32_t kLightMax = 32;
 
+// Insert v into the ascending array b[0..B) (unused entries hold ~0u); the
+// largest entry falls off the end.
+template <int B>
+__device__ __forceinline__ void sorted_insert(uint32_t (&b)[B], uint32_t v) {
+#pragma unroll
+    for (int j = 0; j < B; ++j) {
+        const uint32_t lo = v < b[j] ? v : b[j];
+        const uint32_t hi = v < b[j] ? b[j] : v;
+        b[j] = lo;
+        v = hi;
+    }
+}
+
+__device__ __forceinline__ void add_record(float (&acc)[5], const uint4& a, const uint4& b) {
+    acc[0] = __fadd_rn(acc[0], __uint_as_float(a.w));
+    acc[1] = __fadd_rn(acc[1], __uint_as_float(b.x));
+    acc[2] = __fadd_rn(acc[2], __uint_as_float(b.y));
+    acc[3] = __fadd_rn(acc[3], __uint_as_float(b.z));
+    acc[4] = __fadd_rn(acc[4], __uint_as_float(b.w));
+}
+
+__device__ __forceinline__ void write_voxel(const Params& p, size_t row, const float (&acc)[5],
+                                            int cnt) {
+    const float fc = (float)cnt;
+#pragma unroll
+    for (int c = 0; c < 5; ++c) p.out_feats[row * 5 + c] = __fdiv_rn(acc[c], fc);
+    p.out_counts[row] = cnt;
+}
+
+// Frame and output row of kept voxel g (s_vbase: prefix of kept voxels).
+__device__ __forceinline__ size_t voxel_row(const Params& p, const uint32_t* s_vbase, int F,
+                                            uint32_t g) {
+    int lo = 0, hi = F;  // s_vbase[lo] <= g < s_vbase[hi]
+    while (hi - lo > 1) {
+        const int mid = (lo + hi) >> 1;
+        if (s_vbase[mid] <= g) lo = mid; else hi = mid;
+    }
+    return (size_t)lo * (uint32_t)p.max_voxels + (g - s_vbase[lo]);
+}
+
+template <int B>
 __global__ void __launch_bounds__(kThreads) k_finalize(Params p) {
     __shared__ uint32_t s_vbase[kMaxFrames + 1];
-    __shared__ int64_t s_soff[kMaxSweeps + 1];
-    const int F = p.num_frames, S = p.num_sweeps;
+    pdl_wait();
+    pdl_trigger();
+    const int F = p.num_frames;
     for (int i = threadIdx.x; i < F; i += blockDim.x) s_vbase[i] = p.finfo[i].vbase;
-    for (int i = threadIdx.x; i <= S; i += blockDim.x) s_soff[i] = p.sweep_off[i];
     const uint32_t total = ld_cg(&p.hdr->total_kept);
     if (threadIdx.x == 0) s_vbase[F] = total;
     __syncthreads();
+    const int lane = threadIdx.x & 31;
     const uint32_t gs = gridDim.x * blockDim.x;
     const int K = p.K;
-    for (uint32_t g = blockIdx.x * blockDim.x + threadIdx.x; g < total; g += gs) {
-        int lo = 0, hi = F;  // s_vbase[lo] <= g < s_vbase[hi]
-        while (hi - lo > 1) {
-            const int mid = (lo + hi) >> 1;
-            if (s_vbase[mid] <= g) lo = mid; else hi = mid;
+    for (uint32_t g0 = blockIdx.x * blockDim.x; g0 < total; g0 += gs) {
+        const uint32_t g = g0 + threadIdx.x;
+        const bool act = g < total;
+        uint32_t h = 0, n = 0, off = 0;
+        if (act) {
+            h = p.vid_slot[g];
+            const uint2 s = __ldcg(reinterpret_cast<const uint2*>(slot_key(p, h)));  // seg, -
+            off = s.x;
+            n = ld_cg(slot_cnt(p, h));
         }
-        const int f = lo;
-        const uint32_t vid = g - s_vbase[f];
-        const uint32_t h = p.vid_slot[g];
-        const uint32_t* tk = slot_topk(p, h);
+        const bool heavy = act && n > kLightMax;
+        const uint32_t hm = __ballot_sync(0xFFFFFFFFu, heavy);
+        if (hm) {
+            uint32_t base = 0;
+            if (lane == __ffs(hm) - 1) base = atomicAdd(&p.hdr->num_heavy, (uint32_t)__popc(hm));
+            base = __shfl_sync(0xFFFFFFFFu, base, __ffs(hm) - 1);
+            if (heavy) p.heavy[base + __popc(hm & ((1u << lane) - 1u))] = g;
+        }
+        if (!act || heavy) continue;
+        uint32_t best[B];
+#pragma unroll
+        for (int j = 0; j < B; ++j) best[j] = 0xFFFFFFFFu;
+        for (uint32_t i = 0; i < n; i += 4) {
+            uint32_t v[4];
+#pragma unroll
+            for (int c = 0; c < 4; ++c) v[c] = i + c < n ? __ldg(p.seg + off + i + c) : 0xFFFFFFFFu;
+#pragma unroll
+            for (int c = 0; c < 4; ++c) sorted_insert<B>(best, v[c]);
+        }
+        const int cnt = (int)(n < (uint32_t)K ? n : (uint32_t)K);
         float acc[5] = {0.f, 0.f, 0.f, 0.f, 0.f};
-        int cnt = 0;
-        int s = 0;
-        for (int j0 = 0; j0 < K; j0 += 4) {
-            const uint4 q = __ldcg(reinterpret_cast<const uint4*>(tk + j0));
-            const uint32_t lv[4] = {q.x, q.y, q.z, q.w};
-            bool done = false;
+#pragma unroll
+        for (int j0 = 0; j0 < B; j0 += 4) {
+            if (j0 >= cnt) break;
+            uint4 ra[4], rb[4];
 #pragma unroll
             for (int c = 0; c < 4; ++c) {
-                if (j0 + c >= K || lv[c] == 0u) { done = true; break; }
-                const int64_t idx = (int64_t)(uint32_t)~lv[c];
-                // sweep of idx: indices ascend, so search forward from the last one
-                if (cnt == 0) {
-                    int a = 0, bnd = S;
-                    while (bnd - a > 1) {
-                        const int mid = (a + bnd) >> 1;
-                        if (s_soff[mid] <= idx) a = mid; else bnd = mid;
-                    }
-                    s = a;
-                } else {
-                    while (s + 1 < S && s_soff[s + 1] <= idx) ++s;
+                if (j0 + c < cnt) {
+                    const uint4* rec = p.records + 2 * (size_t)best[j0 + c];
+                    ra[c] = __ldg(rec);
+                    rb[c] = __ldg(rec + 1);
                 }
-                float T[12];
-#pragma unroll
-                for (int e = 0; e < 12; ++e) T[e] = __ldg(p.sweep_tf + (size_t)s * 16 + e);
-                const float* pt = p.points + idx * 5;
-                const float px = __ldg(pt + 0), py = __ldg(pt + 1), pz = __ldg(pt + 2);
-                const float pi = __ldg(pt + 3), pd = __ldg(pt + 4);
-                float x, y, z;
-                compensate(T, px, py, pz, x, y, z);
-                acc[0] = __fadd_rn(acc[0], x);
-                acc[1] = __fadd_rn(acc[1], y);
-                acc[2] = __fadd_rn(acc[2], z);
-                acc[3] = __fadd_rn(acc[3], pi);
-                acc[4] = __fadd_rn(acc[4], pd);
-                ++cnt;
             }
-            if (done) break;
-        }
-        const size_t row = (size_t)f * (uint32_t)p.max_voxels + vid;
-        const float fc = (float)cnt;
 #pragma unroll
-        for (int c = 0; c < 5; ++c) p.out_feats[row * 5 + c] = __fdiv_rn(acc[c], fc);
-        p.out_counts[row] = cnt;
-        // release the slot
-        uint4* sl = reinterpret_cast<uint4*>(p.table + (size_t)h * p.slot_stride);
-        const uint32_t n16 = p.slot_stride / 16;
-        for (uint32_t i = 0; i < n16; ++i) sl[i] = make_uint4(0u, 0u, 0u, 0u);
+            for (int c = 0; c < 4; ++c)
+                if (j0 + c < cnt) add_record(acc, ra[c], rb[c]);
+        }
+        write_voxel(p, voxel_row(p, s_vbase, F, g), acc, cnt);
+        zero_slot(p, h);
+    }
+}
+
+template <int B>
+__global__ void __launch_bounds__(kThreads) k_finalize_heavy(Params p) {
+    __shared__ uint32_t s_vbase[kMaxFrames + 1];
+    pdl_wait();
+    pdl_trigger();
+    const int F = p.num_frames;
+    for (int i = threadIdx.x; i < F; i += blockDim.x) s_vbase[i] = p.finfo[i].vbase;
+    const uint32_t total = ld_cg(&p.hdr->total_kept);
+    if (threadIdx.x == 0) s_vbase[F] = total;
+    __syncthreads();
+    const int lane = threadIdx.x & 31;
+    const uint32_t nh = ld_cg(&p.hdr->num_heavy);
+    const uint32_t gw = (blockIdx.x * blockDim.x + threadIdx.x) >> 5;
+    const uint32_t nw = (gridDim.x * blockDim.x) >> 5;
+    const int K = p.K;
+    for (uint32_t e = gw; e < nh; e += nw) {
+        const uint32_t g = p.heavy[e];
+        const uint32_t h = p.vid_slot[g];
+        const uint32_t off = ld_cg(slot_seg(p, h));
+        const uint32_t n = ld_cg(slot_cnt(p, h));
+        uint32_t best[B];
+#pragma unroll
+        for (int j = 0; j < B; ++j) best[j] = 0xFFFFFFFFu;
+        for (uint32_t i = lane; i < n; i += 32) sorted_insert<B>(best, __ldg(p.seg + off + i));
+        // K rounds of a warp minimum over the lanes' smallest remaining; the
+        // j-th smallest goes to lane j % 32 (second register for j >= 32)
+        const int cnt = (int)(n < (uint32_t)K ? n : (uint32_t)K);
+        uint32_t mine[2] = {0xFFFFFFFFu, 0xFFFFFFFFu};
+        for (int j = 0; j < cnt; ++j) {
+            const uint32_t m = __reduce_min_sync(0xFFFFFFFFu, best[0]);
+            if (lane == (j & 31)) mine[j >> 5] = m;
+            if (best[0] == m) {   // positions are distinct: one lane owns m
+#pragma unroll
+                for (int c = 0; c + 1 < B; ++c) best[c] = best[c + 1];
+                best[B - 1] = 0xFFFFFFFFu;
+            }
+        }
+        float acc[5] = {0.f, 0.f, 0.f, 0.f, 0.f};
+        for (int half = 0; half * 32 < cnt; ++half) {
+            uint4 ra = make_uint4(0u, 0u, 0u, 0u), rb = ra;
+            if (half * 32 + lane < cnt) {
+                const uint4* rec = p.records + 2 * (size_t)mine[half];
+                ra = __ldg(rec);
+                rb = __ldg(rec + 1);
+            }
+            const int m = cnt - half * 32 < 32 ? cnt - half * 32 : 32;
+            for (int j = 0; j < m; ++j) {
+                uint4 a, b;
+                a.w = __shfl_sync(0xFFFFFFFFu, ra.w, j);
+                b.x = __shfl_sync(0xFFFFFFFFu, rb.x, j);
+                b.y = __shfl_sync(0xFFFFFFFFu, rb.y, j);
+                b.z = __shfl_sync(0xFFFFFFFFu, rb.z, j);
+                b.w = __shfl_sync(0xFFFFFFFFu, rb.w, j);
+                add_record(acc, a, b);
+            }
+        }
+        if (lane == 0) {
+            write_voxel(p, voxel_row(p, s_vbase, F, g), acc, cnt);
+            zero_slot(p, h);
+        }
     }
 }
 
 }  // namespace
 
-cudaError_t launch_finalize(const Params& p, int num_sms, cudaStream_t st) {
-    k_finalize<<<num_sms * 4, kThreads, 0, st>>>(p);
-    return cudaGetLastError();
+cudaError_t launch_finalize(const Params& p, int num_sms, bool pdl, cudaStream_t st) {
+    const dim3 grid(num_sms * 8), block(kThreads);
+    if (p.K <= 4) return launch_k(k_finalize<4>, grid, block, 0, st, pdl, p);
+    if (p.K <= 12) return launch_k(k_finalize<12>, grid, block, 0, st, pdl, p);
+    return launch_k(k_finalize<32>, grid, block, 0, st, pdl, p);
+}
+
+cudaError_t launch_finalize_heavy(const Params& p, int num_sms, bool pdl, cudaStream_t st) {
+    const dim3 grid(num_sms * 4), block(kThreads);
+    if (p.K <= 4) return launch_k(k_finalize_heavy<4>, grid, block, 0, st, pdl, p);
+    if (p.K <= 12) return launch_k(k_finalize_heavy<12>, grid, block, 0, st, pdl, p);
+    if (p.K <= 32) return launch_k(k_finalize_heavy<32>, grid, block, 0, st, pdl, p);
+    return launch_k(k_finalize_heavy<kMaxK>, grid, block, 0, st, pdl, p);
 }
 
 }  // namespace mmbev

@@ -1,14 +1,29 @@
 // Internal declarations shared by the kernels of libmmbev (sm_103a).
 //
 // Data layout (one call):
-//   points      caller's float32 [N][5] AoS, read once by the point kernel
-//               through shared-memory tiles (coalesced 16-byte loads).
-//   table       caller's hash table: H = 2^log2 slots of `stride` bytes,
-//               slot = { u64 key+1 (0 = empty), u32 0xFFFFFFFF-minrank
-//               (0 = none), u32 spare, u32 topk[Kp] }; topk holds the
-//               bitwise-NOT of the K smallest point indices of the voxel,
-//               kept sorted by a cascade of atomicMax (largest NOT first =
-//               smallest index first; 0 = empty level).
+//   points      caller's float32 [N][5] AoS, streamed once by the classify
+//               kernel through a 3-stage ring of 40 KB shared-memory tiles,
+//               each tile moved by eight 5 KB cp.async.bulk (TMA) copies.
+//   records     workspace, 32 B per kept point, at position region*32 + (its
+//               rank among the kept points of its 32-point region): {lin,
+//               frame, ROI rank, x', y', z', intensity, dt}. Region g holds
+//               points 32g .. 32g+31, so positions increase with the point
+//               index and "first K by position" is "first K by index".
+//   reg_cnt     workspace, kept points per region.
+//   newlist     workspace, per insert block a sub-list of the voxels that
+//               block created {slot, lin, frame}; the compact kernel
+//               concatenates the sub-lists into the occupied-voxel list.
+//   table       caller's hash table of 16-byte slots: { u64 key+1 (0 =
+//               empty), u32 0xFFFFFFFF-minrank (0 = none), u32 count (points
+//               of the voxel) }. Insert uses the first H slots, H the power of
+//               two >= 1.25 x the kept points of the call (at most the
+//               buffer's capacity, >= 2 x the points). Once the voxels are
+//               listed the key's low word holds the voxel's segment offset.
+//   rec_slot    workspace, per record position {slot, arrival index in the
+//               voxel}, from the insert kernel.
+//   seg         workspace, the record positions of each voxel's points,
+//               voxel after voxel (CSR); a voxel's first K points are its K
+//               smallest positions.
 //   workspace   Header + per-call arrays (see Layout).
 #pragma once
 
@@ -24,21 +39,17 @@ constexpr int kMaxFrames = MMBEV_MAX_FRAMES;
 constexpr int kMaxRoisPerFrame = MMBEV_MAX_ROIS_PER_FRAME;
 constexpr int kMaxK = MMBEV_MAX_PTS_PER_VOXEL;
 
-// Point kernel tiling: 256 threads, 8 points per thread per tile.
-constexpr int kPtsThreads = 256;
-constexpr int kPtsPerThread = 8;
-constexpr int kTile = kPtsThreads * kPtsPerThread;  // 2048 points = 40 KB
+// Point tiles: 2048 points (40 KB) per tile, 64 regions of 32 points.
+constexpr int kTile = 2048;
+constexpr int kTileBytes = kTile * 5 * 4;
+constexpr int kRegion = 32;
 
-// Bucket bitmap ordering: a bucket spans 2^kBucketLog2 consecutive linear
-// indices of one frame; one warp ranks a bucket with two bitmaps in smem.
+// Bucket bitmap ordering: a bucket spans 2^kBucketLog2Max consecutive linear
+// indices of one frame (fewer when the grid is smaller); one warp ranks a
+// bucket with shared-memory bitmaps.
 constexpr int kBucketLog2Max = 13;
 
-// Decoupled look-back scan tile.
-constexpr int kScanThreads = 256;
-constexpr int kScanPerThread = 8;
-constexpr int kScanTile = kScanThreads * kScanPerThread;
-
-// Bounded waits: iterations of a look-back spin before giving up.
+// Bounded waits.
 constexpr uint32_t kSpinLimit = 1u << 22;
 
 constexpr uint32_t kUnset = 0xFFFFFFFFu;
@@ -49,24 +60,28 @@ struct __align__(16) RoiPrep {
     float hl, hw, pad0, pad1;
 };
 
-// Per-frame results of the cap pass.
+// Per-frame results of the frames stage.
 struct __align__(16) FrameInfo {
     uint32_t capped;  // more voxels than max_voxels
     uint32_t rstar;   // rank threshold: ranks < rstar kept, == rstar partly
     uint32_t q;       // how many rank-rstar voxels are kept (smallest lin first)
     uint32_t nvox;    // kept voxels
     uint32_t vbase;   // exclusive prefix of nvox over frames
-    uint32_t pad[3];
+    uint32_t ibase;   // exclusive prefix of the frame's voxel count (item segment)
+    uint32_t pad[2];
 };
 
 // Workspace header; zeroed by the prep kernel at the start of every call.
 struct __align__(16) Header {
-    uint32_t status;       // MMBEV_DEV_* bits
+    uint32_t status;       // MMBEV_DEV_* bits (first word: read by mmbev_get_status)
     uint32_t num_occ;      // occupied slots (unique voxels over all frames)
     uint32_t total_kept;   // kept voxels over all frames
     uint32_t any_capped;   // some frame has more voxels than max_voxels
-    uint32_t scan_ticket;  // tile counter of the look-back scan
-    uint32_t pad[11];
+    uint32_t num_rec;      // kept points (records) of the call
+    uint32_t num_nonempty; // non-empty buckets listed by the scan stage
+    uint32_t seg_total;    // point entries reserved in seg
+    uint32_t num_heavy;    // kept voxels with more than 32 points
+    uint32_t pad[8];
 };
 
 // Everything a kernel needs; passed by value.
@@ -94,11 +109,10 @@ struct Params {
     int32_t bucket_log2;
     uint32_t buckets_per_frame;
     uint32_t num_buckets;   // num_frames * buckets_per_frame
-    uint32_t scan_tiles;
     // hash table
     uint8_t* table;
-    uint32_t table_log2;
-    uint32_t slot_stride;   // bytes
+    uint32_t table_log2;    // the buffer's capacity (log2 slots)
+    int32_t table_log2_fixed;  // > 0: use this many slots instead of sizing by the points
     // workspace arrays
     Header* hdr;
     int64_t* sweep_off;     // [S+1]
@@ -110,16 +124,27 @@ struct Params {
     uint32_t* hist;         // [R] voxels per minimum rank (capped frames)
     uint32_t* frame_u;      // [F] unique voxels per frame
     FrameInfo* finfo;       // [F]
-    unsigned long long* bcnt;  // [B+1] (lo: rank-below count, hi: rank-tie count)
-    unsigned long long* scan_agg;  // [tiles]
-    unsigned long long* scan_inc;  // [tiles]
-    uint32_t* scan_flag;    // [tiles]
+    uint4* records;         // [tiles*2048][2] kept points (see above)
+    uint32_t* reg_cnt;      // [regions] kept points per 32-point region
+    uint2* rec_slot;        // [regions*32] slot and arrival index of each record
+    uint32_t* seg;          // [N] record positions, voxel by voxel
+    uint32_t num_regions;
+    uint4* newlist;         // [regions*32] voxels created, per insert block: slot, lin, frame
+    uint32_t* blockcount;   // [ins_blocks] voxels each insert block created
+    uint32_t ins_blocks;    // grid of the insert kernel
+    unsigned long long* bcnt;   // [B] voxels per bucket (every frame, no classes)
+    unsigned long long* bcnt2;  // [B] capped frames: lo = rank-below, hi = rank-tie
+    unsigned long long* boff;   // [B] exclusive offsets within the frame (lo, hi)
     uint32_t* occ;          // [occ_cap] slot of each unique voxel
     uint32_t* d_bucket;     // [occ_cap]
     uint32_t* d_pos;        // [occ_cap] position inside the bucket
-    uint32_t* items;        // [occ_cap] voxel ids grouped by bucket
+    uint32_t* d_lin;        // [occ_cap] linear index of each unique voxel
+    uint2* items;           // [occ_cap] (slot, lin) grouped by bucket
+    uint32_t* nonempty;     // [B] non-empty bucket ids
     uint32_t* vid_slot;     // [F*max_voxels] slot of each kept voxel, output order
+    uint32_t* heavy;        // [F*max_voxels] kept voxels with more than 32 points
     uint32_t occ_cap;
+    uint32_t rec_cap;
     // outputs
     float* out_feats;
     int32_t* out_coords;
@@ -146,6 +171,11 @@ __device__ __forceinline__ void set_status(Header* hdr, uint32_t bits) {
     atomicOr(&hdr->status, bits);
 }
 
+// Programmatic dependent launch: wait for the preceding kernel's results,
+// and let the next kernel's blocks be scheduled.
+__device__ __forceinline__ void pdl_wait() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
+__device__ __forceinline__ void pdl_trigger() { asm volatile("griddepcontrol.launch_dependents;"); }
+
 // Eq. 6 for one point: ((r0*x + r1*y) + r2*z) + t, every op rounded (no FMA).
 __device__ __forceinline__ void compensate(const float* T, float x, float y, float z,
                                            float& xo, float& yo, float& zo) {
@@ -166,15 +196,77 @@ __device__ __forceinline__ bool roi_contains(const RoiPrep& r, float x, float y)
     return fabsf(u) <= r.hl && fabsf(v) <= r.hw;
 }
 
-// Slot addressing.
+// S2 for one compensated point: range crop, coarse-mask candidates, exact
+// ROI test in rank order, voxel index. `fmask` is the point's frame's coarse
+// mask (coarse^2 cells x mask_words) and `frois` its prepared ROIs, either
+// in shared memory (staged) or in global memory. Returns true and sets lin,
+// rank when the point is kept.
+__device__ __forceinline__ bool classify_point(const Params& p, const uint32_t* fmask,
+                                               const RoiPrep* frois, float x, float y, float z,
+                                               uint32_t& lin, uint32_t& rank) {
+    if (!((p.rmin[0] <= x) && (x < p.rmax[0]) && (p.rmin[1] <= y) && (y < p.rmax[1]) &&
+          (p.rmin[2] <= z) && (z < p.rmax[2])))
+        return false;
+    const int G = p.coarse;
+    const float dx0 = __fsub_rn(x, p.rmin[0]);
+    const float dy0 = __fsub_rn(y, p.rmin[1]);
+    int gx = (int)__fmul_rn(dx0, p.coarse_inv[0]);
+    int gy = (int)__fmul_rn(dy0, p.coarse_inv[1]);
+    gx = min(max(gx, 0), G - 1);
+    gy = min(max(gy, 0), G - 1);
+    const uint32_t* mw = fmask + (gy * G + gx) * p.mask_words;
+    int hit = -1;
+    for (int w = 0; w < p.mask_words && hit < 0; ++w) {
+        uint32_t bits = mw[w];
+        while (bits) {
+            const int b = __ffs(bits) - 1;
+            bits &= bits - 1u;
+            const int r = w * 32 + b;
+            const float4* rp4 = reinterpret_cast<const float4*>(frois + r);
+            const float4 a = rp4[0], c = rp4[1];
+            RoiPrep rp;
+            rp.cx = a.x; rp.cy = a.y; rp.c = a.z; rp.s = a.w; rp.hl = c.x; rp.hw = c.y;
+            if (roi_contains(rp, x, y)) { hit = r; break; }
+        }
+    }
+    if (hit < 0) return false;
+    const uint32_t cx = __float2uint_rz(__fdiv_rn(dx0, p.vs[0]));
+    const uint32_t cy = __float2uint_rz(__fdiv_rn(dy0, p.vs[1]));
+    const uint32_t cz = __float2uint_rz(__fdiv_rn(__fsub_rn(z, p.rmin[2]), p.vs[2]));
+    if (cx >= p.dims[0] || cy >= p.dims[1] || cz >= p.dims[2]) return false;
+    lin = (cz * p.dims[1] + cy) * p.dims[0] + cx;
+    rank = (uint32_t)hit;
+    return true;
+}
+
+// Sweep of global point index i: largest s with off[s] <= i (off nondecreasing).
+__device__ __forceinline__ int find_sweep(const int64_t* off, int nsweeps, int64_t i) {
+    int lo = 0, hi = nsweeps;  // off[lo] <= i < off[hi]
+    while (hi - lo > 1) {
+        const int mid = (lo + hi) >> 1;
+        if (off[mid] <= i) lo = mid; else hi = mid;
+    }
+    return lo;
+}
+
+// Slot addressing (16-byte slots).
+constexpr uint32_t kSlotBytes = 16;
 __device__ __forceinline__ unsigned long long* slot_key(const Params& p, uint32_t h) {
-    return reinterpret_cast<unsigned long long*>(p.table + (size_t)h * p.slot_stride);
+    return reinterpret_cast<unsigned long long*>(p.table + (size_t)h * kSlotBytes);
 }
 __device__ __forceinline__ uint32_t* slot_rank(const Params& p, uint32_t h) {
-    return reinterpret_cast<uint32_t*>(p.table + (size_t)h * p.slot_stride + 8);
+    return reinterpret_cast<uint32_t*>(p.table + (size_t)h * kSlotBytes + 8);
 }
-__device__ __forceinline__ uint32_t* slot_topk(const Params& p, uint32_t h) {
-    return reinterpret_cast<uint32_t*>(p.table + (size_t)h * p.slot_stride + 16);
+__device__ __forceinline__ uint32_t* slot_cnt(const Params& p, uint32_t h) {
+    return reinterpret_cast<uint32_t*>(p.table + (size_t)h * kSlotBytes + 12);
+}
+// valid once the voxel list is built: the key is no longer needed
+__device__ __forceinline__ uint32_t* slot_seg(const Params& p, uint32_t h) {
+    return reinterpret_cast<uint32_t*>(p.table + (size_t)h * kSlotBytes);
+}
+
+__device__ __forceinline__ void zero_slot(const Params& p, uint32_t h) {
+    *reinterpret_cast<uint4*>(p.table + (size_t)h * kSlotBytes) = make_uint4(0u, 0u, 0u, 0u);
 }
 
 // 64-bit mixer (the SplitMix64 finalizer of Steele, Lea and Flood, 2014).
@@ -184,24 +276,56 @@ __device__ __forceinline__ uint64_t mix64(uint64_t z) {
     return z ^ (z >> 31);
 }
 
+__device__ __forceinline__ uint32_t slot_home(uint32_t mask, unsigned long long key1) {
+    return (uint32_t)mix64(key1) & mask;
+}
+
 // Load at L2 (bypassing the non-coherent L1), for words other blocks update.
 __device__ __forceinline__ uint32_t ld_cg(const uint32_t* a) { return __ldcg(a); }
 __device__ __forceinline__ unsigned long long ld_cg(const unsigned long long* a) {
     return __ldcg(a);
 }
 
+__device__ __forceinline__ uint32_t slot_minrank(const Params& p, uint32_t h) {
+    return 0xFFFFFFFFu - ld_cg(slot_rank(p, h));
+}
+
 // ---------------------------------------------------------------- launchers
 
-// All launchers enqueue on `st` and return the cudaGetLastError() result.
+// All launchers enqueue on `st` and return the launch's error code. `pdl`
+// launches the kernel as a programmatic dependent of the preceding one.
 cudaError_t launch_prep(const Params& p, const HostDesc& d, cudaStream_t st);
-cudaError_t launch_points(const Params& p, bool classify_only, cudaStream_t st);
-cudaError_t launch_census(const Params& p, int num_sms, cudaStream_t st);
-cudaError_t launch_frames(const Params& p, cudaStream_t st);
-cudaError_t launch_capped_census(const Params& p, int num_sms, cudaStream_t st);
-cudaError_t launch_scan(const Params& p, cudaStream_t st);
-cudaError_t launch_scatter(const Params& p, int num_sms, cudaStream_t st);
-cudaError_t launch_rank(const Params& p, int num_sms, cudaStream_t st);
-cudaError_t launch_finalize(const Params& p, int num_sms, cudaStream_t st);
+cudaError_t launch_classify(const Params& p, int rmax, int num_sms, bool pdl, cudaStream_t st);
+cudaError_t launch_classify_points(const Params& p, cudaStream_t st);
+cudaError_t launch_insert(const Params& p, bool pdl, cudaStream_t st);
+cudaError_t launch_compact(const Params& p, bool pdl, cudaStream_t st);
+cudaError_t launch_scatter_points(const Params& p, bool pdl, cudaStream_t st);
+uint32_t insert_blocks(int num_sms);
+cudaError_t launch_capped_hist(const Params& p, int num_sms, bool pdl, cudaStream_t st);
+cudaError_t launch_frames(const Params& p, bool pdl, cudaStream_t st);
+cudaError_t launch_capped_census(const Params& p, int num_sms, bool pdl, cudaStream_t st);
+cudaError_t launch_scan(const Params& p, bool pdl, cudaStream_t st);
+cudaError_t launch_scatter(const Params& p, int num_sms, bool pdl, cudaStream_t st);
+cudaError_t launch_rank(const Params& p, int num_sms, bool pdl, cudaStream_t st);
+cudaError_t launch_finalize(const Params& p, int num_sms, bool pdl, cudaStream_t st);
+cudaError_t launch_finalize_heavy(const Params& p, int num_sms, bool pdl, cudaStream_t st);
 cudaError_t launch_zero(void* ptr, size_t bytes, cudaStream_t st);
+
+// Launch `kern` with an optional programmatic-stream-serialization attribute.
+template <typename... KArgs, typename... Args>
+cudaError_t launch_k(void (*kern)(KArgs...), dim3 grid, dim3 block, size_t smem,
+                     cudaStream_t st, bool pdl, Args&&... args) {
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = grid;
+    cfg.blockDim = block;
+    cfg.dynamicSmemBytes = smem;
+    cfg.stream = st;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[0].val.programmaticStreamSerializationAllowed = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = pdl ? 1 : 0;
+    return cudaLaunchKernelEx(&cfg, kern, static_cast<KArgs>(args)...);
+}
 
 }  // namespace mmbev

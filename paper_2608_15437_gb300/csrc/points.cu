@@ -1,322 +1,356 @@
-// Stage 1: the point pass (S1 + S2 + S3 of the path).
+// Stage 1: the classify pass (S1 + S2 of the path).
 //
-// One block takes a tile of 2048 consecutive points:
-//   A. loads the tile's 40 KB of float32 AoS points into shared memory with
-//      coalesced 16-byte streaming loads, stages the tile's sweep transforms;
-//   B. per point: Eq. 6 motion compensation, range crop, Alg. 1 inside-ROI
-//      test (coarse candidate mask, then the exact rotated-box test in rank
-//      order; the first hit is the point's rank), voxel index;
-//   C. ballot/popc compaction of the kept points into a shared queue that
-//      preserves input order;
-//   D. hash insert of the queue: lanes with equal keys are grouped with
-//      __match_any_sync; the group leader probes / claims the slot and lowers
-//      the slot's minimum rank once for the group; every lane then inserts its
-//      point index into the slot's bounded "K smallest indices" list;
-//   E. one atomicAdd per block appends the block's new slots to the
-//      occupied-slot list; per-frame voxel counts are block-aggregated too.
+// A persistent kernel, one block of 1,024 threads (32 warps) per SM,
+// streams a contiguous range of 2,048-point tiles through a ring of 40 KB
+// shared-memory buffers. Each tile arrives as eight 5 KB cp.async.bulk (TMA)
+// copies with an L2 evict-first policy, counted on the buffer's mbarrier: on
+// GB300 a single 40 KB bulk copy per tile streams at about a quarter of HBM
+// bandwidth, eight concurrent ones at nearly all of it. The warps never wait
+// for each other: each warp classifies its own 64 points of a tile, and the
+// last warp to finish a tile (a shared-memory counter) refills that buffer.
+// Per point: Eq. 6 motion compensation, range crop, Alg. 1 inside-ROI test
+// (coarse candidate mask, then the exact rotated-box test in rank order;
+// the first hit is the point's rank) and the voxel index. The masks and
+// prepared ROIs of the (one or two) frames a block's tile range starts with
+// sit in shared memory. Kept points are compacted per 32-point region with
+// a warp ballot, in input order, and written as 32-byte records at
+// position (region)*32 + (rank among the region's kept points), with the
+// compensated features, so later stages never touch the raw points again.
+//
+// The classify-only entry point (per-point outputs for testing S1-S2) uses a
+// plain one-thread-per-point kernel built from the same device functions.
+#include <atomic>
+
 #include "mmbev_internal.cuh"
 
 namespace mmbev {
 namespace {
 
-constexpr int kTfStage = 64;   // sweeps staged in smem per tile
-constexpr int kFrameCnt = 32;  // frames counted in smem per tile
-constexpr int kWarps = kPtsThreads / 32;
+constexpr int kThreads = 1024;
+constexpr int kWarps = kThreads / 32;         // 32
+constexpr int kTfStageMax = 512;              // sweeps whose transforms sit in smem
+constexpr int kMaskSmemWords = 4096;          // one staged frame's coarse mask (16 KB)
+constexpr int kChunks = 8;                    // bulk copies per tile
+constexpr int kChunkBytes = kTileBytes / kChunks;
+static_assert(kTile == kWarps * 2 * kRegion, "a warp covers two regions of a tile");
 
-struct QItem {
-    unsigned long long key;
-    uint32_t idx;
-    uint32_t rank;
+// ---- TMA / mbarrier helpers (inline PTX)
+__device__ __forceinline__ uint32_t smem_addr(const void* p) {
+    return (uint32_t)__cvta_generic_to_shared(p);
+}
+__device__ __forceinline__ void mbar_init(uint64_t* bar, uint32_t count) {
+    asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" ::"r"(smem_addr(bar)), "r"(count)
+                 : "memory");
+}
+__device__ __forceinline__ void mbar_fence_init() {
+    asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+}
+__device__ __forceinline__ void mbar_expect_tx(uint64_t* bar, uint32_t bytes) {
+    asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(smem_addr(bar)),
+                 "r"(bytes)
+                 : "memory");
+}
+__device__ __forceinline__ bool mbar_try_wait(uint64_t* bar, uint32_t parity) {
+    uint32_t ok;
+    asm volatile(
+        "{\n\t.reg .pred p;\n\t"
+        "mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n\t"
+        "selp.u32 %0, 1, 0, p;\n\t}"
+        : "=r"(ok)
+        : "r"(smem_addr(bar)), "r"(parity)
+        : "memory");
+    return ok != 0;
+}
+__device__ __forceinline__ uint64_t evict_first_policy() {
+    uint64_t pol;
+    asm volatile("createpolicy.fractional.L2::evict_first.b64 %0, 1.0;" : "=l"(pol));
+    return pol;
+}
+__device__ __forceinline__ void tma_load(void* dst, const void* src, uint32_t bytes,
+                                         uint64_t* bar, uint64_t pol) {
+    asm volatile(
+        "cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes.L2::cache_hint "
+        "[%0], [%1], %2, [%3], %4;" ::"r"(smem_addr(dst)),
+        "l"(src), "r"(bytes), "r"(smem_addr(bar)), "l"(pol)
+        : "memory");
+}
+
+// Bounded wait on an mbarrier phase; false when the wait gave up.
+__device__ __forceinline__ bool mbar_wait(uint64_t* bar, uint32_t parity) {
+    for (uint32_t i = 0; i < kSpinLimit; ++i)
+        if (mbar_try_wait(bar, parity)) return true;
+    return false;
+}
+
+struct ClsSmem {
+    float* stages;    // [nstages][kTile * 5]
+    uint32_t* mask;   // [2][kMaskSmemWords] coarse masks of the staged frames
+    RoiPrep* rois;    // [2][rmax] prepared ROIs of the staged frames
+    float* tf;        // [S][12] when staged
+    int64_t* soff;    // [S+1]
+    int32_t* sfr;     // [S] frame of each sweep
+    int32_t* sr0;     // [S] first ROI of that frame
+    uint64_t* full;   // [nstages] tile arrived
+    uint32_t* done;   // [nstages] warps finished with the buffer
+    uint32_t* kept;   // [2] kept points of the block, warps finished
 };
-static_assert(kTile * sizeof(QItem) + kTile * sizeof(uint32_t) <= kTile * 5 * sizeof(float),
-              "queue and new-slot list must fit in the point tile");
 
-// Sweep of global point index i: largest s with off[s] <= i (off nondecreasing).
-__device__ __forceinline__ int find_sweep(const int64_t* off, int nsweeps, int64_t i) {
-    int lo = 0, hi = nsweeps;  // off[lo] <= i < off[hi]
-    while (hi - lo > 1) {
-        const int mid = (lo + hi) >> 1;
-        if (off[mid] <= i) lo = mid; else hi = mid;
-    }
-    return lo;
+__host__ __device__ inline size_t align16(size_t o) { return (o + 15) & ~(size_t)15; }
+
+__host__ __device__ inline size_t classify_smem_bytes(int S, int rmax, int nstages) {
+    const bool tf_staged = S <= kTfStageMax;
+    size_t o = (size_t)nstages * kTileBytes + 2 * kMaskSmemWords * 4 + 2 * (size_t)rmax * 32;
+    o += tf_staged ? (size_t)S * 48 : 0;
+    o += (size_t)(S + 1) * 8 + (size_t)S * 8;
+    o = align16(o);
+    return o + (size_t)nstages * 8 + (size_t)nstages * 4 + 8;
 }
 
-// Claim or find the slot of key+1 by linear probing; at most H probes.
-// Returns the slot, sets *is_new when this call claimed it; 0xFFFFFFFF when
-// the table is full.
-__device__ __forceinline__ uint32_t table_insert(const Params& p, unsigned long long key1,
-                                                 bool* is_new) {
-    const uint32_t mask = (uint32_t)((1ull << p.table_log2) - 1ull);
-    uint32_t h = (uint32_t)mix64(key1) & mask;
-    *is_new = false;
-    for (uint64_t probe = 0; probe <= mask; ++probe) {
-        unsigned long long* kp = slot_key(p, h);
-        const unsigned long long cur = ld_cg(kp);
-        if (cur == key1) return h;
-        if (cur == 0ull) {
-            const unsigned long long old = atomicCAS(kp, 0ull, key1);
-            if (old == 0ull) { *is_new = true; return h; }
-            if (old == key1) return h;
-        }
-        h = (h + 1u) & mask;
-    }
-    return kUnset;
+__device__ __forceinline__ ClsSmem carve(unsigned char* smem, int S, int rmax, bool tf_staged,
+                                         int nstages) {
+    ClsSmem s;
+    size_t o = 0;
+    s.stages = reinterpret_cast<float*>(smem);
+    o += (size_t)nstages * kTileBytes;
+    s.mask = reinterpret_cast<uint32_t*>(smem + o);
+    o += 2 * kMaskSmemWords * 4;
+    s.rois = reinterpret_cast<RoiPrep*>(smem + o);
+    o += 2 * (size_t)rmax * 32;
+    s.tf = reinterpret_cast<float*>(smem + o);
+    o += tf_staged ? (size_t)S * 48 : 0;
+    s.soff = reinterpret_cast<int64_t*>(smem + o);
+    o += (size_t)(S + 1) * 8;
+    s.sfr = reinterpret_cast<int32_t*>(smem + o);
+    o += (size_t)S * 4;
+    s.sr0 = reinterpret_cast<int32_t*>(smem + o);
+    o += (size_t)S * 4;
+    o = align16(o);
+    s.full = reinterpret_cast<uint64_t*>(smem + o);
+    o += (size_t)nstages * 8;
+    s.done = reinterpret_cast<uint32_t*>(smem + o);
+    o += (size_t)nstages * 4;
+    s.kept = reinterpret_cast<uint32_t*>(smem + o);
+    return s;
 }
 
-// Insert v = ~index into the slot's sorted list of the K largest values
-// (= the K smallest point indices). Levels only ever grow, so a level read
-// as >= v stays >= v and can be skipped; each atomicMax keeps the larger of
-// (level, v) and carries the smaller one down; an empty level (0) ends it.
-__device__ __forceinline__ void topk_insert(uint32_t* tk, uint32_t v, int K) {
-    int j = 0;
-    while (j < K) {
-        // One round trip reads up to 12 levels.
-        uint32_t lv[12];
-        const int nread = (K - j) < 12 ? (K - j) : 12;
-#pragma unroll
-        for (int c = 0; c < 12; ++c) lv[c] = c < nread ? ld_cg(tk + j + c) : 0u;
-        int first = nread;
-#pragma unroll
-        for (int c = 11; c >= 0; --c)
-            if (c < nread && lv[c] < v) first = c;
-        j += first;
-        if (first < nread) break;
-    }
-    for (; j < K; ++j) {
-        const uint32_t old = atomicMax(tk + j, v);
-        if (old == 0u) return;
-        v = old < v ? old : v;
-    }
-}
-
-template <bool kClassify>
-__global__ void __launch_bounds__(kPtsThreads)
-k_points(Params p) {
-    __shared__ __align__(16) float s_pts[kTile * 5];
-    __shared__ __align__(16) float s_tf[kTfStage][12];
-    __shared__ int64_t s_soff[kTfStage + 1];
-    __shared__ int32_t s_sfr[kTfStage];
-    __shared__ int32_t s_r0[kTfStage];
-    __shared__ uint32_t s_wcnt[kPtsPerThread * kWarps];
-    __shared__ uint32_t s_fcnt[kFrameCnt];
-    __shared__ int s_slo, s_nst;
-    __shared__ uint32_t s_nq, s_nnew, s_occ_base;
-
+__global__ void __launch_bounds__(kThreads, 1) k_classify(Params p, int rmax, int nstages) {
+    extern __shared__ __align__(128) unsigned char smem[];
+    pdl_wait();
+    pdl_trigger();
     const int t = threadIdx.x, lane = t & 31, warp = t >> 5;
-    const int64_t tile_base = (int64_t)blockIdx.x * kTile;
-    const int64_t rem = p.num_points - tile_base;
-    const int n = rem < (int64_t)kTile ? (int)rem : kTile;
-    if (n <= 0) return;
+    const int S = p.num_sweeps;
+    const bool tf_staged = S <= kTfStageMax;
+    ClsSmem sm = carve(smem, S, rmax, tf_staged, nstages);
 
-    // ---- A. stage points and sweep metadata
-    {
-        const float* src = p.points + tile_base * 5;
-        const int nf = n * 5;
-        const int n4 = nf >> 2;
-        const float4* src4 = reinterpret_cast<const float4*>(src);
-        float4* dst4 = reinterpret_cast<float4*>(s_pts);
-        for (int i = t; i < n4; i += kPtsThreads) dst4[i] = __ldcs(src4 + i);
-        for (int i = (n4 << 2) + t; i < nf; i += kPtsThreads) s_pts[i] = __ldcs(src + i);
+    const int64_t N = p.num_points;
+    const int64_t num_tiles = (N + kTile - 1) / kTile;
+    const int64_t full_tiles = N / kTile;
+    const int64_t t_begin = (int64_t)blockIdx.x * num_tiles / gridDim.x;
+    const int64_t t_end = ((int64_t)blockIdx.x + 1) * num_tiles / gridDim.x;
+    if (t_begin >= t_end) return;
+    const int G2W = p.coarse * p.coarse * p.mask_words;
+
+    for (int i = t; i <= S; i += kThreads) sm.soff[i] = p.sweep_off[i];
+    for (int i = t; i < S; i += kThreads) {
+        const int f = p.sweep_frame[i];
+        sm.sfr[i] = f;
+        sm.sr0[i] = p.frame_roi_off[f];
     }
+    if (tf_staged)
+        for (int i = t; i < S * 12; i += kThreads)
+            sm.tf[i] = __ldg(p.sweep_tf + (size_t)(i / 12) * 16 + (i % 12));
+    // the frame of the range's first point and the next one
+    const int f_lo = p.sweep_frame[find_sweep(p.sweep_off, S, t_begin * kTile)];
+    const int n_staged = f_lo + 1 < p.num_frames ? 2 : 1;
+    for (int k = 0; k < n_staged; ++k) {
+        const int f = f_lo + k;
+        const int r0 = p.frame_roi_off[f];
+        const int rn = min(p.frame_roi_off[f + 1] - r0, rmax);
+        const uint32_t* gm = p.masks + (size_t)f * G2W;
+        for (int i = t; i < G2W; i += kThreads) sm.mask[k * kMaskSmemWords + i] = gm[i];
+        for (int i = t; i < rn * 2; i += kThreads)
+            reinterpret_cast<float4*>(sm.rois + (size_t)k * rmax)[i] =
+                reinterpret_cast<const float4*>(p.roi_prep + r0)[i];
+    }
+    const uint64_t pol = evict_first_policy();
     if (t == 0) {
-        const int slo = find_sweep(p.sweep_off, p.num_sweeps, tile_base);
-        const int shi = find_sweep(p.sweep_off, p.num_sweeps, tile_base + n - 1);
-        s_slo = slo;
-        s_nst = shi - slo + 1;
-        s_nq = 0;
-        s_nnew = 0;
-    }
-    if (t < kFrameCnt) s_fcnt[t] = 0u;
-    __syncthreads();
-    const int slo = s_slo, nst = s_nst;
-    const bool staged = nst <= kTfStage;
-    if (staged) {
-        for (int i = t; i < nst * 12; i += kPtsThreads) {
-            const int k = i / 12, c = i % 12;
-            s_tf[k][c] = __ldg(p.sweep_tf + (size_t)(slo + k) * 16 + c);
+        for (int s = 0; s < nstages; ++s) {
+            mbar_init(&sm.full[s], kChunks);
+            sm.done[s] = 0u;
         }
-        for (int i = t; i <= nst; i += kPtsThreads) s_soff[i] = p.sweep_off[slo + i];
-        for (int i = t; i < nst; i += kPtsThreads) {
-            const int f = p.sweep_frame[slo + i];
-            s_sfr[i] = f;
-            s_r0[i] = p.frame_roi_off[f];
-        }
+        sm.kept[0] = sm.kept[1] = 0u;
+        mbar_fence_init();
     }
     __syncthreads();
-    const int f_first = staged ? s_sfr[0] : 0;
+    // lanes 0..kChunks-1 of one warp each move one chunk of a tile
+    auto issue = [&](int stage, int64_t tile) {
+        if (lane < kChunks) {
+            const size_t off = (size_t)lane * kChunkBytes;
+            mbar_expect_tx(&sm.full[stage], kChunkBytes);
+            tma_load(reinterpret_cast<unsigned char*>(sm.stages + (size_t)stage * kTile * 5) + off,
+                     reinterpret_cast<const unsigned char*>(p.points + tile * kTile * 5) + off,
+                     kChunkBytes, &sm.full[stage], pol);
+        }
+    };
+    if (warp == 0)
+        for (int s = 0; s < nstages; ++s) {
+            const int64_t tile = t_begin + s;
+            if (tile < t_end && tile < full_tiles) issue(s, tile);
+        }
 
-    // ---- B. per point
-    const int G = p.coarse, W = p.mask_words;
-    unsigned long long key[kPtsPerThread];
-    uint32_t rank[kPtsPerThread];
-    bool valid[kPtsPerThread];
-#pragma unroll
-    for (int k = 0; k < kPtsPerThread; ++k) {
-        const int j = t + k * kPtsThreads;
-        valid[k] = false;
-        key[k] = 0ull;
-        rank[k] = 0u;
-        if (j >= n) continue;
-        const int64_t idx = tile_base + j;
-        const float* q = s_pts + 5 * j;
-        int sl;
-        const float* T;
-        int f, r0;
-        float Tg[12];
-        if (staged) {
-            sl = 0;
-            while (s_soff[sl + 1] <= idx) ++sl;
-            T = s_tf[sl];
-            f = s_sfr[sl];
-            r0 = s_r0[sl];
-        } else {
-            const int s = find_sweep(p.sweep_off, p.num_sweeps, idx);
-#pragma unroll
-            for (int c = 0; c < 12; ++c) Tg[c] = __ldg(p.sweep_tf + (size_t)s * 16 + c);
-            T = Tg;
-            f = p.sweep_frame[s];
-            r0 = p.frame_roi_off[f];
-        }
-        float x, y, z;
-        compensate(T, q[0], q[1], q[2], x, y, z);
-        if (kClassify) {
-            p.cls_xyz[idx * 3 + 0] = x;
-            p.cls_xyz[idx * 3 + 1] = y;
-            p.cls_xyz[idx * 3 + 2] = z;
-        }
-        bool ok = (p.rmin[0] <= x) && (x < p.rmax[0]) && (p.rmin[1] <= y) && (y < p.rmax[1]) &&
-                  (p.rmin[2] <= z) && (z < p.rmax[2]);
-        int r_hit = -1;
-        if (ok) {
-            int gx = (int)__fmul_rn(__fsub_rn(x, p.rmin[0]), p.coarse_inv[0]);
-            int gy = (int)__fmul_rn(__fsub_rn(y, p.rmin[1]), p.coarse_inv[1]);
-            gx = min(max(gx, 0), G - 1);
-            gy = min(max(gy, 0), G - 1);
-            const uint32_t* mw = p.masks + ((size_t)f * G * G + (size_t)gy * G + gx) * W;
-            for (int w = 0; w < W && r_hit < 0; ++w) {
-                uint32_t bits = __ldg(mw + w);
-                while (bits) {
-                    const int b = __ffs(bits) - 1;
-                    bits &= bits - 1u;
-                    const int r = w * 32 + b;
-                    const RoiPrep rp = p.roi_prep[r0 + r];
-                    if (roi_contains(rp, x, y)) { r_hit = r; break; }
-                }
-            }
-        }
-        uint32_t lin = 0;
-        if (r_hit >= 0) {
-            const uint32_t cx = __float2uint_rz(__fdiv_rn(__fsub_rn(x, p.rmin[0]), p.vs[0]));
-            const uint32_t cy = __float2uint_rz(__fdiv_rn(__fsub_rn(y, p.rmin[1]), p.vs[1]));
-            const uint32_t cz = __float2uint_rz(__fdiv_rn(__fsub_rn(z, p.rmin[2]), p.vs[2]));
-            if (cx < p.dims[0] && cy < p.dims[1] && cz < p.dims[2]) {
-                lin = (cz * p.dims[1] + cy) * p.dims[0] + cx;
-                valid[k] = true;
-                rank[k] = (uint32_t)r_hit;
-                key[k] = ((unsigned long long)(uint32_t)f << 32) | lin;
-            }
-        }
-        if (kClassify) {
-            p.cls_lin[idx] = valid[k] ? (int64_t)lin : (int64_t)-1;
-            p.cls_rank[idx] = valid[k] ? r_hit : -1;
-        }
-    }
-    if (kClassify) return;
-
-    // ---- C. order-preserving compaction into the shared queue
-    uint32_t ballots[kPtsPerThread];
-#pragma unroll
-    for (int k = 0; k < kPtsPerThread; ++k) {
-        ballots[k] = __ballot_sync(0xFFFFFFFFu, valid[k]);
-        if (lane == 0) s_wcnt[k * kWarps + warp] = __popc(ballots[k]);
-    }
-    __syncthreads();
-    if (warp == 0) {
-        // exclusive scan of 64 counts, two per lane, in (k, warp) order
-        const uint32_t a = s_wcnt[2 * lane], b = s_wcnt[2 * lane + 1];
-        uint32_t s = a + b;
-#pragma unroll
-        for (int o = 1; o < 32; o <<= 1) {
-            const uint32_t v = __shfl_up_sync(0xFFFFFFFFu, s, o);
-            if (lane >= o) s += v;
-        }
-        const uint32_t excl = s - (a + b);
-        s_wcnt[2 * lane] = excl;
-        s_wcnt[2 * lane + 1] = excl + a;
-        if (lane == 31) s_nq = s;
-    }
-    __syncthreads();
-    QItem* queue = reinterpret_cast<QItem*>(s_pts);
-    uint32_t* new_slots = reinterpret_cast<uint32_t*>(queue + kTile);
     const uint32_t lt = (1u << lane) - 1u;
-#pragma unroll
-    for (int k = 0; k < kPtsPerThread; ++k) {
-        if (valid[k]) {
-            const uint32_t pos = s_wcnt[k * kWarps + warp] + __popc(ballots[k] & lt);
-            QItem it;
-            it.key = key[k];
-            it.idx = (uint32_t)(tile_base + t + k * kPtsThreads);
-            it.rank = rank[k];
-            queue[pos] = it;
+    uint32_t kept_total = 0;   // this warp's kept points (lane 0)
+    int s = -1;                // sweep of this thread's latest point
+    float T[12];               // that sweep's transform
+    for (int64_t i = 0; t_begin + i < t_end; ++i) {
+        const int64_t tile = t_begin + i;
+        const int st = (int)(i % nstages);
+        const uint32_t parity = (uint32_t)((i / nstages) & 1);
+        float* sp = sm.stages + (size_t)st * kTile * 5;
+        const int64_t base = tile * kTile;
+        const int n = (int)((N - base) < kTile ? (N - base) : kTile);
+        if (tile < full_tiles) {
+            if (!mbar_wait(&sm.full[st], parity)) {
+                if (lane == 0) set_status(p.hdr, MMBEV_DEV_WAIT_TIMEOUT);
+                return;
+            }
+        } else {
+            // the ragged last tile: this warp loads its own 64 points
+            const float* src = p.points + base * 5;
+            for (int k = warp * 320 + lane; k < warp * 320 + 320 && k < n * 5; k += 32)
+                sp[k] = __ldcs(src + k);
+            __syncwarp();
         }
-    }
-    __syncthreads();
-
-    // ---- D. hash insert
-    const uint32_t nq = s_nq;
-    for (uint32_t base = (uint32_t)warp * 32u; base < nq; base += kPtsThreads) {
-        const uint32_t i = base + lane;
-        const bool act = i < nq;
-        const uint32_t am = __ballot_sync(0xFFFFFFFFu, act);
-        if (!act) continue;
-        const QItem it = queue[i];
-        const uint32_t grp = __match_any_sync(am, it.key);
-        const int leader = __ffs(grp) - 1;
-        const uint32_t gmin = __reduce_min_sync(grp, it.rank);
-        uint32_t h = kUnset;
-        if (lane == leader) {
-            bool is_new = false;
-            h = table_insert(p, it.key + 1ull, &is_new);
-            if (h == kUnset) {
-                set_status(p.hdr, MMBEV_DEV_TABLE_FULL);
-            } else {
-                uint32_t* rk = slot_rank(p, h);
-                const uint32_t enc = 0xFFFFFFFFu - gmin;
-                if (ld_cg(rk) < enc) atomicMax(rk, enc);
-                if (is_new) {
-                    const uint32_t slot_i = atomicAdd(&s_nnew, 1u);
-                    new_slots[slot_i] = h;
-                    const uint32_t fo = (uint32_t)(it.key >> 32) - (uint32_t)f_first;
-                    if (staged && fo < (uint32_t)kFrameCnt) atomicAdd(&s_fcnt[fo], 1u);
-                    else atomicAdd(&p.frame_u[it.key >> 32], 1u);
+#pragma unroll
+        for (int k = 0; k < 2; ++k) {
+            const int j = warp * 64 + k * 32 + lane;
+            bool valid = false;
+            uint32_t lin = 0, r = 0, fr = 0;
+            float x = 0.f, y = 0.f, z = 0.f, it = 0.f, dt = 0.f;
+            if (j < n) {
+                const int64_t idx = base + j;
+                int s2 = s < 0 ? find_sweep(sm.soff, S, idx) : s;
+                while (s2 + 1 < S && sm.soff[s2 + 1] <= idx) ++s2;
+                if (s2 != s) {
+                    s = s2;
+                    if (tf_staged) {
+                        const float4* t4 = reinterpret_cast<const float4*>(sm.tf + s * 12);
+                        const float4 a = t4[0], b = t4[1], c = t4[2];
+                        T[0] = a.x; T[1] = a.y; T[2] = a.z; T[3] = a.w;
+                        T[4] = b.x; T[5] = b.y; T[6] = b.z; T[7] = b.w;
+                        T[8] = c.x; T[9] = c.y; T[10] = c.z; T[11] = c.w;
+                    } else {
+#pragma unroll
+                        for (int c = 0; c < 12; ++c) T[c] = __ldg(p.sweep_tf + (size_t)s * 16 + c);
+                    }
                 }
+                const float* q = sp + 5 * j;
+                compensate(T, q[0], q[1], q[2], x, y, z);
+                it = q[3];
+                dt = q[4];
+                const int f = sm.sfr[s];
+                const int slot = f - f_lo;
+                if (slot >= 0 && slot < n_staged) {
+                    valid = classify_point(p, sm.mask + slot * kMaskSmemWords,
+                                           sm.rois + (size_t)slot * rmax, x, y, z, lin, r);
+                } else {
+                    valid = classify_point(p, p.masks + (size_t)f * G2W, p.roi_prep + sm.sr0[s],
+                                           x, y, z, lin, r);
+                }
+                fr = (uint32_t)f;
+            }
+            // compaction in the 32-point region, input order kept
+            const uint32_t ballot = __ballot_sync(0xFFFFFFFFu, valid);
+            const uint32_t region = (uint32_t)(tile * (kTile / kRegion)) + (uint32_t)(warp * 2 + k);
+            if (valid) {
+                uint4* rec = p.records + 2 * ((size_t)region * kRegion + __popc(ballot & lt));
+                rec[0] = make_uint4(lin, fr, r, __float_as_uint(x));
+                rec[1] = make_uint4(__float_as_uint(y), __float_as_uint(z), __float_as_uint(it),
+                                    __float_as_uint(dt));
+            }
+            if (lane == 0) {
+                p.reg_cnt[region] = __popc(ballot);
+                kept_total += __popc(ballot);
             }
         }
-        h = __shfl_sync(grp, h, leader);
-        if (h != kUnset) topk_insert(slot_topk(p, h), ~it.idx, p.K);
+        // the last warp done with this buffer refills it
+        __syncwarp();
+        uint32_t last = 0;
+        if (lane == 0) {
+            // the counter only grows: round i / nstages ends at its kWarps-th arrival
+            last = atomicAdd(&sm.done[st], 1u) == (uint32_t)((i / nstages + 1) * kWarps - 1);
+        }
+        last = __shfl_sync(0xFFFFFFFFu, last, 0);
+        if (last) {
+            const int64_t next = tile + nstages;
+            if (next < t_end && next < full_tiles) issue(st, next);
+        }
     }
-    __syncthreads();
+    // one global add per block: the last warp to leave adds the block's total
+    if (lane == 0) {
+        atomicAdd(&sm.kept[0], kept_total);
+        __threadfence_block();
+        if (atomicAdd(&sm.kept[1], 1u) == (uint32_t)(kWarps - 1)) {
+            const uint32_t tot = atomicAdd(&sm.kept[0], 0u);
+            if (tot) atomicAdd(&p.hdr->num_rec, tot);
+        }
+    }
+}
 
-    // ---- E. publish new slots and per-frame counts
-    const uint32_t nnew = s_nnew;
-    if (t == 0 && nnew > 0) s_occ_base = atomicAdd(&p.hdr->num_occ, nnew);
-    if (staged && t < kFrameCnt && s_fcnt[t] > 0) atomicAdd(&p.frame_u[f_first + t], s_fcnt[t]);
-    __syncthreads();
-    const uint32_t ob = s_occ_base;
-    for (uint32_t i = t; i < nnew; i += kPtsThreads) {
-        if (ob + i < p.occ_cap) p.occ[ob + i] = new_slots[i];
-        else set_status(p.hdr, MMBEV_DEV_BOUNDS);
-    }
+// One thread per point: the per-point view of S1-S2 for testing.
+__global__ void __launch_bounds__(256) k_classify_points(Params p) {
+    pdl_wait();
+    const int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
+    if (i >= p.num_points) return;
+    const int s = find_sweep(p.sweep_off, p.num_sweeps, i);
+    float T[12];
+#pragma unroll
+    for (int c = 0; c < 12; ++c) T[c] = __ldg(p.sweep_tf + (size_t)s * 16 + c);
+    const float* q = p.points + i * 5;
+    float x, y, z;
+    compensate(T, __ldg(q), __ldg(q + 1), __ldg(q + 2), x, y, z);
+    p.cls_xyz[i * 3 + 0] = x;
+    p.cls_xyz[i * 3 + 1] = y;
+    p.cls_xyz[i * 3 + 2] = z;
+    const int f = p.sweep_frame[s];
+    uint32_t lin = 0, r = 0;
+    const bool kept = classify_point(
+        p, p.masks + (size_t)f * p.coarse * p.coarse * p.mask_words,
+        p.roi_prep + p.frame_roi_off[f], x, y, z, lin, r);
+    p.cls_lin[i] = kept ? (int64_t)lin : (int64_t)-1;
+    p.cls_rank[i] = kept ? (int32_t)r : -1;
 }
 
 }  // namespace
 
-cudaError_t launch_points(const Params& p, bool classify_only, cudaStream_t st) {
+cudaError_t launch_classify(const Params& p, int rmax, int num_sms, bool pdl, cudaStream_t st) {
     if (p.num_points <= 0) return cudaSuccess;
-    const int64_t blocks = (p.num_points + kTile - 1) / kTile;
-    if (classify_only) k_points<true><<<(unsigned)blocks, kPtsThreads, 0, st>>>(p);
-    else k_points<false><<<(unsigned)blocks, kPtsThreads, 0, st>>>(p);
-    return cudaGetLastError();
+    if (p.coarse * p.coarse * p.mask_words > kMaskSmemWords) return cudaErrorInvalidValue;
+    if (rmax < 1) rmax = 1;
+    constexpr size_t kSmemLimit = 227 * 1024;
+    int nstages = 4;
+    while (nstages > 2 && classify_smem_bytes(p.num_sweeps, rmax, nstages) > kSmemLimit) --nstages;
+    const size_t smem = classify_smem_bytes(p.num_sweeps, rmax, nstages);
+    if (smem > kSmemLimit) return cudaErrorInvalidValue;
+    static std::atomic<int> configured[64];
+    int dev = 0;
+    cudaError_t e = cudaGetDevice(&dev);
+    if (e != cudaSuccess) return e;
+    if (dev < 0 || dev >= 64 || !configured[dev].load(std::memory_order_acquire)) {
+        e = cudaFuncSetAttribute(k_classify, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                 (int)kSmemLimit);
+        if (e != cudaSuccess) return e;
+        if (dev >= 0 && dev < 64) configured[dev].store(1, std::memory_order_release);
+    }
+    const int64_t tiles = (p.num_points + kTile - 1) / kTile;
+    const int grid = (int)(tiles < num_sms ? tiles : num_sms);
+    return launch_k(k_classify, dim3(grid), dim3(kThreads), smem, st, pdl, p, rmax, nstages);
+}
+
+cudaError_t launch_classify_points(const Params& p, cudaStream_t st) {
+    if (p.num_points <= 0) return cudaSuccess;
+    const int64_t blocks = (p.num_points + 255) / 256;
+    return launch_k(k_classify_points, dim3((unsigned)blocks), dim3(256), 0, st, false, p);
 }
 
 }  // namespace mmbev

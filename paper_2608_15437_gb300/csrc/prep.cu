@@ -19,42 +19,42 @@ constexpr int kPrepThreads = 512;
 constexpr int kZeroBlocks = 64;
 
 // Inclusive cell range of one ROI's padded bounding box, or an empty range.
+// Computed in fp32: the 5 cm pad (plus a relative term) dwarfs the rounding
+// of this bound, of the exact test and of the cell index a point computes.
 struct CellRange { int16_t i0, i1, j0, j1; };
 
 __device__ CellRange roi_cells(const Params& p, const RoiPrep& r) {
     CellRange cr{1, 0, 1, 0};
-    const double c = r.c, s = r.s, hl = r.hl, hw = r.hw;
-    const double cx = r.cx, cy = r.cy;
     // NaN anywhere makes the exact test false for every point: no cells.
-    if (isnan(c) || isnan(s) || isnan(hl) || isnan(hw) || isnan(cx) || isnan(cy)) return cr;
-    const double ex = fabs(c) * hl + fabs(s) * hw;
-    const double ey = fabs(s) * hl + fabs(c) * hw;
-    const double g = p.coarse;
-    double x0 = cx - ex, x1 = cx + ex, y0 = cy - ey, y1 = cy + ey;
+    if (isnan(r.c) || isnan(r.s) || isnan(r.hl) || isnan(r.hw) || isnan(r.cx) || isnan(r.cy))
+        return cr;
+    const float ex = fabsf(r.c) * r.hl + fabsf(r.s) * r.hw;
+    const float ey = fabsf(r.s) * r.hl + fabsf(r.c) * r.hw;
+    const int G = p.coarse;
+    float x0 = r.cx - ex, x1 = r.cx + ex, y0 = r.cy - ey, y1 = r.cy + ey;
     if (!(isfinite(x0) && isfinite(x1) && isfinite(y0) && isfinite(y1))) {
-        // Infinite extents or centre: mark the whole grid (conservative).
-        cr.i0 = 0; cr.i1 = (int16_t)(p.coarse - 1); cr.j0 = 0; cr.j1 = (int16_t)(p.coarse - 1);
+        // infinite extents or centre: mark the whole grid (conservative)
+        cr.i0 = 0; cr.i1 = (int16_t)(G - 1); cr.j0 = 0; cr.j1 = (int16_t)(G - 1);
         return cr;
     }
-    // Pad well beyond the fp32 rounding of the exact test and of the cell
-    // index a point computes for itself.
-    const double span = fabs((double)p.rmin[0]) + fabs((double)p.rmax[0]) +
-                        fabs((double)p.rmin[1]) + fabs((double)p.rmax[1]);
-    const double pad = 0.05 + 1e-4 * (fabs(cx) + fabs(cy) + fabs(ex) + fabs(ey) + span);
+    const float span = fabsf(p.rmin[0]) + fabsf(p.rmax[0]) + fabsf(p.rmin[1]) + fabsf(p.rmax[1]);
+    const float pad = 0.05f + 1e-4f * (fabsf(r.cx) + fabsf(r.cy) + fabsf(ex) + fabsf(ey) + span);
     x0 -= pad; x1 += pad; y0 -= pad; y1 += pad;
-    const double gx = (p.rmax[0] - (double)p.rmin[0]) / g;
-    const double gy = (p.rmax[1] - (double)p.rmin[1]) / g;
-    double fi0 = floor((x0 - p.rmin[0]) / gx), fi1 = floor((x1 - p.rmin[0]) / gx);
-    double fj0 = floor((y0 - p.rmin[1]) / gy), fj1 = floor((y1 - p.rmin[1]) / gy);
-    if (fi1 < 0 || fj1 < 0 || fi0 > g - 1 || fj0 > g - 1 || x1 < x0 || y1 < y0) return cr;
-    cr.i0 = (int16_t)fmax(fi0, 0.0); cr.i1 = (int16_t)fmin(fi1, g - 1);
-    cr.j0 = (int16_t)fmax(fj0, 0.0); cr.j1 = (int16_t)fmin(fj1, g - 1);
+    if (x1 < x0 || y1 < y0) return cr;
+    const float fi0 = floorf((x0 - p.rmin[0]) * p.coarse_inv[0]);
+    const float fi1 = floorf((x1 - p.rmin[0]) * p.coarse_inv[0]);
+    const float fj0 = floorf((y0 - p.rmin[1]) * p.coarse_inv[1]);
+    const float fj1 = floorf((y1 - p.rmin[1]) * p.coarse_inv[1]);
+    if (fi1 < 0.f || fj1 < 0.f || fi0 > (float)(G - 1) || fj0 > (float)(G - 1)) return cr;
+    cr.i0 = (int16_t)fmaxf(fi0, 0.f); cr.i1 = (int16_t)fminf(fi1, (float)(G - 1));
+    cr.j0 = (int16_t)fmaxf(fj0, 0.f); cr.j1 = (int16_t)fminf(fj1, (float)(G - 1));
     return cr;
 }
 
 __global__ void __launch_bounds__(kPrepThreads)
 k_prep(Params p, const __grid_constant__ HostDesc d) {
     extern __shared__ uint32_t s_mask[];  // [coarse^2 * mask_words] for frame blocks
+    __shared__ CellRange s_rng[kMaxRoisPerFrame];
     const int t = threadIdx.x;
     if ((int)blockIdx.x < p.num_frames) {
         const int f = blockIdx.x;
@@ -63,11 +63,9 @@ k_prep(Params p, const __grid_constant__ HostDesc d) {
         const int g2 = p.coarse * p.coarse;
         const int W = p.mask_words;
         for (int i = t; i < g2 * W; i += blockDim.x) s_mask[i] = 0u;
-        __syncthreads();
-        // One warp per ROI: prepare it, then set its bit in every cell of its
-        // padded bounding box.
-        const int warp = t >> 5, lane = t & 31, nwarps = blockDim.x >> 5;
-        for (int r = warp; r < rn; r += nwarps) {
+        // one thread per ROI: cos/sin of the yaw in double, rounded to fp32
+        // (the definition), half-extents grown by the margin, cell range
+        for (int r = t; r < rn; r += blockDim.x) {
             const mmbev_roi_t in = p.rois[r0 + r];
             RoiPrep rp;
             rp.cx = in.cx;
@@ -78,8 +76,14 @@ k_prep(Params p, const __grid_constant__ HostDesc d) {
             rp.hw = __fadd_rn(__fmul_rn(0.5f, in.w), p.margin);
             rp.pad0 = 0.f;
             rp.pad1 = 0.f;
-            if (lane == 0) p.roi_prep[r0 + r] = rp;
-            const CellRange cr = roi_cells(p, rp);
+            p.roi_prep[r0 + r] = rp;
+            s_rng[r] = roi_cells(p, rp);
+        }
+        __syncthreads();
+        // one warp per ROI sets its bit in every cell of its range
+        const int warp = t >> 5, lane = t & 31, nwarps = blockDim.x >> 5;
+        for (int r = warp; r < rn; r += nwarps) {
+            const CellRange cr = s_rng[r];
             const int ni = cr.i1 - cr.i0 + 1, nj = cr.j1 - cr.j0 + 1;
             if (ni <= 0 || nj <= 0) continue;
             const uint32_t bit = 1u << (r & 31);
@@ -90,8 +94,9 @@ k_prep(Params p, const __grid_constant__ HostDesc d) {
             }
         }
         __syncthreads();
-        uint32_t* gm = p.masks + (size_t)f * g2 * W;
-        for (int i = t; i < g2 * W; i += blockDim.x) gm[i] = s_mask[i];
+        uint4* gm = reinterpret_cast<uint4*>(p.masks + (size_t)f * g2 * W);
+        const uint4* sm4 = reinterpret_cast<const uint4*>(s_mask);
+        for (int i = t; i < g2 * W / 4; i += blockDim.x) gm[i] = sm4[i];
         return;
     }
     // Housekeeping blocks: grid-stride over the zero/copy work.
@@ -118,10 +123,16 @@ k_prep(Params p, const __grid_constant__ HostDesc d) {
         for (size_t i = gt; i < (size_t)p.num_rois; i += gs) p.hist[i] = 0u;
     if (p.frame_u)
         for (size_t i = gt; i < (size_t)p.num_frames; i += gs) p.frame_u[i] = 0u;
-    if (p.bcnt)
-        for (size_t i = gt; i <= (size_t)p.num_buckets; i += gs) p.bcnt[i] = 0ull;
-    if (p.scan_flag)
-        for (size_t i = gt; i < (size_t)p.scan_tiles; i += gs) p.scan_flag[i] = 0u;
+    if (p.reg_cnt) {
+        // a classify pass that gives up leaves the regions it did not reach empty
+        uint4* r4 = reinterpret_cast<uint4*>(p.reg_cnt);  // a multiple of 64 counters
+        for (size_t i = gt; i < (size_t)p.num_regions / 4; i += gs) r4[i] = make_uint4(0u, 0u, 0u, 0u);
+    }
+    if (p.bcnt) {
+        uint4* b4 = reinterpret_cast<uint4*>(p.bcnt);  // B u64 counters, B even or padded
+        const size_t n4 = ((size_t)p.num_buckets + 1) / 2;
+        for (size_t i = gt; i < n4; i += gs) b4[i] = make_uint4(0u, 0u, 0u, 0u);
+    }
 }
 
 __global__ void k_zero(uint4* ptr, size_t n16, uint8_t* tail, size_t ntail) {
@@ -134,9 +145,9 @@ __global__ void k_zero(uint4* ptr, size_t n16, uint8_t* tail, size_t ntail) {
 
 }  // namespace
 
-// Largest coarse mask a frame block holds in shared memory: 64 x 64 cells x
-// 13 words (the coarse grid shrinks as the ROI count grows).
-constexpr int kPrepSmemMax = 64 * 64 * 13 * 4;
+// Largest coarse mask a frame block holds in shared memory: 4,096 words (the
+// coarse grid shrinks as the ROI count grows).
+constexpr int kPrepSmemMax = 4096 * 4;
 
 cudaError_t launch_prep(const Params& p, const HostDesc& d, cudaStream_t st) {
     // Raise the dynamic shared memory limit once per device (outside any

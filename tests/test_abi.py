@@ -35,10 +35,10 @@ def test_library_exports_every_declared_symbol(mmbev_lib):
 
 
 def test_sizes_are_host_only(mmbev_lib):
-    # capacity: next power of two >= 2N slots of 16 + 4*round4(K) bytes
-    assert mmbev_lib.table_size(20000, 10) == 65536 * 64
-    assert mmbev_lib.table_size(100, 1) == 1024 * 32
-    assert mmbev_lib.table_size(11110400, 10) == (1 << 25) * 64
+    # capacity: next power of two >= 2N (at least 1024) slots of 16 bytes
+    assert mmbev_lib.table_size(20000, 10) == 65536 * 16
+    assert mmbev_lib.table_size(100, 1) == 1024 * 16
+    assert mmbev_lib.table_size(11110400, 64) == (1 << 25) * 16
     with pytest.raises(ValueError):
         mmbev_lib.table_size(100, 0)
     with pytest.raises(ValueError):
@@ -83,4 +83,4 @@ def test_invalid_arguments_are_rejected_before_launch(mmbev_lib, kw):
 def test_small_buffers_are_rejected_before_launch(mmbev_lib):
     lib = mmbev_lib.load()
     assert _call(lib, ws_bytes=1024) == -3
-    assert _call(lib, table_bytes=64 * 100) == -3   # fewer than 2N slots
+    assert _call(lib, table_bytes=16 * 100) == -3   # fewer than 2N slots

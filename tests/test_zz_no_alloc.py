@@ -55,7 +55,11 @@ def test_no_alloc_matches_workspace_entry_on_two_calls(mmbev_lib, cuda_dev):
 
 
 def test_no_alloc_rejects_calls_beyond_its_array(mmbev_lib, cuda_dev):
-    w = synth.streaming_batch(2)         # 694,400 points: more than the array holds
+    w = synth.concat_frames([synth.nuscenes_frame(s) for s in range(1, 6)], "five")
+    need = (mmbev_lib.table_size(w.num_points, 10) +
+            mmbev_lib.workspace_size(w.num_points, w.rois.shape[0], 1000, 1, w.voxel_size,
+                                     w.pc_range))
+    assert need > 96 * 2**20           # more than the array holds
     pts, tf, rois = to_dev(w, cuda_dev)
     out = mmbev_lib.Outputs.empty(1, 1000, cuda_dev)
     with pytest.raises(mmbev_lib.MMBEVError, match="EWORKSPACE"):
