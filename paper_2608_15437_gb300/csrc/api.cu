@@ -56,8 +56,6 @@ int coarse_for(int mask_words) {
     return 8;
 }
 
-constexpr uint32_t kMaxInsertBlocks = 4096;
-
 constexpr uint32_t kSlotStride = 16;
 
 // Byte offsets of every workspace array for one call shape.
@@ -100,7 +98,7 @@ Layout make_layout(int64_t max_points, int64_t rois_total, int32_t max_rois_fram
     L.rec_slot = take(sizeof(uint2) * TS);
     L.seg = take(sizeof(uint32_t) * U);
     L.newlist = take(16 * TS);
-    L.blockcount = take(sizeof(uint32_t) * kMaxInsertBlocks);
+    L.blockcount = take(sizeof(uint32_t) * L.num_tiles);
     L.bcnt = take(sizeof(unsigned long long) * B2);
     L.bcnt2 = take(sizeof(unsigned long long) * B2);
     L.boff = take(sizeof(unsigned long long) * B2);
@@ -323,8 +321,6 @@ int mmbev_voxelize_roi_batched_ex(const float* points, const int64_t* sweep_offs
 
     const int sms = num_sms();
     if (sms <= 0) return MMBEV_ECUDA;
-    p.ins_blocks = insert_blocks(sms);
-    if (p.ins_blocks > kMaxInsertBlocks) p.ins_blocks = kMaxInsertBlocks;
     cudaEvent_t* ev = opts ? opts->stage_events : nullptr;
     int stage = 0;
     auto mark = [&]() -> cudaError_t {

@@ -1,30 +1,28 @@
 // Stage 2: voxel hash insert and dedup (S3 of the path; Alg. 1 "Voxelize"),
 // stage 3: the occupied-voxel list, stage 4: per-voxel point lists.
 //
-// Insert. Every block owns a contiguous range of 32-point regions; each warp
-// takes one region's kept-point records (at most 32) at a time, with no block
-// barrier in the loop:
+// Insert. One block per 2048-point tile; its warps take the tile's kept-point
+// records in batches of 32 (the next batch's records load while the current
+// batch is inserted), with no block barrier in the loop:
 //   1. lanes holding the same voxel key are grouped with __match_any_sync
 //      (all later warp collectives run on the full warp);
-//   2. the group leader reads the key's home slot (key, minimum rank) in one
-//      round trip; a matching key means found, an empty slot is claimed with
-//      atomicCAS, another key moves on to the next slot (linear probing, at
-//      most H probes). It lowers the slot's minimum ROI rank (stored as
-//      0xFFFFFFFF - rank, so an all-zero slot is empty) with a
-//      fire-and-forget atomicMax only when the group improves it, and adds
-//      the group's size to the slot's point count with one atomicAdd whose
-//      old value numbers the group's points;
+//   2. the group leader claims or finds the key's slot with atomicCAS from
+//      its home slot (linear probing, at most H probes), lowers the slot's
+//      minimum ROI rank (stored as 0xFFFFFFFF - rank, so an all-zero slot is
+//      empty) with a fire-and-forget atomicMax, and adds the group's size to
+//      the slot's point count with one atomicAdd whose old value numbers the
+//      group's points;
 //   3. each lane stores {slot, arrival number} at its record position.
-//   A leader that created the slot appends {slot, lin, frame} to its block's
-//   own sub-list (one shared-memory atomic per warp), so no global counter
-//   is touched. No point ever waits on another point's insertion: the
-//   voxel's first K points are chosen later, from the complete list.
-// Compact. One block per insert block copies that block's sub-list into the
-// dense occupied-voxel list at the sum of the earlier blocks' counts, counts
-// every new voxel into its frame and into its ordering bucket (warp-
-// aggregated, recording its position in the bucket), and reserves the
-// voxel's segment of `seg` (one atomicAdd per block chunk), written into the
-// slot.
+//   A leader that created the slot appends {slot, lin, frame} to its tile's
+//   sub-list (one shared-memory atomic per warp). No point ever waits on
+//   another point's insertion: the voxel's first K points are chosen later,
+//   from the complete list.
+// Compact. One block per tile copies the tile's sub-list into the dense
+// occupied-voxel list at a place taken with one atomicAdd (the list's order
+// is immaterial), counts every new voxel into its frame and into its
+// ordering bucket (warp-aggregated, recording its position in the bucket),
+// and reserves the voxel's segment of `seg` (one atomicAdd per block chunk),
+// written into the slot.
 // Scatter points. Every record's position goes to seg[slot segment +
 // arrival number], so each voxel's points end up contiguous.
 #include "mmbev_internal.cuh"
@@ -33,19 +31,64 @@ namespace mmbev {
 namespace {
 
 constexpr int kThreads = 256;
-constexpr int kBlocksPerSm = 6;
+constexpr int kBlocksPerSm = 8;
 constexpr int kFrameWin = 64;
+constexpr uint32_t kFull = 0xFFFFFFFFu;
+
+// One block per 2048-point tile. The tile's 64 region counts are scanned in
+// shared memory; the tile's kept records are then taken in batches of 32 by
+// the block's warps in turn (record j of the tile lies in the region whose
+// range [excl, incl) holds j, found by a six-step binary search).
+struct TileScan {
+    uint32_t incl[kTile / kRegion];
+    uint32_t excl[kTile / kRegion];
+};
+
+// Threads 0..63 read the counts; every thread must call it (one barrier).
+// Returns the tile's kept records.
+__device__ __forceinline__ uint32_t tile_scan(const Params& p, uint32_t tile, TileScan& ts,
+                                              uint32_t* s_part) {
+    const int t = threadIdx.x, lane = t & 31;
+    uint32_t n = 0, v = 0;
+    if (t < kTile / kRegion) {
+        n = min(ld_cg(&p.reg_cnt[tile * (kTile / kRegion) + t]), (uint32_t)kRegion);
+        v = n;
+#pragma unroll
+        for (int o = 1; o < 32; o <<= 1) {
+            const uint32_t x = __shfl_up_sync(kFull, v, o);
+            if (lane >= o) v += x;
+        }
+        if (lane == 31) s_part[t >> 5] = v;
+    }
+    __syncthreads();
+    if (t < kTile / kRegion) {
+        if (t >= 32) v += s_part[0];
+        ts.incl[t] = v;
+        ts.excl[t] = v - n;
+    }
+    __syncthreads();
+    return ts.incl[kTile / kRegion - 1];
+}
+
+__device__ __forceinline__ uint32_t tile_item_pos(const TileScan& ts, uint32_t tile, uint32_t j) {
+    int l = 0;  // regions whose range ends at or before j
+#pragma unroll
+    for (int step = 32; step >= 1; step >>= 1)
+        if (l + step <= kTile / kRegion && ts.incl[l + step - 1] <= j) l += step;
+    if (l > kTile / kRegion - 1) l = kTile / kRegion - 1;
+    return (tile * (kTile / kRegion) + (uint32_t)l) * kRegion + (j - ts.excl[l]);
+}
 
 __global__ void __launch_bounds__(kThreads, kBlocksPerSm) k_insert(Params p) {
+    __shared__ TileScan ts;
+    __shared__ uint32_t s_part[2];
     __shared__ uint32_t s_nnew;
     pdl_wait();
     pdl_trigger();
     const int t = threadIdx.x, lane = t & 31, warp = t >> 5;
+    const uint32_t tile = blockIdx.x;
     if (t == 0) s_nnew = 0;
-    __syncthreads();
-    const uint32_t RG = p.num_regions;
-    const uint32_t rb = (uint32_t)((uint64_t)blockIdx.x * RG / gridDim.x);
-    const uint32_t re = (uint32_t)((uint64_t)(blockIdx.x + 1) * RG / gridDim.x);
+    const uint32_t total = tile_scan(p, tile, ts, s_part);
     // slots in use: a power of two >= 1.25 x the call's kept points
     uint32_t lg = 10;
     if (p.table_log2_fixed > 0) {
@@ -56,29 +99,30 @@ __global__ void __launch_bounds__(kThreads, kBlocksPerSm) k_insert(Params p) {
     }
     const uint32_t mask = (uint32_t)((1ull << lg) - 1ull);
     const int nwarps = kThreads / 32;
-    uint4* sub = p.newlist + (size_t)rb * kRegion;
-    for (uint32_t g = rb + (uint32_t)warp; g < re; g += (uint32_t)nwarps) {
-        const uint32_t n = min(ld_cg(&p.reg_cnt[g]), (uint32_t)kRegion);
-        if (n == 0) continue;
-        const uint32_t r = g * (uint32_t)kRegion + lane;
-        const uint4* rec = p.records;
-        uint2* rs = p.rec_slot;
-        const bool act = (uint32_t)lane < n;
-        const uint32_t am = __ballot_sync(0xFFFFFFFFu, act);
-        uint4 a = make_uint4(0u, 0u, 0u, 0u);
-        unsigned long long key = ~0ull;
+    const uint32_t lt = (1u << lane) - 1u;
+    // the tile's sub-list of created voxels: room for every record of the tile
+    uint4* sub = p.newlist + (size_t)tile * kTile;
+    // batch j0 is processed while the warp's next batch's records load
+    uint32_t j = (uint32_t)warp * 32u + lane;
+    bool act = j < total;
+    uint32_t pos = act ? tile_item_pos(ts, tile, j) : 0u;
+    uint4 a = act ? __ldcs(p.records + 2 * (size_t)pos) : make_uint4(0u, 0u, 0u, 0u);
+    for (uint32_t j0 = (uint32_t)warp * 32u; j0 < total; j0 += nwarps * 32u) {
+        const uint32_t jn = j0 + nwarps * 32u + lane;
+        const bool actn = jn < total;
+        const uint32_t posn = actn ? tile_item_pos(ts, tile, jn) : 0u;
+        const uint4 an = actn ? __ldcs(p.records + 2 * (size_t)posn) : make_uint4(0u, 0u, 0u, 0u);
+
+        const uint32_t am = __ballot_sync(kFull, act);
+        const unsigned long long key = ((unsigned long long)a.y << 32) | a.x;
         uint32_t grp = 1u << lane;
-        if (act) {
-            a = __ldcs(rec + 2 * r);   // lin, frame, rank, x'
-            key = ((unsigned long long)a.y << 32) | a.x;
-            grp = __match_any_sync(am, key);
-        }
+        if (act) grp = __match_any_sync(am, key);
         const int leader = __ffs(grp) - 1;
         uint32_t gmin_rank = a.z;
-        if (__any_sync(0xFFFFFFFFu, grp != (1u << lane))) {
-            // some voxel appears more than once in this warp
+        if (__any_sync(kFull, grp != (1u << lane))) {
+            // some voxel appears more than once in this batch
             for (int l = 0; l < 32; ++l) {
-                const uint32_t rl = __shfl_sync(0xFFFFFFFFu, a.z, l);
+                const uint32_t rl = __shfl_sync(kFull, a.z, l);
                 if ((grp >> l) & 1u) gmin_rank = rl < gmin_rank ? rl : gmin_rank;
             }
         }
@@ -87,46 +131,41 @@ __global__ void __launch_bounds__(kThreads, kBlocksPerSm) k_insert(Params p) {
         if (act && lane == leader) {
             const unsigned long long key1 = key + 1ull;
             h = slot_home(mask, key1);
-            uint4 s0 = make_uint4(0u, 0u, 0u, 0u);
             bool done = false;
             for (uint32_t probe = 0; probe <= mask; ++probe) {
-                s0 = __ldcg(reinterpret_cast<const uint4*>(slot_key(p, h)));  // key, rank, cnt
-                const unsigned long long cur = ((unsigned long long)s0.y << 32) | s0.x;
-                if (cur == key1) { done = true; break; }
-                if (cur == 0ull) {
-                    const unsigned long long old = atomicCAS(slot_key(p, h), 0ull, key1);
-                    if (old == 0ull) { created = true; done = true; s0.z = 0u; break; }
-                    if (old == key1) { done = true; s0.z = 0u; break; }
-                }
+                const unsigned long long old = atomicCAS(slot_key(p, h), 0ull, key1);
+                if (old == 0ull) { created = true; done = true; break; }
+                if (old == key1) { done = true; break; }
                 h = (h + 1u) & mask;
             }
             if (!done) {
                 set_status(p.hdr, MMBEV_DEV_TABLE_FULL);
                 h = kUnset;
             } else {
-                const uint32_t enc = 0xFFFFFFFFu - gmin_rank;
-                if (enc > s0.z) atomicMax(slot_rank(p, h), enc);
+                atomicMax(slot_rank(p, h), 0xFFFFFFFFu - gmin_rank);
                 base = atomicAdd(slot_cnt(p, h), (uint32_t)__popc(grp));
             }
         }
-        h = __shfl_sync(0xFFFFFFFFu, h, leader);
-        base = __shfl_sync(0xFFFFFFFFu, base, leader);
-        if (act) rs[r] = make_uint2(h, base + __popc(grp & ((1u << lane) - 1u)));
-        // leaders of new slots append to this block's sub-list
-        const uint32_t cm = __ballot_sync(0xFFFFFFFFu, created);
+        h = __shfl_sync(kFull, h, leader);
+        base = __shfl_sync(kFull, base, leader);
+        if (act) p.rec_slot[pos] = make_uint2(h, base + __popc(grp & lt));
+        // leaders of new slots append to the tile's sub-list
+        const uint32_t cm = __ballot_sync(kFull, created);
         if (cm) {
             uint32_t wbase = 0;
             if (lane == __ffs(cm) - 1) wbase = atomicAdd(&s_nnew, (uint32_t)__popc(cm));
-            wbase = __shfl_sync(0xFFFFFFFFu, wbase, __ffs(cm) - 1);
-            if (created) sub[wbase + __popc(cm & ((1u << lane) - 1u))] = make_uint4(h, a.x, a.y, 0u);
+            wbase = __shfl_sync(kFull, wbase, __ffs(cm) - 1);
+            if (created) sub[wbase + __popc(cm & lt)] = make_uint4(h, a.x, a.y, 0u);
         }
+        a = an;
+        pos = posn;
+        act = actn;
     }
     __syncthreads();
-    if (t == 0) p.blockcount[blockIdx.x] = s_nnew;
+    if (t == 0) p.blockcount[tile] = s_nnew;
 }
 
 __global__ void __launch_bounds__(kThreads) k_compact(Params p) {
-    __shared__ uint32_t s_red[kThreads / 32];
     __shared__ uint32_t s_seg[kThreads / 32];
     __shared__ uint32_t s_base, s_segbase;
     __shared__ uint32_t s_fcnt[kFrameWin];
@@ -135,23 +174,14 @@ __global__ void __launch_bounds__(kThreads) k_compact(Params p) {
     pdl_trigger();
     const int t = threadIdx.x, lane = t & 31, warp = t >> 5;
     const uint32_t b = blockIdx.x;
-    // this block's place: the sum of the earlier blocks' counts
-    uint32_t part = 0;
-    for (uint32_t i = t; i < b; i += kThreads) part += p.blockcount[i];
-#pragma unroll
-    for (int o = 16; o > 0; o >>= 1) part += __shfl_xor_sync(0xFFFFFFFFu, part, o);
-    if (lane == 0) s_red[warp] = part;
-    if (t < kFrameWin) s_fcnt[t] = 0;
-    const uint32_t rb = (uint32_t)((uint64_t)b * p.num_regions / p.ins_blocks);
-    const uint4* sub = p.newlist + (size_t)rb * kRegion;
+    const uint4* sub = p.newlist + (size_t)b * kTile;
     const uint32_t n = p.blockcount[b];
-    if (t == 0) s_fmin = n ? sub[0].z : 0u;
-    __syncthreads();
+    if (n == 0) return;
+    if (t < kFrameWin) s_fcnt[t] = 0;
+    // this tile's place in the occupied-voxel list (order is immaterial)
     if (t == 0) {
-        uint32_t s = 0;
-        for (int w = 0; w < kThreads / 32; ++w) s += s_red[w];
-        s_base = s;
-        if (b == p.ins_blocks - 1) p.hdr->num_occ = s + n;
+        s_fmin = sub[0].z;
+        s_base = atomicAdd(&p.hdr->num_occ, n);
     }
     __syncthreads();
     const uint32_t base = s_base;
@@ -214,37 +244,42 @@ __global__ void __launch_bounds__(kThreads) k_compact(Params p) {
     if (t < kFrameWin && s_fcnt[t]) atomicAdd(&p.frame_u[s_fmin + t], s_fcnt[t]);
 }
 
-__global__ void __launch_bounds__(kThreads) k_scatter_points(Params p) {
+__global__ void __launch_bounds__(kThreads, kBlocksPerSm) k_scatter_points(Params p) {
+    __shared__ TileScan ts;
+    __shared__ uint32_t s_part[2];
     pdl_wait();
     pdl_trigger();
+    const uint32_t tile = blockIdx.x;
+    const uint32_t total = tile_scan(p, tile, ts, s_part);
     const uint32_t cap = ld_cg(&p.hdr->seg_total);
-    const size_t npos = (size_t)p.num_regions * kRegion;
-    const size_t gs = (size_t)gridDim.x * blockDim.x;
-    for (size_t r = (size_t)blockIdx.x * blockDim.x + threadIdx.x; r < npos; r += gs) {
-        const uint32_t n = ld_cg(&p.reg_cnt[r / kRegion]);
-        if ((uint32_t)(r % kRegion) >= n) continue;
-        const uint2 hs = p.rec_slot[r];
+    for (uint32_t j = threadIdx.x; j < total; j += blockDim.x) {
+        const uint32_t pos = tile_item_pos(ts, tile, j);
+        const uint2 hs = p.rec_slot[pos];
         if (hs.x == kUnset) continue;
         const uint32_t at = ld_cg(slot_seg(p, hs.x)) + hs.y;
-        if (at < cap) p.seg[at] = (uint32_t)r;
+        if (at < cap) p.seg[at] = pos;
         else set_status(p.hdr, MMBEV_DEV_BOUNDS);
     }
 }
 
 }  // namespace
 
-uint32_t insert_blocks(int num_sms) { return (uint32_t)num_sms * kBlocksPerSm; }
-
 cudaError_t launch_insert(const Params& p, bool pdl, cudaStream_t st) {
-    return launch_k(k_insert, dim3(p.ins_blocks), dim3(kThreads), 0, st, pdl, p);
+    const uint32_t tiles = p.num_regions / (kTile / kRegion);
+    if (tiles == 0) return cudaSuccess;
+    return launch_k(k_insert, dim3(tiles), dim3(kThreads), 0, st, pdl, p);
 }
 
 cudaError_t launch_compact(const Params& p, bool pdl, cudaStream_t st) {
-    return launch_k(k_compact, dim3(p.ins_blocks), dim3(kThreads), 0, st, pdl, p);
+    const uint32_t tiles = p.num_regions / (kTile / kRegion);
+    if (tiles == 0) return cudaSuccess;
+    return launch_k(k_compact, dim3(tiles), dim3(kThreads), 0, st, pdl, p);
 }
 
 cudaError_t launch_scatter_points(const Params& p, bool pdl, cudaStream_t st) {
-    return launch_k(k_scatter_points, dim3(p.ins_blocks), dim3(kThreads), 0, st, pdl, p);
+    const uint32_t tiles = p.num_regions / (kTile / kRegion);
+    if (tiles == 0) return cudaSuccess;
+    return launch_k(k_scatter_points, dim3(tiles), dim3(kThreads), 0, st, pdl, p);
 }
 
 }  // namespace mmbev

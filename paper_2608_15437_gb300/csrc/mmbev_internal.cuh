@@ -10,8 +10,8 @@
 //               points 32g .. 32g+31, so positions increase with the point
 //               index and "first K by position" is "first K by index".
 //   reg_cnt     workspace, kept points per region.
-//   newlist     workspace, per insert block a sub-list of the voxels that
-//               block created {slot, lin, frame}; the compact kernel
+//   newlist     workspace, per tile a sub-list of the voxels that tile's
+//               insert block created {slot, lin, frame}; the compact kernel
 //               concatenates the sub-lists into the occupied-voxel list.
 //   table       caller's hash table of 16-byte slots: { u64 key+1 (0 =
 //               empty), u32 0xFFFFFFFF-minrank (0 = none), u32 count (points
@@ -130,8 +130,7 @@ struct Params {
     uint32_t* seg;          // [N] record positions, voxel by voxel
     uint32_t num_regions;
     uint4* newlist;         // [regions*32] voxels created, per insert block: slot, lin, frame
-    uint32_t* blockcount;   // [ins_blocks] voxels each insert block created
-    uint32_t ins_blocks;    // grid of the insert kernel
+    uint32_t* blockcount;   // [tiles] voxels created by each tile's insert block
     unsigned long long* bcnt;   // [B] voxels per bucket (every frame, no classes)
     unsigned long long* bcnt2;  // [B] capped frames: lo = rank-below, hi = rank-tie
     unsigned long long* boff;   // [B] exclusive offsets within the frame (lo, hi)
@@ -300,7 +299,6 @@ cudaError_t launch_classify_points(const Params& p, cudaStream_t st);
 cudaError_t launch_insert(const Params& p, bool pdl, cudaStream_t st);
 cudaError_t launch_compact(const Params& p, bool pdl, cudaStream_t st);
 cudaError_t launch_scatter_points(const Params& p, bool pdl, cudaStream_t st);
-uint32_t insert_blocks(int num_sms);
 cudaError_t launch_capped_hist(const Params& p, int num_sms, bool pdl, cudaStream_t st);
 cudaError_t launch_frames(const Params& p, bool pdl, cudaStream_t st);
 cudaError_t launch_capped_census(const Params& p, int num_sms, bool pdl, cudaStream_t st);
