@@ -215,7 +215,7 @@ void bind_layout(Params* p, const Layout& L, uint8_t* ws) {
     p->vid_slot = reinterpret_cast<uint32_t*>(ws + L.vid_slot);
     p->heavy = reinterpret_cast<uint32_t*>(ws + L.heavy);
     p->occ_cap = (uint32_t)(p->num_points > 0 ? p->num_points : 1);
-    p->rec_cap = p->occ_cap;
+    p->rec_cap = p->num_regions * (uint32_t)kRegion;
     p->mask_words = L.mask_words;
     p->coarse = L.coarse;
     p->coarse_inv[0] = (float)((double)L.coarse / ((double)p->rmax[0] - (double)p->rmin[0]));

@@ -73,6 +73,7 @@ __global__ void __launch_bounds__(kThreads) k_finalize(Params p) {
     const int F = p.num_frames;
     for (int i = threadIdx.x; i < F; i += blockDim.x) s_vbase[i] = p.finfo[i].vbase;
     const uint32_t total = ld_cg(&p.hdr->total_kept);
+    const uint32_t seg_cap = min(ld_cg(&p.hdr->seg_total), p.occ_cap);  // seg holds N entries
     if (threadIdx.x == 0) s_vbase[F] = total;
     __syncthreads();
     const int lane = threadIdx.x & 31;
@@ -87,6 +88,10 @@ __global__ void __launch_bounds__(kThreads) k_finalize(Params p) {
             const uint2 s = __ldcg(reinterpret_cast<const uint2*>(slot_key(p, h)));  // seg, -
             off = s.x;
             n = ld_cg(slot_cnt(p, h));
+            if (off > seg_cap || n > seg_cap - off) {   // inconsistent lists: report, read nothing
+                set_status(p.hdr, MMBEV_DEV_BOUNDS);
+                n = 0;
+            }
         }
         const bool heavy = act && n > kLightMax;
         const uint32_t hm = __ballot_sync(0xFFFFFFFFu, heavy);
@@ -108,6 +113,7 @@ __global__ void __launch_bounds__(kThreads) k_finalize(Params p) {
             for (int c = 0; c < 4; ++c) sorted_insert<B>(best, v[c]);
         }
         const int cnt = (int)(n < (uint32_t)K ? n : (uint32_t)K);
+        if (cnt > 0 && best[cnt - 1] >= p.rec_cap) set_status(p.hdr, MMBEV_DEV_BOUNDS);
         float acc[5] = {0.f, 0.f, 0.f, 0.f, 0.f};
 #pragma unroll
         for (int j0 = 0; j0 < B; j0 += 4) {
@@ -116,7 +122,7 @@ __global__ void __launch_bounds__(kThreads) k_finalize(Params p) {
 #pragma unroll
             for (int c = 0; c < 4; ++c) {
                 if (j0 + c < cnt) {
-                    const uint4* rec = p.records + 2 * (size_t)best[j0 + c];
+                    const uint4* rec = p.records + 2 * (size_t)min(best[j0 + c], p.rec_cap - 1u);
                     ra[c] = __ldg(rec);
                     rb[c] = __ldg(rec + 1);
                 }
@@ -141,6 +147,7 @@ __global__ void __launch_bounds__(kThreads) k_finalize_heavy(Params p) {
     if (threadIdx.x == 0) s_vbase[F] = total;
     __syncthreads();
     const int lane = threadIdx.x & 31;
+    const uint32_t seg_cap = min(ld_cg(&p.hdr->seg_total), p.occ_cap);  // seg holds N entries
     const uint32_t nh = ld_cg(&p.hdr->num_heavy);
     const uint32_t gw = (blockIdx.x * blockDim.x + threadIdx.x) >> 5;
     const uint32_t nw = (gridDim.x * blockDim.x) >> 5;
@@ -149,7 +156,11 @@ __global__ void __launch_bounds__(kThreads) k_finalize_heavy(Params p) {
         const uint32_t g = p.heavy[e];
         const uint32_t h = p.vid_slot[g];
         const uint32_t off = ld_cg(slot_seg(p, h));
-        const uint32_t n = ld_cg(slot_cnt(p, h));
+        uint32_t n = ld_cg(slot_cnt(p, h));
+        if (off > seg_cap || n > seg_cap - off) {   // inconsistent lists: report, read nothing
+            if (lane == 0) set_status(p.hdr, MMBEV_DEV_BOUNDS);
+            n = 0;
+        }
         uint32_t best[B];
 #pragma unroll
         for (int j = 0; j < B; ++j) best[j] = 0xFFFFFFFFu;
@@ -171,7 +182,8 @@ __global__ void __launch_bounds__(kThreads) k_finalize_heavy(Params p) {
         for (int half = 0; half * 32 < cnt; ++half) {
             uint4 ra = make_uint4(0u, 0u, 0u, 0u), rb = ra;
             if (half * 32 + lane < cnt) {
-                const uint4* rec = p.records + 2 * (size_t)mine[half];
+                if (mine[half] >= p.rec_cap) set_status(p.hdr, MMBEV_DEV_BOUNDS);
+                const uint4* rec = p.records + 2 * (size_t)min(mine[half], p.rec_cap - 1u);
                 ra = __ldg(rec);
                 rb = __ldg(rec + 1);
             }

@@ -251,7 +251,7 @@ __global__ void __launch_bounds__(kThreads, kBlocksPerSm) k_scatter_points(Param
     pdl_trigger();
     const uint32_t tile = blockIdx.x;
     const uint32_t total = tile_scan(p, tile, ts, s_part);
-    const uint32_t cap = ld_cg(&p.hdr->seg_total);
+    const uint32_t cap = min(ld_cg(&p.hdr->seg_total), p.occ_cap);  // seg holds N entries
     for (uint32_t j = threadIdx.x; j < total; j += blockDim.x) {
         const uint32_t pos = tile_item_pos(ts, tile, j);
         const uint2 hs = p.rec_slot[pos];

@@ -143,7 +143,7 @@ struct Params {
     uint32_t* vid_slot;     // [F*max_voxels] slot of each kept voxel, output order
     uint32_t* heavy;        // [F*max_voxels] kept voxels with more than 32 points
     uint32_t occ_cap;
-    uint32_t rec_cap;
+    uint32_t rec_cap;       // record positions of the call (regions * 32)
     // outputs
     float* out_feats;
     int32_t* out_coords;
@@ -195,45 +195,65 @@ __device__ __forceinline__ bool roi_contains(const RoiPrep& r, float x, float y)
     return fabsf(u) <= r.hl && fabsf(v) <= r.hw;
 }
 
-// S2 for one compensated point: range crop, coarse-mask candidates, exact
-// ROI test in rank order, voxel index. `fmask` is the point's frame's coarse
-// mask (coarse^2 cells x mask_words) and `frois` its prepared ROIs, either
-// in shared memory (staged) or in global memory. Returns true and sets lin,
-// rank when the point is kept.
-__device__ __forceinline__ bool classify_point(const Params& p, const uint32_t* fmask,
-                                               const RoiPrep* frois, float x, float y, float z,
-                                               uint32_t& lin, uint32_t& rank) {
+// S2, first part: range crop (half-open box) and the point's coarse BEV cell.
+// Returns false when the point is out of range; `cell` indexes the frame's
+// coarse mask (cells x mask_words words).
+__device__ __forceinline__ bool point_cell(const Params& p, float x, float y, float z,
+                                           int& cell) {
     if (!((p.rmin[0] <= x) && (x < p.rmax[0]) && (p.rmin[1] <= y) && (y < p.rmax[1]) &&
           (p.rmin[2] <= z) && (z < p.rmax[2])))
         return false;
     const int G = p.coarse;
-    const float dx0 = __fsub_rn(x, p.rmin[0]);
-    const float dy0 = __fsub_rn(y, p.rmin[1]);
-    int gx = (int)__fmul_rn(dx0, p.coarse_inv[0]);
-    int gy = (int)__fmul_rn(dy0, p.coarse_inv[1]);
+    int gx = (int)__fmul_rn(__fsub_rn(x, p.rmin[0]), p.coarse_inv[0]);
+    int gy = (int)__fmul_rn(__fsub_rn(y, p.rmin[1]), p.coarse_inv[1]);
     gx = min(max(gx, 0), G - 1);
     gy = min(max(gy, 0), G - 1);
-    const uint32_t* mw = fmask + (gy * G + gx) * p.mask_words;
+    cell = gy * G + gx;
+    return true;
+}
+
+// Exact ROI test of candidate r (prepared ROIs of the point's frame).
+__device__ __forceinline__ bool roi_hit(const RoiPrep* frois, int r, float x, float y) {
+    const float4* rp4 = reinterpret_cast<const float4*>(frois + r);
+    const float4 a = rp4[0], c = rp4[1];
+    RoiPrep rp;
+    rp.cx = a.x; rp.cy = a.y; rp.c = a.z; rp.s = a.w; rp.hl = c.x; rp.hw = c.y;
+    return roi_contains(rp, x, y);
+}
+
+// S2, last part: Eq. 1 voxel index of an in-range point; false when the
+// floor lands on or beyond the grid's far face.
+__device__ __forceinline__ bool voxel_lin(const Params& p, float x, float y, float z,
+                                          uint32_t& lin) {
+    const uint32_t cx = __float2uint_rz(__fdiv_rn(__fsub_rn(x, p.rmin[0]), p.vs[0]));
+    const uint32_t cy = __float2uint_rz(__fdiv_rn(__fsub_rn(y, p.rmin[1]), p.vs[1]));
+    const uint32_t cz = __float2uint_rz(__fdiv_rn(__fsub_rn(z, p.rmin[2]), p.vs[2]));
+    if (cx >= p.dims[0] || cy >= p.dims[1] || cz >= p.dims[2]) return false;
+    lin = (cz * p.dims[1] + cy) * p.dims[0] + cx;
+    return true;
+}
+
+// S2 for one compensated point: range crop, coarse-mask candidates, exact
+// ROI test in rank order, voxel index. `fmask` is the point's frame's coarse
+// mask (coarse^2 cells x mask_words) and `frois` its prepared ROIs. Returns
+// true and sets lin, rank when the point is kept.
+__device__ __forceinline__ bool classify_point(const Params& p, const uint32_t* fmask,
+                                               const RoiPrep* frois, float x, float y, float z,
+                                               uint32_t& lin, uint32_t& rank) {
+    int cell;
+    if (!point_cell(p, x, y, z, cell)) return false;
+    const uint32_t* mw = fmask + cell * p.mask_words;
     int hit = -1;
     for (int w = 0; w < p.mask_words && hit < 0; ++w) {
         uint32_t bits = mw[w];
         while (bits) {
             const int b = __ffs(bits) - 1;
             bits &= bits - 1u;
-            const int r = w * 32 + b;
-            const float4* rp4 = reinterpret_cast<const float4*>(frois + r);
-            const float4 a = rp4[0], c = rp4[1];
-            RoiPrep rp;
-            rp.cx = a.x; rp.cy = a.y; rp.c = a.z; rp.s = a.w; rp.hl = c.x; rp.hw = c.y;
-            if (roi_contains(rp, x, y)) { hit = r; break; }
+            if (roi_hit(frois, w * 32 + b, x, y)) { hit = w * 32 + b; break; }
         }
     }
     if (hit < 0) return false;
-    const uint32_t cx = __float2uint_rz(__fdiv_rn(dx0, p.vs[0]));
-    const uint32_t cy = __float2uint_rz(__fdiv_rn(dy0, p.vs[1]));
-    const uint32_t cz = __float2uint_rz(__fdiv_rn(__fsub_rn(z, p.rmin[2]), p.vs[2]));
-    if (cx >= p.dims[0] || cy >= p.dims[1] || cz >= p.dims[2]) return false;
-    lin = (cz * p.dims[1] + cy) * p.dims[0] + cx;
+    if (!voxel_lin(p, x, y, z, lin)) return false;
     rank = (uint32_t)hit;
     return true;
 }

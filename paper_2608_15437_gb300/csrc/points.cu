@@ -13,7 +13,7 @@
 // the first hit is the point's rank) and the voxel index. The masks and
 // prepared ROIs of the (one or two) frames a block's tile range starts with
 // sit in shared memory. Kept points are compacted per 32-point region with
-// a warp ballot, in input order, and written as 32-byte records at
+// warp ballots, in input order, and written as 32-byte records at
 // position (region)*32 + (rank among the region's kept points), with the
 // compensated features, so later stages never touch the raw points again.
 //
@@ -198,14 +198,46 @@ __global__ void __launch_bounds__(kThreads, 1) k_classify(Params p, int rmax, in
             if (tile < t_end && tile < full_tiles) issue(s, tile);
         }
 
+    // Lane l takes points 2l and 2l+1 of the warp's 64: their ten floats are
+    // five 8-byte shared loads, conflict-free (lane stride 40 bytes). Lanes
+    // 0-15 cover region 2*warp, lanes 16-31 region 2*warp+1.
     const uint32_t lt = (1u << lane) - 1u;
+    const uint32_t half_mask = lane < 16 ? 0x0000FFFFu : 0xFFFF0000u;
     uint32_t kept_total = 0;   // this warp's kept points (lane 0)
-    int s = -1;                // sweep of this thread's latest point
-    float T[12];               // that sweep's transform
-    for (int64_t i = 0; t_begin + i < t_end; ++i) {
-        const int64_t tile = t_begin + i;
-        const int st = (int)(i % nstages);
-        const uint32_t parity = (uint32_t)((i / nstages) & 1);
+    // the sweep of this lane's current point and what depends on it
+    int s = find_sweep(sm.soff, S, t_begin * kTile + warp * 64 + 2 * lane);
+    int64_t next_off = 0;      // first index of the next sweep
+    float T[12];
+    uint32_t fr = 0;
+    const uint32_t* fmask = nullptr;
+    const RoiPrep* frois = nullptr;
+    auto load_sweep = [&]() {
+        next_off = sm.soff[s + 1];
+        if (tf_staged) {
+            const float4* t4 = reinterpret_cast<const float4*>(sm.tf + s * 12);
+            const float4 a = t4[0], b = t4[1], c = t4[2];
+            T[0] = a.x; T[1] = a.y; T[2] = a.z; T[3] = a.w;
+            T[4] = b.x; T[5] = b.y; T[6] = b.z; T[7] = b.w;
+            T[8] = c.x; T[9] = c.y; T[10] = c.z; T[11] = c.w;
+        } else {
+#pragma unroll
+            for (int c = 0; c < 12; ++c) T[c] = __ldg(p.sweep_tf + (size_t)s * 16 + c);
+        }
+        const int f = sm.sfr[s];
+        fr = (uint32_t)f;
+        const int slot = f - f_lo;
+        if (slot >= 0 && slot < n_staged) {
+            fmask = sm.mask + slot * kMaskSmemWords;
+            frois = sm.rois + (size_t)slot * rmax;
+        } else {
+            fmask = p.masks + (size_t)f * G2W;
+            frois = p.roi_prep + sm.sr0[s];
+        }
+    };
+    load_sweep();
+    int st = 0;
+    uint32_t parity = 0, round = 0;
+    for (int64_t tile = t_begin; tile < t_end; ++tile) {
         float* sp = sm.stages + (size_t)st * kTile * 5;
         const int64_t base = tile * kTile;
         const int n = (int)((N - base) < kTile ? (N - base) : kTile);
@@ -221,71 +253,96 @@ __global__ void __launch_bounds__(kThreads, 1) k_classify(Params p, int rmax, in
                 sp[k] = __ldcs(src + k);
             __syncwarp();
         }
+        const int j0 = warp * 64 + 2 * lane;
+        const float2* q2 = reinterpret_cast<const float2*>(sp + 5 * j0);
+        const float2 v0 = q2[0], v1 = q2[1], v2 = q2[2], v3 = q2[3], v4 = q2[4];
+        // the warp is done with the buffer once its reads are complete; the
+        // last warp of the round refills it
+        __threadfence_block();
+        __syncwarp();
+        {
+            uint32_t last = 0;
+            if (lane == 0)  // the counter only grows: a round ends at its kWarps-th arrival
+                last = atomicAdd(&sm.done[st], 1u) == (round + 1u) * kWarps - 1u;
+            last = __shfl_sync(0xFFFFFFFFu, last, 0);
+            if (last) {
+                const int64_t next = tile + nstages;
+                if (next < t_end && next < full_tiles) issue(st, next);
+            }
+        }
+        const float px[2] = {v0.x, v2.y}, py[2] = {v0.y, v3.x}, pz[2] = {v1.x, v3.y};
+        const float pi[2] = {v1.y, v4.x}, pd[2] = {v2.x, v4.y};
+        bool valid[2] = {false, false};
+        uint32_t lin[2] = {0u, 0u}, frk[2] = {0u, 0u};
+        int hit[2] = {-1, -1};
+        float x[2], y[2], z[2];
+        const uint32_t* cm[2] = {nullptr, nullptr};   // the point's coarse-cell mask words
+        const RoiPrep* cr[2] = {frois, frois};         // its frame's ROIs
 #pragma unroll
         for (int k = 0; k < 2; ++k) {
-            const int j = warp * 64 + k * 32 + lane;
-            bool valid = false;
-            uint32_t lin = 0, r = 0, fr = 0;
-            float x = 0.f, y = 0.f, z = 0.f, it = 0.f, dt = 0.f;
-            if (j < n) {
-                const int64_t idx = base + j;
-                int s2 = s < 0 ? find_sweep(sm.soff, S, idx) : s;
-                while (s2 + 1 < S && sm.soff[s2 + 1] <= idx) ++s2;
-                if (s2 != s) {
-                    s = s2;
-                    if (tf_staged) {
-                        const float4* t4 = reinterpret_cast<const float4*>(sm.tf + s * 12);
-                        const float4 a = t4[0], b = t4[1], c = t4[2];
-                        T[0] = a.x; T[1] = a.y; T[2] = a.z; T[3] = a.w;
-                        T[4] = b.x; T[5] = b.y; T[6] = b.z; T[7] = b.w;
-                        T[8] = c.x; T[9] = c.y; T[10] = c.z; T[11] = c.w;
-                    } else {
+            x[k] = y[k] = z[k] = 0.f;
+            if (j0 + k < n) {
+                const int64_t idx = base + j0 + k;
+                if (idx >= next_off) {
+                    while (s + 1 < S && sm.soff[s + 1] <= idx) ++s;
+                    load_sweep();
+                }
+                compensate(T, px[k], py[k], pz[k], x[k], y[k], z[k]);
+                int cell;
+                if (point_cell(p, x[k], y[k], z[k], cell)) cm[k] = fmask + cell * p.mask_words;
+                cr[k] = frois;
+                frk[k] = fr;
+            }
+        }
+        // Alg. 1 ROI test in rank order over the union of the warp's
+        // candidates: each step tests one ROI index for all 64 points (a
+        // broadcast read when the warp's points share a frame); a point keeps
+        // its first hit.
+        for (int w = 0; w < p.mask_words; ++w) {
+            uint32_t m[2];
 #pragma unroll
-                        for (int c = 0; c < 12; ++c) T[c] = __ldg(p.sweep_tf + (size_t)s * 16 + c);
-                    }
-                }
-                const float* q = sp + 5 * j;
-                compensate(T, q[0], q[1], q[2], x, y, z);
-                it = q[3];
-                dt = q[4];
-                const int f = sm.sfr[s];
-                const int slot = f - f_lo;
-                if (slot >= 0 && slot < n_staged) {
-                    valid = classify_point(p, sm.mask + slot * kMaskSmemWords,
-                                           sm.rois + (size_t)slot * rmax, x, y, z, lin, r);
-                } else {
-                    valid = classify_point(p, p.masks + (size_t)f * G2W, p.roi_prep + sm.sr0[s],
-                                           x, y, z, lin, r);
-                }
-                fr = (uint32_t)f;
-            }
-            // compaction in the 32-point region, input order kept
-            const uint32_t ballot = __ballot_sync(0xFFFFFFFFu, valid);
-            const uint32_t region = (uint32_t)(tile * (kTile / kRegion)) + (uint32_t)(warp * 2 + k);
-            if (valid) {
-                uint4* rec = p.records + 2 * ((size_t)region * kRegion + __popc(ballot & lt));
-                rec[0] = make_uint4(lin, fr, r, __float_as_uint(x));
-                rec[1] = make_uint4(__float_as_uint(y), __float_as_uint(z), __float_as_uint(it),
-                                    __float_as_uint(dt));
-            }
-            if (lane == 0) {
-                p.reg_cnt[region] = __popc(ballot);
-                kept_total += __popc(ballot);
+            for (int k = 0; k < 2; ++k) m[k] = (cm[k] && hit[k] < 0) ? cm[k][w] : 0u;
+            uint32_t u = __reduce_or_sync(0xFFFFFFFFu, m[0] | m[1]);
+            while (u) {
+                const int b = __ffs(u) - 1;
+                u &= u - 1u;
+#pragma unroll
+                for (int k = 0; k < 2; ++k)
+                    if (((m[k] >> b) & 1u) && hit[k] < 0 && roi_hit(cr[k], w * 32 + b, x[k], y[k]))
+                        hit[k] = w * 32 + b;
             }
         }
-        // the last warp done with this buffer refills it
-        __syncwarp();
-        uint32_t last = 0;
-        if (lane == 0) {
-            // the counter only grows: round i / nstages ends at its kWarps-th arrival
-            last = atomicAdd(&sm.done[st], 1u) == (uint32_t)((i / nstages + 1) * kWarps - 1);
+#pragma unroll
+        for (int k = 0; k < 2; ++k) valid[k] = hit[k] >= 0 && voxel_lin(p, x[k], y[k], z[k], lin[k]);
+        // compaction in the 32-point regions, input order kept
+        const uint32_t b0 = __ballot_sync(0xFFFFFFFFu, valid[0]);
+        const uint32_t b1 = __ballot_sync(0xFFFFFFFFu, valid[1]);
+        const uint32_t below = lt & half_mask;
+        const uint32_t rank0 = __popc(b0 & below) + __popc(b1 & below);
+        const uint32_t region =
+            (uint32_t)(tile * (kTile / kRegion)) + (uint32_t)(warp * 2) + (lane >> 4);
+#pragma unroll
+        for (int k = 0; k < 2; ++k) {
+            if (valid[k]) {
+                const uint32_t rk = rank0 + (k ? (uint32_t)valid[0] : 0u);
+                uint4* rec = p.records + 2 * ((size_t)region * kRegion + rk);
+                rec[0] = make_uint4(lin[k], frk[k], (uint32_t)hit[k], __float_as_uint(x[k]));
+                rec[1] = make_uint4(__float_as_uint(y[k]), __float_as_uint(z[k]),
+                                    __float_as_uint(pi[k]), __float_as_uint(pd[k]));
+            }
         }
-        last = __shfl_sync(0xFFFFFFFFu, last, 0);
-        if (last) {
-            const int64_t next = tile + nstages;
-            if (next < t_end && next < full_tiles) issue(st, next);
+        if ((lane & 15) == 0) {
+            const uint32_t c = __popc(b0 & half_mask) + __popc(b1 & half_mask);
+            p.reg_cnt[region] = c;
+            kept_total += c;
+        }
+        if (++st == nstages) {
+            st = 0;
+            parity ^= 1u;
+            ++round;
         }
     }
+    kept_total += __shfl_down_sync(0xFFFFFFFFu, kept_total, 16);
     // one global add per block: the last warp to leave adds the block's total
     if (lane == 0) {
         atomicAdd(&sm.kept[0], kept_total);
