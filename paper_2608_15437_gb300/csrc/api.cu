@@ -61,7 +61,7 @@ constexpr uint32_t kSlotStride = 16;
 // Byte offsets of every workspace array for one call shape.
 struct Layout {
     size_t hdr, sweep_off, sweep_frame, fso, fro, roi_prep, masks, hist, frame_u, finfo;
-    size_t records, reg_cnt, rec_slot, seg, newlist, blockcount, bcnt, bcnt2, boff, nonempty, occ, d_bucket,
+    size_t keys, records, reg_cnt, rec_slot, seg, newlist, blockcount, bcnt, bcnt2, boff, nonempty, occ, d_bucket,
         d_pos, d_lin, items, vid_slot, heavy;
     size_t total;
     uint32_t num_buckets, buckets_per_frame, num_tiles;
@@ -93,6 +93,7 @@ Layout make_layout(int64_t max_points, int64_t rois_total, int32_t max_rois_fram
     L.hist = take(sizeof(uint32_t) * R);
     L.frame_u = take(sizeof(uint32_t) * F);
     L.finfo = take(sizeof(FrameInfo) * F);
+    L.keys = take(8 * TS);
     L.records = take(32 * TS);
     L.reg_cnt = take(sizeof(uint32_t) * L.num_tiles * (kTile / kRegion));
     L.rec_slot = take(sizeof(uint2) * TS);
@@ -196,6 +197,7 @@ void bind_layout(Params* p, const Layout& L, uint8_t* ws) {
     p->hist = reinterpret_cast<uint32_t*>(ws + L.hist);
     p->frame_u = reinterpret_cast<uint32_t*>(ws + L.frame_u);
     p->finfo = reinterpret_cast<FrameInfo*>(ws + L.finfo);
+    p->keys = reinterpret_cast<uint2*>(ws + L.keys);
     p->records = reinterpret_cast<uint4*>(ws + L.records);
     p->reg_cnt = reinterpret_cast<uint32_t*>(ws + L.reg_cnt);
     p->rec_slot = reinterpret_cast<uint2*>(ws + L.rec_slot);

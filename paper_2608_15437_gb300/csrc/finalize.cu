@@ -38,12 +38,13 @@ __device__ __forceinline__ void sorted_insert(uint32_t (&b)[B], uint32_t v) {
     }
 }
 
+// record: {x', y', z', intensity} {dt, rank, -, -}
 __device__ __forceinline__ void add_record(float (&acc)[5], const uint4& a, const uint4& b) {
-    acc[0] = __fadd_rn(acc[0], __uint_as_float(a.w));
-    acc[1] = __fadd_rn(acc[1], __uint_as_float(b.x));
-    acc[2] = __fadd_rn(acc[2], __uint_as_float(b.y));
-    acc[3] = __fadd_rn(acc[3], __uint_as_float(b.z));
-    acc[4] = __fadd_rn(acc[4], __uint_as_float(b.w));
+    acc[0] = __fadd_rn(acc[0], __uint_as_float(a.x));
+    acc[1] = __fadd_rn(acc[1], __uint_as_float(a.y));
+    acc[2] = __fadd_rn(acc[2], __uint_as_float(a.z));
+    acc[3] = __fadd_rn(acc[3], __uint_as_float(a.w));
+    acc[4] = __fadd_rn(acc[4], __uint_as_float(b.x));
 }
 
 __device__ __forceinline__ void write_voxel(const Params& p, size_t row, const float (&acc)[5],
@@ -190,11 +191,11 @@ __global__ void __launch_bounds__(kThreads) k_finalize_heavy(Params p) {
             const int m = cnt - half * 32 < 32 ? cnt - half * 32 : 32;
             for (int j = 0; j < m; ++j) {
                 uint4 a, b;
+                a.x = __shfl_sync(0xFFFFFFFFu, ra.x, j);
+                a.y = __shfl_sync(0xFFFFFFFFu, ra.y, j);
+                a.z = __shfl_sync(0xFFFFFFFFu, ra.z, j);
                 a.w = __shfl_sync(0xFFFFFFFFu, ra.w, j);
                 b.x = __shfl_sync(0xFFFFFFFFu, rb.x, j);
-                b.y = __shfl_sync(0xFFFFFFFFu, rb.y, j);
-                b.z = __shfl_sync(0xFFFFFFFFu, rb.z, j);
-                b.w = __shfl_sync(0xFFFFFFFFu, rb.w, j);
                 add_record(acc, a, b);
             }
         }

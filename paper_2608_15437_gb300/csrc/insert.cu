@@ -6,12 +6,11 @@
 // batch is inserted), with no block barrier in the loop:
 //   1. lanes holding the same voxel key are grouped with __match_any_sync
 //      (all later warp collectives run on the full warp);
-//   2. the group leader claims or finds the key's slot with atomicCAS from
-//      its home slot (linear probing, at most H probes), lowers the slot's
-//      minimum ROI rank (stored as 0xFFFFFFFF - rank, so an all-zero slot is
-//      empty) with a fire-and-forget atomicMax, and adds the group's size to
-//      the slot's point count with one atomicAdd whose old value numbers the
-//      group's points;
+//   2. the group leader finds the key's slot from its home slot (linear
+//      probing, at most H probes): a matching key means found, an empty slot
+//      is claimed with atomicCAS; it adds the group's size to the slot's
+//      point count with one atomicAdd whose old value numbers the group's
+//      points (an all-zero slot is empty);
 //   3. each lane stores {slot, arrival number} at its record position.
 //   A leader that created the slot appends {slot, lin, frame} to its tile's
 //   sub-list (one shared-memory atomic per warp). No point ever waits on
@@ -106,26 +105,18 @@ __global__ void __launch_bounds__(kThreads, kBlocksPerSm) k_insert(Params p) {
     uint32_t j = (uint32_t)warp * 32u + lane;
     bool act = j < total;
     uint32_t pos = act ? tile_item_pos(ts, tile, j) : 0u;
-    uint4 a = act ? __ldcs(p.records + 2 * (size_t)pos) : make_uint4(0u, 0u, 0u, 0u);
+    uint2 a = act ? __ldcs(p.keys + pos) : make_uint2(0u, 0u);   // lin, frame
     for (uint32_t j0 = (uint32_t)warp * 32u; j0 < total; j0 += nwarps * 32u) {
         const uint32_t jn = j0 + nwarps * 32u + lane;
         const bool actn = jn < total;
         const uint32_t posn = actn ? tile_item_pos(ts, tile, jn) : 0u;
-        const uint4 an = actn ? __ldcs(p.records + 2 * (size_t)posn) : make_uint4(0u, 0u, 0u, 0u);
+        const uint2 an = actn ? __ldcs(p.keys + posn) : make_uint2(0u, 0u);
 
         const uint32_t am = __ballot_sync(kFull, act);
         const unsigned long long key = ((unsigned long long)a.y << 32) | a.x;
         uint32_t grp = 1u << lane;
         if (act) grp = __match_any_sync(am, key);
         const int leader = __ffs(grp) - 1;
-        uint32_t gmin_rank = a.z;
-        if (__any_sync(kFull, grp != (1u << lane))) {
-            // some voxel appears more than once in this batch
-            for (int l = 0; l < 32; ++l) {
-                const uint32_t rl = __shfl_sync(kFull, a.z, l);
-                if ((grp >> l) & 1u) gmin_rank = rl < gmin_rank ? rl : gmin_rank;
-            }
-        }
         bool created = false;
         uint32_t h = kUnset, base = 0;
         if (act && lane == leader) {
@@ -133,16 +124,19 @@ __global__ void __launch_bounds__(kThreads, kBlocksPerSm) k_insert(Params p) {
             h = slot_home(mask, key1);
             bool done = false;
             for (uint32_t probe = 0; probe <= mask; ++probe) {
-                const unsigned long long old = atomicCAS(slot_key(p, h), 0ull, key1);
-                if (old == 0ull) { created = true; done = true; break; }
-                if (old == key1) { done = true; break; }
+                const unsigned long long cur = __ldcg(slot_key(p, h));
+                if (cur == key1) { done = true; break; }
+                if (cur == 0ull) {
+                    const unsigned long long old = atomicCAS(slot_key(p, h), 0ull, key1);
+                    if (old == 0ull) { created = true; done = true; break; }
+                    if (old == key1) { done = true; break; }
+                }
                 h = (h + 1u) & mask;
             }
             if (!done) {
                 set_status(p.hdr, MMBEV_DEV_TABLE_FULL);
                 h = kUnset;
             } else {
-                atomicMax(slot_rank(p, h), 0xFFFFFFFFu - gmin_rank);
                 base = atomicAdd(slot_cnt(p, h), (uint32_t)__popc(grp));
             }
         }
@@ -250,6 +244,12 @@ __global__ void __launch_bounds__(kThreads, kBlocksPerSm) k_scatter_points(Param
     pdl_wait();
     pdl_trigger();
     const uint32_t tile = blockIdx.x;
+    // frames with more voxels than max_voxels need each voxel's minimum ROI
+    // rank (the cap keeps the smallest (rank, lin)); others never read it
+    int capped = 0;
+    for (int f = threadIdx.x; f < p.num_frames; f += blockDim.x)
+        capped |= ld_cg(&p.frame_u[f]) > (uint32_t)p.max_voxels;
+    capped = __syncthreads_or(capped);
     const uint32_t total = tile_scan(p, tile, ts, s_part);
     const uint32_t cap = min(ld_cg(&p.hdr->seg_total), p.occ_cap);  // seg holds N entries
     for (uint32_t j = threadIdx.x; j < total; j += blockDim.x) {
@@ -259,6 +259,11 @@ __global__ void __launch_bounds__(kThreads, kBlocksPerSm) k_scatter_points(Param
         const uint32_t at = ld_cg(slot_seg(p, hs.x)) + hs.y;
         if (at < cap) p.seg[at] = pos;
         else set_status(p.hdr, MMBEV_DEV_BOUNDS);
+        if (capped) {
+            const uint32_t f = p.keys[pos].y;
+            if (ld_cg(&p.frame_u[f]) > (uint32_t)p.max_voxels)
+                atomicMax(slot_rank(p, hs.x), 0xFFFFFFFFu - p.records[2 * (size_t)pos + 1].y);
+        }
     }
 }
 

@@ -4,11 +4,13 @@
 //   points      caller's float32 [N][5] AoS, streamed once by the classify
 //               kernel through a 3-stage ring of 40 KB shared-memory tiles,
 //               each tile moved by eight 5 KB cp.async.bulk (TMA) copies.
-//   records     workspace, 32 B per kept point, at position region*32 + (its
-//               rank among the kept points of its 32-point region): {lin,
-//               frame, ROI rank, x', y', z', intensity, dt}. Region g holds
-//               points 32g .. 32g+31, so positions increase with the point
-//               index and "first K by position" is "first K by index".
+//   keys        workspace, 8 B per kept point {lin, frame}, at position
+//               region*32 + (its rank among the kept points of its 32-point
+//               region). Region g holds points 32g .. 32g+31, so positions
+//               increase with the point index and "first K by position" is
+//               "first K by index".
+//   records     workspace, 32 B per kept point at the same position:
+//               {x', y', z', intensity} {dt, ROI rank, -, -}.
 //   reg_cnt     workspace, kept points per region.
 //   newlist     workspace, per tile a sub-list of the voxels that tile's
 //               insert block created {slot, lin, frame}; the compact kernel
@@ -124,7 +126,8 @@ struct Params {
     uint32_t* hist;         // [R] voxels per minimum rank (capped frames)
     uint32_t* frame_u;      // [F] unique voxels per frame
     FrameInfo* finfo;       // [F]
-    uint4* records;         // [tiles*2048][2] kept points (see above)
+    uint2* keys;            // [regions*32] voxel key {lin, frame} of each kept point
+    uint4* records;         // [regions*32][2] kept points' features and rank
     uint32_t* reg_cnt;      // [regions] kept points per 32-point region
     uint2* rec_slot;        // [regions*32] slot and arrival index of each record
     uint32_t* seg;          // [N] record positions, voxel by voxel

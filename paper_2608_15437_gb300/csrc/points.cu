@@ -13,9 +13,10 @@
 // the first hit is the point's rank) and the voxel index. The masks and
 // prepared ROIs of the (one or two) frames a block's tile range starts with
 // sit in shared memory. Kept points are compacted per 32-point region with
-// warp ballots, in input order, and written as 32-byte records at
-// position (region)*32 + (rank among the region's kept points), with the
-// compensated features, so later stages never touch the raw points again.
+// warp ballots, in input order: position (region)*32 + (rank among the
+// region's kept points) gets the point's voxel key (8 bytes) and a 32-byte
+// record with the compensated features and the ROI rank, so later stages
+// never touch the raw points again.
 //
 // The classify-only entry point (per-point outputs for testing S1-S2) uses a
 // plain one-thread-per-point kernel built from the same device functions.
@@ -325,10 +326,12 @@ __global__ void __launch_bounds__(kThreads, 1) k_classify(Params p, int rmax, in
         for (int k = 0; k < 2; ++k) {
             if (valid[k]) {
                 const uint32_t rk = rank0 + (k ? (uint32_t)valid[0] : 0u);
-                uint4* rec = p.records + 2 * ((size_t)region * kRegion + rk);
-                rec[0] = make_uint4(lin[k], frk[k], (uint32_t)hit[k], __float_as_uint(x[k]));
-                rec[1] = make_uint4(__float_as_uint(y[k]), __float_as_uint(z[k]),
-                                    __float_as_uint(pi[k]), __float_as_uint(pd[k]));
+                const size_t at = (size_t)region * kRegion + rk;
+                p.keys[at] = make_uint2(lin[k], frk[k]);
+                uint4* rec = p.records + 2 * at;
+                rec[0] = make_uint4(__float_as_uint(x[k]), __float_as_uint(y[k]),
+                                    __float_as_uint(z[k]), __float_as_uint(pi[k]));
+                rec[1] = make_uint4(__float_as_uint(pd[k]), (uint32_t)hit[k], 0u, 0u);
             }
         }
         if ((lane & 15) == 0) {
