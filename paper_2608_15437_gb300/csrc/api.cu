@@ -58,10 +58,12 @@ int coarse_for(int mask_words) {
 
 constexpr uint32_t kSlotStride = 16;
 
+constexpr uint32_t kMaxInsertBlocks = 2048;
+
 // Byte offsets of every workspace array for one call shape.
 struct Layout {
     size_t hdr, sweep_off, sweep_frame, fso, fro, roi_prep, masks, hist, frame_u, finfo;
-    size_t keys, records, reg_cnt, rec_slot, seg, newlist, blockcount, bcnt, bcnt2, boff, nonempty, occ, d_bucket,
+    size_t records, plist, rs, cls_cnt, seg, newlist, blockcount, bcnt, bcnt2, boff, nonempty, occ, d_bucket,
         d_pos, d_lin, items, vid_slot, heavy;
     size_t total;
     uint32_t num_buckets, buckets_per_frame, num_tiles;
@@ -93,13 +95,13 @@ Layout make_layout(int64_t max_points, int64_t rois_total, int32_t max_rois_fram
     L.hist = take(sizeof(uint32_t) * R);
     L.frame_u = take(sizeof(uint32_t) * F);
     L.finfo = take(sizeof(FrameInfo) * F);
-    L.keys = take(8 * TS);
     L.records = take(32 * TS);
-    L.reg_cnt = take(sizeof(uint32_t) * L.num_tiles * (kTile / kRegion));
-    L.rec_slot = take(sizeof(uint2) * TS);
+    L.plist = take(16 * TS);
+    L.rs = take(8 * TS);
+    L.cls_cnt = take(sizeof(uint32_t) * kMaxClsGrid);
     L.seg = take(sizeof(uint32_t) * U);
-    L.newlist = take(16 * TS);
-    L.blockcount = take(sizeof(uint32_t) * L.num_tiles);
+    L.newlist = take(16 * (U + 32 + (size_t)kMaxInsertBlocks * 256));
+    L.blockcount = take(sizeof(uint32_t) * kMaxInsertBlocks);
     L.bcnt = take(sizeof(unsigned long long) * B2);
     L.bcnt2 = take(sizeof(unsigned long long) * B2);
     L.boff = take(sizeof(unsigned long long) * B2);
@@ -197,10 +199,10 @@ void bind_layout(Params* p, const Layout& L, uint8_t* ws) {
     p->hist = reinterpret_cast<uint32_t*>(ws + L.hist);
     p->frame_u = reinterpret_cast<uint32_t*>(ws + L.frame_u);
     p->finfo = reinterpret_cast<FrameInfo*>(ws + L.finfo);
-    p->keys = reinterpret_cast<uint2*>(ws + L.keys);
     p->records = reinterpret_cast<uint4*>(ws + L.records);
-    p->reg_cnt = reinterpret_cast<uint32_t*>(ws + L.reg_cnt);
-    p->rec_slot = reinterpret_cast<uint2*>(ws + L.rec_slot);
+    p->plist = reinterpret_cast<uint4*>(ws + L.plist);
+    p->rs = reinterpret_cast<uint2*>(ws + L.rs);
+    p->cls_cnt = reinterpret_cast<uint32_t*>(ws + L.cls_cnt);
     p->seg = reinterpret_cast<uint32_t*>(ws + L.seg);
     p->num_regions = (uint32_t)((p->num_points + kTile - 1) / kTile) * (kTile / kRegion);
     p->newlist = reinterpret_cast<uint4*>(ws + L.newlist);
@@ -323,6 +325,20 @@ int mmbev_voxelize_roi_batched_ex(const float* points, const int64_t* sweep_offs
 
     const int sms = num_sms();
     if (sms <= 0) return MMBEV_ECUDA;
+    {
+        // classify: one block per SM (at most one per tile); insert: a
+        // persistent grid whose blocks each own a sub-list with room for
+        // every entry their warps can take
+        const uint64_t tiles = ((uint64_t)p.num_points + kTile - 1) / kTile;
+        uint64_t g = tiles < (uint64_t)sms ? tiles : (uint64_t)sms;
+        if (g > (uint64_t)kMaxClsGrid) g = kMaxClsGrid;
+        p.cls_grid = (uint32_t)g;
+        p.ins_blocks = insert_blocks(sms);
+        if (p.ins_blocks > kMaxInsertBlocks) p.ins_blocks = kMaxInsertBlocks;
+        const uint64_t warps = (uint64_t)p.ins_blocks * 8;
+        const uint64_t batches = ((uint64_t)p.num_points + 31) / 32;
+        p.ins_cap = (uint32_t)(256 * ((batches + warps - 1) / warps));
+    }
     cudaEvent_t* ev = opts ? opts->stage_events : nullptr;
     int stage = 0;
     auto mark = [&]() -> cudaError_t {

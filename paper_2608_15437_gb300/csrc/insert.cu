@@ -1,9 +1,14 @@
 // Stage 2: voxel hash insert and dedup (S3 of the path; Alg. 1 "Voxelize"),
 // stage 3: the occupied-voxel list, stage 4: per-voxel point lists.
 //
-// Insert. One block per 2048-point tile; its warps take the tile's kept-point
-// records in batches of 32 (the next batch's records load while the current
-// batch is inserted), with no block barrier in the loop:
+// The classify pass leaves, per classify block, a dense list of its kept
+// points {lin, frame, record position} (in any order). All three kernels
+// here walk the concatenation of those lists; a block finds the list of an
+// entry by binary search over the lists' prefix sums in shared memory.
+//
+// Insert. Persistent blocks; each warp takes 32 consecutive entries at a
+// time (the next 32 load while the current ones are inserted), with no
+// block barrier in the loop:
 //   1. lanes holding the same voxel key are grouped with __match_any_sync
 //      (all later warp collectives run on the full warp);
 //   2. the group leader finds the key's slot from its home slot (linear
@@ -11,19 +16,21 @@
 //      is claimed with atomicCAS; it adds the group's size to the slot's
 //      point count with one atomicAdd whose old value numbers the group's
 //      points (an all-zero slot is empty);
-//   3. each lane stores {slot, arrival number} at its record position.
-//   A leader that created the slot appends {slot, lin, frame} to its tile's
+//   3. each lane stores {slot, arrival number} at its entry.
+//   A leader that created the slot appends {slot, lin, frame} to its block's
 //   sub-list (one shared-memory atomic per warp). No point ever waits on
 //   another point's insertion: the voxel's first K points are chosen later,
 //   from the complete list.
-// Compact. One block per tile copies the tile's sub-list into the dense
-// occupied-voxel list at a place taken with one atomicAdd (the list's order
-// is immaterial), counts every new voxel into its frame and into its
+// Compact. One block per insert block copies that block's sub-list into the
+// dense occupied-voxel list at a place taken with one atomicAdd (the list's
+// order is immaterial), counts every new voxel into its frame and into its
 // ordering bucket (warp-aggregated, recording its position in the bucket),
 // and reserves the voxel's segment of `seg` (one atomicAdd per block chunk),
 // written into the slot.
-// Scatter points. Every record's position goes to seg[slot segment +
-// arrival number], so each voxel's points end up contiguous.
+// Scatter points. Every entry's record position goes to seg[slot segment +
+// arrival number], so each voxel's points end up contiguous. In frames over
+// the voxel cap it also lowers the voxel's minimum ROI rank (stored as
+// 0xFFFFFFFF - rank) with atomicMax.
 #include "mmbev_internal.cuh"
 
 namespace mmbev {
@@ -34,83 +41,95 @@ constexpr int kBlocksPerSm = 8;
 constexpr int kFrameWin = 64;
 constexpr uint32_t kFull = 0xFFFFFFFFu;
 
-// One block per 2048-point tile. The tile's 64 region counts are scanned in
-// shared memory; the tile's kept records are then taken in batches of 32 by
-// the block's warps in turn (record j of the tile lies in the region whose
-// range [excl, incl) holds j, found by a six-step binary search).
-struct TileScan {
-    uint32_t incl[kTile / kRegion];
-    uint32_t excl[kTile / kRegion];
+// Prefix sums of the classify blocks' list lengths (s_off[0..G]) and the
+// first entry of each list (list l starts at tile t_begin(l) * 2048).
+struct Lists {
+    uint32_t off[kMaxClsGrid + 1];
 };
 
-// Threads 0..63 read the counts; every thread must call it (one barrier).
-// Returns the tile's kept records.
-__device__ __forceinline__ uint32_t tile_scan(const Params& p, uint32_t tile, TileScan& ts,
-                                              uint32_t* s_part) {
-    const int t = threadIdx.x, lane = t & 31;
-    uint32_t n = 0, v = 0;
-    if (t < kTile / kRegion) {
-        n = min(ld_cg(&p.reg_cnt[tile * (kTile / kRegion) + t]), (uint32_t)kRegion);
-        v = n;
+// Every thread must call it (one barrier). Returns the entry count.
+__device__ __forceinline__ uint32_t lists_scan(const Params& p, Lists& L, uint32_t* s_part) {
+    const int t = threadIdx.x, lane = t & 31, warp = t >> 5;
+    const uint32_t G = p.cls_grid;
+    const uint64_t T = (uint64_t)p.num_regions / (kTile / kRegion);
+    // kMaxClsGrid <= kThreads * 4: each thread scans up to 4 consecutive lists
+    uint32_t c[4], sum = 0;
 #pragma unroll
-        for (int o = 1; o < 32; o <<= 1) {
-            const uint32_t x = __shfl_up_sync(kFull, v, o);
-            if (lane >= o) v += x;
+    for (int k = 0; k < 4; ++k) {
+        const uint32_t l = (uint32_t)t * 4 + k;
+        c[k] = 0;
+        if (l < G) {
+            const uint64_t room = ((uint64_t)(l + 1) * T / G - (uint64_t)l * T / G) * kTile;
+            c[k] = (uint32_t)min((uint64_t)ld_cg(&p.cls_cnt[l]), room);
         }
-        if (lane == 31) s_part[t >> 5] = v;
+        sum += c[k];
+    }
+    uint32_t v = sum;
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) {
+        const uint32_t x = __shfl_up_sync(kFull, v, o);
+        if (lane >= o) v += x;
+    }
+    if (lane == 31) s_part[warp] = v;
+    __syncthreads();
+    uint32_t wbase = 0;
+    for (int w = 0; w < warp; ++w) wbase += s_part[w];
+    uint32_t run = wbase + v - sum;
+#pragma unroll
+    for (int k = 0; k < 4; ++k) {
+        const uint32_t l = (uint32_t)t * 4 + k;
+        if (l <= G) L.off[l] = run;
+        run += c[k];
     }
     __syncthreads();
-    if (t < kTile / kRegion) {
-        if (t >= 32) v += s_part[0];
-        ts.incl[t] = v;
-        ts.excl[t] = v - n;
-    }
-    __syncthreads();
-    return ts.incl[kTile / kRegion - 1];
+    return L.off[G];
 }
 
-__device__ __forceinline__ uint32_t tile_item_pos(const TileScan& ts, uint32_t tile, uint32_t j) {
-    int l = 0;  // regions whose range ends at or before j
-#pragma unroll
-    for (int step = 32; step >= 1; step >>= 1)
-        if (l + step <= kTile / kRegion && ts.incl[l + step - 1] <= j) l += step;
-    if (l > kTile / kRegion - 1) l = kTile / kRegion - 1;
-    return (tile * (kTile / kRegion) + (uint32_t)l) * kRegion + (j - ts.excl[l]);
+// Entry index (into plist / rs) of the i-th entry of the concatenation.
+__device__ __forceinline__ size_t list_entry(const Params& p, const Lists& L, uint32_t i) {
+    const uint32_t G = p.cls_grid;
+    uint32_t lo = 0, hi = G;  // L.off[lo] <= i < L.off[hi]
+    while (hi - lo > 1) {
+        const uint32_t mid = (lo + hi) >> 1;
+        if (L.off[mid] <= i) lo = mid; else hi = mid;
+    }
+    const uint64_t T = (uint64_t)p.num_regions / (kTile / kRegion);
+    return (size_t)((uint64_t)lo * T / G) * kTile + (i - L.off[lo]);
 }
 
 __global__ void __launch_bounds__(kThreads, kBlocksPerSm) k_insert(Params p) {
-    __shared__ TileScan ts;
-    __shared__ uint32_t s_part[2];
+    __shared__ Lists L;
+    __shared__ uint32_t s_part[kThreads / 32];
     __shared__ uint32_t s_nnew;
     pdl_wait();
     pdl_trigger();
-    const int t = threadIdx.x, lane = t & 31, warp = t >> 5;
-    const uint32_t tile = blockIdx.x;
+    const int t = threadIdx.x, lane = t & 31;
     if (t == 0) s_nnew = 0;
-    const uint32_t total = tile_scan(p, tile, ts, s_part);
+    const uint32_t M = lists_scan(p, L, s_part);
     // slots in use: a power of two >= 1.25 x the call's kept points
     uint32_t lg = 10;
     if (p.table_log2_fixed > 0) {
         lg = (uint32_t)p.table_log2_fixed;
     } else {
-        const uint64_t need = (uint64_t)ld_cg(&p.hdr->num_rec) * 5 / 4;
+        const uint64_t need = (uint64_t)M * 5 / 4;
         while (lg < p.table_log2 && (1ull << lg) < need) ++lg;
     }
     const uint32_t mask = (uint32_t)((1ull << lg) - 1ull);
-    const int nwarps = kThreads / 32;
     const uint32_t lt = (1u << lane) - 1u;
-    // the tile's sub-list of created voxels: room for every record of the tile
-    uint4* sub = p.newlist + (size_t)tile * kTile;
-    // batch j0 is processed while the warp's next batch's records load
-    uint32_t j = (uint32_t)warp * 32u + lane;
-    bool act = j < total;
-    uint32_t pos = act ? tile_item_pos(ts, tile, j) : 0u;
-    uint2 a = act ? __ldcs(p.keys + pos) : make_uint2(0u, 0u);   // lin, frame
-    for (uint32_t j0 = (uint32_t)warp * 32u; j0 < total; j0 += nwarps * 32u) {
-        const uint32_t jn = j0 + nwarps * 32u + lane;
-        const bool actn = jn < total;
-        const uint32_t posn = actn ? tile_item_pos(ts, tile, jn) : 0u;
-        const uint2 an = actn ? __ldcs(p.keys + posn) : make_uint2(0u, 0u);
+    uint4* sub = p.newlist + (size_t)blockIdx.x * p.ins_cap;
+    const uint32_t nb = (M + 31) / 32;
+    const uint32_t gw = (blockIdx.x * kThreads + t) >> 5;
+    const uint32_t W = (gridDim.x * kThreads) >> 5;
+    // batch g is processed while the warp's next batch loads
+    uint32_t g = gw;
+    bool act = g * 32 + lane < M;
+    size_t e = act ? list_entry(p, L, g * 32 + lane) : 0;
+    uint4 a = act ? __ldcs(p.plist + e) : make_uint4(0u, 0u, 0u, 0u);   // lin, frame, pos
+    for (; g < nb; g += W) {
+        const uint32_t in = (g + W) * 32 + lane;
+        const bool actn = g + W < nb && in < M;
+        const size_t en = actn ? list_entry(p, L, in) : 0;
+        const uint4 an = actn ? __ldcs(p.plist + en) : make_uint4(0u, 0u, 0u, 0u);
 
         const uint32_t am = __ballot_sync(kFull, act);
         const unsigned long long key = ((unsigned long long)a.y << 32) | a.x;
@@ -142,21 +161,22 @@ __global__ void __launch_bounds__(kThreads, kBlocksPerSm) k_insert(Params p) {
         }
         h = __shfl_sync(kFull, h, leader);
         base = __shfl_sync(kFull, base, leader);
-        if (act) p.rec_slot[pos] = make_uint2(h, base + __popc(grp & lt));
-        // leaders of new slots append to the tile's sub-list
+        if (act) p.rs[e] = make_uint2(h, base + __popc(grp & lt));
+        // leaders of new slots append to this block's sub-list
         const uint32_t cm = __ballot_sync(kFull, created);
         if (cm) {
             uint32_t wbase = 0;
             if (lane == __ffs(cm) - 1) wbase = atomicAdd(&s_nnew, (uint32_t)__popc(cm));
             wbase = __shfl_sync(kFull, wbase, __ffs(cm) - 1);
-            if (created) sub[wbase + __popc(cm & lt)] = make_uint4(h, a.x, a.y, 0u);
+            const uint32_t at = wbase + __popc(cm & lt);
+            if (created && at < p.ins_cap) sub[at] = make_uint4(h, a.x, a.y, 0u);
         }
         a = an;
-        pos = posn;
+        e = en;
         act = actn;
     }
     __syncthreads();
-    if (t == 0) p.blockcount[tile] = s_nnew;
+    if (t == 0) p.blockcount[blockIdx.x] = min(s_nnew, p.ins_cap);
 }
 
 __global__ void __launch_bounds__(kThreads) k_compact(Params p) {
@@ -168,8 +188,8 @@ __global__ void __launch_bounds__(kThreads) k_compact(Params p) {
     pdl_trigger();
     const int t = threadIdx.x, lane = t & 31, warp = t >> 5;
     const uint32_t b = blockIdx.x;
-    const uint4* sub = p.newlist + (size_t)b * kTile;
-    const uint32_t n = p.blockcount[b];
+    const uint4* sub = p.newlist + (size_t)b * p.ins_cap;
+    const uint32_t n = min(p.blockcount[b], p.ins_cap);
     if (n == 0) return;
     if (t < kFrameWin) s_fcnt[t] = 0;
     // this tile's place in the occupied-voxel list (order is immaterial)
@@ -239,29 +259,31 @@ __global__ void __launch_bounds__(kThreads) k_compact(Params p) {
 }
 
 __global__ void __launch_bounds__(kThreads, kBlocksPerSm) k_scatter_points(Params p) {
-    __shared__ TileScan ts;
-    __shared__ uint32_t s_part[2];
+    __shared__ Lists L;
+    __shared__ uint32_t s_part[kThreads / 32];
     pdl_wait();
     pdl_trigger();
-    const uint32_t tile = blockIdx.x;
     // frames with more voxels than max_voxels need each voxel's minimum ROI
     // rank (the cap keeps the smallest (rank, lin)); others never read it
     int capped = 0;
     for (int f = threadIdx.x; f < p.num_frames; f += blockDim.x)
         capped |= ld_cg(&p.frame_u[f]) > (uint32_t)p.max_voxels;
     capped = __syncthreads_or(capped);
-    const uint32_t total = tile_scan(p, tile, ts, s_part);
+    const uint32_t M = lists_scan(p, L, s_part);
     const uint32_t cap = min(ld_cg(&p.hdr->seg_total), p.occ_cap);  // seg holds N entries
-    for (uint32_t j = threadIdx.x; j < total; j += blockDim.x) {
-        const uint32_t pos = tile_item_pos(ts, tile, j);
-        const uint2 hs = p.rec_slot[pos];
+    const uint32_t gs = gridDim.x * blockDim.x;
+    for (uint32_t i = blockIdx.x * blockDim.x + threadIdx.x; i < M; i += gs) {
+        const size_t e = list_entry(p, L, i);
+        const uint2 hs = p.rs[e];
         if (hs.x == kUnset) continue;
+        const uint32_t pos = p.plist[e].z;
         const uint32_t at = ld_cg(slot_seg(p, hs.x)) + hs.y;
         if (at < cap) p.seg[at] = pos;
         else set_status(p.hdr, MMBEV_DEV_BOUNDS);
         if (capped) {
-            const uint32_t f = p.keys[pos].y;
-            if (ld_cg(&p.frame_u[f]) > (uint32_t)p.max_voxels)
+            const uint32_t f = p.plist[e].y;
+            if (f < (uint32_t)p.num_frames && ld_cg(&p.frame_u[f]) > (uint32_t)p.max_voxels &&
+                pos < p.rec_cap)
                 atomicMax(slot_rank(p, hs.x), 0xFFFFFFFFu - p.records[2 * (size_t)pos + 1].y);
         }
     }
@@ -269,22 +291,18 @@ __global__ void __launch_bounds__(kThreads, kBlocksPerSm) k_scatter_points(Param
 
 }  // namespace
 
+uint32_t insert_blocks(int num_sms) { return (uint32_t)num_sms * kBlocksPerSm; }
+
 cudaError_t launch_insert(const Params& p, bool pdl, cudaStream_t st) {
-    const uint32_t tiles = p.num_regions / (kTile / kRegion);
-    if (tiles == 0) return cudaSuccess;
-    return launch_k(k_insert, dim3(tiles), dim3(kThreads), 0, st, pdl, p);
+    return launch_k(k_insert, dim3(p.ins_blocks), dim3(kThreads), 0, st, pdl, p);
 }
 
 cudaError_t launch_compact(const Params& p, bool pdl, cudaStream_t st) {
-    const uint32_t tiles = p.num_regions / (kTile / kRegion);
-    if (tiles == 0) return cudaSuccess;
-    return launch_k(k_compact, dim3(tiles), dim3(kThreads), 0, st, pdl, p);
+    return launch_k(k_compact, dim3(p.ins_blocks), dim3(kThreads), 0, st, pdl, p);
 }
 
 cudaError_t launch_scatter_points(const Params& p, bool pdl, cudaStream_t st) {
-    const uint32_t tiles = p.num_regions / (kTile / kRegion);
-    if (tiles == 0) return cudaSuccess;
-    return launch_k(k_scatter_points, dim3(tiles), dim3(kThreads), 0, st, pdl, p);
+    return launch_k(k_scatter_points, dim3(p.ins_blocks), dim3(kThreads), 0, st, pdl, p);
 }
 
 }  // namespace mmbev

@@ -4,25 +4,25 @@
 //   points      caller's float32 [N][5] AoS, streamed once by the classify
 //               kernel through a 3-stage ring of 40 KB shared-memory tiles,
 //               each tile moved by eight 5 KB cp.async.bulk (TMA) copies.
-//   keys        workspace, 8 B per kept point {lin, frame}, at position
-//               region*32 + (its rank among the kept points of its 32-point
-//               region). Region g holds points 32g .. 32g+31, so positions
-//               increase with the point index and "first K by position" is
-//               "first K by index".
-//   records     workspace, 32 B per kept point at the same position:
-//               {x', y', z', intensity} {dt, ROI rank, -, -}.
-//   reg_cnt     workspace, kept points per region.
-//   newlist     workspace, per tile a sub-list of the voxels that tile's
-//               insert block created {slot, lin, frame}; the compact kernel
-//               concatenates the sub-lists into the occupied-voxel list.
+//   records     workspace, 32 B per kept point, at position region*32 + (its
+//               rank among the kept points of its 32-point region):
+//               {x', y', z', intensity} {dt, ROI rank, -, -}. Region g holds
+//               points 32g .. 32g+31, so positions increase with the point
+//               index and "first K by position" is "first K by index".
+//   plist       workspace, per classify block a dense list (any order) of its
+//               kept points {lin, frame, position}, starting at the block's
+//               first tile * 2048; cls_cnt holds the lengths.
+//   rs          workspace, parallel to plist: {slot, arrival number of the
+//               point in its voxel}, from the insert kernel.
 //   table       caller's hash table of 16-byte slots: { u64 key+1 (0 =
 //               empty), u32 0xFFFFFFFF-minrank (0 = none), u32 count (points
 //               of the voxel) }. Insert uses the first H slots, H the power of
 //               two >= 1.25 x the kept points of the call (at most the
 //               buffer's capacity, >= 2 x the points). Once the voxels are
 //               listed the key's low word holds the voxel's segment offset.
-//   rec_slot    workspace, per record position {slot, arrival index in the
-//               voxel}, from the insert kernel.
+//   newlist     workspace, per insert block a sub-list of the voxels that
+//               block created {slot, lin, frame}; the compact kernel
+//               concatenates the sub-lists into the occupied-voxel list.
 //   seg         workspace, the record positions of each voxel's points,
 //               voxel after voxel (CSR); a voxel's first K points are its K
 //               smallest positions.
@@ -45,6 +45,9 @@ constexpr int kMaxK = MMBEV_MAX_PTS_PER_VOXEL;
 constexpr int kTile = 2048;
 constexpr int kTileBytes = kTile * 5 * 4;
 constexpr int kRegion = 32;
+
+// Classify blocks (one per SM, at most this many).
+constexpr int kMaxClsGrid = 1000;
 
 // Bucket bitmap ordering: a bucket spans 2^kBucketLog2Max consecutive linear
 // indices of one frame (fewer when the grid is smaller); one warp ranks a
@@ -126,14 +129,17 @@ struct Params {
     uint32_t* hist;         // [R] voxels per minimum rank (capped frames)
     uint32_t* frame_u;      // [F] unique voxels per frame
     FrameInfo* finfo;       // [F]
-    uint2* keys;            // [regions*32] voxel key {lin, frame} of each kept point
     uint4* records;         // [regions*32][2] kept points' features and rank
-    uint32_t* reg_cnt;      // [regions] kept points per 32-point region
-    uint2* rec_slot;        // [regions*32] slot and arrival index of each record
+    uint4* plist;           // [tiles*2048] per classify block: kept {lin, frame, position}
+    uint2* rs;              // [tiles*2048] parallel to plist: {slot, arrival}
+    uint32_t* cls_cnt;      // [kMaxClsGrid] list length of each classify block
+    uint32_t cls_grid;      // classify blocks of the call
     uint32_t* seg;          // [N] record positions, voxel by voxel
     uint32_t num_regions;
-    uint4* newlist;         // [regions*32] voxels created, per insert block: slot, lin, frame
-    uint32_t* blockcount;   // [tiles] voxels created by each tile's insert block
+    uint4* newlist;         // [ins_blocks * ins_cap] voxels created, per insert block
+    uint32_t* blockcount;   // [ins_blocks] voxels each insert block created
+    uint32_t ins_blocks;    // grid of the insert kernel
+    uint32_t ins_cap;       // room of each insert block's sub-list
     unsigned long long* bcnt;   // [B] voxels per bucket (every frame, no classes)
     unsigned long long* bcnt2;  // [B] capped frames: lo = rank-below, hi = rank-tie
     unsigned long long* boff;   // [B] exclusive offsets within the frame (lo, hi)
@@ -320,7 +326,9 @@ cudaError_t launch_prep(const Params& p, const HostDesc& d, cudaStream_t st);
 cudaError_t launch_classify(const Params& p, int rmax, int num_sms, bool pdl, cudaStream_t st);
 cudaError_t launch_classify_points(const Params& p, cudaStream_t st);
 cudaError_t launch_insert(const Params& p, bool pdl, cudaStream_t st);
+cudaError_t launch_insert(const Params& p, bool pdl, cudaStream_t st);
 cudaError_t launch_compact(const Params& p, bool pdl, cudaStream_t st);
+uint32_t insert_blocks(int num_sms);
 cudaError_t launch_scatter_points(const Params& p, bool pdl, cudaStream_t st);
 cudaError_t launch_capped_hist(const Params& p, int num_sms, bool pdl, cudaStream_t st);
 cudaError_t launch_frames(const Params& p, bool pdl, cudaStream_t st);

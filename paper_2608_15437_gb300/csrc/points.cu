@@ -14,9 +14,10 @@
 // prepared ROIs of the (one or two) frames a block's tile range starts with
 // sit in shared memory. Kept points are compacted per 32-point region with
 // warp ballots, in input order: position (region)*32 + (rank among the
-// region's kept points) gets the point's voxel key (8 bytes) and a 32-byte
-// record with the compensated features and the ROI rank, so later stages
-// never touch the raw points again.
+// region's kept points) gets a 32-byte record with the compensated features
+// and the ROI rank, so later stages never touch the raw points again. The
+// block also appends {lin, frame, position} of every kept point to its own
+// dense list (order immaterial) for the hash insert.
 //
 // The classify-only entry point (per-point outputs for testing S1-S2) uses a
 // plain one-thread-per-point kernel built from the same device functions.
@@ -204,7 +205,7 @@ __global__ void __launch_bounds__(kThreads, 1) k_classify(Params p, int rmax, in
     // 0-15 cover region 2*warp, lanes 16-31 region 2*warp+1.
     const uint32_t lt = (1u << lane) - 1u;
     const uint32_t half_mask = lane < 16 ? 0x0000FFFFu : 0xFFFF0000u;
-    uint32_t kept_total = 0;   // this warp's kept points (lane 0)
+    uint4* plist = p.plist + t_begin * kTile;   // room for every point of the range
     // the sweep of this lane's current point and what depends on it
     int s = find_sweep(sm.soff, S, t_begin * kTile + warp * 64 + 2 * lane);
     int64_t next_off = 0;      // first index of the next sweep
@@ -315,29 +316,32 @@ __global__ void __launch_bounds__(kThreads, 1) k_classify(Params p, int rmax, in
         }
 #pragma unroll
         for (int k = 0; k < 2; ++k) valid[k] = hit[k] >= 0 && voxel_lin(p, x[k], y[k], z[k], lin[k]);
-        // compaction in the 32-point regions, input order kept
+        // compaction in the 32-point regions, input order kept: the record
+        // position of a kept point grows with its index
         const uint32_t b0 = __ballot_sync(0xFFFFFFFFu, valid[0]);
         const uint32_t b1 = __ballot_sync(0xFFFFFFFFu, valid[1]);
         const uint32_t below = lt & half_mask;
         const uint32_t rank0 = __popc(b0 & below) + __popc(b1 & below);
         const uint32_t region =
             (uint32_t)(tile * (kTile / kRegion)) + (uint32_t)(warp * 2) + (lane >> 4);
+        // the block's dense list of kept points (any order): one shared
+        // atomic per warp reserves the warp's entries
+        const uint32_t nk = __popc(b0) + __popc(b1);
+        uint32_t lbase = 0;
+        if (lane == 0 && nk) lbase = atomicAdd(&sm.kept[0], nk);
+        lbase = __shfl_sync(0xFFFFFFFFu, lbase, 0);
 #pragma unroll
         for (int k = 0; k < 2; ++k) {
             if (valid[k]) {
                 const uint32_t rk = rank0 + (k ? (uint32_t)valid[0] : 0u);
-                const size_t at = (size_t)region * kRegion + rk;
-                p.keys[at] = make_uint2(lin[k], frk[k]);
-                uint4* rec = p.records + 2 * at;
+                const uint32_t at = region * (uint32_t)kRegion + rk;
+                const uint32_t li = lbase + (k ? __popc(b0) + __popc(b1 & lt) : __popc(b0 & lt));
+                plist[li] = make_uint4(lin[k], frk[k], at, 0u);
+                uint4* rec = p.records + 2 * (size_t)at;
                 rec[0] = make_uint4(__float_as_uint(x[k]), __float_as_uint(y[k]),
                                     __float_as_uint(z[k]), __float_as_uint(pi[k]));
                 rec[1] = make_uint4(__float_as_uint(pd[k]), (uint32_t)hit[k], 0u, 0u);
             }
-        }
-        if ((lane & 15) == 0) {
-            const uint32_t c = __popc(b0 & half_mask) + __popc(b1 & half_mask);
-            p.reg_cnt[region] = c;
-            kept_total += c;
         }
         if (++st == nstages) {
             st = 0;
@@ -345,13 +349,12 @@ __global__ void __launch_bounds__(kThreads, 1) k_classify(Params p, int rmax, in
             ++round;
         }
     }
-    kept_total += __shfl_down_sync(0xFFFFFFFFu, kept_total, 16);
-    // one global add per block: the last warp to leave adds the block's total
+    // the last warp to leave publishes the block's list length
     if (lane == 0) {
-        atomicAdd(&sm.kept[0], kept_total);
         __threadfence_block();
         if (atomicAdd(&sm.kept[1], 1u) == (uint32_t)(kWarps - 1)) {
             const uint32_t tot = atomicAdd(&sm.kept[0], 0u);
+            p.cls_cnt[blockIdx.x] = tot;
             if (tot) atomicAdd(&p.hdr->num_rec, tot);
         }
     }
@@ -402,9 +405,9 @@ cudaError_t launch_classify(const Params& p, int rmax, int num_sms, bool pdl, cu
         if (e != cudaSuccess) return e;
         if (dev >= 0 && dev < 64) configured[dev].store(1, std::memory_order_release);
     }
-    const int64_t tiles = (p.num_points + kTile - 1) / kTile;
-    const int grid = (int)(tiles < num_sms ? tiles : num_sms);
-    return launch_k(k_classify, dim3(grid), dim3(kThreads), smem, st, pdl, p, rmax, nstages);
+    (void)num_sms;
+    return launch_k(k_classify, dim3(p.cls_grid), dim3(kThreads), smem, st, pdl, p, rmax,
+                    nstages);
 }
 
 cudaError_t launch_classify_points(const Params& p, cudaStream_t st) {

@@ -123,11 +123,8 @@ k_prep(Params p, const __grid_constant__ HostDesc d) {
         for (size_t i = gt; i < (size_t)p.num_rois; i += gs) p.hist[i] = 0u;
     if (p.frame_u)
         for (size_t i = gt; i < (size_t)p.num_frames; i += gs) p.frame_u[i] = 0u;
-    if (p.reg_cnt) {
-        // a classify pass that gives up leaves the regions it did not reach empty
-        uint4* r4 = reinterpret_cast<uint4*>(p.reg_cnt);  // a multiple of 64 counters
-        for (size_t i = gt; i < (size_t)p.num_regions / 4; i += gs) r4[i] = make_uint4(0u, 0u, 0u, 0u);
-    }
+    if (p.cls_cnt)  // a classify block that gives up leaves its list empty
+        for (size_t i = gt; i < (size_t)kMaxClsGrid; i += gs) p.cls_cnt[i] = 0u;
     if (p.bcnt) {
         uint4* b4 = reinterpret_cast<uint4*>(p.bcnt);  // B u64 counters, B even or padded
         const size_t n4 = ((size_t)p.num_buckets + 1) / 2;
