@@ -44,6 +44,20 @@ def dist_env():
     return world, rank, local
 
 
+def aggregate_ranks(ms_total: float, e2e_s: float, n_points: float, world: int, device):
+    """Whole-job figures over the ranks: the slowest rank's times (MAX) and
+    the points all ranks processed (SUM). Each rank voxelizes its own frames,
+    so this is the only exchange, and it runs outside the timed regions."""
+    import torch
+    import torch.distributed as dist
+    t = torch.tensor([ms_total, e2e_s], dtype=torch.float64, device=device)
+    pts = torch.tensor([float(n_points)], dtype=torch.float64, device=device)
+    if world > 1:
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+        dist.all_reduce(pts, op=dist.ReduceOp.SUM)
+    return float(t[0].item()), float(t[1].item()), float(pts[0].item())
+
+
 def workload_for_rank(rank: int, frames: int = FRAMES):
     return synth.streaming_batch(frames, base_seed=1000 + FRAMES * rank)
 
@@ -97,7 +111,8 @@ def profile_traffic(stage):
 
 
 class ClockSampler:
-    """nvidia-smi samples (200 ms) while the timed region runs."""
+    """nvidia-smi samples (every 50 ms) from just before the timed region to
+    the end of the per-kernel breakdown run that follows it."""
 
     FIELDS = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
               "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
@@ -113,11 +128,12 @@ class ClockSampler:
         try:
             self.proc = subprocess.Popen(
                 ["nvidia-smi", f"--id={self.gpu}", f"--query-gpu={self.FIELDS}",
-                 "--format=csv,noheader,nounits", "-lms", "200"],
+                 "--format=csv,noheader,nounits", "-lms", "50"],
                 stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
         except OSError:
             self.proc = None
             return
+        self.t0 = time.perf_counter()
         self.thread = threading.Thread(target=self._read, daemon=True)
         self.thread.start()
 
@@ -151,7 +167,8 @@ class ClockSampler:
                     reasons.add(name)
         return {"sm_mhz": float(np.median(sm)) if sm else None,
                 "sm_max_mhz": float(max(smax)) if smax else None,
-                "samples": len(sm), "reasons": sorted(reasons)}
+                "samples": len(sm), "window_s": round(time.perf_counter() - self.t0, 3),
+                "reasons": sorted(reasons)}
 
 
 def cpu_oracle_baseline(w, budget_s: float = 12.0):
@@ -182,7 +199,7 @@ def run_reference(args):
     import oracle
     oracle.build()
     w = workload_for_rank(0)
-    per_step = 2  # frames per step: a bounded sample of the batch
+    per_step = 1  # frames per step: a bounded sample of the batch
     frames = [w.frame(f) for f in range(w.num_frames)]
     in_roi = []
     for fw in frames:  # the metric's numerator per frame, untimed
@@ -270,7 +287,7 @@ def run_gpu(args):
 
     sampler = ClockSampler(dev.index if dev.index is not None else 0)
     sampler.start()
-    time.sleep(0.3)
+    time.sleep(0.1)
     start = torch.cuda.Event(enable_timing=True)
     end = torch.cuda.Event(enable_timing=True)
     # timed region 1, the headline: K back-to-back calls, kernels chained by
@@ -304,16 +321,6 @@ def run_gpu(args):
     stage_ms /= args.steps
     names = mmbev.stage_names()
 
-    # slowest rank decides
-    t_local = torch.tensor([ms_total], dtype=torch.float64, device=dev)
-    pts_local = torch.tensor([float(n_in_roi)], dtype=torch.float64, device=dev)
-    if world > 1:
-        dist.all_reduce(t_local, op=dist.ReduceOp.MAX)
-        dist.all_reduce(pts_local, op=dist.ReduceOp.SUM)
-    ms_max = float(t_local.item())
-    total_pts = float(pts_local.item())
-    ms_step = ms_max / args.steps
-    value = total_pts / (ms_step * 1e-3)
 
     # end to end through the public API: pinned host inputs, H2D, the call,
     # D2H of the per-frame counts and the kept rows
@@ -358,10 +365,12 @@ def run_gpu(args):
     for _ in range(e2e_steps):
         e2e_step()
     torch.cuda.synchronize(dev)
-    e2e_s = torch.tensor([time.perf_counter() - t0], dtype=torch.float64, device=dev)
-    if world > 1:
-        dist.all_reduce(e2e_s, op=dist.ReduceOp.MAX)
-    e2e_value = total_pts / (float(e2e_s.item()) / e2e_steps)
+    e2e_local = time.perf_counter() - t0
+    # slowest rank decides
+    ms_max, e2e_max, total_pts = aggregate_ranks(ms_total, e2e_local, n_in_roi, world, dev)
+    ms_step = ms_max / args.steps
+    value = total_pts / (ms_step * 1e-3)
+    e2e_value = total_pts / (e2e_max / e2e_steps)
     h2d_bytes = w.points.nbytes + w.sweep_tf.nbytes + w.rois.nbytes
 
     if rank == 0:
@@ -404,8 +413,8 @@ def run_gpu(args):
 def main():
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
-    ap.add_argument("--steps", type=int, default=20)
-    ap.add_argument("--warmup", type=int, default=5)
+    ap.add_argument("--steps", type=int, default=1000)
+    ap.add_argument("--warmup", type=int, default=10)
     ap.add_argument("--impl", default="gb300", choices=["gb300", "reference"])
     ap.add_argument("--frames", type=int, default=FRAMES,
                     help="frames per GPU (the headline workload is 32; fewer for small "

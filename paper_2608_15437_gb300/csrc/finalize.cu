@@ -70,7 +70,6 @@ template <int B>
 __global__ void __launch_bounds__(kThreads) k_finalize(Params p) {
     __shared__ uint32_t s_vbase[kMaxFrames + 1];
     pdl_wait();
-    pdl_trigger();
     const int F = p.num_frames;
     for (int i = threadIdx.x; i < F; i += blockDim.x) s_vbase[i] = p.finfo[i].vbase;
     const uint32_t total = ld_cg(&p.hdr->total_kept);
@@ -141,7 +140,6 @@ template <int B>
 __global__ void __launch_bounds__(kThreads) k_finalize_heavy(Params p) {
     __shared__ uint32_t s_vbase[kMaxFrames + 1];
     pdl_wait();
-    pdl_trigger();
     const int F = p.num_frames;
     for (int i = threadIdx.x; i < F; i += blockDim.x) s_vbase[i] = p.finfo[i].vbase;
     const uint32_t total = ld_cg(&p.hdr->total_kept);

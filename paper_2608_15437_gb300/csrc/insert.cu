@@ -102,7 +102,6 @@ __global__ void __launch_bounds__(kThreads, kBlocksPerSm) k_insert(Params p) {
     __shared__ uint32_t s_part[kThreads / 32];
     __shared__ uint32_t s_nnew;
     pdl_wait();
-    pdl_trigger();
     const int t = threadIdx.x, lane = t & 31;
     if (t == 0) s_nnew = 0;
     const uint32_t M = lists_scan(p, L, s_part);
@@ -185,7 +184,6 @@ __global__ void __launch_bounds__(kThreads) k_compact(Params p) {
     __shared__ uint32_t s_fcnt[kFrameWin];
     __shared__ uint32_t s_fmin;
     pdl_wait();
-    pdl_trigger();
     const int t = threadIdx.x, lane = t & 31, warp = t >> 5;
     const uint32_t b = blockIdx.x;
     const uint4* sub = p.newlist + (size_t)b * p.ins_cap;
@@ -262,7 +260,6 @@ __global__ void __launch_bounds__(kThreads, kBlocksPerSm) k_scatter_points(Param
     __shared__ Lists L;
     __shared__ uint32_t s_part[kThreads / 32];
     pdl_wait();
-    pdl_trigger();
     // frames with more voxels than max_voxels need each voxel's minimum ROI
     // rank (the cap keeps the smallest (rank, lin)); others never read it
     int capped = 0;

@@ -179,10 +179,12 @@ __device__ __forceinline__ void set_status(Header* hdr, uint32_t bits) {
     atomicOr(&hdr->status, bits);
 }
 
-// Programmatic dependent launch: wait for the preceding kernel's results,
-// and let the next kernel's blocks be scheduled.
+// Programmatic dependent launch: wait for the preceding kernel's results.
+// No kernel signals its dependents early: they are released as its blocks
+// exit, so waiting blocks of the next kernel never take SM slots from blocks
+// of the running one, while the next launch is still prepared during the
+// running kernel's tail.
 __device__ __forceinline__ void pdl_wait() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
-__device__ __forceinline__ void pdl_trigger() { asm volatile("griddepcontrol.launch_dependents;"); }
 
 // Eq. 6 for one point: ((r0*x + r1*y) + r2*z) + t, every op rounded (no FMA).
 __device__ __forceinline__ void compensate(const float* T, float x, float y, float z,

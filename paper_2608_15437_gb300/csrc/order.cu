@@ -50,7 +50,6 @@ __device__ bool block_any_capped(const Params& p) {
 // ---------------------------------------------------------------- stage 3
 __global__ void __launch_bounds__(kThreads) k_capped_hist(Params p) {
     pdl_wait();
-    pdl_trigger();
     if (!block_any_capped(p)) return;
     const uint32_t U = min(ld_cg(&p.hdr->num_occ), p.occ_cap);
     const uint32_t gs = gridDim.x * blockDim.x;
@@ -69,7 +68,6 @@ __global__ void __launch_bounds__(1024) k_frames(Params p) {
     __shared__ uint32_t s_u[kMaxFrames];
     __shared__ uint32_t s_wsum[2][32];
     pdl_wait();
-    pdl_trigger();
     const int t = threadIdx.x, lane = t & 31, warp = t >> 5;
     const uint32_t maxv = (uint32_t)p.max_voxels;
     const int F = p.num_frames;
@@ -189,7 +187,6 @@ __device__ __forceinline__ uint32_t bucket_add(unsigned long long* cnt, bool min
 
 __global__ void __launch_bounds__(kThreads) k_capped_census(Params p) {
     pdl_wait();
-    pdl_trigger();
     if (ld_cg(&p.hdr->any_capped) == 0u) return;
     const uint32_t U = min(ld_cg(&p.hdr->num_occ), p.occ_cap);
     const int lane = threadIdx.x & 31;
@@ -225,7 +222,6 @@ __global__ void __launch_bounds__(kScanThreads) k_scan(Params p) {
     __shared__ uint32_t s_nz[kScanThreads / 32];
     __shared__ uint32_t s_nzbase;
     pdl_wait();
-    pdl_trigger();
     const int t = threadIdx.x, lane = t & 31, warp = t >> 5;
     const uint32_t f = blockIdx.x;
     const uint32_t Bf = p.buckets_per_frame;
@@ -287,7 +283,6 @@ __global__ void __launch_bounds__(kScanThreads) k_scan(Params p) {
 // ---------------------------------------------------------------- stage 7
 __global__ void __launch_bounds__(kThreads) k_scatter(Params p) {
     pdl_wait();
-    pdl_trigger();
     const uint32_t U = min(ld_cg(&p.hdr->num_occ), p.occ_cap);
     const uint32_t gs = gridDim.x * blockDim.x;
     for (uint32_t d = blockIdx.x * blockDim.x + threadIdx.x; d < U; d += gs) {
@@ -310,7 +305,6 @@ __global__ void __launch_bounds__(kRankWarps * 32) k_rank(Params p) {
     __shared__ uint16_t s_pb[kRankWarps][kBmWords];
     __shared__ uint16_t s_pt[kRankWarps][kBmWords];
     pdl_wait();
-    pdl_trigger();
     const int lane = threadIdx.x & 31, wl = threadIdx.x >> 5;
     uint32_t* bm_below = s_below[wl];
     uint32_t* bm_tie = s_tie[wl];

@@ -138,7 +138,6 @@ __device__ __forceinline__ ClsSmem carve(unsigned char* smem, int S, int rmax, b
 __global__ void __launch_bounds__(kThreads, 1) k_classify(Params p, int rmax, int nstages) {
     extern __shared__ __align__(128) unsigned char smem[];
     pdl_wait();
-    pdl_trigger();
     const int t = threadIdx.x, lane = t & 31, warp = t >> 5;
     const int S = p.num_sweeps;
     const bool tf_staged = S <= kTfStageMax;
