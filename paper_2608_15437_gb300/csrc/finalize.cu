@@ -12,7 +12,8 @@
 //
 // Light kernel: one thread per kept voxel with at most 32 points keeps the K
 // smallest positions in a sorted register array (each position bubbles in
-// with compare-and-swap steps). Voxels with more points go to a list.
+// with compare-and-swap steps; eight positions load at a time). Voxels with
+// more points go to a list.
 // Heavy kernel: one warp per listed voxel; each lane keeps the smallest
 // positions of its share of the segment, then K rounds of a warp minimum
 // pick the voxel's K smallest in ascending order, the lanes fetch those
@@ -39,12 +40,19 @@ __device__ __forceinline__ void sorted_insert(uint32_t (&b)[B], uint32_t v) {
 }
 
 // record: {x', y', z', intensity} {dt, rank, -, -}
-__device__ __forceinline__ void add_record(float (&acc)[5], const uint4& a, const uint4& b) {
+__device__ __forceinline__ void add_record(float (&acc)[5], const uint4& a, float dt) {
     acc[0] = __fadd_rn(acc[0], __uint_as_float(a.x));
     acc[1] = __fadd_rn(acc[1], __uint_as_float(a.y));
     acc[2] = __fadd_rn(acc[2], __uint_as_float(a.z));
     acc[3] = __fadd_rn(acc[3], __uint_as_float(a.w));
-    acc[4] = __fadd_rn(acc[4], __uint_as_float(b.x));
+    acc[4] = __fadd_rn(acc[4], dt);
+}
+
+// Load the features of the record at position q (clamped into the array).
+__device__ __forceinline__ void load_record(const Params& p, uint32_t q, uint4& a, float& dt) {
+    const uint4* rec = p.records + 2 * (size_t)min(q, p.rec_cap - 1u);
+    a = __ldg(rec);
+    dt = __ldg(reinterpret_cast<const float*>(rec + 1));
 }
 
 __device__ __forceinline__ void write_voxel(const Params& p, size_t row, const float (&acc)[5],
@@ -105,31 +113,30 @@ __global__ void __launch_bounds__(kThreads) k_finalize(Params p) {
         uint32_t best[B];
 #pragma unroll
         for (int j = 0; j < B; ++j) best[j] = 0xFFFFFFFFu;
-        for (uint32_t i = 0; i < n; i += 4) {
-            uint32_t v[4];
+        // the segment's positions, eight loads in flight at a time
+        for (uint32_t i = 0; i < n; i += 8) {
+            uint32_t v[8];
 #pragma unroll
-            for (int c = 0; c < 4; ++c) v[c] = i + c < n ? __ldg(p.seg + off + i + c) : 0xFFFFFFFFu;
+            for (int c = 0; c < 8; ++c) v[c] = i + c < n ? __ldg(p.seg + off + i + c) : 0xFFFFFFFFu;
 #pragma unroll
-            for (int c = 0; c < 4; ++c) sorted_insert<B>(best, v[c]);
+            for (int c = 0; c < 8; ++c) sorted_insert<B>(best, v[c]);
         }
         const int cnt = (int)(n < (uint32_t)K ? n : (uint32_t)K);
         if (cnt > 0 && best[cnt - 1] >= p.rec_cap) set_status(p.hdr, MMBEV_DEV_BOUNDS);
+        // the kept records, all loads of a round in flight, summed in order
+        constexpr int R = B < 6 ? B : 6;
         float acc[5] = {0.f, 0.f, 0.f, 0.f, 0.f};
 #pragma unroll
-        for (int j0 = 0; j0 < B; j0 += 4) {
+        for (int j0 = 0; j0 < B; j0 += R) {
             if (j0 >= cnt) break;
-            uint4 ra[4], rb[4];
+            uint4 ra[R];
+            float dt[R];
 #pragma unroll
-            for (int c = 0; c < 4; ++c) {
-                if (j0 + c < cnt) {
-                    const uint4* rec = p.records + 2 * (size_t)min(best[j0 + c], p.rec_cap - 1u);
-                    ra[c] = __ldg(rec);
-                    rb[c] = __ldg(rec + 1);
-                }
-            }
+            for (int c = 0; c < R; ++c)
+                if (j0 + c < cnt) load_record(p, best[j0 + c], ra[c], dt[c]);
 #pragma unroll
-            for (int c = 0; c < 4; ++c)
-                if (j0 + c < cnt) add_record(acc, ra[c], rb[c]);
+            for (int c = 0; c < R; ++c)
+                if (j0 + c < cnt) add_record(acc, ra[c], dt[c]);
         }
         write_voxel(p, voxel_row(p, s_vbase, F, g), acc, cnt);
         zero_slot(p, h);
@@ -163,7 +170,17 @@ __global__ void __launch_bounds__(kThreads) k_finalize_heavy(Params p) {
         uint32_t best[B];
 #pragma unroll
         for (int j = 0; j < B; ++j) best[j] = 0xFFFFFFFFu;
-        for (uint32_t i = lane; i < n; i += 32) sorted_insert<B>(best, __ldg(p.seg + off + i));
+        // each lane takes every 32nd position, eight loads in flight at a time
+        for (uint32_t i0 = lane; i0 < n; i0 += 256) {
+            uint32_t v[8];
+#pragma unroll
+            for (int c = 0; c < 8; ++c) {
+                const uint32_t i = i0 + 32u * c;
+                v[c] = i < n ? __ldg(p.seg + off + i) : 0xFFFFFFFFu;
+            }
+#pragma unroll
+            for (int c = 0; c < 8; ++c) sorted_insert<B>(best, v[c]);
+        }
         // K rounds of a warp minimum over the lanes' smallest remaining; the
         // j-th smallest goes to lane j % 32 (second register for j >= 32)
         const int cnt = (int)(n < (uint32_t)K ? n : (uint32_t)K);
@@ -179,22 +196,20 @@ __global__ void __launch_bounds__(kThreads) k_finalize_heavy(Params p) {
         }
         float acc[5] = {0.f, 0.f, 0.f, 0.f, 0.f};
         for (int half = 0; half * 32 < cnt; ++half) {
-            uint4 ra = make_uint4(0u, 0u, 0u, 0u), rb = ra;
+            uint4 ra = make_uint4(0u, 0u, 0u, 0u);
+            float rdt = 0.f;
             if (half * 32 + lane < cnt) {
                 if (mine[half] >= p.rec_cap) set_status(p.hdr, MMBEV_DEV_BOUNDS);
-                const uint4* rec = p.records + 2 * (size_t)min(mine[half], p.rec_cap - 1u);
-                ra = __ldg(rec);
-                rb = __ldg(rec + 1);
+                load_record(p, mine[half], ra, rdt);
             }
             const int m = cnt - half * 32 < 32 ? cnt - half * 32 : 32;
             for (int j = 0; j < m; ++j) {
-                uint4 a, b;
+                uint4 a;
                 a.x = __shfl_sync(0xFFFFFFFFu, ra.x, j);
                 a.y = __shfl_sync(0xFFFFFFFFu, ra.y, j);
                 a.z = __shfl_sync(0xFFFFFFFFu, ra.z, j);
                 a.w = __shfl_sync(0xFFFFFFFFu, ra.w, j);
-                b.x = __shfl_sync(0xFFFFFFFFu, rb.x, j);
-                add_record(acc, a, b);
+                add_record(acc, a, __shfl_sync(0xFFFFFFFFu, rdt, j));
             }
         }
         if (lane == 0) {
