@@ -215,7 +215,7 @@ __global__ void __launch_bounds__(kThreads) k_capped_census(Params p) {
 // ---------------------------------------------------------------- stage 6
 // One block per frame: boff[b] = sum of the frame's counters before b.
 constexpr int kScanThreads = 1024;
-constexpr int kScanPer = 4;
+constexpr int kScanPer = 12;   // one pass covers 12,288 buckets (a 1440x1440x40 frame has 10,125)
 
 __global__ void __launch_bounds__(kScanThreads) k_scan(Params p) {
     __shared__ unsigned long long s_wsum[kScanThreads / 32];
