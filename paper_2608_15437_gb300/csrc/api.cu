@@ -63,10 +63,10 @@ constexpr uint32_t kMaxInsertBlocks = 2048;
 // Byte offsets of every workspace array for one call shape.
 struct Layout {
     size_t hdr, sweep_off, sweep_frame, fso, fro, roi_prep, masks, hist, frame_u, finfo;
-    size_t records, plist, rs, cls_cnt, seg, newlist, blockcount, bcnt, bcnt2, boff, nonempty, occ, d_bucket,
-        d_pos, d_lin, items, vid_slot, heavy;
+    size_t records, plist, rs, cls_cnt, seg, newlist, blockcount, bcnt, bcnt2, boff, ctot, nonempty, occ, d_bucket,
+        d_pos, d_lin, items, vid_slot, heavy, huge;
     size_t total;
-    uint32_t num_buckets, buckets_per_frame, num_tiles;
+    uint32_t num_buckets, buckets_per_frame, num_tiles, scan_chunks;
     int bucket_log2, mask_words, coarse;
 };
 
@@ -105,6 +105,8 @@ Layout make_layout(int64_t max_points, int64_t rois_total, int32_t max_rois_fram
     L.bcnt = take(sizeof(unsigned long long) * B2);
     L.bcnt2 = take(sizeof(unsigned long long) * B2);
     L.boff = take(sizeof(unsigned long long) * B2);
+    L.scan_chunks = (L.buckets_per_frame + kScanChunk - 1) / kScanChunk;
+    L.ctot = take(sizeof(uint32_t) * F * L.scan_chunks);
     L.nonempty = take(sizeof(uint32_t) * B2);
     L.occ = take(sizeof(uint32_t) * U);
     L.d_bucket = take(sizeof(uint32_t) * U);
@@ -113,6 +115,7 @@ Layout make_layout(int64_t max_points, int64_t rois_total, int32_t max_rois_fram
     L.items = take(sizeof(uint2) * U);
     L.vid_slot = take(sizeof(uint32_t) * (F * (size_t)(max_voxels > 0 ? max_voxels : 1)));
     L.heavy = take(sizeof(uint32_t) * (F * (size_t)(max_voxels > 0 ? max_voxels : 1)));
+    L.huge = take(sizeof(uint32_t) * (F * (size_t)(max_voxels > 0 ? max_voxels : 1)));
     L.total = o;
     return L;
 }
@@ -210,6 +213,8 @@ void bind_layout(Params* p, const Layout& L, uint8_t* ws) {
     p->bcnt = reinterpret_cast<unsigned long long*>(ws + L.bcnt);
     p->bcnt2 = reinterpret_cast<unsigned long long*>(ws + L.bcnt2);
     p->boff = reinterpret_cast<unsigned long long*>(ws + L.boff);
+    p->ctot = reinterpret_cast<uint32_t*>(ws + L.ctot);
+    p->scan_chunks = L.scan_chunks;
     p->nonempty = reinterpret_cast<uint32_t*>(ws + L.nonempty);
     p->occ = reinterpret_cast<uint32_t*>(ws + L.occ);
     p->d_bucket = reinterpret_cast<uint32_t*>(ws + L.d_bucket);
@@ -218,6 +223,7 @@ void bind_layout(Params* p, const Layout& L, uint8_t* ws) {
     p->items = reinterpret_cast<uint2*>(ws + L.items);
     p->vid_slot = reinterpret_cast<uint32_t*>(ws + L.vid_slot);
     p->heavy = reinterpret_cast<uint32_t*>(ws + L.heavy);
+    p->huge = reinterpret_cast<uint32_t*>(ws + L.huge);
     p->occ_cap = (uint32_t)(p->num_points > 0 ? p->num_points : 1);
     p->rec_cap = p->num_regions * (uint32_t)kRegion;
     p->mask_words = L.mask_words;

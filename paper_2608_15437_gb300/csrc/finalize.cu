@@ -17,7 +17,8 @@
 // Heavy kernel: one warp per listed voxel; each lane keeps the smallest
 // positions of its share of the segment, then K rounds of a warp minimum
 // pick the voxel's K smallest in ascending order, the lanes fetch those
-// records in parallel and lane 0 adds them up in order.
+// records in parallel and lane 0 adds them up in order. Voxels with more
+// than 1024 points get a whole block (eight warps' lists merged by one).
 #include "mmbev_internal.cuh"
 
 namespace mmbev {
@@ -25,6 +26,7 @@ namespace {
 
 constexpr int kThreads = 256;
 constexpr uint32_t kLightMax = 32;
+constexpr uint32_t kHugeMin = 1024;   // voxels with more points get a whole block
 
 // Insert v into the ascending array b[0..B) (unused entries hold ~0u); the
 // largest entry falls off the end.
@@ -101,7 +103,8 @@ __global__ void __launch_bounds__(kThreads) k_finalize(Params p) {
                 n = 0;
             }
         }
-        const bool heavy = act && n > kLightMax;
+        const bool heavy = act && n > kLightMax && n <= kHugeMin;
+        const bool huge = act && n > kHugeMin;
         const uint32_t hm = __ballot_sync(0xFFFFFFFFu, heavy);
         if (hm) {
             uint32_t base = 0;
@@ -109,7 +112,8 @@ __global__ void __launch_bounds__(kThreads) k_finalize(Params p) {
             base = __shfl_sync(0xFFFFFFFFu, base, __ffs(hm) - 1);
             if (heavy) p.heavy[base + __popc(hm & ((1u << lane) - 1u))] = g;
         }
-        if (!act || heavy) continue;
+        if (huge) p.huge[atomicAdd(&p.hdr->num_huge, 1u)] = g;  // rare
+        if (!act || heavy || huge) continue;
         uint32_t best[B];
 #pragma unroll
         for (int j = 0; j < B; ++j) best[j] = 0xFFFFFFFFu;
@@ -143,9 +147,34 @@ __global__ void __launch_bounds__(kThreads) k_finalize(Params p) {
     }
 }
 
+// The j-th of a warp's cnt smallest positions sits in lane j % 32 (register
+// j / 32): the lanes load those records in parallel and every lane adds them
+// up in order (lane 0's sum is the one written).
+__device__ __forceinline__ void warp_sum_records(const Params& p, const uint32_t (&mine)[2],
+                                                 int cnt, int lane, float (&acc)[5]) {
+    for (int half = 0; half * 32 < cnt; ++half) {
+        uint4 ra = make_uint4(0u, 0u, 0u, 0u);
+        float rdt = 0.f;
+        if (half * 32 + lane < cnt) {
+            if (mine[half] >= p.rec_cap) set_status(p.hdr, MMBEV_DEV_BOUNDS);
+            load_record(p, mine[half], ra, rdt);
+        }
+        const int m = cnt - half * 32 < 32 ? cnt - half * 32 : 32;
+        for (int j = 0; j < m; ++j) {
+            uint4 a;
+            a.x = __shfl_sync(0xFFFFFFFFu, ra.x, j);
+            a.y = __shfl_sync(0xFFFFFFFFu, ra.y, j);
+            a.z = __shfl_sync(0xFFFFFFFFu, ra.z, j);
+            a.w = __shfl_sync(0xFFFFFFFFu, ra.w, j);
+            add_record(acc, a, __shfl_sync(0xFFFFFFFFu, rdt, j));
+        }
+    }
+}
+
 template <int B>
 __global__ void __launch_bounds__(kThreads) k_finalize_heavy(Params p) {
     __shared__ uint32_t s_vbase[kMaxFrames + 1];
+    __shared__ uint32_t s_cand[kThreads / 32][kMaxK];
     pdl_wait();
     const int F = p.num_frames;
     for (int i = threadIdx.x; i < F; i += blockDim.x) s_vbase[i] = p.finfo[i].vbase;
@@ -154,10 +183,72 @@ __global__ void __launch_bounds__(kThreads) k_finalize_heavy(Params p) {
     __syncthreads();
     const int lane = threadIdx.x & 31;
     const uint32_t seg_cap = min(ld_cg(&p.hdr->seg_total), p.occ_cap);  // seg holds N entries
+    const int K = p.K;
+    // Huge voxels, one block each: every thread keeps the smallest positions
+    // of its share, each warp reduces its threads' to its K smallest, and
+    // warp 0 merges the warps' lists.
+    const uint32_t nhuge = ld_cg(&p.hdr->num_huge);
+    const int warp = threadIdx.x >> 5;
+    for (uint32_t e = blockIdx.x; e < nhuge; e += gridDim.x) {
+        const uint32_t g = p.huge[e];
+        const uint32_t h = p.vid_slot[g];
+        const uint32_t off = ld_cg(slot_seg(p, h));
+        uint32_t n = ld_cg(slot_cnt(p, h));
+        if (off > seg_cap || n > seg_cap - off) {
+            if (threadIdx.x == 0) set_status(p.hdr, MMBEV_DEV_BOUNDS);
+            n = 0;
+        }
+        const int cnt = (int)(n < (uint32_t)K ? n : (uint32_t)K);
+        uint32_t best[B];
+#pragma unroll
+        for (int j = 0; j < B; ++j) best[j] = 0xFFFFFFFFu;
+        for (uint32_t i0 = threadIdx.x; i0 < n; i0 += 8u * kThreads) {
+            uint32_t v[8];
+#pragma unroll
+            for (int c = 0; c < 8; ++c) {
+                const uint32_t i = i0 + (uint32_t)kThreads * c;
+                v[c] = i < n ? __ldg(p.seg + off + i) : 0xFFFFFFFFu;
+            }
+#pragma unroll
+            for (int c = 0; c < 8; ++c) sorted_insert<B>(best, v[c]);
+        }
+        for (int j = 0; j < cnt; ++j) {
+            const uint32_t m = __reduce_min_sync(0xFFFFFFFFu, best[0]);
+            if (lane == 0) s_cand[warp][j] = m;
+            if (best[0] == m) {
+#pragma unroll
+                for (int c = 0; c + 1 < B; ++c) best[c] = best[c + 1];
+                best[B - 1] = 0xFFFFFFFFu;
+            }
+        }
+        __syncthreads();
+        if (warp == 0) {
+#pragma unroll
+            for (int j = 0; j < B; ++j) best[j] = 0xFFFFFFFFu;
+            for (int i = lane; i < (kThreads / 32) * cnt; i += 32)
+                sorted_insert<B>(best, s_cand[i / cnt][i % cnt]);
+            uint32_t mine[2] = {0xFFFFFFFFu, 0xFFFFFFFFu};
+            for (int j = 0; j < cnt; ++j) {
+                const uint32_t m = __reduce_min_sync(0xFFFFFFFFu, best[0]);
+                if (lane == (j & 31)) mine[j >> 5] = m;
+                if (best[0] == m) {
+#pragma unroll
+                    for (int c = 0; c + 1 < B; ++c) best[c] = best[c + 1];
+                    best[B - 1] = 0xFFFFFFFFu;
+                }
+            }
+            float acc[5] = {0.f, 0.f, 0.f, 0.f, 0.f};
+            warp_sum_records(p, mine, cnt, lane, acc);
+            if (lane == 0) {
+                write_voxel(p, voxel_row(p, s_vbase, F, g), acc, cnt);
+                zero_slot(p, h);
+            }
+        }
+        __syncthreads();
+    }
     const uint32_t nh = ld_cg(&p.hdr->num_heavy);
     const uint32_t gw = (blockIdx.x * blockDim.x + threadIdx.x) >> 5;
     const uint32_t nw = (gridDim.x * blockDim.x) >> 5;
-    const int K = p.K;
     for (uint32_t e = gw; e < nh; e += nw) {
         const uint32_t g = p.heavy[e];
         const uint32_t h = p.vid_slot[g];
@@ -195,23 +286,7 @@ __global__ void __launch_bounds__(kThreads) k_finalize_heavy(Params p) {
             }
         }
         float acc[5] = {0.f, 0.f, 0.f, 0.f, 0.f};
-        for (int half = 0; half * 32 < cnt; ++half) {
-            uint4 ra = make_uint4(0u, 0u, 0u, 0u);
-            float rdt = 0.f;
-            if (half * 32 + lane < cnt) {
-                if (mine[half] >= p.rec_cap) set_status(p.hdr, MMBEV_DEV_BOUNDS);
-                load_record(p, mine[half], ra, rdt);
-            }
-            const int m = cnt - half * 32 < 32 ? cnt - half * 32 : 32;
-            for (int j = 0; j < m; ++j) {
-                uint4 a;
-                a.x = __shfl_sync(0xFFFFFFFFu, ra.x, j);
-                a.y = __shfl_sync(0xFFFFFFFFu, ra.y, j);
-                a.z = __shfl_sync(0xFFFFFFFFu, ra.z, j);
-                a.w = __shfl_sync(0xFFFFFFFFu, ra.w, j);
-                add_record(acc, a, __shfl_sync(0xFFFFFFFFu, rdt, j));
-            }
-        }
+        warp_sum_records(p, mine, cnt, lane, acc);
         if (lane == 0) {
             write_voxel(p, voxel_row(p, s_vbase, F, g), acc, cnt);
             zero_slot(p, h);

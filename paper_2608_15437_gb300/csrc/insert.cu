@@ -241,6 +241,11 @@ __global__ void __launch_bounds__(kThreads) k_compact(Params p) {
         if (ok && lane == leader)
             pos = (uint32_t)atomicAdd(&p.bcnt[bk], (unsigned long long)__popc(grp));
         pos = __shfl_sync(0xFFFFFFFFu, pos, leader) + __popc(grp & ((1u << lane) - 1u));
+        // and into its scan chunk (kScanChunk consecutive buckets of a frame)
+        const uint32_t ch = e.z * p.scan_chunks + ((e.y >> p.bucket_log2) / kScanChunk);
+        uint32_t cgrp = 1u << lane;
+        if (ok) cgrp = __match_any_sync(am, ch);
+        if (ok && lane == __ffs(cgrp) - 1) atomicAdd(&p.ctot[ch], (uint32_t)__popc(cgrp));
         if (ok) {
             *slot_seg(p, e.x) = segoff;
             p.occ[d] = e.x;

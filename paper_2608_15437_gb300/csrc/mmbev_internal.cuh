@@ -54,6 +54,10 @@ constexpr int kMaxClsGrid = 1000;
 // bucket with shared-memory bitmaps.
 constexpr int kBucketLog2Max = 13;
 
+// The scan of a frame's bucket counters runs in chunks of this many buckets,
+// one block each; the compact kernel counts voxels per chunk as well.
+constexpr uint32_t kScanChunk = 1024;
+
 // Bounded waits.
 constexpr uint32_t kSpinLimit = 1u << 22;
 
@@ -85,8 +89,9 @@ struct __align__(16) Header {
     uint32_t num_rec;      // kept points (records) of the call
     uint32_t num_nonempty; // non-empty buckets listed by the scan stage
     uint32_t seg_total;    // point entries reserved in seg
-    uint32_t num_heavy;    // kept voxels with more than 32 points
-    uint32_t pad[8];
+    uint32_t num_heavy;    // kept voxels with 33 .. 1024 points
+    uint32_t num_huge;     // kept voxels with more than 1024 points
+    uint32_t pad[7];
 };
 
 // Everything a kernel needs; passed by value.
@@ -143,6 +148,8 @@ struct Params {
     unsigned long long* bcnt;   // [B] voxels per bucket (every frame, no classes)
     unsigned long long* bcnt2;  // [B] capped frames: lo = rank-below, hi = rank-tie
     unsigned long long* boff;   // [B] exclusive offsets within the frame (lo, hi)
+    uint32_t* ctot;         // [F * scan_chunks] voxels per scan chunk (uncapped frames)
+    uint32_t scan_chunks;   // scan chunks per frame
     uint32_t* occ;          // [occ_cap] slot of each unique voxel
     uint32_t* d_bucket;     // [occ_cap]
     uint32_t* d_pos;        // [occ_cap] position inside the bucket
@@ -150,7 +157,8 @@ struct Params {
     uint2* items;           // [occ_cap] (slot, lin) grouped by bucket
     uint32_t* nonempty;     // [B] non-empty bucket ids
     uint32_t* vid_slot;     // [F*max_voxels] slot of each kept voxel, output order
-    uint32_t* heavy;        // [F*max_voxels] kept voxels with more than 32 points
+    uint32_t* heavy;        // [F*max_voxels] kept voxels with 33 .. 1024 points
+    uint32_t* huge;         // [F*max_voxels] kept voxels with more than 1024 points
     uint32_t occ_cap;
     uint32_t rec_cap;       // record positions of the call (regions * 32)
     // outputs

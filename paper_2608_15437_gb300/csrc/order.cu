@@ -26,7 +26,8 @@
 //   frames          (stage 4)  per frame: r*, q, kept count, output base,
 //                              item-segment base
 //   capped census   (stage 5)  per voxel of a capped frame: class, bucket count
-//   scan            (stage 6)  one block per frame: exclusive scan of counters
+//   scan            (stage 6)  one block per chunk of 1024 buckets of a frame:
+//                              exclusive scan of counters
 //   scatter         (stage 7)  voxel ids grouped by bucket
 //   rank            (stage 8)  per non-empty bucket: bitmaps, popcounts, output
 //                              position, coordinates
@@ -214,69 +215,76 @@ __global__ void __launch_bounds__(kThreads) k_capped_census(Params p) {
 
 // ---------------------------------------------------------------- stage 6
 // One block per frame: boff[b] = sum of the frame's counters before b.
-constexpr int kScanThreads = 1024;
-constexpr int kScanPer = 12;   // one pass covers 12,288 buckets (a 1440x1440x40 frame has 10,125)
+constexpr int kScanThreads = (int)kScanChunk;   // one bucket per thread
 
+// One block per (frame, chunk of kScanChunk buckets): the chunk's base is the
+// sum of the frame's earlier chunks (their voxel counts from the compact
+// kernel; capped frames sum their two-class counters instead), then a block
+// scan gives every bucket its exclusive offset within the frame, and the
+// chunk's non-empty buckets are appended to the list with one atomicAdd.
 __global__ void __launch_bounds__(kScanThreads) k_scan(Params p) {
     __shared__ unsigned long long s_wsum[kScanThreads / 32];
     __shared__ uint32_t s_nz[kScanThreads / 32];
+    __shared__ unsigned long long s_base;
     __shared__ uint32_t s_nzbase;
     pdl_wait();
     const int t = threadIdx.x, lane = t & 31, warp = t >> 5;
-    const uint32_t f = blockIdx.x;
+    const uint32_t C = p.scan_chunks;
+    const uint32_t f = blockIdx.x / C, c = blockIdx.x % C;
     const uint32_t Bf = p.buckets_per_frame;
     const size_t b0 = (size_t)f * Bf;
-    const unsigned long long* src = p.finfo[f].capped ? p.bcnt2 : p.bcnt;
-    unsigned long long carry = 0ull;
-    for (uint32_t c = 0; c < Bf; c += kScanThreads * kScanPer) {
-        const uint32_t i0 = c + (uint32_t)t * kScanPer;
-        unsigned long long v[kScanPer], tsum = 0ull;
-        uint32_t nz = 0;
+    const bool capped = p.finfo[f].capped != 0;
+    const unsigned long long* src = capped ? p.bcnt2 : p.bcnt;
+    // the chunk's base
+    unsigned long long part = 0ull;
+    if (!capped) {
+        for (uint32_t k = t; k < c; k += kScanThreads) part += ld_cg(&p.ctot[f * C + k]);
+    } else {
+        for (uint32_t k = t; k < c * kScanChunk; k += kScanThreads) part += src[b0 + k];
+    }
 #pragma unroll
-        for (int k = 0; k < kScanPer; ++k) {
-            v[k] = (i0 + k < Bf) ? src[b0 + i0 + k] : 0ull;
-            tsum += v[k];
-            nz += v[k] != 0ull;
-        }
-        unsigned long long inc = tsum;
-        uint32_t nzi = nz;
+    for (int o = 16; o > 0; o >>= 1) part += __shfl_xor_sync(0xFFFFFFFFu, part, o);
+    if (lane == 0) s_wsum[warp] = part;
+    __syncthreads();
+    if (t == 0) {
+        unsigned long long b = 0ull;
+        for (int w = 0; w < kScanThreads / 32; ++w) b += s_wsum[w];
+        s_base = b;
+    }
+    __syncthreads();
+    const uint32_t i = c * kScanChunk + (uint32_t)t;
+    const unsigned long long v = i < Bf ? src[b0 + i] : 0ull;
+    const uint32_t nz = v != 0ull;
+    unsigned long long inc = v;
+    uint32_t nzi = nz;
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) {
+        const unsigned long long x = __shfl_up_sync(0xFFFFFFFFu, inc, o);
+        const uint32_t y = __shfl_up_sync(0xFFFFFFFFu, nzi, o);
+        if (lane >= o) { inc += x; nzi += y; }
+    }
+    if (lane == 31) { s_wsum[warp] = inc; s_nz[warp] = nzi; }
+    __syncthreads();
+    if (warp == 0) {
+        unsigned long long w = s_wsum[lane];
+        uint32_t z = s_nz[lane];
 #pragma unroll
         for (int o = 1; o < 32; o <<= 1) {
-            const unsigned long long x = __shfl_up_sync(0xFFFFFFFFu, inc, o);
-            const uint32_t y = __shfl_up_sync(0xFFFFFFFFu, nzi, o);
-            if (lane >= o) { inc += x; nzi += y; }
+            const unsigned long long x = __shfl_up_sync(0xFFFFFFFFu, w, o);
+            const uint32_t y = __shfl_up_sync(0xFFFFFFFFu, z, o);
+            if (lane >= o) { w += x; z += y; }
         }
-        if (lane == 31) { s_wsum[warp] = inc; s_nz[warp] = nzi; }
-        __syncthreads();
-        if (warp == 0) {
-            unsigned long long w = s_wsum[lane];
-            uint32_t z = s_nz[lane];
-#pragma unroll
-            for (int o = 1; o < 32; o <<= 1) {
-                const unsigned long long x = __shfl_up_sync(0xFFFFFFFFu, w, o);
-                const uint32_t y = __shfl_up_sync(0xFFFFFFFFu, z, o);
-                if (lane >= o) { w += x; z += y; }
-            }
-            s_wsum[lane] = w;
-            s_nz[lane] = z;
-            if (lane == 31) s_nzbase = z ? atomicAdd(&p.hdr->num_nonempty, z) : 0u;
+        s_wsum[lane] = w;
+        s_nz[lane] = z;
+        if (lane == 31) s_nzbase = z ? atomicAdd(&p.hdr->num_nonempty, z) : 0u;
+    }
+    __syncthreads();
+    if (i < Bf) {
+        p.boff[b0 + i] = s_base + (warp > 0 ? s_wsum[warp - 1] : 0ull) + inc - v;
+        if (nz) {
+            const uint32_t zpos = s_nzbase + (warp > 0 ? s_nz[warp - 1] : 0u) + nzi - 1u;
+            if (zpos < p.num_buckets) p.nonempty[zpos] = (uint32_t)(b0 + i);
         }
-        __syncthreads();
-        unsigned long long run = carry + (warp > 0 ? s_wsum[warp - 1] : 0ull) + inc - tsum;
-        uint32_t zpos = s_nzbase + (warp > 0 ? s_nz[warp - 1] : 0u) + nzi - nz;
-#pragma unroll
-        for (int k = 0; k < kScanPer; ++k) {
-            if (i0 + k < Bf) {
-                p.boff[b0 + i0 + k] = run;
-                if (v[k] != 0ull) {
-                    if (zpos < p.num_buckets) p.nonempty[zpos] = (uint32_t)(b0 + i0 + k);
-                    ++zpos;
-                }
-            }
-            run += v[k];
-        }
-        carry += s_wsum[31];
-        __syncthreads();
     }
 }
 
@@ -419,7 +427,8 @@ cudaError_t launch_capped_census(const Params& p, int num_sms, bool pdl, cudaStr
 }
 
 cudaError_t launch_scan(const Params& p, bool pdl, cudaStream_t st) {
-    return launch_k(k_scan, dim3(p.num_frames), dim3(kScanThreads), 0, st, pdl, p);
+    return launch_k(k_scan, dim3(p.num_frames * p.scan_chunks), dim3(kScanThreads), 0, st, pdl,
+                    p);
 }
 
 cudaError_t launch_scatter(const Params& p, int num_sms, bool pdl, cudaStream_t st) {

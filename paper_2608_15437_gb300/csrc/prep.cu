@@ -123,6 +123,8 @@ k_prep(Params p, const __grid_constant__ HostDesc d) {
         for (size_t i = gt; i < (size_t)p.num_rois; i += gs) p.hist[i] = 0u;
     if (p.frame_u)
         for (size_t i = gt; i < (size_t)p.num_frames; i += gs) p.frame_u[i] = 0u;
+    if (p.ctot)
+        for (size_t i = gt; i < (size_t)p.num_frames * p.scan_chunks; i += gs) p.ctot[i] = 0u;
     if (p.cls_cnt)  // a classify block that gives up leaves its list empty
         for (size_t i = gt; i < (size_t)kMaxClsGrid; i += gs) p.cls_cnt[i] = 0u;
     if (p.bcnt) {
