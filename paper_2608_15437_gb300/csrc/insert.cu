@@ -190,7 +190,7 @@ __global__ void __launch_bounds__(kThreads) k_compact(Params p) {
     const uint32_t n = min(p.blockcount[b], p.ins_cap);
     if (n == 0) return;
     if (t < kFrameWin) s_fcnt[t] = 0;
-    // this tile's place in the occupied-voxel list (order is immaterial)
+    // this block's place in the occupied-voxel list (order is immaterial)
     if (t == 0) {
         s_fmin = sub[0].z;
         s_base = atomicAdd(&p.hdr->num_occ, n);

@@ -2,8 +2,9 @@
 //
 // Data layout (one call):
 //   points      caller's float32 [N][5] AoS, streamed once by the classify
-//               kernel through a 3-stage ring of 40 KB shared-memory tiles,
-//               each tile moved by eight 5 KB cp.async.bulk (TMA) copies.
+//               kernel through a ring of (up to four) 40 KB shared-memory
+//               tiles, each tile moved by eight 5 KB cp.async.bulk (TMA)
+//               copies.
 //   records     workspace, 32 B per kept point, at position region*32 + (its
 //               rank among the kept points of its 32-point region):
 //               {x', y', z', intensity} {dt, ROI rank, -, -}. Region g holds

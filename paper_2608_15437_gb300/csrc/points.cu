@@ -7,7 +7,8 @@
 // GB300 a single 40 KB bulk copy per tile streams at about a quarter of HBM
 // bandwidth, eight concurrent ones at nearly all of it. The warps never wait
 // for each other: each warp classifies its own 64 points of a tile, and the
-// last warp to finish a tile (a shared-memory counter) refills that buffer.
+// last warp to have read its points from a buffer (a shared-memory counter)
+// refills it with the tile one ring length ahead.
 // Per point: Eq. 6 motion compensation, range crop, Alg. 1 inside-ROI test
 // (coarse candidate mask, then the exact rotated-box test in rank order;
 // the first hit is the point's rank) and the voxel index. The masks and
