@@ -55,12 +55,16 @@ def _load():
         i32, i64, f32 = ctypes.c_int32, ctypes.c_int64, ctypes.c_float
         lib.oracle_classify.argtypes = [P, P, i32, P, P, i32, f32, P, P, P, P, P]
         lib.oracle_classify.restype = ctypes.c_int
+        u64 = ctypes.c_uint64
         lib.oracle_voxelize_roi.argtypes = [P, P, i32, P, P, i32, f32, P, P,
-                                            i32, i32, P, P, P, P]
+                                            i32, i32, f32, u64, P, P, P, P]
         lib.oracle_voxelize_roi.restype = ctypes.c_int
         lib.oracle_voxelize_roi_batched.argtypes = [P, P, i32, P, P, i32, f32, P, P,
-                                                    i32, i32, i32, P, P, P, P, P, P]
+                                                    i32, i32, f32, u64, i32, P, P, P, P,
+                                                    P, P]
         lib.oracle_voxelize_roi_batched.restype = ctypes.c_int
+        lib.oracle_splitmix64.argtypes = [u64, u64]
+        lib.oracle_splitmix64.restype = u64
         _lib = lib
     return _lib
 
@@ -95,9 +99,16 @@ def classify(points, sweep_offsets, sweep_tf, rois, roi_margin, voxel_size, pc_r
     return xyz, lin, rank
 
 
+def splitmix64(seed, n):
+    """The n-th output (n >= 1) of the SplitMix64 stream seeded with `seed`."""
+    return int(_load().oracle_splitmix64(int(seed) & (2**64 - 1), int(n) & (2**64 - 1)))
+
+
 def voxelize_roi(points, sweep_offsets, sweep_tf, rois, roi_margin, voxel_size,
-                 pc_range, max_pts_per_voxel, max_voxels):
-    """One frame. Returns (feats [nvox,5], coords [nvox,3] (z,y,x), counts [nvox])."""
+                 pc_range, max_pts_per_voxel, max_voxels, rho_out=0.0, seed=0):
+    """One frame. Returns (feats [nvox,5], coords [nvox,3] (z,y,x), counts [nvox]).
+    rho_out: keep probability of points inside no ROI (Alg. 1), drawn from
+    SplitMix64(seed) per frame-local point index."""
     lib = _load()
     points = _c(points, np.float32).reshape(-1, 5)
     so = _c(sweep_offsets, np.int64)
@@ -112,7 +123,8 @@ def voxelize_roi(points, sweep_offsets, sweep_tf, rois, roi_margin, voxel_size,
     nvox = np.zeros(1, np.int32)
     rc = lib.oracle_voxelize_roi(_ptr(points), _ptr(so), len(so) - 1, _ptr(tf), _ptr(rois),
                                  rois.shape[0], float(roi_margin), _ptr(vs), _ptr(rg),
-                                 int(max_pts_per_voxel), mv, _ptr(feats), _ptr(coords),
+                                 int(max_pts_per_voxel), mv, float(rho_out),
+                                 int(seed) & (2**64 - 1), _ptr(feats), _ptr(coords),
                                  _ptr(counts), _ptr(nvox))
     if rc != 0:
         raise ValueError(f"oracle_voxelize_roi failed with status {rc}")
@@ -122,7 +134,7 @@ def voxelize_roi(points, sweep_offsets, sweep_tf, rois, roi_margin, voxel_size,
 
 def voxelize_roi_batched(points, sweep_offsets, sweep_tf, rois, roi_margin, voxel_size,
                          pc_range, max_pts_per_voxel, max_voxels, frame_sweep_offsets,
-                         frame_roi_offsets):
+                         frame_roi_offsets, rho_out=0.0, seed=0):
     """Independent frames in one call. Returns a list of per-frame
     (feats, coords, counts) tuples."""
     lib = _load()
@@ -143,7 +155,8 @@ def voxelize_roi_batched(points, sweep_offsets, sweep_tf, rois, roi_margin, voxe
     nvox = np.zeros(max(nf, 1), np.int32)
     rc = lib.oracle_voxelize_roi_batched(
         _ptr(points), _ptr(so), len(so) - 1, _ptr(tf), _ptr(rois), rois.shape[0],
-        float(roi_margin), _ptr(vs), _ptr(rg), int(max_pts_per_voxel), mv, nf,
+        float(roi_margin), _ptr(vs), _ptr(rg), int(max_pts_per_voxel), mv, float(rho_out),
+        int(seed) & (2**64 - 1), nf,
         _ptr(fso), _ptr(fro), _ptr(feats), _ptr(coords), _ptr(counts), _ptr(nvox))
     if rc != 0:
         raise ValueError(f"oracle_voxelize_roi_batched failed with status {rc}")

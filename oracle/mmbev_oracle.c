@@ -20,8 +20,13 @@
  *   3. Alg. 1 (inside-any-box test) with the boxes of Eq. 1: a point is kept
  *      when it lies inside some ROI box, the box grown by the margin r on each
  *      half-extent. The ROIs arrive in criticality order (Sec. IV-C); the
- *      point's rank is the index of the first box that contains it. The
- *      out-of-ROI keep probability of Alg. 1 is taken as zero.
+ *      point's rank is the index of the first box that contains it. A point
+ *      inside no box is kept with probability rho_out (Alg. 1), decided by
+ *      one draw of a counter-based generator: SplitMix64 (Steele, Lea and
+ *      Flood, OOPSLA 2014) seeded with `seed`, its (j+1)-th output for the
+ *      frame's j-th point; the point is kept when the top 24 bits of that
+ *      output are below floor(rho_out * 2^24). Such a background point has
+ *      rank R (the frame's ROI count): below every ROI in criticality.
  *   4. Hard voxelization (Sec. IV-F): voxel c = floor((p' - min) / size) per
  *      axis, dropped when c >= n; linear index lin = (cz*ny + cy)*nx + cx.
  *      Each voxel keeps the K points with the smallest input index. When more
@@ -60,6 +65,28 @@ typedef struct {
     int64_t n;
     int32_t minrank;
 } voxel_t;
+
+/* SplitMix64: the n-th output (n >= 1) of the stream that starts at state
+ * `seed` is the finalizer applied to seed + n * 0x9E3779B97F4A7C15. */
+static uint64_t splitmix64_nth(uint64_t seed, uint64_t n)
+{
+    uint64_t z = seed + n * 0x9E3779B97F4A7C15ull;
+    z = (z ^ (z >> 30)) * 0xBF58476D1CE4E5B9ull;
+    z = (z ^ (z >> 27)) * 0x94D049BB133111EBull;
+    return z ^ (z >> 31);
+}
+
+/* Exposed for the pins: the n-th output of the stream seeded with `seed`. */
+uint64_t oracle_splitmix64(uint64_t seed, uint64_t n) { return splitmix64_nth(seed, n); }
+
+/* floor(rho * 2^24) for rho in [0, 1], the keep threshold of a draw's top
+ * 24 bits. */
+static uint32_t keep_threshold(float rho)
+{
+    if (!(rho > 0.0f)) return 0u;
+    if (rho >= 1.0f) return 1u << 24;
+    return (uint32_t)floor((double)rho * 16777216.0);
+}
 
 /* Grid extent along one axis: round((max - min) / size) in double. */
 static int64_t grid_dim(float lo, float hi, float size)
@@ -182,6 +209,7 @@ int oracle_voxelize_roi(const float *points, const int64_t *sweep_offsets,
                         const oracle_roi_t *rois, int32_t num_rois, float margin,
                         const float voxel_size[3], const float range[6],
                         int32_t max_pts_per_voxel, int32_t max_voxels,
+                        float rho_out, uint64_t seed,
                         float *out_feats, int32_t *out_coords,
                         int32_t *out_counts, int32_t *out_nvox)
 {
@@ -190,6 +218,8 @@ int oracle_voxelize_roi(const float *points, const int64_t *sweep_offsets,
         return ORACLE_EINVAL;
     if (validate_grid(voxel_size, range, dims) != ORACLE_OK) return ORACLE_EINVAL;
     if (!(margin >= 0.0f)) return ORACLE_EINVAL;
+    if (!(rho_out >= 0.0f && rho_out <= 1.0f)) return ORACLE_EINVAL;
+    const uint32_t thr = keep_threshold(rho_out);
 
     int64_t first = num_sweeps > 0 ? sweep_offsets[0] : 0;
     int64_t last = num_sweeps > 0 ? sweep_offsets[num_sweeps] : 0;
@@ -212,7 +242,12 @@ int oracle_voxelize_roi(const float *points, const int64_t *sweep_offsets,
             for (int32_t r = 0; r < num_rois; ++r) {
                 if (inside_roi(&rois[r], margin, x, y)) { rank = r; break; }
             }
-            if (rank < 0) continue;
+            if (rank < 0) {
+                /* outside every ROI: kept with probability rho_out */
+                const uint64_t j = (uint64_t)(i - first);
+                if (thr == 0u || (uint32_t)(splitmix64_nth(seed, j + 1) >> 40) >= thr) continue;
+                rank = num_rois;
+            }
             int64_t cx = (int64_t)floorf((x - range[0]) / voxel_size[0]);
             int64_t cy = (int64_t)floorf((y - range[1]) / voxel_size[1]);
             int64_t cz = (int64_t)floorf((z - range[2]) / voxel_size[2]);
@@ -279,14 +314,16 @@ int oracle_voxelize_roi(const float *points, const int64_t *sweep_offsets,
 }
 
 /* Batched form: num_frames independent frames, each an oracle_voxelize_roi
- * call on its own sweeps and ROIs; frame f writes rows starting at
+ * call on its own sweeps and ROIs (the draws use frame-local point indices,
+ * so a batch equals its frames run alone); frame f writes rows starting at
  * f*max_voxels and out_nvox[f]. */
 int oracle_voxelize_roi_batched(const float *points, const int64_t *sweep_offsets,
                                 int32_t num_sweeps, const float *sweep_tf,
                                 const oracle_roi_t *rois, int32_t num_rois,
                                 float margin, const float voxel_size[3],
                                 const float range[6], int32_t max_pts_per_voxel,
-                                int32_t max_voxels, int32_t num_frames,
+                                int32_t max_voxels, float rho_out, uint64_t seed,
+                                int32_t num_frames,
                                 const int32_t *frame_sweep_offsets,
                                 const int32_t *frame_roi_offsets,
                                 float *out_feats, int32_t *out_coords,
@@ -304,7 +341,7 @@ int oracle_voxelize_roi_batched(const float *points, const int64_t *sweep_offset
         int rc = oracle_voxelize_roi(points, sweep_offsets + s0, s1 - s0,
                                      sweep_tf + 16 * (int64_t)s0, rois + r0, r1 - r0,
                                      margin, voxel_size, range, max_pts_per_voxel,
-                                     max_voxels, out_feats + 5 * row,
+                                     max_voxels, rho_out, seed, out_feats + 5 * row,
                                      out_coords + 3 * row, out_counts + row,
                                      out_nvox + f);
         if (rc != ORACLE_OK) return rc;

@@ -575,3 +575,84 @@ def test_tiny_matches_stored_oracle_output(oracle_mod):
     assert c.tolist() == g["coords"]
     assert n.tolist() == g["counts"]
     assert [[float.hex(float(v)) for v in row] for row in f] == g["feats_hex"]
+
+
+# ------------------------------------------------------------------ rho_out (Alg. 1)
+
+def _vox(oracle_mod, w, rho_out=0.0, seed=0, max_pts_per_voxel=None, max_voxels=None):
+    return oracle_mod.voxelize_roi(
+        w.points, w.sweep_offsets, w.sweep_tf, w.rois, w.roi_margin, w.voxel_size, w.pc_range,
+        w.max_pts_per_voxel if max_pts_per_voxel is None else max_pts_per_voxel,
+        w.max_voxels if max_voxels is None else max_voxels, rho_out=rho_out, seed=seed)
+
+
+def test_splitmix64_matches_the_published_stream(oracle_mod):
+    # pins the counter-based generator that decides out-of-ROI keeps
+    ref = json.load(open(os.path.join(GOLDEN, "splitmix64_seed0.json")))
+    got = [oracle_mod.splitmix64(ref["seed"], n + 1) for n in range(len(ref["outputs"]))]
+    assert got == [int(h, 16) for h in ref["outputs"]]
+
+
+def _frame_without_rois():
+    w = synth.nuscenes_frame(1)
+    return w.with_rois(np.zeros((0, 5), np.float32))
+
+
+def test_rho_zero_keeps_only_roi_points(oracle_mod):
+    w = synth.nuscenes_frame(1)
+    a = _vox(oracle_mod, w)
+    b = _vox(oracle_mod, w, rho_out=0.0, seed=99)
+    for x, y in zip(a, b):
+        assert np.array_equal(x.view(np.uint32), y.view(np.uint32))
+
+
+def test_rho_one_is_dense_voxelization(oracle_mod):
+    # every in-range point kept: the same output as one box covering the range
+    w = _frame_without_rois()
+    dense = synth.roi_coverage("full")
+    got = _vox(oracle_mod, w, rho_out=1.0, seed=5)
+    want = _vox(oracle_mod, dense)
+    for x, y in zip(got, want):
+        assert np.array_equal(x.view(np.uint32), y.view(np.uint32))
+
+
+def test_rho_below_one_draw_keeps_nothing(oracle_mod):
+    # floor(rho * 2^24) = 0: no draw can pass
+    w = _frame_without_rois()
+    f, c, n = _vox(oracle_mod, w, rho_out=1e-9, seed=5)
+    assert len(c) == 0
+
+
+def test_background_keep_fraction_follows_rho(oracle_mod):
+    w = _frame_without_rois()
+    dense = synth.roi_coverage("full")
+    big = dict(max_pts_per_voxel=1 << 20, max_voxels=1 << 20)
+    in_range = int(_vox(oracle_mod, dense, **big)[2].sum())
+    for rho in (0.1, 0.5):
+        kept = int(_vox(oracle_mod, w, rho_out=rho, seed=11, **big)[2].sum())
+        sd = np.sqrt(in_range * rho * (1 - rho))
+        assert abs(kept - rho * in_range) < 5 * sd, (rho, kept, in_range)
+
+
+def test_background_voxels_rank_below_every_roi(oracle_mod):
+    # capped to the voxels that hold an ROI point, rho = 1 keeps exactly them
+    w = synth.nuscenes_frame(1)
+    roi_only = _vox(oracle_mod, w)
+    u = len(roi_only[1])
+    got = _vox(oracle_mod, w, rho_out=1.0, seed=3, max_voxels=u)
+    assert np.array_equal(got[1], roi_only[1])
+    full = _vox(oracle_mod, w, rho_out=1.0, seed=3)
+    assert len(full[1]) > u
+
+
+def test_draws_use_frame_local_indices(oracle_mod):
+    frames = [synth.nuscenes_frame(s) for s in (1, 2)]
+    b = synth.concat_frames(frames, "two")
+    out = oracle_mod.voxelize_roi_batched(
+        b.points, b.sweep_offsets, b.sweep_tf, b.rois, b.roi_margin, b.voxel_size, b.pc_range,
+        b.max_pts_per_voxel, b.max_voxels, b.frame_sweep_offsets, b.frame_roi_offsets,
+        rho_out=0.25, seed=17)
+    for fw, got in zip(frames, out):
+        want = _vox(oracle_mod, fw, rho_out=0.25, seed=17)
+        for x, y in zip(got, want):
+            assert np.array_equal(x.view(np.uint32), y.view(np.uint32))
