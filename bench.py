@@ -260,7 +260,8 @@ def run_gpu(args):
     rois = torch.from_numpy(w.rois).to(dev)
     rmax = int(np.max(np.diff(w.frame_roi_offsets)))
     vx = mmbev.Voxelizer(w.num_points, rmax, w.max_voxels, w.num_frames, w.voxel_size,
-                         w.pc_range, w.max_pts_per_voxel, w.roi_margin, device=dev)
+                         w.pc_range, w.max_pts_per_voxel, w.roi_margin, device=dev,
+                         rho_out=args.rho_out, seed=args.seed)
     # the metric's numerator: in-ROI points, counted by the library's own
     # per-point classification of these inputs (S1-S2), once, untimed
     _, lin, _ = mmbev.classify_points(pts, w.sweep_offsets, tf, rois, w.roi_margin, w.voxel_size,
@@ -386,6 +387,7 @@ def run_gpu(args):
             "data": "synthetic", "config": workload_desc(w),
             "us_per_frame": 1e3 * ms_step / w.num_frames,
             "in_roi_points_per_gpu": n_in_roi, "voxels_out_per_gpu": u_out,
+            "rho_out": args.rho_out,
             "path_hbm_gbs": path_bytes / (ms_step * 1e-3) / 1e9,
             "path_frac_of_peak": path_bytes / (ms_step * 1e-3) / 1e9 / peak,
             "stage_us": {n: round(1e3 * t, 2) for n, t in zip(names, stage_ms)},
@@ -416,6 +418,10 @@ def main():
     ap.add_argument("--steps", type=int, default=1000)
     ap.add_argument("--warmup", type=int, default=10)
     ap.add_argument("--impl", default="gb300", choices=["gb300", "reference"])
+    ap.add_argument("--rho-out", type=float, default=0.0,
+                    help="keep probability of points inside no ROI (Alg. 1); the headline "
+                         "workload uses 0")
+    ap.add_argument("--seed", type=int, default=0, help="seed of the rho_out draws")
     ap.add_argument("--frames", type=int, default=FRAMES,
                     help="frames per GPU (the headline workload is 32; fewer for small "
                          "profiling cases)")

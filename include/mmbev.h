@@ -214,11 +214,24 @@ int mmbev_get_status(const void *workspace, size_t workspace_bytes,
  *                     instead of the power of two >= 1.25 x the call's kept
  *                     points (at most table_bytes / 16; a full table sets
  *                     MMBEV_DEV_TABLE_FULL).
+ *   rho_out           keep probability, in [0, 1], of an in-range point inside
+ *                     no ROI (Alg. 1; the other entry points use 0). The draw
+ *                     for the j-th point of a frame (0-based, within that
+ *                     frame) is the (j+1)-th output of SplitMix64 (Steele,
+ *                     Lea and Flood, OOPSLA 2014) seeded with `seed`; the
+ *                     point is kept when the output's top 24 bits are below
+ *                     floor(rho_out * 2^24). A kept background point has rank
+ *                     R_f (the frame's ROI count), below every ROI, so the
+ *                     voxel cap drops background-only voxels first.
+ *                     Outside [0, 1] or NaN: MMBEV_EINVAL.
+ *   seed              the generator's seed.
  */
 #define MMBEV_NUM_STAGES 13
 typedef struct mmbev_exec_opts {
     cudaEvent_t *stage_events;
     int32_t table_log2_override;
+    float rho_out;
+    uint64_t seed;
 } mmbev_exec_opts_t;
 
 int mmbev_voxelize_roi_batched_ex(const float *points, const int64_t *sweep_offsets,

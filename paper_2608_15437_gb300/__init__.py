@@ -35,7 +35,8 @@ class MMBEVError(RuntimeError):
 
 
 class _ExecOpts(ctypes.Structure):
-    _fields_ = [("stage_events", ctypes.c_void_p), ("table_log2_override", ctypes.c_int32)]
+    _fields_ = [("stage_events", ctypes.c_void_p), ("table_log2_override", ctypes.c_int32),
+                ("rho_out", ctypes.c_float), ("seed", ctypes.c_uint64)]
 
 
 def load():
@@ -194,14 +195,17 @@ def voxelize_roi_batched(points: torch.Tensor, sweep_offsets, sweep_tf: torch.Te
                          max_pts_per_voxel: int, max_voxels: int, frame_sweep_offsets,
                          frame_roi_offsets, *, table: torch.Tensor, workspace: torch.Tensor,
                          out: Outputs | None = None, stream=None, stage_events=None,
-                         table_log2_override: int = 0) -> Outputs:
+                         table_log2_override: int = 0, rho_out: float = 0.0,
+                         seed: int = 0) -> Outputs:
     """Voxelize F independent frames in one call (``mmbev_voxelize_roi_batched``).
 
     points [N,5] float32, sweep_tf [S,16] float32 and rois [R,5] float32 live
     on the device; sweep_offsets [S+1], frame_sweep_offsets [F+1] and
     frame_roi_offsets [F+1] are host arrays. ``stage_events``, a list of
     NUM_STAGES + 1 ``torch.cuda.Event(enable_timing=True)`` already recorded
-    once, brackets each kernel of the call.
+    once, brackets each kernel of the call. ``rho_out`` keeps points inside
+    no ROI with that probability (SplitMix64 draws keyed by ``seed`` and the
+    point's index within its frame).
     """
     lib = load()
     so = _host(sweep_offsets, np.int64)
@@ -219,10 +223,11 @@ def voxelize_roi_batched(points: torch.Tensor, sweep_offsets, sweep_tf: torch.Te
             _dptr(out.feats), _dptr(out.coords), _dptr(out.counts), _dptr(out.nvox),
             _dptr(table, torch.uint8, "table"), table.numel(),
             _dptr(workspace, torch.uint8, "workspace"), workspace.numel(), _stream(stream)]
-    if stage_events is None and not table_log2_override:
+    if stage_events is None and not table_log2_override and not rho_out:
         rc = lib.mmbev_voxelize_roi_batched(*args)
     else:
-        opts = _ExecOpts(None, int(table_log2_override))
+        opts = _ExecOpts(None, int(table_log2_override), float(rho_out),
+                         int(seed) & (2**64 - 1))
         if stage_events is not None:
             assert len(stage_events) == NUM_STAGES + 1
             arr = (ctypes.c_void_p * len(stage_events))(*[e.cuda_event for e in stage_events])
@@ -310,7 +315,9 @@ class Voxelizer:
     batched entry point on device tensors."""
 
     def __init__(self, max_points, max_rois_per_frame, max_voxels, num_frames, voxel_size,
-                 pc_range, max_pts_per_voxel, roi_margin, device="cuda"):
+                 pc_range, max_pts_per_voxel, roi_margin, device="cuda", rho_out=0.0, seed=0):
+        self.rho_out = float(rho_out)
+        self.seed = int(seed)
         self.voxel_size = _host(voxel_size, np.float32)
         self.pc_range = _host(pc_range, np.float32)
         self.max_voxels = int(max_voxels)
@@ -328,7 +335,8 @@ class Voxelizer:
                                     self.voxel_size, self.pc_range, self.K, self.max_voxels,
                                     frame_sweep_offsets, frame_roi_offsets, table=self.table,
                                     workspace=self.workspace, out=self.out, stream=stream,
-                                    stage_events=stage_events)
+                                    stage_events=stage_events, rho_out=self.rho_out,
+                                    seed=self.seed)
 
     def status(self) -> int:
         return get_status(self.workspace)

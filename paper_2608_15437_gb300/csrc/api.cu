@@ -92,7 +92,7 @@ Layout make_layout(int64_t max_points, int64_t rois_total, int32_t max_rois_fram
     L.fro = take(sizeof(int32_t) * (F + 1));
     L.roi_prep = take(sizeof(RoiPrep) * R);
     L.masks = take(sizeof(uint32_t) * F * L.coarse * L.coarse * L.mask_words);
-    L.hist = take(sizeof(uint32_t) * R);
+    L.hist = take(sizeof(uint32_t) * (R + F));
     L.frame_u = take(sizeof(uint32_t) * F);
     L.finfo = take(sizeof(FrameInfo) * F);
     L.records = take(32 * TS);
@@ -320,6 +320,15 @@ int mmbev_voxelize_roi_batched_ex(const float* points, const int64_t* sweep_offs
     while (lg < 31 && (2ull << lg) <= fit) ++lg;
     if ((1ull << lg) > fit) return MMBEV_EWORKSPACE;
     p.table_log2_fixed = 0;
+    p.rho_thr = 0u;
+    p.seed = 0ull;
+    if (opts) {
+        const float rho = opts->rho_out;
+        if (!(rho >= 0.0f && rho <= 1.0f)) return MMBEV_EINVAL;
+        // floor(rho * 2^24); rho = 1 keeps every draw
+        p.rho_thr = rho >= 1.0f ? (1u << 24) : (uint32_t)std::floor((double)rho * 16777216.0);
+        p.seed = opts->seed;
+    }
     if (opts && opts->table_log2_override > 0) {
         if (opts->table_log2_override > (int32_t)lg) return MMBEV_EWORKSPACE;
         p.table_log2_fixed = opts->table_log2_override;

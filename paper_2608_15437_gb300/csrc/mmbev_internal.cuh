@@ -116,6 +116,8 @@ struct Params {
     uint32_t cells;         // nx*ny*nz
     int32_t K;
     int32_t max_voxels;
+    uint32_t rho_thr;       // keep a point inside no ROI when its draw's top 24 bits < rho_thr
+    uint64_t seed;          // SplitMix64 seed of those draws
     // bucket ordering
     int32_t bucket_log2;
     uint32_t buckets_per_frame;
@@ -132,7 +134,7 @@ struct Params {
     int32_t* frame_roi_off;    // [F+1]
     RoiPrep* roi_prep;      // [R]
     uint32_t* masks;        // [F][coarse^2][mask_words]
-    uint32_t* hist;         // [R] voxels per minimum rank (capped frames)
+    uint32_t* hist;         // [R + F] voxels per minimum rank 0 .. R_f (capped frames)
     uint32_t* frame_u;      // [F] unique voxels per frame
     FrameInfo* finfo;       // [F]
     uint4* records;         // [regions*32][2] kept points' features and rank
@@ -306,6 +308,15 @@ __device__ __forceinline__ uint32_t* slot_seg(const Params& p, uint32_t h) {
 
 __device__ __forceinline__ void zero_slot(const Params& p, uint32_t h) {
     *reinterpret_cast<uint4*>(p.table + (size_t)h * kSlotBytes) = make_uint4(0u, 0u, 0u, 0u);
+}
+
+// The n-th output (n >= 1) of SplitMix64 (Steele, Lea and Flood, OOPSLA
+// 2014) started at state `seed`: the finalizer of seed + n * golden gamma.
+__device__ __forceinline__ uint64_t splitmix64_nth(uint64_t seed, uint64_t n) {
+    uint64_t z = seed + n * 0x9E3779B97F4A7C15ull;
+    z = (z ^ (z >> 30)) * 0xBF58476D1CE4E5B9ull;
+    z = (z ^ (z >> 27)) * 0x94D049BB133111EBull;
+    return z ^ (z >> 31);
 }
 
 // 64-bit mixer (the SplitMix64 finalizer of Steele, Lea and Flood, 2014).

@@ -57,8 +57,10 @@ __global__ void __launch_bounds__(kThreads) k_capped_hist(Params p) {
     for (uint32_t d = blockIdx.x * blockDim.x + threadIdx.x; d < U; d += gs) {
         const uint32_t f = p.d_bucket[d] / p.buckets_per_frame;
         if (ld_cg(&p.frame_u[f]) <= (uint32_t)p.max_voxels) continue;
-        const uint32_t r = slot_minrank(p, p.occ[d]);
-        atomicAdd(&p.hist[p.frame_roi_off[f] + r], 1u);
+        const int r0 = p.frame_roi_off[f];
+        const uint32_t rn = (uint32_t)(p.frame_roi_off[f + 1] - r0);  // background rank
+        const uint32_t r = min(slot_minrank(p, p.occ[d]), rn);
+        atomicAdd(&p.hist[r0 + f + r], 1u);
     }
 }
 
@@ -84,8 +86,9 @@ __global__ void __launch_bounds__(1024) k_frames(Params p) {
         } else {
             fi.capped = 1;
             fi.nvox = maxv;
-            const int r0 = p.frame_roi_off[f];
-            const int rn = p.frame_roi_off[f + 1] - r0;
+            // ranks 0 .. R_f (R_f: points kept outside every ROI)
+            const int r0 = p.frame_roi_off[f] + f;
+            const int rn = p.frame_roi_off[f + 1] - p.frame_roi_off[f] + 1;
             uint32_t run = 0;  // voxels with a rank below this chunk
             fi.rstar = (uint32_t)rn;
             fi.q = 0;

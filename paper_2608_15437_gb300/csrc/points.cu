@@ -11,7 +11,8 @@
 // refills it with the tile one ring length ahead.
 // Per point: Eq. 6 motion compensation, range crop, Alg. 1 inside-ROI test
 // (coarse candidate mask, then the exact rotated-box test in rank order;
-// the first hit is the point's rank) and the voxel index. The masks and
+// the first hit is the point's rank; a point inside no ROI is kept with
+// probability rho_out and rank R_f) and the voxel index. The masks and
 // prepared ROIs of the (one or two) frames a block's tile range starts with
 // sit in shared memory. Kept points are compacted per 32-point region with
 // warp ballots, in input order: position (region)*32 + (rank among the
@@ -312,6 +313,18 @@ __global__ void __launch_bounds__(kThreads, 1) k_classify(Params p, int rmax, in
                 for (int k = 0; k < 2; ++k)
                     if (((m[k] >> b) & 1u) && hit[k] < 0 && roi_hit(cr[k], w * 32 + b, x[k], y[k]))
                         hit[k] = w * 32 + b;
+            }
+        }
+        // Alg. 1: an in-range point inside no ROI is kept with probability
+        // rho_out (a SplitMix64 draw keyed by its index within the frame)
+        if (p.rho_thr) {
+#pragma unroll
+            for (int k = 0; k < 2; ++k) {
+                if (hit[k] >= 0 || !cm[k]) continue;
+                const uint32_t f = frk[k];
+                const int64_t j = base + j0 + k - sm.soff[p.frame_sweep_off[f]];
+                if ((uint32_t)(splitmix64_nth(p.seed, (uint64_t)j + 1ull) >> 40) < p.rho_thr)
+                    hit[k] = p.frame_roi_off[f + 1] - p.frame_roi_off[f];  // rank R_f
             }
         }
 #pragma unroll

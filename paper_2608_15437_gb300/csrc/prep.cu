@@ -120,7 +120,7 @@ k_prep(Params p, const __grid_constant__ HostDesc d) {
         p.sweep_frame[s] = lo;
     }
     if (p.hist)
-        for (size_t i = gt; i < (size_t)p.num_rois; i += gs) p.hist[i] = 0u;
+        for (size_t i = gt; i < (size_t)p.num_rois + p.num_frames; i += gs) p.hist[i] = 0u;
     if (p.frame_u)
         for (size_t i = gt; i < (size_t)p.num_frames; i += gs) p.frame_u[i] = 0u;
     if (p.ctot)

@@ -17,7 +17,7 @@ def to_dev(w, dev, rois=None):
 
 
 def run_gpu(mmbev, w, dev, K=None, maxv=None, table_log2_override=0, table=None, workspace=None,
-            stream=None):
+            stream=None, rho_out=0.0, seed=0):
     """Batched C-ABI call on w; returns (per-frame list of (feats, coords,
     counts), device status, table, workspace)."""
     import torch
@@ -34,7 +34,8 @@ def run_gpu(mmbev, w, dev, K=None, maxv=None, table_log2_override=0, table=None,
     out = mmbev.voxelize_roi_batched(pts, w.sweep_offsets, tf, rois, w.roi_margin, w.voxel_size,
                                      w.pc_range, K, maxv, w.frame_sweep_offsets,
                                      w.frame_roi_offsets, table=table, workspace=workspace,
-                                     table_log2_override=table_log2_override, stream=stream)
+                                     table_log2_override=table_log2_override, stream=stream,
+                                     rho_out=rho_out, seed=seed)
     torch.cuda.synchronize(dev)
     status = mmbev.get_status(workspace)
     nvox = out.nvox.cpu().numpy()
@@ -42,12 +43,12 @@ def run_gpu(mmbev, w, dev, K=None, maxv=None, table_log2_override=0, table=None,
     return frames, status, table, workspace
 
 
-def run_oracle(oracle, w, K=None, maxv=None):
+def run_oracle(oracle, w, K=None, maxv=None, rho_out=0.0, seed=0):
     K = w.max_pts_per_voxel if K is None else K
     maxv = w.max_voxels if maxv is None else maxv
     return oracle.voxelize_roi_batched(w.points, w.sweep_offsets, w.sweep_tf, w.rois, w.roi_margin,
                                        w.voxel_size, w.pc_range, K, maxv, w.frame_sweep_offsets,
-                                       w.frame_roi_offsets)
+                                       w.frame_roi_offsets, rho_out=rho_out, seed=seed)
 
 
 def assert_frames_equal(got, want, label=""):

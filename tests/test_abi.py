@@ -84,3 +84,20 @@ def test_small_buffers_are_rejected_before_launch(mmbev_lib):
     lib = mmbev_lib.load()
     assert _call(lib, ws_bytes=1024) == -3
     assert _call(lib, table_bytes=16 * 100) == -3   # fewer than 2N slots
+
+
+@pytest.mark.parametrize("rho", [-0.1, 1.5, float("nan")])
+def test_rho_out_outside_unit_interval_is_rejected(mmbev_lib, rho):
+    lib = mmbev_lib.load()
+    so = np.asarray((0, 100), np.int64)
+    fso = np.asarray([0, 1], np.int32)
+    fro = np.asarray([0, 1], np.int32)
+    P = ctypes.c_void_p
+    fake = P(0x7e0000000000)
+    opts = mmbev_lib._ExecOpts(None, 0, rho, 1)
+    rc = lib.mmbev_voxelize_roi_batched_ex(
+        fake, so.ctypes.data_as(P), 1, fake, fake, 1, 0.5, TINY_VS.ctypes.data_as(P),
+        TINY_RG.ctypes.data_as(P), 10, 100, 1, fso.ctypes.data_as(P), fro.ctypes.data_as(P),
+        fake, fake, fake, fake, P(0x7f1000000000), 1 << 30, P(0x7f0000000000), 1 << 30, None,
+        ctypes.byref(opts))
+    assert rc == -1

@@ -346,3 +346,49 @@ def test_workspace_too_small_is_rejected(mmbev_lib, cuda_dev):
         mmbev_lib.voxelize_roi_batched(pts, w.sweep_offsets, tf, rois, 0.5, w.voxel_size,
                                        w.pc_range, 10, 16000, w.frame_sweep_offsets,
                                        w.frame_roi_offsets, table=table, workspace=ws)
+
+
+# ------------------------------------------------------------------ rho_out (Alg. 1)
+
+@pytest.mark.gpu
+@pytest.mark.parametrize("rho", [0.1, 0.5, 1.0])
+def test_rho_out_parity(oracle_mod, mmbev_lib, cuda_dev, rho):
+    # points inside no ROI kept with probability rho (SplitMix64 draws), rank R_f
+    w = synth.nuscenes_frame(1)
+    got, status, table, _ = run_gpu(mmbev_lib, w, cuda_dev, rho_out=rho, seed=7)
+    assert status == 0
+    want = run_oracle(oracle_mod, w, rho_out=rho, seed=7)
+    assert assert_frames_equal(got, want, f"rho={rho}") == 1.0
+    assert _table_is_clean(table)
+
+
+@pytest.mark.gpu
+def test_rho_out_with_the_cap(oracle_mod, mmbev_lib, cuda_dev):
+    # rho = 1 with a cap below the voxel count: background-only voxels (rank
+    # R_f) go first, then the rank-tie split by lin
+    w = synth.nuscenes_frame(1)
+    for maxv in (9000, 30000):
+        got, status, table, _ = run_gpu(mmbev_lib, w, cuda_dev, maxv=maxv, rho_out=1.0, seed=3)
+        assert status == 0
+        want = run_oracle(oracle_mod, w, maxv=maxv, rho_out=1.0, seed=3)
+        assert len(want[0][1]) == maxv
+        assert assert_frames_equal(got, want, f"rho cap {maxv}") == 1.0
+        assert _table_is_clean(table)
+
+
+@pytest.mark.gpu
+def test_rho_out_batched_frames(oracle_mod, mmbev_lib, cuda_dev):
+    # draws use frame-local indices: a batch equals its frames
+    w = synth.concat_frames([synth.nuscenes_frame(s) for s in (1, 2, 3)], "three")
+    got, status, _, _ = run_gpu(mmbev_lib, w, cuda_dev, rho_out=0.3, seed=12345)
+    assert status == 0
+    want = run_oracle(oracle_mod, w, rho_out=0.3, seed=12345)
+    assert assert_frames_equal(got, want, "rho batch") == 1.0
+
+
+@pytest.mark.gpu
+def test_rho_out_seed_changes_the_draws(mmbev_lib, cuda_dev):
+    w = synth.nuscenes_frame(1).with_rois(np.zeros((0, 5), np.float32))
+    a, _, _, _ = run_gpu(mmbev_lib, w, cuda_dev, rho_out=0.5, seed=1)
+    b, _, _, _ = run_gpu(mmbev_lib, w, cuda_dev, rho_out=0.5, seed=2)
+    assert not np.array_equal(a[0][1], b[0][1])
