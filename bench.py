@@ -255,6 +255,8 @@ def run_gpu(args):
     mmbev.load()
 
     w = workload_for_rank(rank, args.frames)
+    if args.pillars:   # the same frames on a pillar grid (nz = 1)
+        w.voxel_size = np.array([0.075, 0.075, 8.0], np.float32)
     pts = torch.from_numpy(w.points).to(dev)
     tf = torch.from_numpy(w.sweep_tf).to(dev)
     rois = torch.from_numpy(w.rois).to(dev)
@@ -272,13 +274,24 @@ def run_gpu(args):
 
     stream = torch.cuda.current_stream(dev)
     nstage = mmbev.NUM_STAGES
+    # ScatterToBEV (Alg. 1, last step), part of the step with --bev
+    dims = [int(round((float(w.pc_range[a + 3]) - float(w.pc_range[a])) / float(w.voxel_size[a])))
+            for a in range(3)]
+    canvas = (torch.empty((w.num_frames, dims[2] * 5, dims[1], dims[0]), dtype=torch.float32,
+                          device=dev) if args.bev else None)
+
+    def step(**kw):
+        out = vx(pts, w.sweep_offsets, tf, rois, w.frame_sweep_offsets, w.frame_roi_offsets, **kw)
+        if canvas is not None:
+            mmbev.scatter_bev(out, w.max_voxels, dims, canvas=canvas)
+        return out
     step_ev = [[torch.cuda.Event(enable_timing=True) for _ in range(nstage + 1)]
                for _ in range(args.steps)]
     for evs in step_ev:
         for e in evs:
             e.record(stream)  # materialise the events before handing them to the library
     for _ in range(args.warmup):
-        vx(pts, w.sweep_offsets, tf, rois, w.frame_sweep_offsets, w.frame_roi_offsets)
+        step()
     torch.cuda.synchronize(dev)
     status = vx.status()
     if status != 0:
@@ -298,7 +311,7 @@ def run_gpu(args):
     torch.cuda.synchronize(dev)
     start.record(stream)
     for k in range(args.steps):
-        vx(pts, w.sweep_offsets, tf, rois, w.frame_sweep_offsets, w.frame_roi_offsets)
+        step()
     end.record(stream)
     torch.cuda.synchronize(dev)
     if world > 1:
@@ -307,9 +320,18 @@ def run_gpu(args):
     # timed region 2, the per-kernel breakdown: the same K calls with a CUDA
     # event on the launching stream between consecutive kernels
     for k in range(args.steps):
-        vx(pts, w.sweep_offsets, tf, rois, w.frame_sweep_offsets, w.frame_roi_offsets,
-           stage_events=step_ev[k])
+        step(stage_events=step_ev[k])
     torch.cuda.synchronize(dev)
+    bev_us = None
+    if canvas is not None:   # ScatterToBEV alone, on the last call's outputs
+        b0 = torch.cuda.Event(enable_timing=True)
+        b1 = torch.cuda.Event(enable_timing=True)
+        b0.record(stream)
+        for k in range(args.steps):
+            mmbev.scatter_bev(vx.out, w.max_voxels, dims, canvas=canvas)
+        b1.record(stream)
+        torch.cuda.synchronize(dev)
+        bev_us = 1e3 * b0.elapsed_time(b1) / args.steps
     clocks = sampler.stop()
     status = vx.status()
     if status != 0:
@@ -388,6 +410,10 @@ def run_gpu(args):
             "us_per_frame": 1e3 * ms_step / w.num_frames,
             "in_roi_points_per_gpu": n_in_roi, "voxels_out_per_gpu": u_out,
             "rho_out": args.rho_out,
+            "grid": dims,
+            "scatter_bev": (None if bev_us is None else
+                            {"us": round(bev_us, 2), "canvas_mb": round(canvas.numel() * 4 / 1e6, 1),
+                             "canvas_gbs": round(canvas.numel() * 4 / (bev_us * 1e-6) / 1e9, 1)}),
             "path_hbm_gbs": path_bytes / (ms_step * 1e-3) / 1e9,
             "path_frac_of_peak": path_bytes / (ms_step * 1e-3) / 1e9 / peak,
             "stage_us": {n: round(1e3 * t, 2) for n, t in zip(names, stage_ms)},
@@ -422,6 +448,10 @@ def main():
                     help="keep probability of points inside no ROI (Alg. 1); the headline "
                          "workload uses 0")
     ap.add_argument("--seed", type=int, default=0, help="seed of the rho_out draws")
+    ap.add_argument("--pillars", action="store_true",
+                    help="the same frames on a 0.075 x 0.075 x 8 m pillar grid (nz = 1)")
+    ap.add_argument("--bev", action="store_true",
+                    help="add ScatterToBEV (a dense [F, nz*5, ny, nx] canvas) to every step")
     ap.add_argument("--frames", type=int, default=FRAMES,
                     help="frames per GPU (the headline workload is 32; fewer for small "
                          "profiling cases)")

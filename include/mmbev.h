@@ -26,7 +26,8 @@
  *     |u| <= hl and |v| <= hw. l runs along the heading, w across it, yaw is
  *     counter-clockwise from +x. The point's rank is the first ROI (in array
  *     order = criticality order) that contains it; a point in no ROI is
- *     dropped (the out-of-ROI keep rate of Alg. 1 is zero).
+ *     dropped, except that mmbev_voxelize_roi_batched_ex can keep such points
+ *     at the rate rho_out of Alg. 1 (see mmbev_exec_opts_t).
  *   - Voxel: c_a = (int)floorf((p'_a - min_a) / size_a), dropped if
  *     c_a >= n_a, with n_a = (int)llround(((double)max_a - min_a) / size_a);
  *     lin = (cz*ny + cy)*nx + cx.
@@ -288,6 +289,27 @@ const char *mmbev_stage_name(int32_t stage);
 
 /* Library version string. */
 const char *mmbev_version(void);
+
+/*
+ * ScatterToBEV (Alg. 1, last step): the voxel features of F frames written
+ * into a dense, zero-initialized canvas by voxel coordinate.
+ *   feats, coords, nvox  device, the outputs of a voxelize call: feats
+ *               [F*max_voxels][5] fp32, coords [F*max_voxels][3] int32
+ *               (z, y, x), nvox [F] int32; frame f's rows start at
+ *               f*max_voxels and rows >= nvox[f] are ignored.
+ *   dims        host, the grid (nx, ny, nz), each >= 1.
+ *   canvas      device fp32 [F][nz*5][ny][nx]: channel cz*5 + c of cell
+ *               (cy, cx) holds feature c of voxel (cz, cy, cx); for a pillar
+ *               grid (nz = 1) that is the usual [5][ny][nx] BEV map. The call
+ *               zero-fills it first. canvas_bytes must be at least
+ *               F*nz*5*ny*nx*4 (else MMBEV_EWORKSPACE) and the canvas 16-byte
+ *               aligned (else MMBEV_EINVAL).
+ * Voxels whose coordinates lie outside dims are skipped. Asynchronous on
+ * `stream`; the library owns no memory.
+ */
+int mmbev_scatter_bev(const float *feats, const int32_t *coords, const int32_t *nvox,
+                      int32_t num_frames, int32_t max_voxels, const int32_t dims[3],
+                      float *canvas, size_t canvas_bytes, cudaStream_t stream);
 
 #ifdef __cplusplus
 }

@@ -168,6 +168,21 @@ def voxelize_roi_batched(points, sweep_offsets, sweep_tf, rois, roi_margin, voxe
     return out
 
 
+def scatter_bev(frames, dims):
+    """ScatterToBEV (Alg. 1, last step), written out: a zero canvas
+    [F, nz*5, ny, nx] and, for every kept voxel (cz, cy, cx) of frame f, its
+    feature c at channel cz*5 + c of cell (cy, cx). `frames` is the list of
+    per-frame (feats, coords, counts) a voxelize call returns."""
+    nx, ny, nz = (int(d) for d in dims)
+    canvas = np.zeros((len(frames), nz * 5, ny, nx), np.float32)
+    for f, (feats, coords, _) in enumerate(frames):
+        for v in range(len(coords)):
+            cz, cy, cx = (int(c) for c in coords[v])
+            for c in range(5):
+                canvas[f, cz * 5 + c, cy, cx] = feats[v, c]
+    return canvas
+
+
 def grid_dims(voxel_size, pc_range):
     """(nx, ny, nz) = round-half-away((max - min) / size) in double, as the
     oracle's llround does for these positive extents."""

@@ -61,6 +61,8 @@ def load():
     batched = vox + [i32, P, P, P, P, P, P, P, sz, P, sz, P]
     lib.mmbev_voxelize_roi_batched.argtypes = batched
     lib.mmbev_voxelize_roi_batched.restype = ctypes.c_int
+    lib.mmbev_scatter_bev.argtypes = [P, P, P, i32, i32, P, P, ctypes.c_size_t, P]
+    lib.mmbev_scatter_bev.restype = ctypes.c_int
     lib.mmbev_voxelize_roi_batched_ex.argtypes = batched + [ctypes.POINTER(_ExecOpts)]
     lib.mmbev_voxelize_roi_batched_ex.restype = ctypes.c_int
     lib.mmbev_classify_points.argtypes = [P, P, i32, P, P, i32, f32, P, P, i32, P, P,
@@ -308,6 +310,24 @@ def classify_points(points: torch.Tensor, sweep_offsets, sweep_tf: torch.Tensor,
         workspace.numel(), _stream(stream))
     _check(rc, "mmbev_classify_points")
     return xyz[:n], lin[:n], rank[:n]
+
+
+def scatter_bev(out: "Outputs", max_voxels: int, dims, canvas: torch.Tensor | None = None,
+                stream=None) -> torch.Tensor:
+    """ScatterToBEV (``mmbev_scatter_bev``): the voxels of a voxelize call's
+    outputs written into a zero-filled fp32 canvas [F, nz*5, ny, nx] (channel
+    cz*5 + c of cell (cy, cx) holds feature c of voxel (cz, cy, cx))."""
+    lib = load()
+    nx, ny, nz = (int(d) for d in dims)
+    nf = out.nvox.numel()
+    if canvas is None:
+        canvas = torch.empty((nf, nz * 5, ny, nx), dtype=torch.float32, device=out.feats.device)
+    d = np.asarray([nx, ny, nz], np.int32)
+    rc = lib.mmbev_scatter_bev(_dptr(out.feats), _dptr(out.coords), _dptr(out.nvox), nf,
+                               int(max_voxels), _hptr(d), _dptr(canvas, torch.float32, "canvas"),
+                               canvas.numel() * 4, _stream(stream))
+    _check(rc, "mmbev_scatter_bev")
+    return canvas
 
 
 class Voxelizer:

@@ -101,3 +101,17 @@ def test_rho_out_outside_unit_interval_is_rejected(mmbev_lib, rho):
         fake, fake, fake, fake, P(0x7f1000000000), 1 << 30, P(0x7f0000000000), 1 << 30, None,
         ctypes.byref(opts))
     assert rc == -1
+
+
+def test_scatter_bev_checks_the_canvas(mmbev_lib):
+    lib = mmbev_lib.load()
+    P = ctypes.c_void_p
+    fake = P(0x7e0000000000)
+    dims = np.asarray([512, 512, 1], np.int32)
+    need = 2 * 512 * 512 * 5 * 4
+    args = (fake, fake, fake, 2, 100, dims.ctypes.data_as(P))
+    assert lib.mmbev_scatter_bev(*args, P(0x7f0000000000), need - 16, None) == -3
+    assert lib.mmbev_scatter_bev(*args, P(0x7f0000000004), need, None) == -1
+    bad = np.asarray([512, 0, 1], np.int32)
+    assert lib.mmbev_scatter_bev(fake, fake, fake, 2, 100, bad.ctypes.data_as(P),
+                                 P(0x7f0000000000), need, None) == -1

@@ -392,3 +392,54 @@ def test_rho_out_seed_changes_the_draws(mmbev_lib, cuda_dev):
     a, _, _, _ = run_gpu(mmbev_lib, w, cuda_dev, rho_out=0.5, seed=1)
     b, _, _, _ = run_gpu(mmbev_lib, w, cuda_dev, rho_out=0.5, seed=2)
     assert not np.array_equal(a[0][1], b[0][1])
+
+
+# ------------------------------------------------------------------ ScatterToBEV (Alg. 1)
+
+@pytest.mark.gpu
+@pytest.mark.parametrize("name", ["tiny", "nuscenes_pillars"])
+def test_scatter_bev_parity(oracle_mod, mmbev_lib, cuda_dev, name):
+    import torch
+    if name == "tiny":
+        w = synth.tiny(0)
+    else:  # the nuScenes frame on a pillar grid (0.075 x 0.075 x 8 m)
+        base = synth.nuscenes_frame(1)
+        w = synth.concat_frames([base, synth.nuscenes_frame(2)], "two")
+        w.voxel_size = np.array([0.075, 0.075, 8.0], np.float32)
+    got, status, _, _ = run_gpu(mmbev_lib, w, cuda_dev)
+    assert status == 0
+    want = run_oracle(oracle_mod, w)
+    assert_frames_equal(got, want, name)
+    dims = oracle_mod.grid_dims(w.voxel_size, w.pc_range)
+    # the GPU scatter on the GPU voxelize outputs vs the oracle scatter of
+    # the oracle's voxelize outputs
+    pts, tf, rois = to_dev(w, cuda_dev)
+    vx = mmbev_lib.Voxelizer(w.num_points, int(np.max(np.diff(w.frame_roi_offsets))), w.max_voxels,
+                             w.num_frames, w.voxel_size, w.pc_range, w.max_pts_per_voxel,
+                             w.roi_margin, device=cuda_dev)
+    out = vx(pts, w.sweep_offsets, tf, rois, w.frame_sweep_offsets, w.frame_roi_offsets)
+    canvas = mmbev_lib.scatter_bev(out, w.max_voxels, dims)
+    torch.cuda.synchronize(cuda_dev)
+    ref = oracle_mod.scatter_bev(want, dims)
+    assert np.array_equal(canvas.cpu().numpy().view(np.uint32), ref.view(np.uint32))
+
+
+@pytest.mark.gpu
+def test_scatter_bev_refills_zeros_and_skips_bad_coords(oracle_mod, mmbev_lib, cuda_dev):
+    import torch
+    dims = (8, 4, 2)
+    out = mmbev_lib.Outputs.empty(2, 3, device=cuda_dev)
+    feats = torch.arange(30, dtype=torch.float32, device=cuda_dev).reshape(6, 5) + 1
+    coords = torch.tensor([[0, 1, 2], [1, 3, 7], [0, 4, 0], [1, 0, 0], [5, 0, 0], [0, 0, 0]],
+                          dtype=torch.int32, device=cuda_dev)   # row 2 and 4: outside dims
+    out.feats.copy_(feats)
+    out.coords.copy_(coords)
+    out.nvox.copy_(torch.tensor([3, 2], dtype=torch.int32))
+    canvas = torch.full((2, 10, 4, 8), 7.0, device=cuda_dev)    # stale contents get cleared
+    mmbev_lib.scatter_bev(out, 3, dims, canvas=canvas)
+    torch.cuda.synchronize(cuda_dev)
+    f = feats.cpu().numpy()
+    c = coords.cpu().numpy()
+    frames = [(f[0:2], c[0:2], None), (f[3:4], c[3:4], None)]   # valid rows of each frame
+    ref = oracle_mod.scatter_bev(frames, dims)
+    assert np.array_equal(canvas.cpu().numpy(), ref)

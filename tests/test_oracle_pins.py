@@ -656,3 +656,31 @@ def test_draws_use_frame_local_indices(oracle_mod):
         want = _vox(oracle_mod, fw, rho_out=0.25, seed=17)
         for x, y in zip(got, want):
             assert np.array_equal(x.view(np.uint32), y.view(np.uint32))
+
+
+# ------------------------------------------------------------------ ScatterToBEV (Alg. 1)
+
+def test_scatter_bev_places_features_by_coordinate(oracle_mod):
+    feats = np.array([[1, 2, 3, 4, 5], [6, 7, 8, 9, 10]], np.float32)
+    coords = np.array([[0, 2, 3], [1, 0, 1]], np.int32)   # (z, y, x)
+    canvas = oracle_mod.scatter_bev([(feats, coords, np.array([1, 1], np.int32))], (4, 3, 2))
+    assert canvas.shape == (1, 10, 3, 4)
+    assert list(canvas[0, 0:5, 2, 3]) == [1, 2, 3, 4, 5]
+    assert list(canvas[0, 5:10, 0, 1]) == [6, 7, 8, 9, 10]
+    assert np.count_nonzero(canvas) == 10
+
+
+def test_scatter_bev_pillars_is_the_bev_map(oracle_mod):
+    # nz = 1: channel c of cell (cy, cx) is feature c; the canvas sums to the features
+    w = synth.tiny(0)
+    out = oracle_mod.voxelize_roi(w.points, w.sweep_offsets, w.sweep_tf, w.rois, w.roi_margin,
+                                  w.voxel_size, w.pc_range, w.max_pts_per_voxel, w.max_voxels)
+    dims = oracle_mod.grid_dims(w.voxel_size, w.pc_range)
+    canvas = oracle_mod.scatter_bev([out], dims)
+    feats, coords, _ = out
+    assert canvas.shape == (1, 5, dims[1], dims[0])
+    assert np.allclose(canvas.sum(axis=(0, 2, 3), dtype=np.float64), feats.sum(0, dtype=np.float64))
+    occupied = np.count_nonzero(np.any(canvas[0] != 0, axis=0))
+    assert occupied <= len(coords)
+    for v in (0, len(coords) // 2, len(coords) - 1):
+        assert np.array_equal(canvas[0, :, coords[v, 1], coords[v, 2]], feats[v])
