@@ -63,6 +63,10 @@ def _load():
                                                     i32, i32, f32, u64, i32, P, P, P, P,
                                                     P, P]
         lib.oracle_voxelize_roi_batched.restype = ctypes.c_int
+        lib.oracle_build_rois.argtypes = [P, i32, P, P, P]
+        lib.oracle_build_rois.restype = ctypes.c_int
+        lib.oracle_crit_thresholds.argtypes = [P, P, P]
+        lib.oracle_crit_thresholds.restype = None
         lib.oracle_splitmix64.argtypes = [u64, u64]
         lib.oracle_splitmix64.restype = u64
         _lib = lib
@@ -166,6 +170,45 @@ def voxelize_roi_batched(points, sweep_offsets, sweep_tf, rois, roi_margin, voxe
         r0 = f * mv
         out.append((feats[r0:r0 + k].copy(), coords[r0:r0 + k].copy(), counts[r0:r0 + k].copy()))
     return out
+
+
+CRIT_FIELDS = ("v_ego", "dt", "a_brake", "d_min", "theta_max_deg", "theta_min_deg", "v_wide",
+               "v_narrow", "tau_vru", "tau_motor", "r_coll")
+CLS_MOTOR, CLS_VRU, CLS_STATIC = 0, 1, 2
+
+
+def _crit_params(params):
+    return np.asarray([float(params[k]) for k in CRIT_FIELDS], np.float32)
+
+
+def build_rois(objects, params):
+    """Temporal ROIs and criticality ranking of one frame (Sec. IV-C, Eq. 1,
+    3-5, 8). objects: [n, 8] float32 rows (cx, cy, w, l, yaw, vx, vy, cls).
+    Returns (rois [2n, 5] in rank order, flags [n]: bit 0 Geom, bit 1 Safety)."""
+    lib = _load()
+    obj = np.ascontiguousarray(objects, np.float32).reshape(-1, 8)
+    n = obj.shape[0]
+    rec = np.zeros(n, dtype=[("f", np.float32, 7), ("cls", np.int32)])
+    rec["f"] = obj[:, :7]
+    rec["cls"] = obj[:, 7].astype(np.int32)
+    q = _crit_params(params)
+    rois = np.zeros((max(2 * n, 1), 5), np.float32)
+    flags = np.zeros(max(n, 1), np.int32)
+    rc = lib.oracle_build_rois(rec.ctypes.data_as(ctypes.c_void_p), n, _ptr(q), _ptr(rois),
+                               _ptr(flags))
+    if rc != 0:
+        raise ValueError(f"oracle_build_rois failed with status {rc}")
+    return rois[:2 * n].copy(), flags[:n].copy()
+
+
+def crit_thresholds(params):
+    """(dmax, tan(theta)) of Eq. 4 and the cone, as fp32."""
+    lib = _load()
+    q = _crit_params(params)
+    d = np.zeros(1, np.float32)
+    t = np.zeros(1, np.float32)
+    lib.oracle_crit_thresholds(_ptr(q), _ptr(d), _ptr(t))
+    return float(d[0]), float(t[0])
 
 
 def scatter_bev(frames, dims):

@@ -348,3 +348,103 @@ int oracle_voxelize_roi_batched(const float *points, const int64_t *sweep_offset
     }
     return ORACLE_OK;
 }
+
+/*
+ * Temporal-ROI construction and criticality ranking (Sec. IV-C; Eq. 1, 3-5,
+ * 8), one frame. Each object (previous-frame detection, in the current ego
+ * frame: x forward, y left) gives two ROIs, its box and the box moved by the
+ * relative velocity (vx - v_ego, vy) times dt (Eq. 1's b and b + v dt), in
+ * that order. Objects are ranked mandatory first (Geom or Safety), then by
+ * TTC, squared distance and input index, all ascending.
+ *   Geom (Eq. 3-4): x >= 0, |p|^2 <= dmax^2 and |y| <= x * tan(theta), with
+ *     dmax = max(d_min, v_ego^2 / (2 a_brake)) and theta(v_ego) = theta_max
+ *     below v_wide, theta_min above v_narrow, linear in between (both in
+ *     double, then fp32).
+ *   Safety (Eq. 5, 8): class not static and TTC <= tau (VRU or motorized),
+ *     TTC = t* = -(p.v)/|v|^2 when t* > 0 and |p + t* v|^2 <= r_coll^2, else
+ *     infinity.
+ * Arithmetic in fp32, every product and sum rounded, in the order written.
+ */
+typedef struct { float cx, cy, w, l, yaw, vx, vy; int32_t cls; } oracle_object_t;
+typedef struct {
+    float v_ego, dt, a_brake, d_min, theta_max_deg, theta_min_deg, v_wide, v_narrow;
+    float tau_vru, tau_motor, r_coll;
+} oracle_crit_params_t;
+
+typedef struct { int32_t mand; float ttc, d2; int32_t idx; } crit_key_t;
+
+static int cmp_crit(const void *a, const void *b)
+{
+    const crit_key_t *u = (const crit_key_t *)a, *v = (const crit_key_t *)b;
+    if (u->mand != v->mand) return u->mand > v->mand ? -1 : 1;
+    if (u->ttc != v->ttc) return u->ttc < v->ttc ? -1 : 1;
+    if (u->d2 != v->d2) return u->d2 < v->d2 ? -1 : 1;
+    return u->idx < v->idx ? -1 : (u->idx > v->idx);
+}
+
+/* The frame-independent thresholds, in double, rounded to fp32. */
+void oracle_crit_thresholds(const oracle_crit_params_t *q, float *dmax, float *tan_theta)
+{
+    double v = q->v_ego;
+    double dm = v * v / (2.0 * q->a_brake);
+    if (dm < q->d_min) dm = q->d_min;
+    double th;
+    if (v <= q->v_wide) th = q->theta_max_deg;
+    else if (v >= q->v_narrow) th = q->theta_min_deg;
+    else th = q->theta_max_deg + (q->theta_min_deg - q->theta_max_deg) *
+                                 (v - q->v_wide) / (q->v_narrow - q->v_wide);
+    *dmax = (float)dm;
+    *tan_theta = (float)tan(th * 3.14159265358979323846 / 180.0);
+}
+
+int oracle_build_rois(const oracle_object_t *obj, int32_t n, const oracle_crit_params_t *q,
+                      oracle_roi_t *out_rois, int32_t *out_flags)
+{
+    if (n < 0 || !(q->a_brake > 0.0f) || !(q->v_narrow > q->v_wide) || !(q->dt >= 0.0f))
+        return ORACLE_EINVAL;
+    float dmax, tant;
+    oracle_crit_thresholds(q, &dmax, &tant);
+    const float dmax2 = dmax * dmax, r2 = q->r_coll * q->r_coll;
+    crit_key_t *key = (crit_key_t *)malloc(sizeof(crit_key_t) * (size_t)(n > 0 ? n : 1));
+    if (!key) return ORACLE_ENOMEM;
+    for (int32_t i = 0; i < n; ++i) {
+        const oracle_object_t *o = &obj[i];
+        const float px = o->cx, py = o->cy;
+        const float rvx = o->vx - q->v_ego, rvy = o->vy;
+        float a, b;
+        a = px * px; b = py * py; const float d2 = a + b;
+        const int geom = px >= 0.0f && d2 <= dmax2 && fabsf(py) <= px * tant;
+        float ttc = INFINITY;
+        a = rvx * rvx; b = rvy * rvy; const float vv = a + b;
+        if (vv > 0.0f) {
+            a = px * rvx; b = py * rvy; const float pv = a + b;
+            const float t = -pv / vv;
+            if (t > 0.0f) {
+                a = t * rvx; const float ex = px + a;
+                b = t * rvy; const float ey = py + b;
+                a = ex * ex; b = ey * ey;
+                if (a + b <= r2) ttc = t;
+            }
+        }
+        const float tau = o->cls == 1 ? q->tau_vru : q->tau_motor;
+        const int safety = o->cls != 2 && ttc <= tau;
+        out_flags[i] = geom | (safety << 1);
+        key[i].mand = geom || safety;
+        key[i].ttc = ttc;
+        key[i].d2 = d2;
+        key[i].idx = i;
+    }
+    qsort(key, (size_t)n, sizeof(crit_key_t), cmp_crit);
+    for (int32_t k = 0; k < n; ++k) {
+        const oracle_object_t *o = &obj[key[k].idx];
+        const float rvx = o->vx - q->v_ego, rvy = o->vy;
+        oracle_roi_t r = {o->cx, o->cy, o->w, o->l, o->yaw};
+        out_rois[2 * k] = r;
+        float m;
+        m = rvx * q->dt; r.cx = o->cx + m;
+        m = rvy * q->dt; r.cy = o->cy + m;
+        out_rois[2 * k + 1] = r;
+    }
+    free(key);
+    return ORACLE_OK;
+}

@@ -684,3 +684,71 @@ def test_scatter_bev_pillars_is_the_bev_map(oracle_mod):
     assert occupied <= len(coords)
     for v in (0, len(coords) // 2, len(coords) - 1):
         assert np.array_equal(canvas[0, :, coords[v, 1], coords[v, 2]], feats[v])
+
+
+# ------------------------------------------------------------------ temporal ROIs, criticality (Sec. IV-C)
+
+CRIT = dict(v_ego=10.0, dt=0.1, a_brake=6.0, d_min=10.0, theta_max_deg=60.0, theta_min_deg=15.0,
+            v_wide=5.0, v_narrow=30.0, tau_vru=1.5, tau_motor=2.5, r_coll=2.0)
+
+
+def _obj(cx, cy, vx=0.0, vy=0.0, cls=0, w=2.0, l=4.5, yaw=0.0):
+    return [cx, cy, w, l, yaw, vx, vy, cls]
+
+
+def test_braking_distance_and_cone(oracle_mod):
+    # Eq. 4: dmax = max(d_min, v^2 / (2 a)); the cone half-angle spans 60 .. 15 deg
+    d, t = oracle_mod.crit_thresholds(dict(CRIT, v_ego=10.0))
+    assert d == pytest.approx(10.0) and t == pytest.approx(np.tan(np.radians(51.0)), rel=1e-6)
+    d, t = oracle_mod.crit_thresholds(dict(CRIT, v_ego=20.0))
+    assert d == pytest.approx(400.0 / 12.0, rel=1e-6)
+    assert oracle_mod.crit_thresholds(dict(CRIT, v_ego=0.0))[1] == pytest.approx(np.sqrt(3), rel=1e-6)
+    assert oracle_mod.crit_thresholds(dict(CRIT, v_ego=40.0))[1] == pytest.approx(
+        np.tan(np.radians(15.0)), rel=1e-6)
+
+
+def test_time_to_collision_closed_forms(oracle_mod):
+    # ego at 10 m/s: a parked car 20 m ahead closes at 10 m/s, t* = 2 s
+    objs = np.array([_obj(20, 0, cls=0), _obj(20, 0, cls=1), _obj(20, 5, cls=0),
+                     _obj(20, 0, vx=15.0, cls=0), _obj(20, 0, cls=2)], np.float32)
+    _, flags = oracle_mod.build_rois(objs, CRIT)
+    assert flags[0] == 2          # Safety: TTC 2 <= 2.5 (motorized)
+    assert flags[1] == 0          # VRU threshold 1.5 < 2
+    assert flags[2] == 0          # passes 5 m to the side: beyond r_coll
+    assert flags[3] == 0          # pulling away: t* < 0
+    assert flags[4] == 0          # static: geometry only, and it is out of the cone range
+
+
+def test_geometry_cone_is_inclusive_and_forward(oracle_mod):
+    d, t = oracle_mod.crit_thresholds(CRIT)
+    x = np.float32(5.0)
+    y_edge = np.float32(x * np.float32(t))
+    objs = np.array([_obj(x, y_edge, vx=10.0), _obj(x, np.nextafter(y_edge, np.float32(1e9)), vx=10.0),
+                     _obj(-1.0, 0.0, vx=10.0), _obj(9.9, 0.0, vx=10.0), _obj(10.1, 0.0, vx=10.0)],
+                    np.float32)   # vx = v_ego: no relative motion, no TTC
+    _, flags = oracle_mod.build_rois(objs, CRIT)
+    assert list(flags) == [1, 0, 0, 1, 0]
+
+
+def test_ranking_mandatory_then_ttc_then_distance(oracle_mod):
+    objs = np.array([_obj(30, 20, vx=10.0),            # optional, far
+                     _obj(3, 1, vx=10.0),              # optional? in the cone and near: Geom
+                     _obj(20, 0, cls=0),               # Safety, TTC 2.0
+                     _obj(15, 0, cls=0),               # Safety, TTC 1.5
+                     _obj(8, 25, vx=10.0)], np.float32)   # optional, nearer than the first
+    rois, flags = oracle_mod.build_rois(objs, CRIT)
+    order = [int(np.argmin(np.abs(objs[:, 0] - r[0]) + np.abs(objs[:, 1] - r[1]))) for r in rois[::2]]
+    # mandatory (TTC 1.5, TTC 2.0, then the Geom-only one with TTC inf), then optional by distance
+    assert order == [3, 2, 1, 4, 0]
+    assert list(flags) == [0, 1, 2, 2, 0]
+
+
+def test_each_object_gives_its_box_and_the_extrapolated_box(oracle_mod):
+    objs = np.array([_obj(12.0, -3.0, vx=4.0, vy=1.5, cls=1, w=0.8, l=0.9, yaw=0.3)], np.float32)
+    rois, _ = oracle_mod.build_rois(objs, CRIT)
+    assert rois.shape == (2, 5)
+    assert list(rois[0]) == [12.0, -3.0, 0.8, 0.9, np.float32(0.3)]
+    rvx, rvy = np.float32(4.0 - 10.0), np.float32(1.5)
+    assert rois[1][0] == np.float32(12.0) + rvx * np.float32(0.1)
+    assert rois[1][1] == np.float32(-3.0) + rvy * np.float32(0.1)
+    assert list(rois[1][2:]) == list(rois[0][2:])
