@@ -264,14 +264,6 @@ def run_gpu(args):
     vx = mmbev.Voxelizer(w.num_points, rmax, w.max_voxels, w.num_frames, w.voxel_size,
                          w.pc_range, w.max_pts_per_voxel, w.roi_margin, device=dev,
                          rho_out=args.rho_out, seed=args.seed)
-    # the metric's numerator: in-ROI points, counted by the library's own
-    # per-point classification of these inputs (S1-S2), once, untimed
-    _, lin, _ = mmbev.classify_points(pts, w.sweep_offsets, tf, rois, w.roi_margin, w.voxel_size,
-                                      w.pc_range, w.frame_sweep_offsets, w.frame_roi_offsets,
-                                      workspace=vx.workspace)
-    n_in_roi = int((lin >= 0).sum().item())
-    del lin
-
     stream = torch.cuda.current_stream(dev)
     nstage = mmbev.NUM_STAGES
     # ScatterToBEV (Alg. 1, last step), part of the step with --bev
@@ -280,8 +272,46 @@ def run_gpu(args):
     canvas = (torch.empty((w.num_frames, dims[2] * 5, dims[1], dims[0]), dtype=torch.float32,
                           device=dev) if args.bev else None)
 
+    # Temporal ROIs (Sec. IV-C), part of the step with --build-rois: every
+    # frame's ROI boxes become previous-frame objects with seeded velocities,
+    # and the device builds the ranked table the call then uses
+    crit = dict(v_ego=10.0, dt=0.1, a_brake=6.0, d_min=10.0, theta_max_deg=60.0,
+                theta_min_deg=15.0, v_wide=5.0, v_narrow=30.0, tau_vru=1.5, tau_motor=2.5,
+                r_coll=2.0)
+    roi_off = w.frame_roi_offsets
+    objs_d = None
+    if args.build_rois:
+        orng = np.random.default_rng(4242 + rank)
+        objs = np.zeros((w.rois.shape[0], 8), np.float32)
+        objs[:, :5] = w.rois
+        objs[:, 5] = orng.uniform(-5, 20, len(objs))
+        objs[:, 6] = orng.uniform(-3, 3, len(objs))
+        objs[:, 7] = orng.integers(0, 3, len(objs))
+        objs_d = mmbev.pack_objects(torch.from_numpy(objs).to(dev))
+        rois_buf = (torch.empty((2 * len(objs), 5), dtype=torch.float32, device=dev),
+                    torch.empty(len(objs), dtype=torch.int32, device=dev))
+        obj_off = np.asarray(w.frame_roi_offsets, np.int32)
+        roi_off = (2 * obj_off).astype(np.int32)
+        rmax = 2 * rmax
+        vx = mmbev.Voxelizer(w.num_points, rmax, w.max_voxels, w.num_frames, w.voxel_size,
+                             w.pc_range, w.max_pts_per_voxel, w.roi_margin, device=dev,
+                             rho_out=args.rho_out, seed=args.seed)
+
+    # the metric's numerator: in-ROI points, counted by the library's own
+    # per-point classification of these inputs (S1-S2) with the ROI table the
+    # step uses, once, untimed
+    rois_used = rois if objs_d is None else mmbev.build_rois(objs_d, obj_off, crit)[0]
+    _, lin, _ = mmbev.classify_points(pts, w.sweep_offsets, tf, rois_used, w.roi_margin,
+                                      w.voxel_size, w.pc_range, w.frame_sweep_offsets, roi_off,
+                                      workspace=vx.workspace)
+    n_in_roi = int((lin >= 0).sum().item())
+    del lin
+
     def step(**kw):
-        out = vx(pts, w.sweep_offsets, tf, rois, w.frame_sweep_offsets, w.frame_roi_offsets, **kw)
+        rl = rois
+        if objs_d is not None:
+            rl = mmbev.build_rois(objs_d, obj_off, crit, out=rois_buf)[0]
+        out = vx(pts, w.sweep_offsets, tf, rl, w.frame_sweep_offsets, roi_off, **kw)
         if canvas is not None:
             mmbev.scatter_bev(out, w.max_voxels, dims, canvas=canvas)
         return out
@@ -322,6 +352,16 @@ def run_gpu(args):
     for k in range(args.steps):
         step(stage_events=step_ev[k])
     torch.cuda.synchronize(dev)
+    rois_us = None
+    if objs_d is not None:   # the ROI construction alone
+        r0e = torch.cuda.Event(enable_timing=True)
+        r1e = torch.cuda.Event(enable_timing=True)
+        r0e.record(stream)
+        for k in range(args.steps):
+            mmbev.build_rois(objs_d, obj_off, crit, out=rois_buf)
+        r1e.record(stream)
+        torch.cuda.synchronize(dev)
+        rois_us = 1e3 * r0e.elapsed_time(r1e) / args.steps
     bev_us = None
     if canvas is not None:   # ScatterToBEV alone, on the last call's outputs
         b0 = torch.cuda.Event(enable_timing=True)
@@ -361,12 +401,20 @@ def run_gpu(args):
     e2e_steps = max(3, min(args.steps, 10))
     d2h_bytes = 0
 
+    h_objs = objs_d.cpu().pin_memory() if objs_d is not None else None   # packed layout
+    d_objs = torch.empty_like(objs_d) if objs_d is not None else None
+
     def e2e_step():
         nonlocal d2h_bytes
         d_pts.copy_(h_pts, non_blocking=True)
         d_tf.copy_(h_tf, non_blocking=True)
-        d_rois.copy_(h_rois, non_blocking=True)
-        out = vx(d_pts, w.sweep_offsets, d_tf, d_rois, w.frame_sweep_offsets, w.frame_roi_offsets)
+        if d_objs is None:
+            d_rois.copy_(h_rois, non_blocking=True)
+            rl = d_rois
+        else:   # the previous frame's objects go up; the ROI table is built on the device
+            d_objs.copy_(h_objs, non_blocking=True)
+            rl = mmbev.build_rois(d_objs, obj_off, crit, out=rois_buf)[0]
+        out = vx(d_pts, w.sweep_offsets, d_tf, rl, w.frame_sweep_offsets, roi_off)
         h_nvox.copy_(out.nvox, non_blocking=True)
         torch.cuda.current_stream(dev).synchronize()
         nb = 0
@@ -394,7 +442,8 @@ def run_gpu(args):
     ms_step = ms_max / args.steps
     value = total_pts / (ms_step * 1e-3)
     e2e_value = total_pts / (e2e_max / e2e_steps)
-    h2d_bytes = w.points.nbytes + w.sweep_tf.nbytes + w.rois.nbytes
+    h2d_bytes = w.points.nbytes + w.sweep_tf.nbytes + (
+        w.rois.nbytes if objs_d is None else objs.nbytes)
 
     if rank == 0:
         peak, peak_kind = read_peaks()
@@ -411,6 +460,8 @@ def run_gpu(args):
             "in_roi_points_per_gpu": n_in_roi, "voxels_out_per_gpu": u_out,
             "rho_out": args.rho_out,
             "grid": dims,
+            "build_rois": (None if rois_us is None else
+                           {"us": round(rois_us, 2), "objects": int(objs_d.shape[0])}),
             "scatter_bev": (None if bev_us is None else
                             {"us": round(bev_us, 2), "canvas_mb": round(canvas.numel() * 4 / 1e6, 1),
                              "canvas_gbs": round(canvas.numel() * 4 / (bev_us * 1e-6) / 1e9, 1)}),
@@ -450,6 +501,9 @@ def main():
     ap.add_argument("--seed", type=int, default=0, help="seed of the rho_out draws")
     ap.add_argument("--pillars", action="store_true",
                     help="the same frames on a 0.075 x 0.075 x 8 m pillar grid (nz = 1)")
+    ap.add_argument("--build-rois", action="store_true",
+                    help="build every frame's ROI table on the device from previous-frame "
+                         "objects (Sec. IV-C) as part of the step")
     ap.add_argument("--bev", action="store_true",
                     help="add ScatterToBEV (a dense [F, nz*5, ny, nx] canvas) to every step")
     ap.add_argument("--frames", type=int, default=FRAMES,

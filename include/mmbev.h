@@ -291,6 +291,52 @@ const char *mmbev_stage_name(int32_t stage);
 const char *mmbev_version(void);
 
 /*
+ * Temporal ROIs and criticality ranking (Sec. IV-C; Eq. 1, 3-5, 8): the ROI
+ * table a voxelize call takes, built on the device from the previous frame's
+ * detections.
+ *   objects     device, per frame its detections in the current ego frame
+ *               (x forward, y left, metres): box (cx, cy, w, l, yaw), ground
+ *               velocity (vx, vy) in m/s along the ego axes, class
+ *               MMBEV_CLS_*. Frame f owns objects [off[f], off[f+1]),
+ *               at most MMBEV_MAX_ROIS_PER_FRAME / 2 of them.
+ *   frame_obj_offsets  host, [num_frames + 1], off[0] = 0, nondecreasing.
+ *   params      host: ego speed v_ego along +x, dt of Eq. 1, a_brake and
+ *               d_min of Eq. 4, the cone half-angle theta (theta_max_deg at
+ *               or below v_wide, theta_min_deg at or above v_narrow, linear
+ *               in between; the paper bounds it by 60 and 15 degrees), the
+ *               TTC thresholds tau of Eq. 5 for vulnerable and motorized
+ *               classes (static objects are geometry-critical only), and
+ *               r_coll of Eq. 8. The paper leaves a_brake, d_min, the theta
+ *               breakpoints and r_coll open.
+ *   out_rois    device, [2 * off[num_frames]]: frame f's ROIs at
+ *               [2*off[f], 2*off[f+1]) in rank order, so 2*off serves as
+ *               the voxelize call's frame_roi_offsets. Each object gives two
+ *               ROIs, its box and its box moved by the relative velocity
+ *               (vx - v_ego, vy) times dt (Eq. 1's b and b + v dt).
+ *   out_flags   device [off[num_frames]] or NULL: per object (input order)
+ *               bit 0 Geom, bit 1 Safety.
+ * Ranking: mandatory objects (Geom or Safety) first, then ascending TTC,
+ * then ascending squared distance, then input index. Geom: x >= 0,
+ * x^2 + y^2 <= dmax^2, |y| <= x * tan(theta), dmax = max(d_min, v_ego^2 /
+ * (2 a_brake)) and tan(theta) evaluated in double then rounded to fp32.
+ * TTC: relative velocity v = (vx - v_ego, vy); t* = -(p.v)/|v|^2; TTC = t*
+ * when t* > 0 and |p + t* v|^2 <= r_coll^2, else infinity. All other
+ * arithmetic is fp32, every product and sum rounded in the order written.
+ */
+#define MMBEV_CLS_MOTOR 0
+#define MMBEV_CLS_VRU 1
+#define MMBEV_CLS_STATIC 2
+typedef struct { float cx, cy, w, l, yaw, vx, vy; int32_t cls; } mmbev_object_t;
+typedef struct {
+    float v_ego, dt, a_brake, d_min, theta_max_deg, theta_min_deg, v_wide, v_narrow;
+    float tau_vru, tau_motor, r_coll;
+} mmbev_crit_params_t;
+
+int mmbev_build_rois(const mmbev_object_t *objects, const int32_t *frame_obj_offsets,
+                     int32_t num_frames, const mmbev_crit_params_t *params,
+                     mmbev_roi_t *out_rois, int32_t *out_flags, cudaStream_t stream);
+
+/*
  * ScatterToBEV (Alg. 1, last step): the voxel features of F frames written
  * into a dense, zero-initialized canvas by voxel coordinate.
  *   feats, coords, nvox  device, the outputs of a voxelize call: feats

@@ -385,14 +385,15 @@ static int cmp_crit(const void *a, const void *b)
 /* The frame-independent thresholds, in double, rounded to fp32. */
 void oracle_crit_thresholds(const oracle_crit_params_t *q, float *dmax, float *tan_theta)
 {
-    double v = q->v_ego;
-    double dm = v * v / (2.0 * q->a_brake);
-    if (dm < q->d_min) dm = q->d_min;
+    const double v = q->v_ego;
+    double dm = v * v / (2.0 * (double)q->a_brake);
+    if (dm < (double)q->d_min) dm = q->d_min;
     double th;
-    if (v <= q->v_wide) th = q->theta_max_deg;
-    else if (v >= q->v_narrow) th = q->theta_min_deg;
-    else th = q->theta_max_deg + (q->theta_min_deg - q->theta_max_deg) *
-                                 (v - q->v_wide) / (q->v_narrow - q->v_wide);
+    if (v <= (double)q->v_wide) th = q->theta_max_deg;
+    else if (v >= (double)q->v_narrow) th = q->theta_min_deg;
+    else th = (double)q->theta_max_deg +
+              ((double)q->theta_min_deg - (double)q->theta_max_deg) * (v - (double)q->v_wide) /
+                  ((double)q->v_narrow - (double)q->v_wide);
     *dmax = (float)dm;
     *tan_theta = (float)tan(th * 3.14159265358979323846 / 180.0);
 }

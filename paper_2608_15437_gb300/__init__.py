@@ -61,6 +61,8 @@ def load():
     batched = vox + [i32, P, P, P, P, P, P, P, sz, P, sz, P]
     lib.mmbev_voxelize_roi_batched.argtypes = batched
     lib.mmbev_voxelize_roi_batched.restype = ctypes.c_int
+    lib.mmbev_build_rois.argtypes = [P, P, i32, P, P, P, P]
+    lib.mmbev_build_rois.restype = ctypes.c_int
     lib.mmbev_scatter_bev.argtypes = [P, P, P, i32, i32, P, P, ctypes.c_size_t, P]
     lib.mmbev_scatter_bev.restype = ctypes.c_int
     lib.mmbev_voxelize_roi_batched_ex.argtypes = batched + [ctypes.POINTER(_ExecOpts)]
@@ -310,6 +312,45 @@ def classify_points(points: torch.Tensor, sweep_offsets, sweep_tf: torch.Tensor,
         workspace.numel(), _stream(stream))
     _check(rc, "mmbev_classify_points")
     return xyz[:n], lin[:n], rank[:n]
+
+
+CRIT_FIELDS = ("v_ego", "dt", "a_brake", "d_min", "theta_max_deg", "theta_min_deg", "v_wide",
+               "v_narrow", "tau_vru", "tau_motor", "r_coll")
+CLS_MOTOR, CLS_VRU, CLS_STATIC = 0, 1, 2
+
+
+def pack_objects(objects: torch.Tensor) -> torch.Tensor:
+    """float32 [n, 8] rows (cx, cy, w, l, yaw, vx, vy, class) on the device ->
+    the ``mmbev_object_t`` layout (the class as int32 bits in column 7)."""
+    n = objects.shape[0]
+    packed = torch.empty((max(n, 1), 8), dtype=torch.float32, device=objects.device)
+    if n:
+        packed[:n, :7] = objects[:, :7]
+        packed.view(torch.int32)[:n, 7] = objects[:, 7].to(torch.int32)
+    return packed[:n]
+
+
+def build_rois(packed: torch.Tensor, frame_obj_offsets, params: dict, out=None, stream=None):
+    """Temporal ROIs and criticality ranking (``mmbev_build_rois``).
+
+    packed: device objects from ``pack_objects`` (class 0 motorized,
+    1 vulnerable, 2 static); frame_obj_offsets: host [F+1]; params: the
+    CRIT_FIELDS; out: optional (rois, flags) to fill. Returns (rois [2n, 5]
+    float32 in rank order per frame, flags [n] int32, frame_roi_offsets =
+    2 * offsets)."""
+    lib = load()
+    off = _host(frame_obj_offsets, np.int32)
+    n = packed.shape[0]
+    dev = packed.device
+    if out is None:
+        out = (torch.empty((max(2 * n, 1), 5), dtype=torch.float32, device=dev),
+               torch.empty(max(n, 1), dtype=torch.int32, device=dev))
+    rois, flags = out
+    q = np.asarray([float(params[k]) for k in CRIT_FIELDS], np.float32)
+    rc = lib.mmbev_build_rois(_dptr(packed) if n else None, _hptr(off), len(off) - 1, _hptr(q),
+                              _dptr(rois), _dptr(flags), _stream(stream))
+    _check(rc, "mmbev_build_rois")
+    return rois[:2 * n], flags[:n], (2 * off).astype(np.int32)
 
 
 def scatter_bev(out: "Outputs", max_voxels: int, dims, canvas: torch.Tensor | None = None,

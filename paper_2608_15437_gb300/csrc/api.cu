@@ -91,7 +91,15 @@ Layout make_layout(int64_t max_points, int64_t rois_total, int32_t max_rois_fram
     L.fso = take(sizeof(int32_t) * (F + 1));
     L.fro = take(sizeof(int32_t) * (F + 1));
     L.roi_prep = take(sizeof(RoiPrep) * R);
-    L.masks = take(sizeof(uint32_t) * F * L.coarse * L.coarse * L.mask_words);
+    // room for the largest mask any call with at most max_rois_frame ROIs per
+    // frame selects (fewer ROIs can pick a finer grid), so the size is
+    // monotone in max_rois_frame
+    size_t mask_words_frame = 0;
+    for (int w = 1; w <= L.mask_words; ++w) {
+        const size_t c = (size_t)coarse_for(w);
+        if (c * c * (size_t)w > mask_words_frame) mask_words_frame = c * c * (size_t)w;
+    }
+    L.masks = take(sizeof(uint32_t) * F * mask_words_frame);
     L.hist = take(sizeof(uint32_t) * (R + F));
     L.frame_u = take(sizeof(uint32_t) * F);
     L.finfo = take(sizeof(FrameInfo) * F);

@@ -115,3 +115,32 @@ def test_scatter_bev_checks_the_canvas(mmbev_lib):
     bad = np.asarray([512, 0, 1], np.int32)
     assert lib.mmbev_scatter_bev(fake, fake, fake, 2, 100, bad.ctypes.data_as(P),
                                  P(0x7f0000000000), need, None) == -1
+
+
+def test_build_rois_validates_on_the_host(mmbev_lib):
+    lib = mmbev_lib.load()
+    P = ctypes.c_void_p
+    fake = P(0x7e0000000000)
+    good = dict(v_ego=10.0, dt=0.1, a_brake=6.0, d_min=10.0, theta_max_deg=60.0,
+                theta_min_deg=15.0, v_wide=5.0, v_narrow=30.0, tau_vru=1.5, tau_motor=2.5,
+                r_coll=2.0)
+
+    def call(off, **kw):
+        q = np.asarray([float(dict(good, **kw)[k]) for k in mmbev_lib.CRIT_FIELDS], np.float32)
+        off = np.asarray(off, np.int32)
+        return lib.mmbev_build_rois(fake, off.ctypes.data_as(P), len(off) - 1,
+                                    q.ctypes.data_as(P), fake, fake, None)
+    assert call([0, 513]) == -1                 # more objects than half the ROI limit
+    assert call([0, 5, 3]) == -1                # offsets decrease
+    assert call([1, 5]) == -1                   # must start at 0
+    assert call([0, 5], a_brake=0.0) == -1
+    assert call([0, 5], v_narrow=4.0) == -1
+    assert call([0, 5], dt=float("nan")) == -1
+    assert call([0, 0]) == 0                    # nothing to do: no launch
+
+
+def test_workspace_size_is_monotone_in_the_roi_count(mmbev_lib):
+    # a workspace sized for up to R ROIs per frame serves every call with fewer
+    sizes = [mmbev_lib.workspace_size(20000, r, 16000, 4, TINY_VS, TINY_RG)
+             for r in (1, 32, 33, 64, 128, 129, 512, 1024)]
+    assert sizes == sorted(sizes)

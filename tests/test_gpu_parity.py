@@ -443,3 +443,73 @@ def test_scatter_bev_refills_zeros_and_skips_bad_coords(oracle_mod, mmbev_lib, c
     frames = [(f[0:2], c[0:2], None), (f[3:4], c[3:4], None)]   # valid rows of each frame
     ref = oracle_mod.scatter_bev(frames, dims)
     assert np.array_equal(canvas.cpu().numpy(), ref)
+
+
+# ------------------------------------------------------------------ temporal ROIs, criticality (Sec. IV-C)
+
+CRIT = dict(v_ego=12.0, dt=0.1, a_brake=6.0, d_min=10.0, theta_max_deg=60.0, theta_min_deg=15.0,
+            v_wide=5.0, v_narrow=30.0, tau_vru=1.5, tau_motor=2.5, r_coll=2.0)
+
+
+def _random_objects(rng, n):
+    o = np.zeros((n, 8), np.float32)
+    o[:, 0] = rng.uniform(-40, 40, n)
+    o[:, 1] = rng.uniform(-40, 40, n)
+    o[:, 2] = rng.uniform(0.5, 3.0, n)
+    o[:, 3] = rng.uniform(0.5, 6.0, n)
+    o[:, 4] = rng.uniform(-np.pi, np.pi, n)
+    o[:, 5] = rng.uniform(-15, 25, n)
+    o[:, 6] = rng.uniform(-5, 5, n)
+    o[:, 7] = rng.integers(0, 3, n)
+    # a few exact ties in distance and TTC-free objects moving with the ego
+    o[: n // 8, 5] = CRIT["v_ego"]
+    o[: n // 8, 6] = 0.0
+    if n > 4:
+        o[1, :2] = o[0, :2]
+    return o
+
+
+@pytest.mark.gpu
+def test_build_rois_parity(oracle_mod, mmbev_lib, cuda_dev):
+    import torch
+    rng = np.random.default_rng(21)
+    counts = [0, 37, 512, 1, 200]
+    objs = np.concatenate([_random_objects(rng, n) for n in counts]).astype(np.float32)
+    off = np.concatenate([[0], np.cumsum(counts)]).astype(np.int32)
+    for params in (CRIT, dict(CRIT, v_ego=0.0), dict(CRIT, v_ego=35.0, dt=0.0)):
+        rois, flags, roff = mmbev_lib.build_rois(
+            mmbev_lib.pack_objects(torch.from_numpy(objs).to(cuda_dev)), off, params)
+        torch.cuda.synchronize(cuda_dev)
+        rois, flags = rois.cpu().numpy(), flags.cpu().numpy()
+        assert np.array_equal(roff, 2 * off)
+        for f in range(len(counts)):
+            want_r, want_f = oracle_mod.build_rois(objs[off[f]:off[f + 1]], params)
+            assert np.array_equal(rois[2 * off[f]:2 * off[f + 1]].view(np.uint32), want_r.view(np.uint32))
+            assert np.array_equal(flags[off[f]:off[f + 1]], want_f)
+
+
+@pytest.mark.gpu
+def test_built_rois_drive_the_voxelization(oracle_mod, mmbev_lib, cuda_dev):
+    # the ROI table from the previous frame's detections feeds the call directly
+    import torch
+    frames = [synth.nuscenes_frame(s) for s in (1, 2)]
+    rng = np.random.default_rng(5)
+    objs = [_random_objects(rng, 40) for _ in frames]
+    for o in objs:
+        o[:, 0:2] = rng.uniform(-30, 30, (len(o), 2))
+    allobj = np.concatenate(objs)
+    off = np.array([0, 40, 80], np.int32)
+    rois_d, _, roff = mmbev_lib.build_rois(
+        mmbev_lib.pack_objects(torch.from_numpy(allobj).to(cuda_dev)), off, CRIT)
+    w = synth.concat_frames([fw.with_rois(oracle_mod.build_rois(o, CRIT)[0])
+                             for fw, o in zip(frames, objs)], "built")
+    assert np.array_equal(w.frame_roi_offsets, roff)
+    pts, tf, _ = to_dev(w, cuda_dev)
+    vx = mmbev_lib.Voxelizer(w.num_points, 80, w.max_voxels, 2, w.voxel_size, w.pc_range,
+                             w.max_pts_per_voxel, w.roi_margin, device=cuda_dev)
+    out = vx(pts, w.sweep_offsets, tf, rois_d, w.frame_sweep_offsets, roff)
+    torch.cuda.synchronize(cuda_dev)
+    assert vx.status() == 0
+    got = [out.frame(f, w.max_voxels) for f in range(2)]
+    want = run_oracle(oracle_mod, w)
+    assert assert_frames_equal(got, want, "built rois") == 1.0
