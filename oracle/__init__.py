@@ -211,6 +211,50 @@ def crit_thresholds(params):
     return float(d[0]), float(t[0])
 
 
+def voxel_components(frames, dims):
+    """Connected components of each frame's kept voxels under 26-connectivity
+    (voxels sharing a face, an edge or a corner): the voxel-grid proposer of
+    the paper's robot deployment, written out with a dict and union-find.
+    Each voxel's label is the smallest output row (within its frame) of its
+    component. Returns per frame (labels [n], components [k, 8] rows of
+    (label, size, zmin, ymin, xmin, zmax, ymax, xmax) sorted by label)."""
+    nx, ny, nz = (int(d) for d in dims)
+    out = []
+    for feats, coords, _ in frames:
+        n = len(coords)
+        at = {tuple(int(c) for c in coords[v]): v for v in range(n)}
+        parent = list(range(n))
+
+        def find(x):
+            while parent[x] != x:
+                parent[x] = parent[parent[x]]
+                x = parent[x]
+            return x
+
+        for v in range(n):
+            z, y, x = (int(c) for c in coords[v])
+            for dz in (-1, 0, 1):
+                for dy in (-1, 0, 1):
+                    for dx in (-1, 0, 1):
+                        u = at.get((z + dz, y + dy, x + dx))
+                        if u is None or u == v:
+                            continue
+                        a, b = find(v), find(u)
+                        if a != b:
+                            parent[max(a, b)] = min(a, b)
+        labels = np.array([find(v) for v in range(n)], np.int32)
+        comps = {}
+        for v in range(n):
+            z, y, x = (int(c) for c in coords[v])
+            r = comps.setdefault(int(labels[v]), [int(labels[v]), 0, z, y, x, z, y, x])
+            r[1] += 1
+            r[2], r[3], r[4] = min(r[2], z), min(r[3], y), min(r[4], x)
+            r[5], r[6], r[7] = max(r[5], z), max(r[6], y), max(r[7], x)
+        comp = np.array([comps[k] for k in sorted(comps)], np.int32).reshape(-1, 8)
+        out.append((labels, comp))
+    return out
+
+
 def scatter_bev(frames, dims):
     """ScatterToBEV (Alg. 1, last step), written out: a zero canvas
     [F, nz*5, ny, nx] and, for every kept voxel (cz, cy, cx) of frame f, its

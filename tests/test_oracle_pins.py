@@ -752,3 +752,35 @@ def test_each_object_gives_its_box_and_the_extrapolated_box(oracle_mod):
     assert rois[1][0] == np.float32(12.0) + rvx * np.float32(0.1)
     assert rois[1][1] == np.float32(-3.0) + rvy * np.float32(0.1)
     assert list(rois[1][2:]) == list(rois[0][2:])
+
+
+# ------------------------------------------------------------------ voxel-grid components (proposer)
+
+def _cc(oracle_mod, coords, dims=(16, 16, 4)):
+    coords = np.asarray(coords, np.int32).reshape(-1, 3)
+    feats = np.zeros((len(coords), 5), np.float32)
+    return oracle_mod.voxel_components([(feats, coords, None)], dims)[0]
+
+
+def test_components_use_26_connectivity(oracle_mod):
+    # face, edge and corner neighbours join; a gap of one cell separates
+    labels, comp = _cc(oracle_mod, [[0, 0, 0], [0, 0, 1], [0, 1, 2], [1, 2, 3], [1, 2, 5]])
+    assert list(labels) == [0, 0, 0, 0, 4]
+    assert comp.tolist() == [[0, 4, 0, 0, 0, 1, 2, 3], [4, 1, 1, 2, 5, 1, 2, 5]]
+
+
+def test_component_label_is_the_smallest_row(oracle_mod):
+    # rows listed out of spatial order: the label is the smallest row index
+    labels, comp = _cc(oracle_mod, [[0, 5, 5], [0, 9, 9], [0, 5, 6], [0, 9, 8], [0, 5, 7]])
+    assert list(labels) == [0, 1, 0, 1, 0]
+    assert comp[:, 0].tolist() == [0, 1] and comp[:, 1].tolist() == [3, 2]
+
+
+def test_component_sizes_sum_to_the_voxels(oracle_mod):
+    w = synth.nuscenes_frame(1)
+    out = _vox(oracle_mod, w)
+    dims = oracle_mod.grid_dims(w.voxel_size, w.pc_range)
+    labels, comp = oracle_mod.voxel_components([out], dims)[0]
+    assert comp[:, 1].sum() == len(out[1])
+    assert np.all(labels[comp[:, 0]] == comp[:, 0])   # roots label themselves
+    assert np.all(labels <= np.arange(len(labels)))
