@@ -362,6 +362,19 @@ def run_gpu(args):
         r1e.record(stream)
         torch.cuda.synchronize(dev)
         rois_us = 1e3 * r0e.elapsed_time(r1e) / args.steps
+    cc_us = cc_n = None
+    if args.components:   # the voxel-grid proposer alone, on the last call's outputs
+        need = mmbev.components_table_bytes(w.num_frames, w.max_voxels)
+        cc_table = torch.zeros(need, dtype=torch.uint8, device=dev) if need else None
+        c0e = torch.cuda.Event(enable_timing=True)
+        c1e = torch.cuda.Event(enable_timing=True)
+        c0e.record(stream)
+        for k in range(args.steps):
+            cc = mmbev.voxel_components(vx.out, w.max_voxels, dims, cc_table)
+        c1e.record(stream)
+        torch.cuda.synchronize(dev)
+        cc_us = 1e3 * c0e.elapsed_time(c1e) / args.steps
+        cc_n = int(cc[2].sum().item())
     bev_us = None
     if canvas is not None:   # ScatterToBEV alone, on the last call's outputs
         b0 = torch.cuda.Event(enable_timing=True)
@@ -460,6 +473,7 @@ def run_gpu(args):
             "in_roi_points_per_gpu": n_in_roi, "voxels_out_per_gpu": u_out,
             "rho_out": args.rho_out,
             "grid": dims,
+            "components": (None if cc_us is None else {"us": round(cc_us, 2), "components": cc_n}),
             "build_rois": (None if rois_us is None else
                            {"us": round(rois_us, 2), "objects": int(objs_d.shape[0])}),
             "scatter_bev": (None if bev_us is None else
@@ -504,6 +518,8 @@ def main():
     ap.add_argument("--build-rois", action="store_true",
                     help="build every frame's ROI table on the device from previous-frame "
                          "objects (Sec. IV-C) as part of the step")
+    ap.add_argument("--components", action="store_true",
+                    help="also time the voxel-grid connected-component proposer on the outputs")
     ap.add_argument("--bev", action="store_true",
                     help="add ScatterToBEV (a dense [F, nz*5, ny, nx] canvas) to every step")
     ap.add_argument("--frames", type=int, default=FRAMES,

@@ -91,6 +91,7 @@ typedef enum mmbev_status {
 #define MMBEV_DEV_TABLE_FULL   0x1u  /* a voxel key found no free slot */
 #define MMBEV_DEV_WAIT_TIMEOUT 0x2u  /* an internal inter-block wait gave up */
 #define MMBEV_DEV_BOUNDS       0x4u  /* an internal index failed its bounds check */
+#define MMBEV_DEV_UNSORTED     0x8u  /* components: a frame's rows do not ascend by linear index */
 
 /* Limits of one call. */
 #define MMBEV_MAX_SWEEPS          2048
@@ -335,6 +336,43 @@ typedef struct {
 int mmbev_build_rois(const mmbev_object_t *objects, const int32_t *frame_obj_offsets,
                      int32_t num_frames, const mmbev_crit_params_t *params,
                      mmbev_roi_t *out_rois, int32_t *out_flags, cudaStream_t stream);
+
+/*
+ * Voxel-grid connected components (the object-cluster proposer of the
+ * paper's robot deployment): the kept voxels of each frame joined under
+ * 26-connectivity (voxels sharing a face, an edge or a corner).
+ *   coords, nvox  device, a voxelize call's outputs ([F*max_voxels][3] (z, y,
+ *               x) int32, [F] int32); rows >= nvox[f] are ignored. A frame's
+ *               rows must ascend by linear index (as voxelize writes them;
+ *               else MMBEV_DEV_UNSORTED is set and the labels are undefined).
+ *   dims        host (nx, ny, nz).
+ *   table, table_bytes  only when max_voxels > 262,144 (else ignored, may
+ *               be NULL): the caller's all-zero device buffer, 16-byte
+ *               aligned, of at least mmbev_components_table_size(F,
+ *               max_voxels) bytes (else MMBEV_EWORKSPACE): per frame a hash
+ *               region of 8-byte slots, then 4 bytes of scratch per row. All
+ *               zero again when the work completes.
+ *   out_labels  device int32 [F*max_voxels]: for each kept row, the row
+ *               (within its frame) of its component's root, the smallest
+ *               row of the component; -1 for rows >= nvox[f] and rows whose
+ *               coordinates lie outside the grid.
+ *   out_comp    device int32 [F*max_voxels][7] or NULL: at each root row the
+ *               component's voxel count and bounding box (zmin, ymin, xmin,
+ *               zmax, ymax, xmax); other rows are unspecified.
+ *   out_ncomp   device int32 [F]: components per frame.
+ *   out_status  device uint32 or NULL: MMBEV_DEV_* bits, reset by the call.
+ * mmbev_components_table_size returns that table size: 0 when no table is
+ * needed, and for sizes out of range; max_voxels <= 2^28. With max_voxels <=
+ * 262,144 the work is one launch of one thread-block cluster per frame (the
+ * frame's union-find in the cluster's shared memory, neighbours found by
+ * the rows' order), else five launches over a frame grid.
+ * Asynchronous on `stream`.
+ */
+size_t mmbev_components_table_size(int32_t num_frames, int32_t max_voxels);
+int mmbev_voxel_components(const int32_t *coords, const int32_t *nvox, int32_t num_frames,
+                           int32_t max_voxels, const int32_t dims[3], void *table,
+                           size_t table_bytes, int32_t *out_labels, int32_t *out_comp,
+                           int32_t *out_ncomp, uint32_t *out_status, cudaStream_t stream);
 
 /*
  * ScatterToBEV (Alg. 1, last step): the voxel features of F frames written

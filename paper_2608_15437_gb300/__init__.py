@@ -61,6 +61,10 @@ def load():
     batched = vox + [i32, P, P, P, P, P, P, P, sz, P, sz, P]
     lib.mmbev_voxelize_roi_batched.argtypes = batched
     lib.mmbev_voxelize_roi_batched.restype = ctypes.c_int
+    lib.mmbev_components_table_size.argtypes = [i32, i32]
+    lib.mmbev_components_table_size.restype = sz
+    lib.mmbev_voxel_components.argtypes = [P, P, i32, i32, P, P, ctypes.c_size_t, P, P, P, P, P]
+    lib.mmbev_voxel_components.restype = ctypes.c_int
     lib.mmbev_build_rois.argtypes = [P, P, i32, P, P, P, P]
     lib.mmbev_build_rois.restype = ctypes.c_int
     lib.mmbev_scatter_bev.argtypes = [P, P, P, i32, i32, P, P, ctypes.c_size_t, P]
@@ -317,6 +321,37 @@ def classify_points(points: torch.Tensor, sweep_offsets, sweep_tf: torch.Tensor,
 CRIT_FIELDS = ("v_ego", "dt", "a_brake", "d_min", "theta_max_deg", "theta_min_deg", "v_wide",
                "v_narrow", "tau_vru", "tau_motor", "r_coll")
 CLS_MOTOR, CLS_VRU, CLS_STATIC = 0, 1, 2
+
+
+def components_table_bytes(num_frames: int, max_voxels: int) -> int:
+    """Bytes of all-zero table ``voxel_components`` needs (0: none, as for
+    every cap up to 262,144 voxels a frame)."""
+    return int(load().mmbev_components_table_size(int(num_frames), int(max_voxels)))
+
+
+def voxel_components(out: "Outputs", max_voxels: int, dims, table: torch.Tensor | None = None,
+                     stream=None):
+    """Connected components of the kept voxels (``mmbev_voxel_components``,
+    26-connectivity). table: None when ``components_table_bytes`` is 0, else
+    an all-zero uint8 device buffer of at least that size. Returns (labels [F*max_voxels] int32: the frame-local root row, -1
+    for unused rows; comp [F*max_voxels, 7] int32: size and box at root rows;
+    ncomp [F] int32; status [1] uint32)."""
+    lib = load()
+    nf = out.nvox.numel()
+    dev = out.coords.device
+    rows = max(nf * int(max_voxels), 1)
+    labels = torch.empty(rows, dtype=torch.int32, device=dev)
+    comp = torch.empty((rows, 7), dtype=torch.int32, device=dev)
+    ncomp = torch.empty(max(nf, 1), dtype=torch.int32, device=dev)
+    status = torch.zeros(1, dtype=torch.int32, device=dev)
+    d = np.asarray([int(x) for x in dims], np.int32)
+    rc = lib.mmbev_voxel_components(_dptr(out.coords), _dptr(out.nvox), nf, int(max_voxels),
+                                    _hptr(d), _dptr(table, torch.uint8, "table"),
+                                    0 if table is None else table.numel(),
+                                    _dptr(labels), _dptr(comp), _dptr(ncomp), _dptr(status),
+                                    _stream(stream))
+    _check(rc, "mmbev_voxel_components")
+    return labels, comp, ncomp[:nf], status
 
 
 def pack_objects(objects: torch.Tensor) -> torch.Tensor:

@@ -144,3 +144,31 @@ def test_workspace_size_is_monotone_in_the_roi_count(mmbev_lib):
     sizes = [mmbev_lib.workspace_size(20000, r, 16000, 4, TINY_VS, TINY_RG)
              for r in (1, 32, 33, 64, 128, 129, 512, 1024)]
     assert sizes == sorted(sizes)
+
+
+def test_voxel_components_checks_the_table(mmbev_lib):
+    lib = mmbev_lib.load()
+    P = ctypes.c_void_p
+    fake = P(0x7e0000000000)
+    dims = np.asarray([512, 512, 1], np.int32)
+    # caps up to 8 x 32,768 rows take the cluster path: no table
+    assert lib.mmbev_components_table_size(2, 16000) == 0
+    assert lib.mmbev_components_table_size(1, 262144) == 0
+    # larger caps: per frame 2^k >= 4 * cap slots of 8 bytes, then the scratch
+    maxv = 300000
+    H = 1 << 21
+    need = 2 * H * 8 + 4 * 2 * maxv
+    assert lib.mmbev_components_table_size(2, maxv) == need
+    assert lib.mmbev_components_table_size(-1, 10) == 0
+    assert lib.mmbev_components_table_size(1, (1 << 28) + 1) == 0
+    args = (fake, fake, 2, maxv, dims.ctypes.data_as(P))
+    tail = (fake, fake, fake, None, None)
+    assert lib.mmbev_voxel_components(*args, P(0x7f1000000000), need - 4, *tail) == -3
+    assert lib.mmbev_voxel_components(*args, P(0x7f1000000008), need, *tail) == -1
+    assert lib.mmbev_voxel_components(*args, None, need, *tail) == -1
+    bad = np.asarray([512, 512, 0], np.int32)
+    assert lib.mmbev_voxel_components(fake, fake, 2, 16000, bad.ctypes.data_as(P),
+                                      None, 0, *tail) == -1
+    assert lib.mmbev_voxel_components(fake, fake, 2, (1 << 28) + 1, dims.ctypes.data_as(P),
+                                      None, 0, *tail) == -1
+

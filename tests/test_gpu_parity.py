@@ -513,3 +513,120 @@ def test_built_rois_drive_the_voxelization(oracle_mod, mmbev_lib, cuda_dev):
     got = [out.frame(f, w.max_voxels) for f in range(2)]
     want = run_oracle(oracle_mod, w)
     assert assert_frames_equal(got, want, "built rois") == 1.0
+
+
+# ------------------------------------------------------------------ voxel-grid components (proposer)
+
+def _components_case(name):
+    """(workload, per-frame voxel cap) of a components parity case."""
+    if name == "tiny":
+        return synth.tiny(0), None
+    if name == "nuscenes":
+        return synth.nuscenes_frame(1), None
+    if name == "two_frames":
+        return synth.concat_frames([synth.nuscenes_frame(s) for s in (1, 2)], "two"), None
+    if name == "with_empty":   # a frame with no ROI (no kept voxel) between two
+        return synth.concat_frames([synth.nuscenes_frame(1), synth.roi_coverage(0),
+                                    synth.tiny(3)], "with_empty"), None
+    if name == "multi_launch":   # a cap above 8 x 40,960 rows: the five-launch path
+        return synth.concat_frames([synth.tiny(0), synth.tiny(5)], "two_tiny"), 400_000
+    if name == "batch32":   # the full 32-frame batch, as the bench times it
+        return synth.streaming_batch(32), None
+    raise KeyError(name)
+
+
+@pytest.mark.gpu
+@pytest.mark.parametrize("name", ["tiny", "nuscenes", "two_frames", "with_empty", "multi_launch",
+                                  "batch32"])
+def test_voxel_components_parity(oracle_mod, mmbev_lib, cuda_dev, name):
+    import torch
+    w, maxv = _components_case(name)
+    maxv = w.max_voxels if maxv is None else maxv
+    pts, tf, rois = to_dev(w, cuda_dev)
+    vx = mmbev_lib.Voxelizer(w.num_points, int(np.max(np.diff(w.frame_roi_offsets))), maxv,
+                             w.num_frames, w.voxel_size, w.pc_range, w.max_pts_per_voxel,
+                             w.roi_margin, device=cuda_dev)
+    out = vx(pts, w.sweep_offsets, tf, rois, w.frame_sweep_offsets, w.frame_roi_offsets)
+    dims = oracle_mod.grid_dims(w.voxel_size, w.pc_range)
+    need = mmbev_lib.components_table_bytes(w.num_frames, maxv)
+    table = torch.zeros(need, dtype=torch.uint8, device=cuda_dev) if need else None
+    # twice on the same table: the first call must leave it all-zero
+    for _ in range(2):
+        labels, comp, ncomp, status = mmbev_lib.voxel_components(out, maxv, dims, table)
+        torch.cuda.synchronize(cuda_dev)
+        assert int(status.item()) == 0
+        assert table is None or _table_is_clean(table)
+    want = oracle_mod.voxel_components(run_oracle(oracle_mod, w, maxv=maxv), dims)
+    labels, comp, ncomp = labels.cpu().numpy(), comp.cpu().numpy(), ncomp.cpu().numpy()
+    nvox = out.nvox.cpu().numpy()
+    for f, (wl, wc) in enumerate(want):
+        r0 = f * maxv
+        assert nvox[f] == len(wl)
+        assert np.array_equal(labels[r0:r0 + nvox[f]], wl)
+        assert np.all(labels[r0 + nvox[f]:r0 + maxv] == -1)
+        assert ncomp[f] == len(wc)
+        got = np.concatenate([wc[:, :1], comp[r0 + wc[:, 0]]], axis=1)
+        assert np.array_equal(got, wc)
+
+
+class _CoordsOut:
+    """The two fields of a voxelize output that voxel_components reads."""
+    def __init__(self, coords, nvox):
+        self.coords, self.nvox = coords, nvox
+
+
+@pytest.mark.gpu
+def test_voxel_components_dense_blocks(oracle_mod, mmbev_lib, cuda_dev):
+    """Solid blocks of voxels, rows in ascending index: every voxel has all 13
+    earlier neighbours, and every CTA of the frame's cluster starts inside a
+    block, so many pairs reach the previous CTA; plus isolated voxels and two
+    blocks that touch only at a corner."""
+    import torch
+    dims = (1440, 1440, 40)   # (nx, ny, nz)
+    cells = set()
+    for z in range(2, 18):
+        for y in range(100, 130):
+            for x in range(200, 230):
+                cells.add((z, y, x))
+    for z in range(18, 22):   # a second block meeting the first at one corner
+        for y in range(130, 140):
+            for x in range(230, 240):
+                cells.add((z, y, x))
+    rng = np.random.default_rng(11)
+    for _ in range(300):   # scattered voxels, mostly isolated
+        cells.add((int(rng.integers(0, 40)), int(rng.integers(0, 1440)), int(rng.integers(0, 1440))))
+    nx, ny, nz = dims
+    coords = np.array(sorted(cells, key=lambda c: (c[0] * ny + c[1]) * nx + c[2]), np.int32)
+    nv, maxv = len(coords), 20000
+    assert nv <= maxv
+    cbuf = np.zeros((maxv, 3), np.int32)
+    cbuf[:nv] = coords
+    out = _CoordsOut(torch.from_numpy(cbuf).to(cuda_dev),
+                     torch.tensor([nv], dtype=torch.int32, device=cuda_dev))
+    assert mmbev_lib.components_table_bytes(1, maxv) == 0   # the cluster path: no table
+    labels, comp, ncomp, status = mmbev_lib.voxel_components(out, maxv, dims)
+    torch.cuda.synchronize(cuda_dev)
+    assert int(status.item()) == 0
+    (wl, wc), = oracle_mod.voxel_components([(None, coords, None)], dims)
+    labels = labels.cpu().numpy()
+    assert np.array_equal(labels[:nv], wl)
+    assert np.all(labels[nv:] == -1)
+    assert int(ncomp.cpu()[0]) == len(wc)
+    got = np.concatenate([wc[:, :1], comp.cpu().numpy()[wc[:, 0]]], axis=1)
+    assert np.array_equal(got, wc)
+    # the two blocks are one component (corner contact is 26-connected)
+    row = {tuple(c): i for i, c in enumerate(coords.tolist())}
+    assert labels[row[(2, 100, 200)]] == labels[row[(21, 139, 239)]]
+    assert np.sum(labels[:nv] == labels[row[(2, 100, 200)]]) >= 30 * 30 * 16 + 4 * 10 * 10
+
+
+@pytest.mark.gpu
+def test_voxel_components_flags_unsorted_rows(mmbev_lib, cuda_dev):
+    """Rows that do not ascend by linear index set MMBEV_DEV_UNSORTED."""
+    import torch
+    cbuf = np.array([[0, 0, 5], [0, 0, 2], [0, 0, 3], [0, 0, 0]], np.int32)
+    out = _CoordsOut(torch.from_numpy(cbuf).to(cuda_dev),
+                     torch.tensor([3], dtype=torch.int32, device=cuda_dev))
+    _, _, _, status = mmbev_lib.voxel_components(out, 4, (8, 8, 1))
+    torch.cuda.synchronize(cuda_dev)
+    assert int(status.item()) & 0x8
