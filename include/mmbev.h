@@ -339,7 +339,7 @@ int mmbev_build_rois(const mmbev_object_t *objects, const int32_t *frame_obj_off
 
 /*
  * Voxel-grid connected components (the object-cluster proposer of the
- * paper's robot deployment): the kept voxels of each frame joined under
+ * paper's robot deployment, Sec. VI-F): the kept voxels of each frame joined under
  * 26-connectivity (voxels sharing a face, an edge or a corner).
  *   coords, nvox  device, a voxelize call's outputs ([F*max_voxels][3] (z, y,
  *               x) int32, [F] int32); rows >= nvox[f] are ignored. A frame's

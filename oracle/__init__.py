@@ -214,7 +214,8 @@ def crit_thresholds(params):
 def voxel_components(frames, dims):
     """Connected components of each frame's kept voxels under 26-connectivity
     (voxels sharing a face, an edge or a corner): the voxel-grid proposer of
-    the paper's robot deployment, written out with a dict and union-find.
+    the paper's robot deployment (Sec. VI-F), written out with a dict and
+    union-find.
     Each voxel's label is the smallest output row (within its frame) of its
     component. Returns per frame (labels [n], components [k, 8] rows of
     (label, size, zmin, ymin, xmin, zmax, ymax, xmax) sorted by label)."""

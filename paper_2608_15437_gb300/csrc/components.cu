@@ -1,5 +1,6 @@
 // Voxel-grid connected components (the proposer of the paper's robot
-// deployment): occupied voxels of each frame joined under 26-connectivity.
+// deployment, Sec. VI-F): occupied voxels of each frame joined under
+// 26-connectivity.
 //
 // Union-find over each frame's kept rows. Rows ascend by linear index within
 // a frame, so a voxel's neighbours with smaller rows are the 13 with a

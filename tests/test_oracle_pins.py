@@ -784,3 +784,35 @@ def test_component_sizes_sum_to_the_voxels(oracle_mod):
     assert comp[:, 1].sum() == len(out[1])
     assert np.all(labels[comp[:, 0]] == comp[:, 0])   # roots label themselves
     assert np.all(labels <= np.arange(len(labels)))
+
+
+@pytest.mark.parametrize("density", [0.05, 0.2, 0.45])
+def test_components_match_textbook_26_connected_labelling(oracle_mod, density):
+    """The partition, sizes and boxes equal scipy.ndimage.label with a full
+    3x3x3 structuring element (26-connectivity) on a small dense grid."""
+    ndimage = pytest.importorskip("scipy.ndimage")
+    rng = np.random.default_rng(int(density * 100))
+    nz, ny, nx = 6, 14, 17
+    occ = rng.random((nz, ny, nx)) < density
+    zs, ys, xs = np.nonzero(occ)                       # ascending linear index
+    coords = np.stack([zs, ys, xs], 1).astype(np.int32)
+    perm = rng.permutation(len(coords))                # rows in any order
+    coords = coords[perm]
+    labels, comp = _cc(oracle_mod, coords, dims=(nx, ny, nz))
+    ref, nref = ndimage.label(occ, structure=np.ones((3, 3, 3), bool))
+    ref_of_row = ref[coords[:, 0], coords[:, 1], coords[:, 2]]
+    assert len(comp) == nref
+    # same partition: the map oracle label -> scipy label is a bijection
+    pairs = set(zip(labels.tolist(), ref_of_row.tolist()))
+    assert len(pairs) == nref
+    assert len({p[0] for p in pairs}) == nref and len({p[1] for p in pairs}) == nref
+    # each label is the smallest row of its component
+    for lab in np.unique(labels):
+        assert lab == np.min(np.nonzero(labels == lab)[0])
+    # sizes and bounding boxes
+    for row in comp:
+        lab, size = int(row[0]), int(row[1])
+        r = ref_of_row[lab]
+        cz, cy, cx = np.nonzero(ref == r)
+        assert size == len(cz)
+        assert row[2:].tolist() == [cz.min(), cy.min(), cx.min(), cz.max(), cy.max(), cx.max()]
