@@ -399,18 +399,16 @@ def run_gpu(args):
 
 
     # end to end through the public API: pinned host inputs, H2D, the call,
-    # D2H of the per-frame counts and the kept rows
+    # then every frame's kept rows packed by the device straight into a
+    # pinned host buffer (offsets and 36-byte records), and one sync
     h_pts = torch.from_numpy(w.points).pin_memory()
     h_tf = torch.from_numpy(w.sweep_tf).pin_memory()
     h_rois = torch.from_numpy(w.rois).pin_memory()
     d_pts = torch.empty_like(pts)
     d_tf = torch.empty_like(tf)
     d_rois = torch.empty_like(rois)
-    h_nvox = torch.empty(w.num_frames, dtype=torch.int32).pin_memory()
-    mv = w.max_voxels
-    h_feats = torch.empty((w.num_frames * mv, 5), dtype=torch.float32).pin_memory()
-    h_coords = torch.empty((w.num_frames * mv, 3), dtype=torch.int32).pin_memory()
-    h_counts = torch.empty(w.num_frames * mv, dtype=torch.int32).pin_memory()
+    h_packed = torch.empty(mmbev.pack_bytes(w.num_frames, w.max_voxels),
+                           dtype=torch.uint8).pin_memory()
     e2e_steps = max(3, min(args.steps, 10))
     d2h_bytes = 0
 
@@ -419,27 +417,19 @@ def run_gpu(args):
 
     def e2e_step():
         nonlocal d2h_bytes
-        d_pts.copy_(h_pts, non_blocking=True)
-        d_tf.copy_(h_tf, non_blocking=True)
-        if d_objs is None:
-            d_rois.copy_(h_rois, non_blocking=True)
-            rl = d_rois
+        if d_objs is None:   # host inputs: chunks go up while earlier ones are voxelized
+            out = vx.run_host(h_pts, w.sweep_offsets, h_tf, h_rois, w.frame_sweep_offsets,
+                              roi_off, chunk_frames=args.e2e_chunk)
         else:   # the previous frame's objects go up; the ROI table is built on the device
+            d_pts.copy_(h_pts, non_blocking=True)
+            d_tf.copy_(h_tf, non_blocking=True)
             d_objs.copy_(h_objs, non_blocking=True)
             rl = mmbev.build_rois(d_objs, obj_off, crit, out=rois_buf)[0]
-        out = vx(d_pts, w.sweep_offsets, d_tf, rl, w.frame_sweep_offsets, roi_off)
-        h_nvox.copy_(out.nvox, non_blocking=True)
+            out = vx(d_pts, w.sweep_offsets, d_tf, rl, w.frame_sweep_offsets, roi_off)
+        mmbev.pack_voxels(out, w.max_voxels, h_packed)
         torch.cuda.current_stream(dev).synchronize()
-        nb = 0
-        for f in range(w.num_frames):
-            n = int(h_nvox[f])
-            r0 = f * mv
-            h_feats[r0:r0 + n].copy_(out.feats[r0:r0 + n], non_blocking=True)
-            h_coords[r0:r0 + n].copy_(out.coords[r0:r0 + n], non_blocking=True)
-            h_counts[r0:r0 + n].copy_(out.counts[r0:r0 + n], non_blocking=True)
-            nb += n * BYTES_PER_VOXEL
-        torch.cuda.current_stream(dev).synchronize()
-        d2h_bytes = nb + 4 * w.num_frames
+        total = int(h_packed[4 * w.num_frames:4 * w.num_frames + 4].view(torch.int32)[0])
+        d2h_bytes = 4 * (w.num_frames + 1) + BYTES_PER_VOXEL * total
 
     e2e_step()
     if world > 1:
@@ -518,6 +508,8 @@ def main():
     ap.add_argument("--build-rois", action="store_true",
                     help="build every frame's ROI table on the device from previous-frame "
                          "objects (Sec. IV-C) as part of the step")
+    ap.add_argument("--e2e-chunk", type=int, default=8,
+                    help="frames per host-to-device chunk in the end-to-end leg")
     ap.add_argument("--components", action="store_true",
                     help="also time the voxel-grid connected-component proposer on the outputs")
     ap.add_argument("--bev", action="store_true",

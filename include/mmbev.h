@@ -236,6 +236,33 @@ typedef struct mmbev_exec_opts {
     uint64_t seed;
 } mmbev_exec_opts_t;
 
+/*
+ * The batched call with its inputs in host memory (pinned, for the copies
+ * to overlap): frames go up in chunks of chunk_frames on copy_stream, and
+ * each chunk is voxelized on `stream` as soon as its copy has landed, so the
+ * transfers of later chunks overlap the work on earlier ones. The results
+ * are those of mmbev_voxelize_roi_batched_ex on the same inputs (frames are
+ * independent; the draws of opts->rho_out use frame-local indices).
+ *   h_points, h_sweep_tf, h_rois  host, as points, sweep_tf, rois above.
+ *   d_points, d_sweep_tf, d_rois  device staging of the same sizes, written
+ *               by the call.
+ *   sweep_offsets, frame_*_offsets  host, as above; checked before any copy.
+ *   chunk_frames  frames a chunk (>= 1).
+ *   copy_stream  the stream of the copies (the call's own `stream` makes it
+ *               serial).
+ * Everything else as mmbev_voxelize_roi_batched_ex; opts->stage_events must
+ * be NULL. The workspace status accumulates over the chunks.
+ */
+int mmbev_voxelize_roi_batched_host(
+    const float *h_points, const int64_t *sweep_offsets, int32_t num_sweeps,
+    const float *h_sweep_tf, const mmbev_roi_t *h_rois, int32_t num_rois, float roi_margin,
+    const float voxel_size[3], const float range[6], int32_t max_pts_per_voxel,
+    int32_t max_voxels, int32_t num_frames, const int32_t *frame_sweep_offsets,
+    const int32_t *frame_roi_offsets, float *d_points, float *d_sweep_tf, mmbev_roi_t *d_rois,
+    float *out_feats, int32_t *out_coords, int32_t *out_counts, int32_t *out_nvox, void *table,
+    size_t table_bytes, void *workspace, size_t workspace_bytes, int32_t chunk_frames,
+    cudaStream_t stream, cudaStream_t copy_stream, const mmbev_exec_opts_t *opts);
+
 int mmbev_voxelize_roi_batched_ex(const float *points, const int64_t *sweep_offsets,
                                   int32_t num_sweeps, const float *sweep_tf,
                                   const mmbev_roi_t *rois, int32_t num_rois,
@@ -373,6 +400,26 @@ int mmbev_voxel_components(const int32_t *coords, const int32_t *nvox, int32_t n
                            int32_t max_voxels, const int32_t dims[3], void *table,
                            size_t table_bytes, int32_t *out_labels, int32_t *out_comp,
                            int32_t *out_ncomp, uint32_t *out_status, cudaStream_t stream);
+
+/*
+ * Packing of a voxelize call's outputs for the host: every frame's kept rows
+ * [0, nvox[f]) gathered, frame after frame, into one contiguous buffer, so
+ * the result crosses to the host in one transfer (or, with dst in pinned
+ * host memory, is written there by the device directly).
+ *   feats, coords, counts, nvox  device, a voxelize call's outputs (frame f's
+ *               rows start at f*max_voxels).
+ *   dst, dst_bytes  device memory or pinned host memory, 4-byte aligned, at
+ *               least mmbev_pack_size(F, max_voxels) bytes (else
+ *               MMBEV_EWORKSPACE): int32 off[F+1] (off[f] = the first record
+ *               of frame f, off[F] = the total T), then T records of nine
+ *               4-byte words: the five fp32 means, then z, y, x and the point
+ *               count as int32.
+ * Asynchronous on `stream`; one kernel.
+ */
+size_t mmbev_pack_size(int32_t num_frames, int32_t max_voxels);
+int mmbev_pack_voxels(const float *feats, const int32_t *coords, const int32_t *counts,
+                      const int32_t *nvox, int32_t num_frames, int32_t max_voxels, void *dst,
+                      size_t dst_bytes, cudaStream_t stream);
 
 /*
  * ScatterToBEV (Alg. 1, last step): the voxel features of F frames written

@@ -61,6 +61,10 @@ def load():
     batched = vox + [i32, P, P, P, P, P, P, P, sz, P, sz, P]
     lib.mmbev_voxelize_roi_batched.argtypes = batched
     lib.mmbev_voxelize_roi_batched.restype = ctypes.c_int
+    lib.mmbev_pack_size.argtypes = [i32, i32]
+    lib.mmbev_pack_size.restype = sz
+    lib.mmbev_pack_voxels.argtypes = [P, P, P, P, i32, i32, P, sz, P]
+    lib.mmbev_pack_voxels.restype = ctypes.c_int
     lib.mmbev_components_table_size.argtypes = [i32, i32]
     lib.mmbev_components_table_size.restype = sz
     lib.mmbev_voxel_components.argtypes = [P, P, i32, i32, P, P, ctypes.c_size_t, P, P, P, P, P]
@@ -71,6 +75,10 @@ def load():
     lib.mmbev_scatter_bev.restype = ctypes.c_int
     lib.mmbev_voxelize_roi_batched_ex.argtypes = batched + [ctypes.POINTER(_ExecOpts)]
     lib.mmbev_voxelize_roi_batched_ex.restype = ctypes.c_int
+    lib.mmbev_voxelize_roi_batched_host.argtypes = (
+        [P, P, i32, P, P, i32, f32, P, P, i32, i32, i32, P, P, P, P, P, P, P, P, P, P, sz, P, sz,
+         i32, P, P, ctypes.POINTER(_ExecOpts)])
+    lib.mmbev_voxelize_roi_batched_host.restype = ctypes.c_int
     lib.mmbev_classify_points.argtypes = [P, P, i32, P, P, i32, f32, P, P, i32, P, P,
                                           P, P, P, P, sz, P]
     lib.mmbev_classify_points.restype = ctypes.c_int
@@ -323,6 +331,38 @@ CRIT_FIELDS = ("v_ego", "dt", "a_brake", "d_min", "theta_max_deg", "theta_min_de
 CLS_MOTOR, CLS_VRU, CLS_STATIC = 0, 1, 2
 
 
+def pack_bytes(num_frames: int, max_voxels: int) -> int:
+    """Bytes ``pack_voxels`` may write for this batch shape."""
+    return int(load().mmbev_pack_size(int(num_frames), int(max_voxels)))
+
+
+def pack_voxels(out: "Outputs", max_voxels: int, dst: torch.Tensor, stream=None) -> None:
+    """Gather every frame's kept rows into dst (``mmbev_pack_voxels``): a
+    uint8 tensor of at least ``pack_bytes`` bytes, on the device or in pinned
+    host memory (the device then writes it directly). Read it back with
+    ``unpack``."""
+    lib = load()
+    nf = out.nvox.numel()
+    if dst.dtype != torch.uint8 or not dst.is_contiguous():
+        raise ValueError("dst must be a contiguous uint8 tensor")
+    if not dst.is_cuda and not dst.is_pinned():
+        raise ValueError("dst must be on the device or in pinned host memory")
+    rc = lib.mmbev_pack_voxels(_dptr(out.feats), _dptr(out.coords), _dptr(out.counts),
+                               _dptr(out.nvox), nf, int(max_voxels),
+                               ctypes.c_void_p(dst.data_ptr()), dst.numel(), _stream(stream))
+    _check(rc, "mmbev_pack_voxels")
+
+
+def unpack(dst: torch.Tensor, num_frames: int):
+    """Views of a packed buffer: (off [F+1] int32, feats [T,5] fp32, coords
+    [T,3] int32, counts [T] int32)."""
+    words = dst.view(torch.int32)
+    off = words[:num_frames + 1]
+    total = int(off[-1])
+    rec = words[num_frames + 1:num_frames + 1 + 9 * total].view(total, 9)
+    return off, rec[:, :5].view(torch.float32), rec[:, 5:8], rec[:, 8]
+
+
 def components_table_bytes(num_frames: int, max_voxels: int) -> int:
     """Bytes of all-zero table ``voxel_components`` needs (0: none, as for
     every cap up to 262,144 voxels a frame)."""
@@ -433,6 +473,45 @@ class Voxelizer:
                                     workspace=self.workspace, out=self.out, stream=stream,
                                     stage_events=stage_events, rho_out=self.rho_out,
                                     seed=self.seed)
+
+    def run_host(self, h_points: torch.Tensor, sweep_offsets, h_sweep_tf: torch.Tensor,
+                 h_rois: torch.Tensor, frame_sweep_offsets, frame_roi_offsets,
+                 chunk_frames: int = 8, stream=None) -> Outputs:
+        """The batched call on pinned host inputs
+        (``mmbev_voxelize_roi_batched_host``): chunks of ``chunk_frames``
+        frames go up on a side stream while earlier chunks are voxelized.
+        Device staging is allocated on first use and kept."""
+        lib = load()
+        so = _host(sweep_offsets, np.int64)
+        fso = _host(frame_sweep_offsets, np.int32)
+        fro = _host(frame_roi_offsets, np.int32)
+        for name, t in (("h_points", h_points), ("h_sweep_tf", h_sweep_tf), ("h_rois", h_rois)):
+            if t.is_cuda or t.dtype != torch.float32 or not t.is_contiguous():
+                raise ValueError(f"{name} must be a contiguous float32 host tensor")
+        dev = self.out.nvox.device
+        need = (h_points.shape, h_sweep_tf.shape, h_rois.shape)
+        if getattr(self, "_staging_shape", None) != need:
+            self._staging = tuple(torch.empty(sh, dtype=torch.float32, device=dev) for sh in need)
+            self._staging_shape = need
+            self._copy_stream = torch.cuda.Stream(device=dev)
+        d_pts, d_tf, d_rois = self._staging
+        st = stream if stream is not None else torch.cuda.current_stream(dev)
+        # the staging buffers are reused across calls: copies of this call
+        # start after the previous work on `st` has read them
+        self._copy_stream.wait_stream(st)
+        opts = _ExecOpts(None, 0, float(self.rho_out), int(self.seed) & (2**64 - 1))
+        nr = h_rois.shape[0] if h_rois.dim() > 1 else h_rois.numel() // 5
+        rc = lib.mmbev_voxelize_roi_batched_host(
+            ctypes.c_void_p(h_points.data_ptr()), _hptr(so), len(so) - 1,
+            ctypes.c_void_p(h_sweep_tf.data_ptr()), ctypes.c_void_p(h_rois.data_ptr()), nr,
+            self.margin, _hptr(self.voxel_size), _hptr(self.pc_range), self.K, self.max_voxels,
+            len(fso) - 1, _hptr(fso), _hptr(fro), _dptr(d_pts), _dptr(d_tf), _dptr(d_rois),
+            _dptr(self.out.feats), _dptr(self.out.coords), _dptr(self.out.counts),
+            _dptr(self.out.nvox), _dptr(self.table), self.table.numel(), _dptr(self.workspace),
+            self.workspace.numel(), int(chunk_frames), _stream(st), _stream(self._copy_stream),
+            ctypes.byref(opts))
+        _check(rc, "mmbev_voxelize_roi_batched_host")
+        return self.out
 
     def status(self) -> int:
         return get_status(self.workspace)

@@ -5,6 +5,8 @@
 #include <cstring>
 #include <atomic>
 
+#include <vector>
+
 #include "mmbev_internal.cuh"
 
 namespace mmbev {
@@ -286,19 +288,24 @@ int mmbev_table_clear(void* table, size_t table_bytes, cudaStream_t stream) {
     return launch_zero(table, table_bytes, stream) == cudaSuccess ? MMBEV_OK : MMBEV_ECUDA;
 }
 
-int mmbev_voxelize_roi_batched_ex(const float* points, const int64_t* sweep_offsets,
-                                  int32_t num_sweeps, const float* sweep_tf,
-                                  const mmbev_roi_t* rois, int32_t num_rois, float roi_margin,
-                                  const float voxel_size[3], const float range[6],
-                                  int32_t max_pts_per_voxel, int32_t max_voxels,
-                                  int32_t num_frames, const int32_t* frame_sweep_offsets,
-                                  const int32_t* frame_roi_offsets, float* out_feats,
-                                  int32_t* out_coords, int32_t* out_counts, int32_t* out_nvox,
-                                  void* table, size_t table_bytes, void* workspace,
-                                  size_t workspace_bytes, cudaStream_t stream,
-                                  const mmbev_exec_opts_t* opts) {
+}  // extern "C"
+
+namespace {
+
+// The batched call; keep_status: leave the workspace's status word as it is
+// (the chunks after the first of a host-input call).
+int voxelize_batched(const float* points, const int64_t* sweep_offsets, int32_t num_sweeps,
+                     const float* sweep_tf, const mmbev_roi_t* rois, int32_t num_rois,
+                     float roi_margin, const float voxel_size[3], const float range[6],
+                     int32_t max_pts_per_voxel, int32_t max_voxels, int32_t num_frames,
+                     const int32_t* frame_sweep_offsets, const int32_t* frame_roi_offsets,
+                     float* out_feats, int32_t* out_coords, int32_t* out_counts,
+                     int32_t* out_nvox, void* table, size_t table_bytes, void* workspace,
+                     size_t workspace_bytes, cudaStream_t stream, const mmbev_exec_opts_t* opts,
+                     bool keep_status) {
     HostDesc desc;  // ~25 KB; consumed by the prep launch's parameter copy
     Params p;
+    p.keep_status = keep_status ? 1 : 0;
     Grid g;
     int32_t rmax = 0;
     if (max_pts_per_voxel < 1 || max_pts_per_voxel > kMaxK || max_voxels < 0) return MMBEV_EINVAL;
@@ -402,6 +409,111 @@ int mmbev_voxelize_roi_batched_ex(const float* points, const int64_t* sweep_offs
         if ((e = mark()) != cudaSuccess) break;
     } while (0);
     return e == cudaSuccess ? MMBEV_OK : MMBEV_ECUDA;
+}
+
+}  // namespace
+
+extern "C" {
+
+int mmbev_voxelize_roi_batched_ex(const float* points, const int64_t* sweep_offsets,
+                                  int32_t num_sweeps, const float* sweep_tf,
+                                  const mmbev_roi_t* rois, int32_t num_rois, float roi_margin,
+                                  const float voxel_size[3], const float range[6],
+                                  int32_t max_pts_per_voxel, int32_t max_voxels,
+                                  int32_t num_frames, const int32_t* frame_sweep_offsets,
+                                  const int32_t* frame_roi_offsets, float* out_feats,
+                                  int32_t* out_coords, int32_t* out_counts, int32_t* out_nvox,
+                                  void* table, size_t table_bytes, void* workspace,
+                                  size_t workspace_bytes, cudaStream_t stream,
+                                  const mmbev_exec_opts_t* opts) {
+    return voxelize_batched(points, sweep_offsets, num_sweeps, sweep_tf, rois, num_rois,
+                            roi_margin, voxel_size, range, max_pts_per_voxel, max_voxels,
+                            num_frames, frame_sweep_offsets, frame_roi_offsets, out_feats,
+                            out_coords, out_counts, out_nvox, table, table_bytes, workspace,
+                            workspace_bytes, stream, opts, false);
+}
+
+int mmbev_voxelize_roi_batched_host(
+    const float* h_points, const int64_t* sweep_offsets, int32_t num_sweeps,
+    const float* h_sweep_tf, const mmbev_roi_t* h_rois, int32_t num_rois, float roi_margin,
+    const float voxel_size[3], const float range[6], int32_t max_pts_per_voxel,
+    int32_t max_voxels, int32_t num_frames, const int32_t* frame_sweep_offsets,
+    const int32_t* frame_roi_offsets, float* d_points, float* d_sweep_tf, mmbev_roi_t* d_rois,
+    float* out_feats, int32_t* out_coords, int32_t* out_counts, int32_t* out_nvox, void* table,
+    size_t table_bytes, void* workspace, size_t workspace_bytes, int32_t chunk_frames,
+    cudaStream_t stream, cudaStream_t copy_stream, const mmbev_exec_opts_t* opts) {
+    if (num_frames < 1 || num_frames > kMaxFrames || chunk_frames < 1) return MMBEV_EINVAL;
+    if (num_sweeps < 0 || num_sweeps > kMaxSweeps || num_rois < 0) return MMBEV_EINVAL;
+    if (!out_nvox) return MMBEV_EINVAL;
+    if (!sweep_offsets || !frame_sweep_offsets || !frame_roi_offsets) return MMBEV_EINVAL;
+    if (opts && opts->stage_events) return MMBEV_EINVAL;   // stage events need a single call
+    if (max_voxels < 0 || (int64_t)max_voxels * num_frames > 0x7FFFFFFFll) return MMBEV_EINVAL;
+    // the offsets this entry slices by: checked before any copy
+    if (frame_sweep_offsets[0] != 0 || frame_sweep_offsets[num_frames] != num_sweeps ||
+        frame_roi_offsets[0] != 0 || frame_roi_offsets[num_frames] != num_rois ||
+        sweep_offsets[0] != 0)
+        return MMBEV_EINVAL;
+    for (int32_t f = 0; f < num_frames; ++f)
+        if (frame_sweep_offsets[f + 1] < frame_sweep_offsets[f] ||
+            frame_roi_offsets[f + 1] < frame_roi_offsets[f])
+            return MMBEV_EINVAL;
+    for (int32_t s = 0; s < num_sweeps; ++s)
+        if (sweep_offsets[s + 1] < sweep_offsets[s]) return MMBEV_EINVAL;
+    const int64_t n = sweep_offsets[num_sweeps];
+    if ((n > 0 && (!h_points || !d_points)) || (num_sweeps > 0 && (!h_sweep_tf || !d_sweep_tf)) ||
+        (num_rois > 0 && (!h_rois || !d_rois)))
+        return MMBEV_EINVAL;
+
+    const int32_t nchunks = (num_frames + chunk_frames - 1) / chunk_frames;
+    std::vector<cudaEvent_t> ev((size_t)nchunks, nullptr);
+    std::vector<int64_t> so;
+    std::vector<int32_t> fso, fro;
+    int rc = MMBEV_OK;
+    for (int32_t c = 0; c < nchunks && rc == MMBEV_OK; ++c) {
+        const int32_t f0 = c * chunk_frames, f1 = std::min(num_frames, f0 + chunk_frames);
+        const int32_t s0 = frame_sweep_offsets[f0], s1 = frame_sweep_offsets[f1];
+        const int32_t r0 = frame_roi_offsets[f0], r1 = frame_roi_offsets[f1];
+        const int64_t p0 = sweep_offsets[s0], p1 = sweep_offsets[s1];
+        // the chunk's inputs go up on the copy stream; the compute stream
+        // waits for them only
+        cudaError_t e = cudaEventCreateWithFlags(&ev[(size_t)c], cudaEventDisableTiming);
+        if (e == cudaSuccess && p1 > p0)
+            e = cudaMemcpyAsync(d_points + 5 * p0, h_points + 5 * p0,
+                                sizeof(float) * 5 * (size_t)(p1 - p0), cudaMemcpyHostToDevice,
+                                copy_stream);
+        if (e == cudaSuccess && s1 > s0)
+            e = cudaMemcpyAsync(d_sweep_tf + 16 * (size_t)s0, h_sweep_tf + 16 * (size_t)s0,
+                                sizeof(float) * 16 * (size_t)(s1 - s0), cudaMemcpyHostToDevice,
+                                copy_stream);
+        if (e == cudaSuccess && r1 > r0)
+            e = cudaMemcpyAsync(d_rois + r0, h_rois + r0, sizeof(mmbev_roi_t) * (size_t)(r1 - r0),
+                                cudaMemcpyHostToDevice, copy_stream);
+        if (e == cudaSuccess) e = cudaEventRecord(ev[(size_t)c], copy_stream);
+        if (e == cudaSuccess) e = cudaStreamWaitEvent(stream, ev[(size_t)c], 0);
+        if (e != cudaSuccess) {
+            rc = MMBEV_ECUDA;
+            break;
+        }
+        // the chunk's offsets, rebased (taken by value at launch)
+        so.assign(sweep_offsets + s0, sweep_offsets + s1 + 1);
+        for (int64_t& v : so) v -= p0;
+        fso.assign(frame_sweep_offsets + f0, frame_sweep_offsets + f1 + 1);
+        for (int32_t& v : fso) v -= s0;
+        fro.assign(frame_roi_offsets + f0, frame_roi_offsets + f1 + 1);
+        for (int32_t& v : fro) v -= r0;
+        const size_t row0 = (size_t)f0 * (size_t)max_voxels;
+        rc = voxelize_batched(
+            d_points ? d_points + 5 * p0 : nullptr, so.data(), s1 - s0,
+            d_sweep_tf ? d_sweep_tf + 16 * (size_t)s0 : nullptr, d_rois ? d_rois + r0 : nullptr,
+            r1 - r0, roi_margin, voxel_size, range, max_pts_per_voxel, max_voxels, f1 - f0,
+            fso.data(), fro.data(), out_feats ? out_feats + 5 * row0 : nullptr,
+            out_coords ? out_coords + 3 * row0 : nullptr,
+            out_counts ? out_counts + row0 : nullptr, out_nvox + f0, table, table_bytes,
+            workspace, workspace_bytes, stream, opts, c > 0);
+    }
+    for (cudaEvent_t x : ev)
+        if (x) cudaEventDestroy(x);   // released once the work recorded on it is done
+    return rc;
 }
 
 int mmbev_voxelize_roi_batched(const float* points, const int64_t* sweep_offsets,

@@ -118,6 +118,7 @@ struct Params {
     int32_t max_voxels;
     uint32_t rho_thr;       // keep a point inside no ROI when its draw's top 24 bits < rho_thr
     uint64_t seed;          // SplitMix64 seed of those draws
+    int32_t keep_status = 0;  // prep leaves the status word as it is (later chunks of a call)
     // bucket ordering
     int32_t bucket_log2;
     uint32_t buckets_per_frame;

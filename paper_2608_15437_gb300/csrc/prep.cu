@@ -104,7 +104,8 @@ k_prep(Params p, const __grid_constant__ HostDesc d) {
     const int nz = gridDim.x - p.num_frames;
     const size_t gt = (size_t)zb * blockDim.x + t;
     const size_t gs = (size_t)nz * blockDim.x;
-    if (gt < sizeof(Header) / 4) reinterpret_cast<uint32_t*>(p.hdr)[gt] = 0u;
+    if (gt < sizeof(Header) / 4 && !(gt == 0 && p.keep_status))   // word 0: the status
+        reinterpret_cast<uint32_t*>(p.hdr)[gt] = 0u;
     for (size_t i = gt; i <= (size_t)p.num_sweeps; i += gs) p.sweep_off[i] = d.sweep_off[i];
     for (size_t i = gt; i <= (size_t)p.num_frames; i += gs) {
         p.frame_sweep_off[i] = d.frame_sweep_off[i];

@@ -172,3 +172,45 @@ def test_voxel_components_checks_the_table(mmbev_lib):
     assert lib.mmbev_voxel_components(fake, fake, 2, (1 << 28) + 1, dims.ctypes.data_as(P),
                                       None, 0, *tail) == -1
 
+
+
+def test_pack_voxels_checks_its_arguments(mmbev_lib):
+    lib = mmbev_lib.load()
+    P = ctypes.c_void_p
+    fake = P(0x7e0000000000)
+    # off[F+1] then 36 bytes a row of the cap
+    assert lib.mmbev_pack_size(2, 1000) == 4 * 3 + 36 * 2 * 1000
+    assert lib.mmbev_pack_size(0, 1000) == 4
+    assert lib.mmbev_pack_size(-1, 10) == 0
+    need = lib.mmbev_pack_size(2, 1000)
+    args = (fake, fake, fake, fake, 2, 1000)
+    assert lib.mmbev_pack_voxels(*args, P(0x7f2000000000), need - 4, None) == -3
+    assert lib.mmbev_pack_voxels(*args, P(0x7f2000000002), need, None) == -1   # not 4-byte aligned
+    assert lib.mmbev_pack_voxels(*args, None, need, None) == -1
+    assert lib.mmbev_pack_voxels(fake, fake, fake, fake, -1, 1000, P(0x7f2000000000), need,
+                                 None) == -1
+
+
+def test_host_input_call_checks_offsets_before_copying(mmbev_lib):
+    lib = mmbev_lib.load()
+    P = ctypes.c_void_p
+    fake = P(0x7e0000000000)
+    vs = np.asarray([0.2, 0.2, 8.0], np.float32)
+    rg = np.asarray([-51.2, -51.2, -5.0, 51.2, 51.2, 3.0], np.float32)
+    so = np.asarray([0, 100, 250], np.int64)
+
+    def call(fso, fro, chunk=1, nsw=2, nroi=3, so=so):
+        fso = np.asarray(fso, np.int32)
+        fro = np.asarray(fro, np.int32)
+        return lib.mmbev_voxelize_roi_batched_host(
+            fake, so.ctypes.data_as(P), nsw, fake, fake, nroi, 0.5, vs.ctypes.data_as(P),
+            rg.ctypes.data_as(P), 10, 1000, len(fso) - 1, fso.ctypes.data_as(P),
+            fro.ctypes.data_as(P), fake, fake, fake, fake, fake, fake, fake, fake, 1 << 20, fake,
+            1 << 20, chunk, None, None, None)
+
+    assert call([0, 1, 2], [0, 1, 3], chunk=0) == -1           # chunk_frames < 1
+    assert call([1, 1, 2], [0, 1, 3]) == -1                     # frames must start at sweep 0
+    assert call([0, 1, 3], [0, 1, 3]) == -1                     # last frame past the sweeps
+    assert call([0, 2, 1], [0, 1, 3], nsw=1) == -1              # decreasing
+    assert call([0, 1, 2], [0, 2, 1], nroi=1) == -1             # decreasing ROI offsets
+    assert call([0, 1, 2], [0, 1, 3], so=np.asarray([0, 100, 50], np.int64)) == -1

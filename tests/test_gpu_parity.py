@@ -630,3 +630,74 @@ def test_voxel_components_flags_unsorted_rows(mmbev_lib, cuda_dev):
     _, _, _, status = mmbev_lib.voxel_components(out, 4, (8, 8, 1))
     torch.cuda.synchronize(cuda_dev)
     assert int(status.item()) & 0x8
+
+
+@pytest.mark.gpu
+@pytest.mark.parametrize("where", ["device", "pinned_host"])
+def test_pack_voxels_gathers_every_frame(mmbev_lib, cuda_dev, where):
+    """The packed buffer holds off[F+1] and every frame's kept rows in order,
+    bit for bit, whether it lives on the device or in pinned host memory."""
+    import torch
+    w = synth.concat_frames([synth.nuscenes_frame(1), synth.roi_coverage(0), synth.tiny(3),
+                             synth.nuscenes_frame(2)], "pack4")
+    pts, tf, rois = to_dev(w, cuda_dev)
+    vx = mmbev_lib.Voxelizer(w.num_points, int(np.max(np.diff(w.frame_roi_offsets))), w.max_voxels,
+                             w.num_frames, w.voxel_size, w.pc_range, w.max_pts_per_voxel,
+                             w.roi_margin, device=cuda_dev)
+    out = vx(pts, w.sweep_offsets, tf, rois, w.frame_sweep_offsets, w.frame_roi_offsets)
+    nbytes = mmbev_lib.pack_bytes(w.num_frames, w.max_voxels)
+    if where == "device":
+        dst = torch.full((nbytes,), 0xAB, dtype=torch.uint8, device=cuda_dev)
+    else:
+        dst = torch.full((nbytes,), 0xAB, dtype=torch.uint8).pin_memory()
+    mmbev_lib.pack_voxels(out, w.max_voxels, dst)
+    torch.cuda.synchronize(cuda_dev)
+    off, feats, coords, counts = mmbev_lib.unpack(dst.cpu() if dst.is_cuda else dst, w.num_frames)
+    off = off.numpy()
+    nvox = out.nvox.cpu().numpy()
+    assert off[0] == 0 and np.array_equal(np.diff(off), nvox)
+    assert nvox[1] == 0   # the frame with no ROI
+    for f in range(w.num_frames):
+        ef, ec, en = out.frame(f, w.max_voxels)
+        a, b = off[f], off[f + 1]
+        assert np.array_equal(feats[a:b].numpy().view(np.uint32), ef.view(np.uint32))
+        assert np.array_equal(coords[a:b].numpy(), ec)
+        assert np.array_equal(counts[a:b].numpy(), en)
+    # nothing written past the last record
+    tail = (dst.cpu() if dst.is_cuda else dst)[4 * (w.num_frames + 1) + 36 * int(off[-1]):]
+    assert bool((tail == 0xAB).all())
+
+
+@pytest.mark.gpu
+@pytest.mark.parametrize("chunk", [1, 3, 5, 8])
+@pytest.mark.parametrize("rho", [0.0, 0.3])
+def test_host_input_call_equals_device_input_call(mmbev_lib, cuda_dev, chunk, rho):
+    """mmbev_voxelize_roi_batched_host (pinned host inputs, chunked copies on
+    a side stream) gives exactly the outputs of the device-input call, for
+    chunk sizes that do and do not divide the frame count."""
+    import torch
+    w = synth.concat_frames([synth.nuscenes_frame(s) for s in (1, 2, 3)] + [synth.roi_coverage(0)]
+                            + [synth.tiny(s) for s in (4, 5)] + [synth.nuscenes_frame(6)],
+                            "seven")
+    pts, tf, rois = to_dev(w, cuda_dev)
+    rmax = int(np.max(np.diff(w.frame_roi_offsets)))
+    mk = lambda: mmbev_lib.Voxelizer(w.num_points, rmax, w.max_voxels, w.num_frames, w.voxel_size,
+                                     w.pc_range, w.max_pts_per_voxel, w.roi_margin,
+                                     device=cuda_dev, rho_out=rho, seed=9)
+    ref = mk()
+    want = ref(pts, w.sweep_offsets, tf, rois, w.frame_sweep_offsets, w.frame_roi_offsets)
+    vx = mk()
+    h_pts = torch.from_numpy(np.ascontiguousarray(w.points)).pin_memory()
+    h_tf = torch.from_numpy(np.ascontiguousarray(w.sweep_tf)).pin_memory()
+    h_rois = torch.from_numpy(np.ascontiguousarray(w.rois, np.float32).reshape(-1, 5)).pin_memory()
+    for _ in range(2):   # twice: the staging is reused
+        got = vx.run_host(h_pts, w.sweep_offsets, h_tf, h_rois, w.frame_sweep_offsets,
+                          w.frame_roi_offsets, chunk_frames=chunk)
+        torch.cuda.synchronize(cuda_dev)
+        assert vx.status() == 0
+        assert torch.equal(got.nvox, want.nvox)
+        for f in range(w.num_frames):
+            gf, gc, gn = got.frame(f, w.max_voxels)
+            ef, ec, en = want.frame(f, w.max_voxels)
+            assert np.array_equal(gf.view(np.uint32), ef.view(np.uint32))
+            assert np.array_equal(gc, ec) and np.array_equal(gn, en)
