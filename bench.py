@@ -307,13 +307,25 @@ def run_gpu(args):
     n_in_roi = int((lin >= 0).sum().item())
     del lin
 
+    # with --bev the outputs are double-buffered, so each step's scatter only
+    # clears the previous step's cells (the canvas then equals a full fill
+    # and scatter of the step's outputs)
+    bev_outs = [vx.out, mmbev.Outputs.empty(w.num_frames, w.max_voxels, dev)] if args.bev else None
+    bev_prev = [None]
+
     def step(**kw):
         rl = rois
         if objs_d is not None:
             rl = mmbev.build_rois(objs_d, obj_off, crit, out=rois_buf)[0]
+        if canvas is not None:
+            vx.out = bev_outs[1] if vx.out is bev_outs[0] else bev_outs[0]
         out = vx(pts, w.sweep_offsets, tf, rl, w.frame_sweep_offsets, roi_off, **kw)
         if canvas is not None:
-            mmbev.scatter_bev(out, w.max_voxels, dims, canvas=canvas)
+            if bev_prev[0] is None or args.bev_full:
+                mmbev.scatter_bev(out, w.max_voxels, dims, canvas=canvas)
+            else:
+                mmbev.scatter_bev_update(bev_prev[0], out, w.max_voxels, dims, canvas)
+            bev_prev[0] = out
         return out
     step_ev = [[torch.cuda.Event(enable_timing=True) for _ in range(nstage + 1)]
                for _ in range(args.steps)]
@@ -375,8 +387,8 @@ def run_gpu(args):
         torch.cuda.synchronize(dev)
         cc_us = 1e3 * c0e.elapsed_time(c1e) / args.steps
         cc_n = int(cc[2].sum().item())
-    bev_us = None
-    if canvas is not None:   # ScatterToBEV alone, on the last call's outputs
+    bev_us = bev_upd_us = None
+    if canvas is not None:   # ScatterToBEV alone, on the last calls' outputs
         b0 = torch.cuda.Event(enable_timing=True)
         b1 = torch.cuda.Event(enable_timing=True)
         b0.record(stream)
@@ -385,6 +397,13 @@ def run_gpu(args):
         b1.record(stream)
         torch.cuda.synchronize(dev)
         bev_us = 1e3 * b0.elapsed_time(b1) / args.steps
+        b0.record(stream)   # the update form, alternating the two output buffers
+        for k in range(args.steps):
+            mmbev.scatter_bev_update(bev_outs[k % 2], bev_outs[(k + 1) % 2], w.max_voxels, dims,
+                                     canvas)
+        b1.record(stream)
+        torch.cuda.synchronize(dev)
+        bev_upd_us = 1e3 * b0.elapsed_time(b1) / args.steps
     clocks = sampler.stop()
     status = vx.status()
     if status != 0:
@@ -468,7 +487,9 @@ def run_gpu(args):
                            {"us": round(rois_us, 2), "objects": int(objs_d.shape[0])}),
             "scatter_bev": (None if bev_us is None else
                             {"us": round(bev_us, 2), "canvas_mb": round(canvas.numel() * 4 / 1e6, 1),
-                             "canvas_gbs": round(canvas.numel() * 4 / (bev_us * 1e-6) / 1e9, 1)}),
+                             "canvas_gbs": round(canvas.numel() * 4 / (bev_us * 1e-6) / 1e9, 1),
+                             "update_us": round(bev_upd_us, 2),
+                             "in_step": "full" if args.bev_full else "update"}),
             "path_hbm_gbs": path_bytes / (ms_step * 1e-3) / 1e9,
             "path_frac_of_peak": path_bytes / (ms_step * 1e-3) / 1e9 / peak,
             "stage_us": {n: round(1e3 * t, 2) for n, t in zip(names, stage_ms)},
@@ -514,6 +535,9 @@ def main():
                     help="also time the voxel-grid connected-component proposer on the outputs")
     ap.add_argument("--bev", action="store_true",
                     help="add ScatterToBEV (a dense [F, nz*5, ny, nx] canvas) to every step")
+    ap.add_argument("--bev-full", action="store_true",
+                    help="with --bev: fill the whole canvas every step instead of clearing the "
+                         "previous step's cells")
     ap.add_argument("--frames", type=int, default=FRAMES,
                     help="frames per GPU (the headline workload is 32; fewer for small "
                          "profiling cases)")

@@ -442,6 +442,20 @@ int mmbev_scatter_bev(const float *feats, const int32_t *coords, const int32_t *
                       int32_t num_frames, int32_t max_voxels, const int32_t dims[3],
                       float *canvas, size_t canvas_bytes, cudaStream_t stream);
 
+/*
+ * ScatterToBEV for a stream of calls: a canvas that holds exactly the
+ * scatter of the previous outputs (prev_coords, prev_nvox: device, the same
+ * shapes as coords, nvox; both NULL for an all-zero canvas) gets the cells of
+ * those voxels zeroed, then the new voxels written. The canvas equals the
+ * one mmbev_scatter_bev gives for (feats, coords, nvox), without the fill of
+ * the whole canvas. prev and the new outputs must not alias. Other arguments
+ * and errors as mmbev_scatter_bev.
+ */
+int mmbev_scatter_bev_update(const int32_t *prev_coords, const int32_t *prev_nvox,
+                             const float *feats, const int32_t *coords, const int32_t *nvox,
+                             int32_t num_frames, int32_t max_voxels, const int32_t dims[3],
+                             float *canvas, size_t canvas_bytes, cudaStream_t stream);
+
 #ifdef __cplusplus
 }
 #endif

@@ -72,6 +72,8 @@ def load():
     lib.mmbev_build_rois.argtypes = [P, P, i32, P, P, P, P]
     lib.mmbev_build_rois.restype = ctypes.c_int
     lib.mmbev_scatter_bev.argtypes = [P, P, P, i32, i32, P, P, ctypes.c_size_t, P]
+    lib.mmbev_scatter_bev_update.argtypes = [P, P, P, P, P, i32, i32, P, P, ctypes.c_size_t, P]
+    lib.mmbev_scatter_bev_update.restype = ctypes.c_int
     lib.mmbev_scatter_bev.restype = ctypes.c_int
     lib.mmbev_voxelize_roi_batched_ex.argtypes = batched + [ctypes.POINTER(_ExecOpts)]
     lib.mmbev_voxelize_roi_batched_ex.restype = ctypes.c_int
@@ -443,6 +445,25 @@ def scatter_bev(out: "Outputs", max_voxels: int, dims, canvas: torch.Tensor | No
                                int(max_voxels), _hptr(d), _dptr(canvas, torch.float32, "canvas"),
                                canvas.numel() * 4, _stream(stream))
     _check(rc, "mmbev_scatter_bev")
+    return canvas
+
+
+def scatter_bev_update(prev: "Outputs | None", out: "Outputs", max_voxels: int, dims,
+                       canvas: torch.Tensor, stream=None) -> torch.Tensor:
+    """ScatterToBEV into a canvas that holds exactly the scatter of ``prev``
+    (``mmbev_scatter_bev_update``; None: an all-zero canvas): the cells of
+    prev's voxels are zeroed, then out's written, giving the canvas
+    ``scatter_bev(out)`` would. ``prev`` and ``out`` must be different
+    buffers (double-buffer the outputs)."""
+    lib = load()
+    nx, ny, nz = (int(d) for d in dims)
+    nf = out.nvox.numel()
+    d = np.asarray([nx, ny, nz], np.int32)
+    rc = lib.mmbev_scatter_bev_update(
+        None if prev is None else _dptr(prev.coords), None if prev is None else _dptr(prev.nvox),
+        _dptr(out.feats), _dptr(out.coords), _dptr(out.nvox), nf, int(max_voxels), _hptr(d),
+        _dptr(canvas, torch.float32, "canvas"), canvas.numel() * 4, _stream(stream))
+    _check(rc, "mmbev_scatter_bev_update")
     return canvas
 
 

@@ -214,3 +214,18 @@ def test_host_input_call_checks_offsets_before_copying(mmbev_lib):
     assert call([0, 2, 1], [0, 1, 3], nsw=1) == -1              # decreasing
     assert call([0, 1, 2], [0, 2, 1], nroi=1) == -1             # decreasing ROI offsets
     assert call([0, 1, 2], [0, 1, 3], so=np.asarray([0, 100, 50], np.int64)) == -1
+
+
+def test_scatter_bev_update_checks_its_arguments(mmbev_lib):
+    lib = mmbev_lib.load()
+    P = ctypes.c_void_p
+    fake = P(0x7e0000000000)
+    dims = np.asarray([100, 50, 2], np.int32)
+    need = 2 * 100 * 50 * 2 * 5 * 4
+    args = (fake, fake, fake, 2, 10, dims.ctypes.data_as(P))
+    assert lib.mmbev_scatter_bev_update(fake, fake, *args, P(0x7f3000000000), need - 4, None) == -3
+    assert lib.mmbev_scatter_bev_update(fake, fake, *args, P(0x7f3000000004), need, None) == -1
+    assert lib.mmbev_scatter_bev_update(fake, None, *args, P(0x7f3000000000), need, None) == -1
+    bad = np.asarray([100, 0, 2], np.int32)
+    assert lib.mmbev_scatter_bev_update(None, None, fake, fake, fake, 2, 10, bad.ctypes.data_as(P),
+                                        P(0x7f3000000000), need, None) == -1

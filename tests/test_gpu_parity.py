@@ -701,3 +701,37 @@ def test_host_input_call_equals_device_input_call(mmbev_lib, cuda_dev, chunk, rh
             ef, ec, en = want.frame(f, w.max_voxels)
             assert np.array_equal(gf.view(np.uint32), ef.view(np.uint32))
             assert np.array_equal(gc, ec) and np.array_equal(gn, en)
+
+
+@pytest.mark.gpu
+def test_scatter_bev_update_equals_a_fresh_scatter(oracle_mod, mmbev_lib, cuda_dev):
+    """A stream of frames through the update entry (previous cells cleared,
+    new ones written) leaves, after every call, the canvas a fresh fill and
+    scatter gives, bit for bit, and equal to the oracle's scatter."""
+    import torch
+    seqs = [[synth.nuscenes_frame(s) for s in (1, 2)], [synth.nuscenes_frame(s) for s in (3, 4)],
+            [synth.roi_coverage(0), synth.nuscenes_frame(5)],
+            [synth.nuscenes_frame(6), synth.nuscenes_frame(6)]]
+    ws = [synth.concat_frames(fr, f"seq{i}") for i, fr in enumerate(seqs)]
+    for w in ws:   # a pillar grid keeps the canvas small
+        w.voxel_size = np.array([0.075, 0.075, 8.0], np.float32)
+    w0 = ws[0]
+    dims = oracle_mod.grid_dims(w0.voxel_size, w0.pc_range)
+    rmax = max(int(np.max(np.diff(w.frame_roi_offsets))) for w in ws)
+    npts = max(w.num_points for w in ws)
+    vxs = [mmbev_lib.Voxelizer(npts, rmax, w0.max_voxels, 2, w0.voxel_size, w0.pc_range,
+                               w0.max_pts_per_voxel, w0.roi_margin, device=cuda_dev)
+           for _ in range(2)]                           # double-buffered outputs
+    canvas = torch.zeros((2, dims[2] * 5, dims[1], dims[0]), device=cuda_dev)   # all-zero start
+    prev = None
+    for i, w in enumerate(ws):
+        pts, tf, rois = to_dev(w, cuda_dev)
+        out = vxs[i % 2](pts, w.sweep_offsets, tf, rois, w.frame_sweep_offsets,
+                         w.frame_roi_offsets)
+        mmbev_lib.scatter_bev_update(prev, out, w0.max_voxels, dims, canvas)
+        fresh = mmbev_lib.scatter_bev(out, w0.max_voxels, dims)
+        torch.cuda.synchronize(cuda_dev)
+        assert torch.equal(canvas.view(torch.int32), fresh.view(torch.int32)), f"call {i}"
+        ref = oracle_mod.scatter_bev(run_oracle(oracle_mod, w), dims)
+        assert np.array_equal(canvas.cpu().numpy().view(np.uint32), ref.view(np.uint32))
+        prev = out
