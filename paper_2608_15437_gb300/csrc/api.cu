@@ -124,8 +124,9 @@ Layout make_layout(int64_t max_points, int64_t rois_total, int32_t max_rois_fram
     L.d_lin = take(sizeof(uint32_t) * U);
     L.items = take(sizeof(uint2) * U);
     L.vid_slot = take(sizeof(uint32_t) * (F * (size_t)(max_voxels > 0 ? max_voxels : 1)));
-    L.heavy = take(sizeof(uint32_t) * (F * (size_t)(max_voxels > 0 ? max_voxels : 1)));
-    L.huge = take(sizeof(uint32_t) * (F * (size_t)(max_voxels > 0 ? max_voxels : 1)));
+    // slots with more than kLightMax (kHugeMin) of the at most U points
+    L.heavy = take(sizeof(uint32_t) * (U / (kLightMax + 1) + 1));
+    L.huge = take(sizeof(uint32_t) * (U / (kHugeMin + 1) + 1));
     L.total = o;
     return L;
 }
@@ -252,7 +253,7 @@ void bind_layout(Params* p, const Layout& L, uint8_t* ws) {
 
 const char* const kStageNames[MMBEV_NUM_STAGES] = {
     "prep", "classify", "insert", "compact", "scatter_points", "capped_hist", "frames",
-    "capped_census", "scan", "scatter", "rank", "finalize", "finalize_heavy"};
+    "capped_census", "scan", "scatter", "rank", "finalize"};
 
 }  // namespace
 }  // namespace mmbev
@@ -404,8 +405,6 @@ int voxelize_batched(const float* points, const int64_t* sweep_offsets, int32_t 
         if ((e = launch_rank(p, sms, pdl, stream)) != cudaSuccess) break;
         if ((e = mark()) != cudaSuccess) break;
         if ((e = launch_finalize(p, sms, pdl, stream)) != cudaSuccess) break;
-        if ((e = mark()) != cudaSuccess) break;
-        if ((e = launch_finalize_heavy(p, sms, pdl, stream)) != cudaSuccess) break;
         if ((e = mark()) != cudaSuccess) break;
     } while (0);
     return e == cudaSuccess ? MMBEV_OK : MMBEV_ECUDA;

@@ -10,23 +10,23 @@
 // and divided once by the count; the feature row and the count are written
 // and the slot is returned to the all-zero state.
 //
-// Light kernel: one thread per kept voxel with at most 32 points keeps the K
-// smallest positions in a sorted register array (each position bubbles in
-// with compare-and-swap steps; eight positions load at a time). Voxels with
-// more points go to a list.
-// Heavy kernel: one warp per listed voxel; each lane keeps the smallest
+// One launch, two roles. Light blocks: one thread per kept voxel with at
+// most 32 points keeps the K smallest positions in a sorted register array
+// (each position bubbles in with compare-and-swap steps; eight positions load
+// at a time); the others are skipped. Heavy blocks (the first block indices,
+// so they are dispatched first), over the slots the compact stage listed: one
+// warp per voxel with 33 to 1024 points, where each lane keeps the smallest
 // positions of its share of the segment, then K rounds of a warp minimum
 // pick the voxel's K smallest in ascending order, the lanes fetch those
-// records in parallel and lane 0 adds them up in order. Voxels with more
-// than 1024 points get a whole block (eight warps' lists merged by one).
+// records in parallel and lane 0 adds them up in order; a whole block per
+// voxel with more than 1024 points (eight warps' lists merged by one). The
+// heavy voxels' work so overlaps the light voxels'.
 #include "mmbev_internal.cuh"
 
 namespace mmbev {
 namespace {
 
 constexpr int kThreads = 256;
-constexpr uint32_t kLightMax = 32;
-constexpr uint32_t kHugeMin = 1024;   // voxels with more points get a whole block
 
 // Insert v into the ascending array b[0..B) (unused entries hold ~0u); the
 // largest entry falls off the end.
@@ -76,20 +76,14 @@ __device__ __forceinline__ size_t voxel_row(const Params& p, const uint32_t* s_v
     return (size_t)lo * (uint32_t)p.max_voxels + (g - s_vbase[lo]);
 }
 
+// Light role: block lb of nlb.
 template <int B>
-__global__ void __launch_bounds__(kThreads) k_finalize(Params p) {
-    __shared__ uint32_t s_vbase[kMaxFrames + 1];
-    pdl_wait();
-    const int F = p.num_frames;
-    for (int i = threadIdx.x; i < F; i += blockDim.x) s_vbase[i] = p.finfo[i].vbase;
-    const uint32_t total = ld_cg(&p.hdr->total_kept);
-    const uint32_t seg_cap = min(ld_cg(&p.hdr->seg_total), p.occ_cap);  // seg holds N entries
-    if (threadIdx.x == 0) s_vbase[F] = total;
-    __syncthreads();
-    const int lane = threadIdx.x & 31;
-    const uint32_t gs = gridDim.x * blockDim.x;
+__device__ __forceinline__ void finalize_light(const Params& p, const uint32_t* s_vbase, int F,
+                                               uint32_t total, uint32_t seg_cap, uint32_t lb,
+                                               uint32_t nlb) {
+    const uint32_t gs = nlb * blockDim.x;
     const int K = p.K;
-    for (uint32_t g0 = blockIdx.x * blockDim.x; g0 < total; g0 += gs) {
+    for (uint32_t g0 = lb * blockDim.x; g0 < total; g0 += gs) {
         const uint32_t g = g0 + threadIdx.x;
         const bool act = g < total;
         uint32_t h = 0, n = 0, off = 0;
@@ -103,17 +97,9 @@ __global__ void __launch_bounds__(kThreads) k_finalize(Params p) {
                 n = 0;
             }
         }
-        const bool heavy = act && n > kLightMax && n <= kHugeMin;
-        const bool huge = act && n > kHugeMin;
-        const uint32_t hm = __ballot_sync(0xFFFFFFFFu, heavy);
-        if (hm) {
-            uint32_t base = 0;
-            if (lane == __ffs(hm) - 1) base = atomicAdd(&p.hdr->num_heavy, (uint32_t)__popc(hm));
-            base = __shfl_sync(0xFFFFFFFFu, base, __ffs(hm) - 1);
-            if (heavy) p.heavy[base + __popc(hm & ((1u << lane) - 1u))] = g;
-        }
-        if (huge) p.huge[atomicAdd(&p.hdr->num_huge, 1u)] = g;  // rare
-        if (!act || heavy || huge) continue;
+        // heavy and huge voxels are the heavy role's; a count of 0 is a slot
+        // that role has already returned to zero (a kept voxel has a point)
+        if (!act || n == 0 || n > kLightMax) continue;
         uint32_t best[B];
 #pragma unroll
         for (int j = 0; j < B; ++j) best[j] = 0xFFFFFFFFu;
@@ -171,29 +157,30 @@ __device__ __forceinline__ void warp_sum_records(const Params& p, const uint32_t
     }
 }
 
+// Heavy role: block hb of nhb (block-uniform, so its barriers are safe), over
+// the slots the compact stage listed; the rank stage left each kept voxel's
+// output index in its slot, and a listed slot the cap dropped is all-zero.
 template <int B>
-__global__ void __launch_bounds__(kThreads) k_finalize_heavy(Params p) {
-    __shared__ uint32_t s_vbase[kMaxFrames + 1];
-    __shared__ uint32_t s_cand[kThreads / 32][kMaxK];
-    pdl_wait();
-    const int F = p.num_frames;
-    for (int i = threadIdx.x; i < F; i += blockDim.x) s_vbase[i] = p.finfo[i].vbase;
-    const uint32_t total = ld_cg(&p.hdr->total_kept);
-    if (threadIdx.x == 0) s_vbase[F] = total;
-    __syncthreads();
+__device__ __forceinline__ void finalize_heavy(const Params& p, const uint32_t* s_vbase, int F,
+                                               uint32_t total, uint32_t seg_cap, uint32_t hb,
+                                               uint32_t nhb, uint32_t (*s_cand)[kMaxK]) {
     const int lane = threadIdx.x & 31;
-    const uint32_t seg_cap = min(ld_cg(&p.hdr->seg_total), p.occ_cap);  // seg holds N entries
     const int K = p.K;
     // Huge voxels, one block each: every thread keeps the smallest positions
     // of its share, each warp reduces its threads' to its K smallest, and
     // warp 0 merges the warps' lists.
     const uint32_t nhuge = ld_cg(&p.hdr->num_huge);
     const int warp = threadIdx.x >> 5;
-    for (uint32_t e = blockIdx.x; e < nhuge; e += gridDim.x) {
-        const uint32_t g = p.huge[e];
-        const uint32_t h = p.vid_slot[g];
+    for (uint32_t e = hb; e < nhuge; e += nhb) {
+        const uint32_t h = p.huge[e];
         const uint32_t off = ld_cg(slot_seg(p, h));
         uint32_t n = ld_cg(slot_cnt(p, h));
+        if (n == 0) continue;   // dropped by the cap (the same for the whole block)
+        const uint32_t g = ld_cg(slot_rank(p, h));
+        if (g >= total) {
+            if (threadIdx.x == 0) set_status(p.hdr, MMBEV_DEV_BOUNDS);
+            continue;
+        }
         if (off > seg_cap || n > seg_cap - off) {
             if (threadIdx.x == 0) set_status(p.hdr, MMBEV_DEV_BOUNDS);
             n = 0;
@@ -247,13 +234,18 @@ __global__ void __launch_bounds__(kThreads) k_finalize_heavy(Params p) {
         __syncthreads();
     }
     const uint32_t nh = ld_cg(&p.hdr->num_heavy);
-    const uint32_t gw = (blockIdx.x * blockDim.x + threadIdx.x) >> 5;
-    const uint32_t nw = (gridDim.x * blockDim.x) >> 5;
+    const uint32_t gw = (hb * blockDim.x + threadIdx.x) >> 5;
+    const uint32_t nw = (nhb * blockDim.x) >> 5;
     for (uint32_t e = gw; e < nh; e += nw) {
-        const uint32_t g = p.heavy[e];
-        const uint32_t h = p.vid_slot[g];
+        const uint32_t h = p.heavy[e];
         const uint32_t off = ld_cg(slot_seg(p, h));
         uint32_t n = ld_cg(slot_cnt(p, h));
+        if (n == 0) continue;   // dropped by the cap (the same for the whole warp)
+        const uint32_t g = ld_cg(slot_rank(p, h));
+        if (g >= total) {
+            if (lane == 0) set_status(p.hdr, MMBEV_DEV_BOUNDS);
+            continue;
+        }
         if (off > seg_cap || n > seg_cap - off) {   // inconsistent lists: report, read nothing
             if (lane == 0) set_status(p.hdr, MMBEV_DEV_BOUNDS);
             n = 0;
@@ -294,21 +286,33 @@ __global__ void __launch_bounds__(kThreads) k_finalize_heavy(Params p) {
     }
 }
 
+template <int BL, int BH>
+__global__ void __launch_bounds__(kThreads) k_finalize(Params p, uint32_t heavy_blocks) {
+    __shared__ uint32_t s_vbase[kMaxFrames + 1];
+    __shared__ uint32_t s_cand[kThreads / 32][kMaxK];
+    pdl_wait();
+    const int F = p.num_frames;
+    for (int i = threadIdx.x; i < F; i += blockDim.x) s_vbase[i] = p.finfo[i].vbase;
+    const uint32_t total = ld_cg(&p.hdr->total_kept);
+    const uint32_t seg_cap = min(ld_cg(&p.hdr->seg_total), p.occ_cap);  // seg holds N entries
+    if (threadIdx.x == 0) s_vbase[F] = total;
+    __syncthreads();
+    if (blockIdx.x < heavy_blocks)
+        finalize_heavy<BH>(p, s_vbase, F, total, seg_cap, blockIdx.x, heavy_blocks, s_cand);
+    else
+        finalize_light<BL>(p, s_vbase, F, total, seg_cap, blockIdx.x - heavy_blocks,
+                           gridDim.x - heavy_blocks);
+}
+
 }  // namespace
 
 cudaError_t launch_finalize(const Params& p, int num_sms, bool pdl, cudaStream_t st) {
-    const dim3 grid(num_sms * 8), block(kThreads);
-    if (p.K <= 4) return launch_k(k_finalize<4>, grid, block, 0, st, pdl, p);
-    if (p.K <= 12) return launch_k(k_finalize<12>, grid, block, 0, st, pdl, p);
-    return launch_k(k_finalize<32>, grid, block, 0, st, pdl, p);
-}
-
-cudaError_t launch_finalize_heavy(const Params& p, int num_sms, bool pdl, cudaStream_t st) {
-    const dim3 grid(num_sms * 4), block(kThreads);
-    if (p.K <= 4) return launch_k(k_finalize_heavy<4>, grid, block, 0, st, pdl, p);
-    if (p.K <= 12) return launch_k(k_finalize_heavy<12>, grid, block, 0, st, pdl, p);
-    if (p.K <= 32) return launch_k(k_finalize_heavy<32>, grid, block, 0, st, pdl, p);
-    return launch_k(k_finalize_heavy<kMaxK>, grid, block, 0, st, pdl, p);
+    const uint32_t heavy = (uint32_t)num_sms * 4;
+    const dim3 grid(num_sms * 12), block(kThreads);
+    if (p.K <= 4) return launch_k(k_finalize<4, 4>, grid, block, 0, st, pdl, p, heavy);
+    if (p.K <= 12) return launch_k(k_finalize<12, 12>, grid, block, 0, st, pdl, p, heavy);
+    if (p.K <= 32) return launch_k(k_finalize<32, 32>, grid, block, 0, st, pdl, p, heavy);
+    return launch_k(k_finalize<32, kMaxK>, grid, block, 0, st, pdl, p, heavy);
 }
 
 }  // namespace mmbev

@@ -246,6 +246,25 @@ __global__ void __launch_bounds__(kThreads) k_compact(Params p) {
         uint32_t cgrp = 1u << lane;
         if (ok) cgrp = __match_any_sync(am, ch);
         if (ok && lane == __ffs(cgrp) - 1) atomicAdd(&p.ctot[ch], (uint32_t)__popc(cgrp));
+        // slots with more than kLightMax points, for the finalize stage's heavy
+        // role (counts sum to at most occ_cap points: the lists have room)
+        const bool heavy = ok && cnt > kLightMax && cnt <= kHugeMin;
+        const uint32_t hm = __ballot_sync(0xFFFFFFFFu, heavy);
+        if (hm) {
+            const int hl = __ffs(hm) - 1;
+            uint32_t hb = 0;
+            if (lane == hl) hb = atomicAdd(&p.hdr->num_heavy, (uint32_t)__popc(hm));
+            hb = __shfl_sync(0xFFFFFFFFu, hb, hl) + __popc(hm & ((1u << lane) - 1u));
+            if (heavy) {
+                if (hb < p.occ_cap / (kLightMax + 1) + 1) p.heavy[hb] = e.x;
+                else set_status(p.hdr, MMBEV_DEV_BOUNDS);
+            }
+        }
+        if (ok && cnt > kHugeMin) {   // rare
+            const uint32_t hu = atomicAdd(&p.hdr->num_huge, 1u);
+            if (hu < p.occ_cap / (kHugeMin + 1) + 1) p.huge[hu] = e.x;
+            else set_status(p.hdr, MMBEV_DEV_BOUNDS);
+        }
         if (ok) {
             *slot_seg(p, e.x) = segoff;
             p.occ[d] = e.x;

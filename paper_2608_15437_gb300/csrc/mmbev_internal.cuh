@@ -360,7 +360,12 @@ cudaError_t launch_scan(const Params& p, bool pdl, cudaStream_t st);
 cudaError_t launch_scatter(const Params& p, int num_sms, bool pdl, cudaStream_t st);
 cudaError_t launch_rank(const Params& p, int num_sms, bool pdl, cudaStream_t st);
 cudaError_t launch_finalize(const Params& p, int num_sms, bool pdl, cudaStream_t st);
-cudaError_t launch_finalize_heavy(const Params& p, int num_sms, bool pdl, cudaStream_t st);
+
+// Voxels with more points than kLightMax are "heavy" (a warp each in the
+// finalize stage), with more than kHugeMin "huge" (a block each); the compact
+// stage lists their slots.
+constexpr uint32_t kLightMax = 32;
+constexpr uint32_t kHugeMin = 1024;
 cudaError_t launch_zero(void* ptr, size_t bytes, cudaStream_t st);
 
 // Launch `kern` with an optional programmatic-stream-serialization attribute.

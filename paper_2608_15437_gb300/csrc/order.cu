@@ -399,6 +399,10 @@ __global__ void __launch_bounds__(kRankWarps * 32) k_rank(Params p) {
             else { kept = true; vid = A + (c < fi.q ? c : fi.q); }
             if (kept && vid < fi.nvox) {
                 p.vid_slot[fi.vbase + vid] = h;
+                // the slot's rank word is not read past this stage: it now
+                // holds the voxel's output index, for the finalize stage's
+                // heavy role (which starts from the slot)
+                *slot_rank(p, h) = fi.vbase + vid;
                 const size_t row = (size_t)f * (uint32_t)p.max_voxels + vid;
                 const uint32_t cx = lin % nx;
                 const uint32_t cy = (lin / nx) % ny;
