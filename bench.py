@@ -438,14 +438,14 @@ def run_gpu(args):
         nonlocal d2h_bytes
         if d_objs is None:   # host inputs: chunks go up while earlier ones are voxelized
             out = vx.run_host(h_pts, w.sweep_offsets, h_tf, h_rois, w.frame_sweep_offsets,
-                              roi_off, chunk_frames=args.e2e_chunk)
+                              roi_off, chunk_frames=args.e2e_chunk, pack_dst=h_packed)
         else:   # the previous frame's objects go up; the ROI table is built on the device
             d_pts.copy_(h_pts, non_blocking=True)
             d_tf.copy_(h_tf, non_blocking=True)
             d_objs.copy_(h_objs, non_blocking=True)
             rl = mmbev.build_rois(d_objs, obj_off, crit, out=rois_buf)[0]
             out = vx(d_pts, w.sweep_offsets, d_tf, rl, w.frame_sweep_offsets, roi_off)
-        mmbev.pack_voxels(out, w.max_voxels, h_packed)
+            mmbev.pack_voxels(out, w.max_voxels, h_packed)
         torch.cuda.current_stream(dev).synchronize()
         total = int(h_packed[4 * w.num_frames:4 * w.num_frames + 4].view(torch.int32)[0])
         d2h_bytes = 4 * (w.num_frames + 1) + BYTES_PER_VOXEL * total

@@ -247,6 +247,11 @@ typedef struct mmbev_exec_opts {
  *   d_points, d_sweep_tf, d_rois  device staging of the same sizes, written
  *               by the call.
  *   sweep_offsets, frame_*_offsets  host, as above; checked before any copy.
+ *   pack_dst, pack_bytes  NULL, or device or pinned host memory of at least
+ *               mmbev_pack_size(F, max_voxels) bytes: each chunk's kept rows
+ *               are packed there (mmbev_pack_voxels' layout) as soon as the
+ *               chunk is done, so the results cross to the host while later
+ *               chunks go up and run.
  *   chunk_frames  frames a chunk (>= 1).
  *   copy_stream  the stream of the copies (the call's own `stream` makes it
  *               serial).
@@ -260,8 +265,9 @@ int mmbev_voxelize_roi_batched_host(
     int32_t max_voxels, int32_t num_frames, const int32_t *frame_sweep_offsets,
     const int32_t *frame_roi_offsets, float *d_points, float *d_sweep_tf, mmbev_roi_t *d_rois,
     float *out_feats, int32_t *out_coords, int32_t *out_counts, int32_t *out_nvox, void *table,
-    size_t table_bytes, void *workspace, size_t workspace_bytes, int32_t chunk_frames,
-    cudaStream_t stream, cudaStream_t copy_stream, const mmbev_exec_opts_t *opts);
+    size_t table_bytes, void *workspace, size_t workspace_bytes, void *pack_dst,
+    size_t pack_bytes, int32_t chunk_frames, cudaStream_t stream, cudaStream_t copy_stream,
+    const mmbev_exec_opts_t *opts);
 
 int mmbev_voxelize_roi_batched_ex(const float *points, const int64_t *sweep_offsets,
                                   int32_t num_sweeps, const float *sweep_tf,

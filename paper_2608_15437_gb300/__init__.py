@@ -79,7 +79,7 @@ def load():
     lib.mmbev_voxelize_roi_batched_ex.restype = ctypes.c_int
     lib.mmbev_voxelize_roi_batched_host.argtypes = (
         [P, P, i32, P, P, i32, f32, P, P, i32, i32, i32, P, P, P, P, P, P, P, P, P, P, sz, P, sz,
-         i32, P, P, ctypes.POINTER(_ExecOpts)])
+         P, sz, i32, P, P, ctypes.POINTER(_ExecOpts)])
     lib.mmbev_voxelize_roi_batched_host.restype = ctypes.c_int
     lib.mmbev_classify_points.argtypes = [P, P, i32, P, P, i32, f32, P, P, i32, P, P,
                                           P, P, P, P, sz, P]
@@ -497,11 +497,16 @@ class Voxelizer:
 
     def run_host(self, h_points: torch.Tensor, sweep_offsets, h_sweep_tf: torch.Tensor,
                  h_rois: torch.Tensor, frame_sweep_offsets, frame_roi_offsets,
-                 chunk_frames: int = 8, stream=None) -> Outputs:
+                 chunk_frames: int = 8, stream=None, pack_dst: torch.Tensor | None = None) -> Outputs:
         """The batched call on pinned host inputs
         (``mmbev_voxelize_roi_batched_host``): chunks of ``chunk_frames``
         frames go up on a side stream while earlier chunks are voxelized.
+        With ``pack_dst`` (a uint8 tensor of ``pack_bytes``, on the device or
+        pinned), each chunk's kept rows are packed there as it completes.
         Device staging is allocated on first use and kept."""
+        if pack_dst is not None and (pack_dst.dtype != torch.uint8 or not pack_dst.is_contiguous()
+                                     or not (pack_dst.is_cuda or pack_dst.is_pinned())):
+            raise ValueError("pack_dst must be a contiguous uint8 device or pinned tensor")
         lib = load()
         so = _host(sweep_offsets, np.int64)
         fso = _host(frame_sweep_offsets, np.int32)
@@ -529,7 +534,10 @@ class Voxelizer:
             len(fso) - 1, _hptr(fso), _hptr(fro), _dptr(d_pts), _dptr(d_tf), _dptr(d_rois),
             _dptr(self.out.feats), _dptr(self.out.coords), _dptr(self.out.counts),
             _dptr(self.out.nvox), _dptr(self.table), self.table.numel(), _dptr(self.workspace),
-            self.workspace.numel(), int(chunk_frames), _stream(st), _stream(self._copy_stream),
+            self.workspace.numel(),
+            None if pack_dst is None else ctypes.c_void_p(pack_dst.data_ptr()),
+            0 if pack_dst is None else pack_dst.numel(), int(chunk_frames), _stream(st),
+            _stream(self._copy_stream),
             ctypes.byref(opts))
         _check(rc, "mmbev_voxelize_roi_batched_host")
         return self.out

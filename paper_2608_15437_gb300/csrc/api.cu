@@ -131,20 +131,6 @@ Layout make_layout(int64_t max_points, int64_t rois_total, int32_t max_rois_fram
     return L;
 }
 
-int num_sms() {
-    static std::atomic<int> cache[64];
-    int dev = 0;
-    if (cudaGetDevice(&dev) != cudaSuccess) return 0;
-    if (dev >= 0 && dev < 64) {
-        const int c = cache[dev].load(std::memory_order_relaxed);
-        if (c > 0) return c;
-    }
-    int n = 0;
-    if (cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess) return 0;
-    if (dev >= 0 && dev < 64) cache[dev].store(n, std::memory_order_relaxed);
-    return n;
-}
-
 // Validation shared by the full path and the classify-only path. Fills the
 // call-shape fields of Params and the host descriptor.
 int validate_common(const float* points, const int64_t* sweep_offsets, int32_t num_sweeps,
@@ -256,6 +242,21 @@ const char* const kStageNames[MMBEV_NUM_STAGES] = {
     "capped_census", "scan", "scatter", "rank", "finalize"};
 
 }  // namespace
+
+int num_sms() {
+    static std::atomic<int> cache[64];
+    int dev = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess) return 0;
+    if (dev >= 0 && dev < 64) {
+        const int c = cache[dev].load(std::memory_order_relaxed);
+        if (c > 0) return c;
+    }
+    int n = 0;
+    if (cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess) return 0;
+    if (dev >= 0 && dev < 64) cache[dev].store(n, std::memory_order_relaxed);
+    return n;
+}
+
 }  // namespace mmbev
 
 using namespace mmbev;
@@ -439,8 +440,9 @@ int mmbev_voxelize_roi_batched_host(
     int32_t max_voxels, int32_t num_frames, const int32_t* frame_sweep_offsets,
     const int32_t* frame_roi_offsets, float* d_points, float* d_sweep_tf, mmbev_roi_t* d_rois,
     float* out_feats, int32_t* out_coords, int32_t* out_counts, int32_t* out_nvox, void* table,
-    size_t table_bytes, void* workspace, size_t workspace_bytes, int32_t chunk_frames,
-    cudaStream_t stream, cudaStream_t copy_stream, const mmbev_exec_opts_t* opts) {
+    size_t table_bytes, void* workspace, size_t workspace_bytes, void* pack_dst,
+    size_t pack_bytes, int32_t chunk_frames, cudaStream_t stream, cudaStream_t copy_stream,
+    const mmbev_exec_opts_t* opts) {
     if (num_frames < 1 || num_frames > kMaxFrames || chunk_frames < 1) return MMBEV_EINVAL;
     if (num_sweeps < 0 || num_sweeps > kMaxSweeps || num_rois < 0) return MMBEV_EINVAL;
     if (!out_nvox) return MMBEV_EINVAL;
@@ -458,6 +460,9 @@ int mmbev_voxelize_roi_batched_host(
             return MMBEV_EINVAL;
     for (int32_t s = 0; s < num_sweeps; ++s)
         if (sweep_offsets[s + 1] < sweep_offsets[s]) return MMBEV_EINVAL;
+    if (pack_dst && ((reinterpret_cast<uintptr_t>(pack_dst) & 3u) || max_voxels == 0))
+        return MMBEV_EINVAL;
+    if (pack_dst && pack_bytes < mmbev_pack_size(num_frames, max_voxels)) return MMBEV_EWORKSPACE;
     const int64_t n = sweep_offsets[num_sweeps];
     if ((n > 0 && (!h_points || !d_points)) || (num_sweeps > 0 && (!h_sweep_tf || !d_sweep_tf)) ||
         (num_rois > 0 && (!h_rois || !d_rois)))
@@ -509,6 +514,12 @@ int mmbev_voxelize_roi_batched_host(
             out_coords ? out_coords + 3 * row0 : nullptr,
             out_counts ? out_counts + row0 : nullptr, out_nvox + f0, table, table_bytes,
             workspace, workspace_bytes, stream, opts, c > 0);
+        // the chunk's kept rows into the packed buffer (offsets of frames
+        // f0..f1 and their records), while later chunks go up and run
+        if (rc == MMBEV_OK && pack_dst &&
+            launch_pack(out_feats, out_coords, out_counts, out_nvox, num_frames, f0, f1,
+                        max_voxels, pack_dst, stream) != cudaSuccess)
+            rc = MMBEV_ECUDA;
     }
     for (cudaEvent_t x : ev)
         if (x) cudaEventDestroy(x);   // released once the work recorded on it is done

@@ -360,6 +360,12 @@ cudaError_t launch_scan(const Params& p, bool pdl, cudaStream_t st);
 cudaError_t launch_scatter(const Params& p, int num_sms, bool pdl, cudaStream_t st);
 cudaError_t launch_rank(const Params& p, int num_sms, bool pdl, cudaStream_t st);
 cudaError_t launch_finalize(const Params& p, int num_sms, bool pdl, cudaStream_t st);
+// Kept rows of frames [f0, f1) of a call's outputs into a packed buffer
+// (mmbev_pack_voxels' layout for F frames).
+cudaError_t launch_pack(const float* feats, const int32_t* coords, const int32_t* counts,
+                        const int32_t* nvox, int32_t F, int32_t f0, int32_t f1,
+                        int32_t max_voxels, void* dst, cudaStream_t stream);
+int num_sms();   // of the current device, cached
 
 // Voxels with more points than kLightMax are "heavy" (a warp each in the
 // finalize stage), with more than kHugeMin "huge" (a block each); the compact

@@ -10,7 +10,9 @@
 // One kernel: every block scans nvox into shared memory (F <= 1024 frames),
 // then each warp takes 32 consecutive records at a time: a lane finds its
 // record's frame by binary search, and the warp writes the 288 words of the
-// 32 records as nine stores of 32 consecutive words.
+// 32 records as nine stores of 32 consecutive words. A launch may cover a
+// range of frames [f0, f1): it writes off[f0..f1] and those frames' records,
+// so a batch can be packed chunk by chunk as its chunks complete.
 #include <cstdint>
 
 #include "mmbev_internal.cuh"
@@ -24,19 +26,19 @@ constexpr int kPackPer = (kMaxFrames + kPackThreads - 1) / kPackThreads;   // fr
 __global__ void __launch_bounds__(kPackThreads)
 k_pack(const float* __restrict__ feats, const int32_t* __restrict__ coords,
        const int32_t* __restrict__ counts, const int32_t* __restrict__ nvox, int32_t F,
-       int32_t max_voxels, int32_t* dst) {
+       int32_t f0, int32_t f1, int32_t max_voxels, int32_t* dst) {
     __shared__ int32_t s_off[kMaxFrames + 1];
     __shared__ int32_t s_warp[kPackThreads / 32];
     const int t = threadIdx.x, lane = t & 31, wid = t >> 5;
 
-    // exclusive prefix of min(max(nvox[f], 0), max_voxels): kPackPer frames a
-    // thread, then a scan across the block
+    // exclusive prefix of min(max(nvox[f], 0), max_voxels) over frames
+    // [0, f1): kPackPer frames a thread, then a scan across the block
     int32_t mine[kPackPer];
     int32_t sum = 0;
 #pragma unroll
     for (int i = 0; i < kPackPer; ++i) {
         const int f = t * kPackPer + i;
-        mine[i] = f < F ? min(max(__ldg(nvox + f), 0), max_voxels) : 0;
+        mine[i] = f < f1 ? min(max(__ldg(nvox + f), 0), max_voxels) : 0;
         sum += mine[i];
     }
     int32_t incl = sum;
@@ -52,23 +54,24 @@ k_pack(const float* __restrict__ feats, const int32_t* __restrict__ coords,
 #pragma unroll
     for (int i = 0; i < kPackPer; ++i) {
         const int f = t * kPackPer + i;
-        if (f < F) s_off[f] = before;
+        if (f < f1) s_off[f] = before;
         before += mine[i];
     }
-    if (t == kPackThreads - 1) s_off[F] = before;   // the last thread's running sum is T
+    if (t == kPackThreads - 1) s_off[f1] = before;   // the last thread's running sum
     __syncthreads();
-    const int32_t T = s_off[F];
+    const int32_t T = s_off[f1];   // records before frame f1
     if (blockIdx.x == 0)
-        for (int f = t; f <= F; f += kPackThreads) dst[f] = s_off[f];
+        for (int f = f0 + t; f <= f1; f += kPackThreads) dst[f] = s_off[f];
 
     uint32_t* rec = reinterpret_cast<uint32_t*>(dst + F + 1);
     const size_t nwarps = (size_t)gridDim.x * (kPackThreads / 32);
-    for (size_t p0 = ((size_t)blockIdx.x * (kPackThreads / 32) + wid) * 32; p0 < (size_t)T;
+    const size_t first = (size_t)s_off[f0];   // this range's records: [first, T)
+    for (size_t p0 = first + ((size_t)blockIdx.x * (kPackThreads / 32) + wid) * 32; p0 < (size_t)T;
          p0 += nwarps * 32) {
         const size_t p = p0 + lane;
         unsigned long long src = 0;
         if (p < (size_t)T) {
-            int lo = 0, hi = F;   // the last f with s_off[f] <= p
+            int lo = f0, hi = f1;   // the last f with s_off[f] <= p
             while (hi - lo > 1) {
                 const int mid = (lo + hi) >> 1;
                 if ((size_t)s_off[mid] <= p) lo = mid;
@@ -77,7 +80,7 @@ k_pack(const float* __restrict__ feats, const int32_t* __restrict__ coords,
             src = (unsigned long long)lo * (unsigned long long)max_voxels + (p - (size_t)s_off[lo]);
         }
         const int nrec = (int)min((size_t)32, (size_t)T - p0);
-        uint32_t* out = rec + p0 * 9;
+        uint32_t* out = rec + p0 * 9;   // record p0 of the whole batch
 #pragma unroll
         for (int k = 0; k < 9; ++k) {
             const int w = k * 32 + lane;   // word of the warp's block of 32 records
@@ -94,6 +97,18 @@ k_pack(const float* __restrict__ feats, const int32_t* __restrict__ coords,
 }
 
 }  // namespace
+
+cudaError_t launch_pack(const float* feats, const int32_t* coords, const int32_t* counts,
+                        const int32_t* nvox, int32_t F, int32_t f0, int32_t f1,
+                        int32_t max_voxels, void* dst, cudaStream_t stream) {
+    const int sms = num_sms();
+    if (sms <= 0) return cudaErrorInvalidDevice;
+    k_pack<<<(unsigned)sms * 2, kPackThreads, 0, stream>>>(feats, coords, counts, nvox, F, f0, f1,
+                                                            max_voxels,
+                                                            static_cast<int32_t*>(dst));
+    return cudaGetLastError();
+}
+
 }  // namespace mmbev
 
 using namespace mmbev;
@@ -113,12 +128,8 @@ extern "C" int mmbev_pack_voxels(const float* feats, const int32_t* coords, cons
     if (!dst || (reinterpret_cast<uintptr_t>(dst) & 3u)) return MMBEV_EINVAL;
     if (dst_bytes < mmbev_pack_size(num_frames, max_voxels)) return MMBEV_EWORKSPACE;
     if (num_frames > 0 && (!feats || !coords || !counts || !nvox)) return MMBEV_EINVAL;
-    int dev = 0, sms = 0;
-    if (cudaGetDevice(&dev) != cudaSuccess) return MMBEV_ECUDA;
-    if (cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess)
-        return MMBEV_ECUDA;
-    k_pack<<<(unsigned)sms * 2, kPackThreads, 0, stream>>>(feats, coords, counts, nvox,
-                                                            num_frames, max_voxels,
-                                                            static_cast<int32_t*>(dst));
-    return cudaGetLastError() == cudaSuccess ? MMBEV_OK : MMBEV_ECUDA;
+    return launch_pack(feats, coords, counts, nvox, num_frames, 0, num_frames, max_voxels, dst,
+                       stream) == cudaSuccess
+               ? MMBEV_OK
+               : MMBEV_ECUDA;
 }

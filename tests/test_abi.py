@@ -206,7 +206,7 @@ def test_host_input_call_checks_offsets_before_copying(mmbev_lib):
             fake, so.ctypes.data_as(P), nsw, fake, fake, nroi, 0.5, vs.ctypes.data_as(P),
             rg.ctypes.data_as(P), 10, 1000, len(fso) - 1, fso.ctypes.data_as(P),
             fro.ctypes.data_as(P), fake, fake, fake, fake, fake, fake, fake, fake, 1 << 20, fake,
-            1 << 20, chunk, None, None, None)
+            1 << 20, None, 0, chunk, None, None, None)
 
     assert call([0, 1, 2], [0, 1, 3], chunk=0) == -1           # chunk_frames < 1
     assert call([1, 1, 2], [0, 1, 3]) == -1                     # frames must start at sweep 0

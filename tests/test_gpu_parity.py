@@ -690,12 +690,22 @@ def test_host_input_call_equals_device_input_call(mmbev_lib, cuda_dev, chunk, rh
     h_pts = torch.from_numpy(np.ascontiguousarray(w.points)).pin_memory()
     h_tf = torch.from_numpy(np.ascontiguousarray(w.sweep_tf)).pin_memory()
     h_rois = torch.from_numpy(np.ascontiguousarray(w.rois, np.float32).reshape(-1, 5)).pin_memory()
-    for _ in range(2):   # twice: the staging is reused
+    nb = mmbev_lib.pack_bytes(w.num_frames, w.max_voxels)
+    ref_pack = torch.zeros(nb, dtype=torch.uint8).pin_memory()
+    mmbev_lib.pack_voxels(want, w.max_voxels, ref_pack)
+    for it in range(2):   # twice: the staging is reused
+        packed = torch.full((nb,), 0xCD, dtype=torch.uint8).pin_memory()
         got = vx.run_host(h_pts, w.sweep_offsets, h_tf, h_rois, w.frame_sweep_offsets,
-                          w.frame_roi_offsets, chunk_frames=chunk)
+                          w.frame_roi_offsets, chunk_frames=chunk,
+                          pack_dst=packed if it == 1 else None)
         torch.cuda.synchronize(cuda_dev)
         assert vx.status() == 0
         assert torch.equal(got.nvox, want.nvox)
+        if it == 1:   # packed chunk by chunk = packed in one go
+            total = int(ref_pack[4 * w.num_frames:4 * w.num_frames + 4].view(torch.int32)[0])
+            used = 4 * (w.num_frames + 1) + 36 * total
+            assert torch.equal(packed[:used], ref_pack[:used])
+            assert bool((packed[used:] == 0xCD).all())
         for f in range(w.num_frames):
             gf, gc, gn = got.frame(f, w.max_voxels)
             ef, ec, en = want.frame(f, w.max_voxels)
