@@ -514,6 +514,74 @@ def run_gpu(args):
     return 0
 
 
+SMALL_CONFIGS = ("tiny", "nuscenes", "ouster", "roi_0", "roi_8", "roi_32", "roi_128", "roi_full")
+
+
+def run_small_configs(args):
+    """The single-frame configs (tiny, nuScenes- and Ouster-shaped, the ROI
+    coverage sweep): L2-resident, so reported as warm us per call, eager and
+    replayed from a CUDA graph, with no roofline claim. One JSON line."""
+    import torch
+
+    import paper_2608_15437_gb300 as mmbev
+
+    dev = torch.device("cuda", 0)
+    mmbev.load()
+    rows = {}
+    for name in SMALL_CONFIGS:
+        w = synth.CONFIGS[name]()
+        pts = torch.from_numpy(w.points).to(dev)
+        tf = torch.from_numpy(w.sweep_tf).to(dev)
+        rois = torch.from_numpy(np.ascontiguousarray(w.rois, np.float32).reshape(-1, 5)).to(dev)
+        rmax = max(1, int(np.max(np.diff(w.frame_roi_offsets))))
+        vx = mmbev.Voxelizer(w.num_points, rmax, w.max_voxels, w.num_frames, w.voxel_size,
+                             w.pc_range, w.max_pts_per_voxel, w.roi_margin, device=dev)
+
+        def call():
+            return vx(pts, w.sweep_offsets, tf, rois, w.frame_sweep_offsets, w.frame_roi_offsets)
+
+        for _ in range(max(3, args.warmup)):
+            call()
+        torch.cuda.synchronize(dev)
+        if vx.status() != 0:
+            raise RuntimeError(f"{name}: device status {vx.status():#x}")
+        _, lin, _ = mmbev.classify_points(pts, w.sweep_offsets, tf, rois, w.roi_margin,
+                                          w.voxel_size, w.pc_range, w.frame_sweep_offsets,
+                                          w.frame_roi_offsets, workspace=vx.workspace)
+        n_in = int((lin >= 0).sum().item())
+        nvox = int(vx.out.nvox.sum().item())
+        reps = max(20, min(args.steps, 200))
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        e0.record()
+        for _ in range(reps):
+            call()
+        e1.record()
+        torch.cuda.synchronize(dev)
+        eager = 1e3 * e0.elapsed_time(e1) / reps
+        g = torch.cuda.CUDAGraph()
+        cs = torch.cuda.Stream(dev)
+        with torch.cuda.graph(g, stream=cs):
+            call()
+        g.replay()
+        torch.cuda.synchronize(dev)
+        e0.record()
+        for _ in range(reps):
+            g.replay()
+        e1.record()
+        torch.cuda.synchronize(dev)
+        graph = 1e3 * e0.elapsed_time(e1) / reps
+        if vx.status() != 0:
+            raise RuntimeError(f"{name}: device status {vx.status():#x}")
+        rows[name] = {"points": int(w.num_points), "in_roi_points": n_in, "voxels": nvox,
+                      "rois": int(w.rois.reshape(-1, 5).shape[0]), "us_eager": round(eager, 2),
+                      "us_graph": round(graph, 2),
+                      "in_roi_points_per_s_graph": round(n_in / (graph * 1e-6), 1)}
+    print(json.dumps({"metric": "us per single-frame call (warm; eager and CUDA-graph replay)",
+                      "unit": "us", "n_gpus": 1, "data": "synthetic",
+                      "higher_is_better": False, "configs": rows}))
+    return 0
+
+
 def main():
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
@@ -541,7 +609,12 @@ def main():
     ap.add_argument("--frames", type=int, default=FRAMES,
                     help="frames per GPU (the headline workload is 32; fewer for small "
                          "profiling cases)")
+    ap.add_argument("--small-configs", action="store_true",
+                    help="instead of the headline: warm us per call of the single-frame "
+                         "configs (tiny, nuScenes, Ouster, ROI sweep)")
     args = ap.parse_args()
+    if args.small_configs:
+        return run_small_configs(args)
     if args.impl == "reference":
         return run_reference(args)
     return run_gpu(args)

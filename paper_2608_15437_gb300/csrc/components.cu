@@ -547,15 +547,20 @@ __device__ __forceinline__ int cc_window_lo(const CcArgs& a, size_t base, int n,
 template <class Lins>
 __device__ __forceinline__ void cc_cluster_joins(const CcArgs& a, const Lins& S, int lo, int f,
                                                  int nv, int v0, int v1, int R, int32_t* s_par,
-                                                 unsigned long long* s_set) {
+                                                 unsigned long long* s_set, int* s_next) {
     cg::cluster_group cl = cg::this_cluster();
     const size_t base = (size_t)f * (size_t)a.maxv;
     const int t = threadIdx.x, lane = t & 31;
     const LocalPar L{smem_addr(s_par), v0};
 
-    // 2. joins within this CTA's rows, on its own shared memory (whole warps
-    // iterate together); pairs reaching an earlier CTA wait
-    for (int w0 = v0 + (t & ~31); w0 < v1; w0 += kClThreads) {
+    // 2. joins within this CTA's rows, on its own shared memory; each warp
+    // takes the next 32 rows from a shared counter (join chains vary in
+    // length), and pairs reaching an earlier CTA wait
+    for (;;) {
+        int w0 = 0;
+        if (lane == 0) w0 = atomicAdd(s_next, 32);
+        w0 = __shfl_sync(0xFFFFFFFFu, w0, 0);
+        if (w0 >= v1) break;
         const int v = w0 + lane;
         int z = 0, y = 0, x = 0;
         const bool active = v < v1 && cc_coords(a, base + (size_t)v, z, y, x);
@@ -620,6 +625,7 @@ __global__ void __launch_bounds__(kClThreads, 1) k_cc_cluster(CcArgs a, int C, i
     // [kClSet] distinct pairs of roots, [rcap] parents, [kClLinMax] linear
     // indices of the rows [lo, v1)
     extern __shared__ unsigned long long s_dyn[];
+    __shared__ int s_next;   // the next row of the join phase
     unsigned long long* s_set = s_dyn;
     int32_t* s_par = reinterpret_cast<int32_t*>(s_dyn + kClSet);
     uint32_t* s_lin = reinterpret_cast<uint32_t*>(s_par + rcap);
@@ -632,6 +638,7 @@ __global__ void __launch_bounds__(kClThreads, 1) k_cc_cluster(CcArgs a, int C, i
     const size_t base = (size_t)f * (size_t)a.maxv;
     const int t = threadIdx.x, lane = t & 31;
     if (rank == 0 && t == 0) a.ncomp[f] = 0;
+    if (t == 0) s_next = v0;
     for (int i = t; i < kClSet; i += kClThreads) s_set[i] = 0ull;
 
     // the window of rows any of this CTA's rows may neighbour: from the
@@ -659,8 +666,8 @@ __global__ void __launch_bounds__(kClThreads, 1) k_cc_cluster(CcArgs a, int C, i
     cc_fill_unused(a, base, nv, rank * kClThreads + t, C * kClThreads);
     __syncthreads();
 
-    if (in_smem) cc_cluster_joins(a, SmemLins{s_lin, lo}, lo, f, nv, v0, v1, R, s_par, s_set);
-    else cc_cluster_joins(a, GL, lo, f, nv, v0, v1, R, s_par, s_set);
+    if (in_smem) cc_cluster_joins(a, SmemLins{s_lin, lo}, lo, f, nv, v0, v1, R, s_par, s_set, &s_next);
+    else cc_cluster_joins(a, GL, lo, f, nv, v0, v1, R, s_par, s_set, &s_next);
 
     // 6. labels, components (this CTA's rows only: no other CTA's memory is
     // touched past the last barrier)
