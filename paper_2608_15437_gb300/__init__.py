@@ -497,7 +497,8 @@ class Voxelizer:
 
     def run_host(self, h_points: torch.Tensor, sweep_offsets, h_sweep_tf: torch.Tensor,
                  h_rois: torch.Tensor, frame_sweep_offsets, frame_roi_offsets,
-                 chunk_frames: int = 8, stream=None, pack_dst: torch.Tensor | None = None) -> Outputs:
+                 chunk_frames: int = 8, stream=None, pack_dst: torch.Tensor | None = None,
+                 table_log2_override: int = 0) -> Outputs:
         """The batched call on pinned host inputs
         (``mmbev_voxelize_roi_batched_host``): chunks of ``chunk_frames``
         frames go up on a side stream while earlier chunks are voxelized.
@@ -525,7 +526,8 @@ class Voxelizer:
         # the staging buffers are reused across calls: copies of this call
         # start after the previous work on `st` has read them
         self._copy_stream.wait_stream(st)
-        opts = _ExecOpts(None, 0, float(self.rho_out), int(self.seed) & (2**64 - 1))
+        opts = _ExecOpts(None, int(table_log2_override), float(self.rho_out),
+                         int(self.seed) & (2**64 - 1))
         nr = h_rois.shape[0] if h_rois.dim() > 1 else h_rois.numel() // 5
         rc = lib.mmbev_voxelize_roi_batched_host(
             ctypes.c_void_p(h_points.data_ptr()), _hptr(so), len(so) - 1,

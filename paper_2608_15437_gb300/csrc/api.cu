@@ -168,7 +168,7 @@ int validate_common(const float* points, const int64_t* sweep_offsets, int32_t n
         d->frame_sweep_off[f] = fso[f];
         d->frame_roi_off[f] = fro[f];
     }
-    std::memset(p, 0, sizeof(Params));
+    *p = Params{};
     p->points = points;
     p->sweep_tf = sweep_tf;
     p->rois = rois;
@@ -307,7 +307,6 @@ int voxelize_batched(const float* points, const int64_t* sweep_offsets, int32_t 
                      bool keep_status) {
     HostDesc desc;  // ~25 KB; consumed by the prep launch's parameter copy
     Params p;
-    p.keep_status = keep_status ? 1 : 0;
     Grid g;
     int32_t rmax = 0;
     if (max_pts_per_voxel < 1 || max_pts_per_voxel > kMaxK || max_voxels < 0) return MMBEV_EINVAL;
@@ -320,6 +319,7 @@ int voxelize_batched(const float* points, const int64_t* sweep_offsets, int32_t 
                              roi_margin, voxel_size, range, num_frames, frame_sweep_offsets,
                              frame_roi_offsets, &p, &desc, &g, &rmax);
     if (rc != MMBEV_OK) return rc;
+    p.keep_status = keep_status ? 1 : 0;   // after validation, which resets p
     const Layout L = make_layout(p.num_points, num_rois, rmax, max_voxels, num_frames, g);
     if (L.total > workspace_bytes) return MMBEV_EWORKSPACE;
     bind_layout(&p, L, static_cast<uint8_t*>(workspace));

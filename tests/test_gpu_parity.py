@@ -745,3 +745,28 @@ def test_scatter_bev_update_equals_a_fresh_scatter(oracle_mod, mmbev_lib, cuda_d
         ref = oracle_mod.scatter_bev(run_oracle(oracle_mod, w), dims)
         assert np.array_equal(canvas.cpu().numpy().view(np.uint32), ref.view(np.uint32))
         prev = out
+
+
+@pytest.mark.gpu
+def test_host_input_call_keeps_an_early_chunks_status(mmbev_lib, cuda_dev):
+    """The workspace status accumulates over the chunks of a host-input call:
+    a table overflow in the first chunk is still reported after a later chunk
+    that fits."""
+    import torch
+    w = synth.concat_frames([synth.nuscenes_frame(1), synth.tiny(2)], "big_then_small")
+    rmax = int(np.max(np.diff(w.frame_roi_offsets)))
+    vx = mmbev_lib.Voxelizer(w.num_points, rmax, w.max_voxels, w.num_frames, w.voxel_size,
+                             w.pc_range, w.max_pts_per_voxel, w.roi_margin, device=cuda_dev)
+    h_pts = torch.from_numpy(np.ascontiguousarray(w.points)).pin_memory()
+    h_tf = torch.from_numpy(np.ascontiguousarray(w.sweep_tf)).pin_memory()
+    h_rois = torch.from_numpy(np.ascontiguousarray(w.rois, np.float32).reshape(-1, 5)).pin_memory()
+    # 1024 slots: too few for the first frame's voxels, enough for the second's
+    vx.run_host(h_pts, w.sweep_offsets, h_tf, h_rois, w.frame_sweep_offsets, w.frame_roi_offsets,
+                chunk_frames=1, table_log2_override=10)
+    torch.cuda.synchronize(cuda_dev)
+    assert vx.status() & mmbev_lib.DEV_TABLE_FULL   # from the first chunk
+    # the next call starts clean: the first chunk resets the status
+    vx.run_host(h_pts, w.sweep_offsets, h_tf, h_rois, w.frame_sweep_offsets, w.frame_roi_offsets,
+                chunk_frames=1)
+    torch.cuda.synchronize(cuda_dev)
+    assert vx.status() == 0
