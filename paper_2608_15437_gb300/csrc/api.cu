@@ -184,6 +184,8 @@ int validate_common(const float* points, const int64_t* sweep_offsets, int32_t n
         p->dims[a] = g->dims[a];
     }
     p->cells = (uint32_t)g->cells;
+    p->div_nx = udiv_make(g->dims[0]);
+    p->div_ny = udiv_make(g->dims[1]);
     *max_rois_frame = rmax;
     return MMBEV_OK;
 }

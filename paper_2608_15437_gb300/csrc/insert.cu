@@ -41,10 +41,12 @@ constexpr int kBlocksPerSm = 8;
 constexpr int kFrameWin = 64;
 constexpr uint32_t kFull = 0xFFFFFFFFu;
 
-// Prefix sums of the classify blocks' list lengths (s_off[0..G]) and the
-// first entry of each list (list l starts at tile t_begin(l) * 2048).
+// Prefix sums of the classify blocks' list lengths (off[0..G]) and the
+// first plist entry of each list (list l starts at tile t_begin(l) * 2048;
+// record positions, and so entries, fit in 32 bits).
 struct Lists {
     uint32_t off[kMaxClsGrid + 1];
+    uint32_t start[kMaxClsGrid];
 };
 
 // Every thread must call it (one barrier). Returns the entry count.
@@ -59,8 +61,10 @@ __device__ __forceinline__ uint32_t lists_scan(const Params& p, Lists& L, uint32
         const uint32_t l = (uint32_t)t * 4 + k;
         c[k] = 0;
         if (l < G) {
-            const uint64_t room = ((uint64_t)(l + 1) * T / G - (uint64_t)l * T / G) * kTile;
+            const uint64_t t0 = (uint64_t)l * T / G;
+            const uint64_t room = ((uint64_t)(l + 1) * T / G - t0) * kTile;
             c[k] = (uint32_t)min((uint64_t)ld_cg(&p.cls_cnt[l]), room);
+            L.start[l] = (uint32_t)(t0 * kTile);
         }
         sum += c[k];
     }
@@ -93,8 +97,7 @@ __device__ __forceinline__ size_t list_entry(const Params& p, const Lists& L, ui
         const uint32_t mid = (lo + hi) >> 1;
         if (L.off[mid] <= i) lo = mid; else hi = mid;
     }
-    const uint64_t T = (uint64_t)p.num_regions / (kTile / kRegion);
-    return (size_t)((uint64_t)lo * T / G) * kTile + (i - L.off[lo]);
+    return (size_t)L.start[lo] + (i - L.off[lo]);
 }
 
 __global__ void __launch_bounds__(kThreads, kBlocksPerSm) k_insert(Params p) {

@@ -64,6 +64,29 @@ constexpr uint32_t kSpinLimit = 1u << 22;
 
 constexpr uint32_t kUnset = 0xFFFFFFFFu;
 
+// Unsigned 32-bit division by a divisor fixed for the whole call, by one
+// multiply-high and two shifts (Granlund and Montgomery, "Division by
+// Invariant Integers using Multiplication", PLDI 1994, Fig. 4.1): with
+// l = ceil(log2 d) and m = floor(2^32 (2^l - d) / d) + 1 (32 bits),
+// n / d = (t + ((n - t) >> min(l, 1))) >> max(l - 1, 0), t = mulhi(m, n),
+// exact for every 1 <= d < 2^32 and 0 <= n < 2^32.
+struct UDiv {
+    uint32_t m, s1, s2;
+};
+inline UDiv udiv_make(uint32_t d) {
+    uint32_t l = 0;
+    while (l < 32 && (1ull << l) < (uint64_t)d) ++l;
+    UDiv u;
+    u.m = (uint32_t)((((1ull << l) - d) << 32) / d + 1ull);
+    u.s1 = l < 1 ? l : 1u;
+    u.s2 = l > 1 ? l - 1u : 0u;
+    return u;
+}
+__device__ __forceinline__ uint32_t udiv(const UDiv& u, uint32_t n) {
+    const uint32_t t = __umulhi(u.m, n);
+    return (t + ((n - t) >> u.s1)) >> u.s2;
+}
+
 // Prepared ROI: centre, cos/sin of yaw, half-extents grown by the margin.
 struct __align__(16) RoiPrep {
     float cx, cy, c, s;
@@ -114,6 +137,7 @@ struct Params {
     float coarse_inv[2];    // coarse cells per metre along x, y
     uint32_t dims[3];       // nx, ny, nz
     uint32_t cells;         // nx*ny*nz
+    UDiv div_nx, div_ny;    // division by nx and by ny (voxel coordinates from lin)
     int32_t K;
     int32_t max_voxels;
     uint32_t rho_thr;       // keep a point inside no ROI when its draw's top 24 bits < rho_thr

@@ -309,6 +309,23 @@ __global__ void __launch_bounds__(kThreads) k_scatter(Params p) {
 }
 
 // ---------------------------------------------------------------- stage 8
+// Output row `vid` of frame f (call-wide index g) is the voxel in slot h with
+// linear index lin: its slot and coordinates.
+__device__ __forceinline__ void write_rank(const Params& p, uint32_t g, uint32_t f, uint32_t vid,
+                                           uint32_t h, uint32_t lin) {
+    p.vid_slot[g] = h;
+    // the slot's rank word is not read past this stage: it now holds the
+    // voxel's output index, for the finalize stage's heavy role (which starts
+    // from the slot)
+    *slot_rank(p, h) = g;
+    const size_t row = (size_t)f * (uint32_t)p.max_voxels + vid;
+    const uint32_t q = udiv(p.div_nx, lin);      // cz * ny + cy
+    const uint32_t cz = udiv(p.div_ny, q);
+    p.out_coords[row * 3 + 0] = (int32_t)cz;
+    p.out_coords[row * 3 + 1] = (int32_t)(q - cz * p.dims[1]);
+    p.out_coords[row * 3 + 2] = (int32_t)(lin - q * p.dims[0]);
+}
+
 // One warp per non-empty bucket (the scan's list), assigned round-robin.
 __global__ void __launch_bounds__(kRankWarps * 32) k_rank(Params p) {
     __shared__ uint32_t s_below[kRankWarps][kBmWords];
@@ -326,7 +343,6 @@ __global__ void __launch_bounds__(kRankWarps * 32) k_rank(Params p) {
     const uint32_t lbmask = (1u << p.bucket_log2) - 1u;
     const uint32_t U = min(ld_cg(&p.hdr->num_occ), p.occ_cap);
     const uint32_t NE = min(ld_cg(&p.hdr->num_nonempty), p.num_buckets);
-    const uint32_t nx = p.dims[0], ny = p.dims[1];
     const uint32_t Bf = p.buckets_per_frame;
     const uint32_t gw = blockIdx.x * kRankWarps + wl;
     const uint32_t nw = gridDim.x * kRankWarps;
@@ -342,6 +358,26 @@ __global__ void __launch_bounds__(kRankWarps * 32) k_rank(Params p) {
         const uint64_t start = (uint64_t)fi.ibase + a0 + c0;
         if (start + n > U) {
             if (lane == 0) set_status(p.hdr, MMBEV_DEV_BOUNDS);
+            continue;
+        }
+        if (!capped && n <= 32) {
+            // a bucket of at most 32 voxels in a frame under the cap (most
+            // buckets): lane i holds item i, and its rank in the bucket is
+            // the number of the bucket's (distinct) linear indices below its
+            // own, counted over the warp with shuffles
+            uint2 it = make_uint2(0u, 0u);
+            if ((uint32_t)lane < n) it = p.items[start + lane];
+            const uint32_t key = (uint32_t)lane < n ? (it.y & lbmask) : 0xFFFFFFFFu;
+            uint32_t r = 0;
+            for (uint32_t j = 0; j < n; ++j) r += __shfl_sync(0xFFFFFFFFu, key, j) < key;
+            if ((uint32_t)lane < n) {
+                const uint32_t vid = a0 + r;
+                if (vid < fi.nvox) write_rank(p, fi.vbase + vid, f, vid, it.x, it.y);
+                else {
+                    set_status(p.hdr, MMBEV_DEV_BOUNDS);
+                    zero_slot(p, it.x);
+                }
+            }
             continue;
         }
         for (int w = lane; w < nwords; w += 32) {
@@ -398,18 +434,7 @@ __global__ void __launch_bounds__(kRankWarps * 32) k_rank(Params p) {
             if (tie) { kept = c < fi.q; vid = A + c; }
             else { kept = true; vid = A + (c < fi.q ? c : fi.q); }
             if (kept && vid < fi.nvox) {
-                p.vid_slot[fi.vbase + vid] = h;
-                // the slot's rank word is not read past this stage: it now
-                // holds the voxel's output index, for the finalize stage's
-                // heavy role (which starts from the slot)
-                *slot_rank(p, h) = fi.vbase + vid;
-                const size_t row = (size_t)f * (uint32_t)p.max_voxels + vid;
-                const uint32_t cx = lin % nx;
-                const uint32_t cy = (lin / nx) % ny;
-                const uint32_t cz = lin / (nx * ny);
-                p.out_coords[row * 3 + 0] = (int32_t)cz;
-                p.out_coords[row * 3 + 1] = (int32_t)cy;
-                p.out_coords[row * 3 + 2] = (int32_t)cx;
+                write_rank(p, fi.vbase + vid, f, vid, h, lin);
             } else {
                 if (kept) set_status(p.hdr, MMBEV_DEV_BOUNDS);
                 zero_slot(p, h);  // dropped by the cap: release the slot
