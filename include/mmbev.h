@@ -228,7 +228,7 @@ int mmbev_get_status(const void *workspace, size_t workspace_bytes,
  *                     Outside [0, 1] or NaN: MMBEV_EINVAL.
  *   seed              the generator's seed.
  */
-#define MMBEV_NUM_STAGES 12
+#define MMBEV_NUM_STAGES 11
 typedef struct mmbev_exec_opts {
     cudaEvent_t *stage_events;
     int32_t table_log2_override;

@@ -240,7 +240,7 @@ void bind_layout(Params* p, const Layout& L, uint8_t* ws) {
     } while (0)
 
 const char* const kStageNames[MMBEV_NUM_STAGES] = {
-    "prep", "classify", "insert", "compact", "scatter_points", "capped_hist", "frames",
+    "prep", "classify", "insert", "compact", "scatter_points", "frames",
     "capped_census", "scan", "scatter", "rank", "finalize"};
 
 }  // namespace
@@ -395,9 +395,7 @@ int voxelize_batched(const float* points, const int64_t* sweep_offsets, int32_t 
         if ((e = mark()) != cudaSuccess) break;
         if ((e = launch_scatter_points(p, pdl, stream)) != cudaSuccess) break;
         if ((e = mark()) != cudaSuccess) break;
-        if ((e = launch_capped_hist(p, sms, pdl, stream)) != cudaSuccess) break;
-        if ((e = mark()) != cudaSuccess) break;
-        if ((e = launch_frames(p, pdl, stream)) != cudaSuccess) break;
+        if ((e = launch_frames(p, sms, pdl, stream)) != cudaSuccess) break;
         if ((e = mark()) != cudaSuccess) break;
         if ((e = launch_capped_census(p, sms, pdl, stream)) != cudaSuccess) break;
         if ((e = mark()) != cudaSuccess) break;

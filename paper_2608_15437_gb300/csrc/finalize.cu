@@ -307,8 +307,10 @@ __global__ void __launch_bounds__(kThreads) k_finalize(Params p, uint32_t heavy_
 }  // namespace
 
 cudaError_t launch_finalize(const Params& p, int num_sms, bool pdl, cudaStream_t st) {
-    const uint32_t heavy = (uint32_t)num_sms * 4;
-    const dim3 grid(num_sms * 12), block(kThreads);
+    // two heavy blocks per SM, six light ones: at 64 registers four blocks
+    // fit an SM, so the light blocks start while the heavy ones run
+    const uint32_t heavy = (uint32_t)num_sms * 2;
+    const dim3 grid(num_sms * 8), block(kThreads);
     if (p.K <= 4) return launch_k(k_finalize<4, 4>, grid, block, 0, st, pdl, p, heavy);
     if (p.K <= 12) return launch_k(k_finalize<12, 12>, grid, block, 0, st, pdl, p, heavy);
     if (p.K <= 32) return launch_k(k_finalize<32, 32>, grid, block, 0, st, pdl, p, heavy);

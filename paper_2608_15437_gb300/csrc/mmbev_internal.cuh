@@ -115,7 +115,8 @@ struct __align__(16) Header {
     uint32_t seg_total;    // point entries reserved in seg
     uint32_t num_heavy;    // kept voxels with 33 .. 1024 points
     uint32_t num_huge;     // kept voxels with more than 1024 points
-    uint32_t pad[7];
+    uint32_t frames_done;  // blocks of the frames stage that finished their histogram share
+    uint32_t pad[6];
 };
 
 // Everything a kernel needs; passed by value.
@@ -377,8 +378,7 @@ cudaError_t launch_insert(const Params& p, bool pdl, cudaStream_t st);
 cudaError_t launch_compact(const Params& p, bool pdl, cudaStream_t st);
 uint32_t insert_blocks(int num_sms);
 cudaError_t launch_scatter_points(const Params& p, bool pdl, cudaStream_t st);
-cudaError_t launch_capped_hist(const Params& p, int num_sms, bool pdl, cudaStream_t st);
-cudaError_t launch_frames(const Params& p, bool pdl, cudaStream_t st);
+cudaError_t launch_frames(const Params& p, int num_sms, bool pdl, cudaStream_t st);
 cudaError_t launch_capped_census(const Params& p, int num_sms, bool pdl, cudaStream_t st);
 cudaError_t launch_scan(const Params& p, bool pdl, cudaStream_t st);
 cudaError_t launch_scatter(const Params& p, int num_sms, bool pdl, cudaStream_t st);

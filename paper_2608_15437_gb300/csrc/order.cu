@@ -22,9 +22,9 @@
 // voxel's output position is A + min(c, q), where A counts below-voxels and
 // c counts tie-voxels with a smaller lin in the same frame.
 //
-//   capped hist     (stage 3)  rank histogram of capped frames
-//   frames          (stage 4)  per frame: r*, q, kept count, output base,
-//                              item-segment base
+//   frames          (stages 3-4) rank histogram of capped frames, then (the
+//                              last block) per frame: r*, q, kept count,
+//                              output base, item-segment base
 //   capped census   (stage 5)  per voxel of a capped frame: class, bucket count
 //   scan            (stage 6)  one block per chunk of 1024 buckets of a frame:
 //                              exclusive scan of counters
@@ -48,34 +48,18 @@ __device__ bool block_any_capped(const Params& p) {
     return __syncthreads_or(mine) != 0;
 }
 
-// ---------------------------------------------------------------- stage 3
-__global__ void __launch_bounds__(kThreads) k_capped_hist(Params p) {
-    pdl_wait();
-    if (!block_any_capped(p)) return;
-    const uint32_t U = min(ld_cg(&p.hdr->num_occ), p.occ_cap);
-    const uint32_t gs = gridDim.x * blockDim.x;
-    for (uint32_t d = blockIdx.x * blockDim.x + threadIdx.x; d < U; d += gs) {
-        const uint32_t f = p.d_bucket[d] / p.buckets_per_frame;
-        if (ld_cg(&p.frame_u[f]) <= (uint32_t)p.max_voxels) continue;
-        const int r0 = p.frame_roi_off[f];
-        const uint32_t rn = (uint32_t)(p.frame_roi_off[f + 1] - r0);  // background rank
-        const uint32_t r = min(slot_minrank(p, p.occ[d]), rn);
-        atomicAdd(&p.hist[r0 + f + r], 1u);
-    }
-}
-
-// ---------------------------------------------------------------- stage 4
-// One block; F <= 1024 frames.
-__global__ void __launch_bounds__(1024) k_frames(Params p) {
-    __shared__ uint32_t s_nvox[kMaxFrames];
-    __shared__ uint32_t s_u[kMaxFrames];
-    __shared__ uint32_t s_wsum[2][32];
-    pdl_wait();
+// ---------------------------------------------------------------- stages 3-4
+// Per frame: r*, q, kept count, output base, item-segment base, from the
+// minimum-rank histogram of the capped frames (F <= 1024 frames). Run by one
+// block of any multiple of 32 threads.
+__device__ void frames_body(const Params& p, uint32_t* s_nvox, uint32_t* s_u,
+                            uint32_t (*s_wsum)[32]) {
     const int t = threadIdx.x, lane = t & 31, warp = t >> 5;
+    const int nwarps = (int)(blockDim.x >> 5);
     const uint32_t maxv = (uint32_t)p.max_voxels;
     const int F = p.num_frames;
     uint32_t any_capped = 0;
-    for (int f = warp; f < F; f += 32) {
+    for (int f = warp; f < F; f += nwarps) {
         const uint32_t u = ld_cg(&p.frame_u[f]);
         FrameInfo fi{};
         if (u <= maxv) {
@@ -93,7 +77,7 @@ __global__ void __launch_bounds__(1024) k_frames(Params p) {
             fi.rstar = (uint32_t)rn;
             fi.q = 0;
             for (int c = 0; c < rn; c += 32) {
-                const uint32_t v = (c + lane < rn) ? p.hist[r0 + c + lane] : 0u;
+                const uint32_t v = (c + lane < rn) ? ld_cg(&p.hist[r0 + c + lane]) : 0u;
                 uint32_t inc = v;
 #pragma unroll
                 for (int o = 1; o < 32; o <<= 1) {
@@ -127,7 +111,7 @@ __global__ void __launch_bounds__(1024) k_frames(Params p) {
     __syncthreads();
     // exclusive scans over frames of nvox (output rows) and u (item segments)
     uint32_t carry_v = 0, carry_u = 0;
-    for (int c = 0; c < F; c += 1024) {
+    for (int c = 0; c < F; c += (int)blockDim.x) {
         const int f = c + t;
         const uint32_t v = f < F ? s_nvox[f] : 0u;
         const uint32_t u = f < F ? s_u[f] : 0u;
@@ -141,7 +125,8 @@ __global__ void __launch_bounds__(1024) k_frames(Params p) {
         if (lane == 31) { s_wsum[0][warp] = iv; s_wsum[1][warp] = iu; }
         __syncthreads();
         if (warp == 0) {
-            uint32_t a = s_wsum[0][lane], b = s_wsum[1][lane];
+            uint32_t a = lane < nwarps ? s_wsum[0][lane] : 0u;
+            uint32_t b = lane < nwarps ? s_wsum[1][lane] : 0u;
 #pragma unroll
             for (int o = 1; o < 32; o <<= 1) {
                 const uint32_t xa = __shfl_up_sync(0xFFFFFFFFu, a, o);
@@ -164,6 +149,36 @@ __global__ void __launch_bounds__(1024) k_frames(Params p) {
         __syncthreads();
     }
     if (t == 0) p.hdr->total_kept = carry_v;
+}
+
+// Every block adds the minimum ranks of its share of the voxels of capped
+// frames to their frame's histogram (nothing when no frame is capped); the
+// last block to finish, told by a counter, then runs the per-frame stage.
+__global__ void __launch_bounds__(kThreads) k_frames(Params p) {
+    __shared__ uint32_t s_nvox[kMaxFrames];
+    __shared__ uint32_t s_u[kMaxFrames];
+    __shared__ uint32_t s_wsum[2][32];
+    __shared__ uint32_t s_last;
+    pdl_wait();
+    if (block_any_capped(p)) {
+        const uint32_t U = min(ld_cg(&p.hdr->num_occ), p.occ_cap);
+        const uint32_t gs = gridDim.x * blockDim.x;
+        for (uint32_t d = blockIdx.x * blockDim.x + threadIdx.x; d < U; d += gs) {
+            const uint32_t f = p.d_bucket[d] / p.buckets_per_frame;
+            if (ld_cg(&p.frame_u[f]) <= (uint32_t)p.max_voxels) continue;
+            const int r0 = p.frame_roi_off[f];
+            const uint32_t rn = (uint32_t)(p.frame_roi_off[f + 1] - r0);  // background rank
+            const uint32_t r = min(slot_minrank(p, p.occ[d]), rn);
+            atomicAdd(&p.hist[r0 + f + r], 1u);
+        }
+    }
+    __threadfence();
+    __syncthreads();
+    if (threadIdx.x == 0) s_last = atomicAdd(&p.hdr->frames_done, 1u) == gridDim.x - 1u;
+    __syncthreads();
+    if (!s_last) return;
+    __threadfence();
+    frames_body(p, s_nvox, s_u, s_wsum);
 }
 
 // ---------------------------------------------------------------- stage 5
@@ -446,12 +461,8 @@ __global__ void __launch_bounds__(kRankWarps * 32) k_rank(Params p) {
 
 }  // namespace
 
-cudaError_t launch_capped_hist(const Params& p, int num_sms, bool pdl, cudaStream_t st) {
-    return launch_k(k_capped_hist, dim3(num_sms * 2), dim3(kThreads), 0, st, pdl, p);
-}
-
-cudaError_t launch_frames(const Params& p, bool pdl, cudaStream_t st) {
-    return launch_k(k_frames, dim3(1), dim3(1024), 0, st, pdl, p);
+cudaError_t launch_frames(const Params& p, int num_sms, bool pdl, cudaStream_t st) {
+    return launch_k(k_frames, dim3(num_sms * 2), dim3(kThreads), 0, st, pdl, p);
 }
 
 cudaError_t launch_capped_census(const Params& p, int num_sms, bool pdl, cudaStream_t st) {

@@ -6,9 +6,12 @@
 // copies with an L2 evict-first policy, counted on the buffer's mbarrier: on
 // GB300 a single 40 KB bulk copy per tile streams at about a quarter of HBM
 // bandwidth, eight concurrent ones at nearly all of it. The warps never wait
-// for each other: each warp classifies its own 64 points of a tile, and the
-// last warp to have read its points from a buffer (a shared-memory counter)
-// refills it with the tile one ring length ahead.
+// for each other: they take 64-point chunks (32 to a tile) in increasing
+// order from a shared-memory counter, each as soon as it has finished the
+// last, and whichever warp finishes the last chunk of a buffer's tile (a
+// shared-memory counter) refills it with the tile one ring length ahead. A
+// fixed chunk per warp and tile would make every tile wait for its slowest
+// chunk: chunks whose points meet many ROIs cost several times the others.
 // Per point: Eq. 6 motion compensation, range crop, Alg. 1 inside-ROI test
 // (coarse candidate mask, then the exact rotated-box test in rank order;
 // the first hit is the point's rank; a point inside no ROI is kept with
@@ -96,7 +99,7 @@ struct ClsSmem {
     int32_t* sr0;     // [S] first ROI of that frame
     uint64_t* full;   // [nstages] tile arrived
     uint32_t* done;   // [nstages] warps finished with the buffer
-    uint32_t* kept;   // [2] kept points of the block, warps finished
+    uint32_t* kept;   // [4] kept points of the block, warps finished, next chunk, -
 };
 
 __host__ __device__ inline size_t align16(size_t o) { return (o + 15) & ~(size_t)15; }
@@ -107,7 +110,7 @@ __host__ __device__ inline size_t classify_smem_bytes(int S, int rmax, int nstag
     o += tf_staged ? (size_t)S * 48 : 0;
     o += (size_t)(S + 1) * 8 + (size_t)S * 8;
     o = align16(o);
-    return o + (size_t)nstages * 8 + (size_t)nstages * 4 + 8;
+    return o + (size_t)nstages * 8 + (size_t)nstages * 4 + 16;
 }
 
 __device__ __forceinline__ ClsSmem carve(unsigned char* smem, int S, int rmax, bool tf_staged,
@@ -135,6 +138,241 @@ __device__ __forceinline__ ClsSmem carve(unsigned char* smem, int S, int rmax, b
     o += (size_t)nstages * 4;
     s.kept = reinterpret_cast<uint32_t*>(smem + o);
     return s;
+}
+
+// Lanes 0..kChunks-1 of one warp each move one chunk of a tile into
+// buffer `stage`.
+__device__ __forceinline__ void issue_tile(const Params& p, const ClsSmem& sm, int stage,
+                                           int64_t tile, int lane, uint64_t pol) {
+    if (lane < kChunks) {
+        const size_t off = (size_t)lane * kChunkBytes;
+        mbar_expect_tx(&sm.full[stage], kChunkBytes);
+        tma_load(reinterpret_cast<unsigned char*>(sm.stages + (size_t)stage * kTile * 5) + off,
+                 reinterpret_cast<const unsigned char*>(p.points + tile * kTile * 5) + off,
+                 kChunkBytes, &sm.full[stage], pol);
+    }
+}
+
+// The block's tile range, chunk after chunk. Work is handed out in chunks of
+// 64 points (a tile holds 32), in increasing order, from a shared-memory
+// counter: a warp takes the next chunk as soon as it is done with its
+// current one, so warps whose points meet many ROIs do not hold the others
+// back. A buffer is refilled, with the tile one ring length ahead, by
+// whichever warp finishes the last of its 32 chunks. Within a chunk, lane l
+// takes points 2l and 2l+1: their ten floats are five 8-byte shared loads,
+// conflict-free (lane stride 40 bytes). Lanes 0-15 cover the chunk's first
+// 32-point region, lanes 16-31 its second. kStaged: every frame of the range
+// has its mask and ROIs in shared memory. Point indices fit in 32 bits (the
+// host rejects more points). Returns false when a wait gave up.
+template <bool kStaged>
+__device__ __forceinline__ bool classify_range(const Params& p, const ClsSmem& sm, int rmax,
+                                               int nstages, int64_t t_begin, int64_t t_end,
+                                               int f_lo, int n_staged) {
+    const int lane = threadIdx.x & 31;
+    const int S = p.num_sweeps;
+    const bool tf_staged = S <= kTfStageMax;
+    const uint32_t N = (uint32_t)p.num_points;
+    const uint32_t full_tiles = N / kTile;
+    const int G2W = p.coarse * p.coarse * p.mask_words;
+    const uint64_t pol = evict_first_policy();
+    const uint32_t lt = (1u << lane) - 1u;
+    const uint32_t half_mask = lane < 16 ? 0x0000FFFFu : 0xFFFF0000u;
+    uint4* plist = p.plist + t_begin * kTile;   // room for every point of the range
+    const uint32_t nchunks = (uint32_t)(t_end - t_begin) * (uint32_t)kWarps;
+    const uint32_t tb = (uint32_t)t_begin;
+    // the sweep of this lane's current point and what depends on it (points
+    // only move forward: chunks are taken in increasing order)
+    int s = find_sweep(sm.soff, S, t_begin * kTile);
+    uint32_t next_off = 0;     // first index of the next sweep
+    float T[12];
+    uint32_t fr = 0;
+    uint32_t moff = 0, roff = 0;           // staged: the frame's mask / ROI offsets in shared memory
+    const uint32_t* fmask = nullptr;       // not staged: its mask and ROIs in global memory
+    const RoiPrep* frois = nullptr;
+    auto load_sweep = [&]() {
+        next_off = (uint32_t)sm.soff[s + 1];
+        if (tf_staged) {
+            const float4* t4 = reinterpret_cast<const float4*>(sm.tf + s * 12);
+            const float4 a = t4[0], b = t4[1], c = t4[2];
+            T[0] = a.x; T[1] = a.y; T[2] = a.z; T[3] = a.w;
+            T[4] = b.x; T[5] = b.y; T[6] = b.z; T[7] = b.w;
+            T[8] = c.x; T[9] = c.y; T[10] = c.z; T[11] = c.w;
+        } else {
+#pragma unroll
+            for (int c = 0; c < 12; ++c) T[c] = __ldg(p.sweep_tf + (size_t)s * 16 + c);
+        }
+        const int f = sm.sfr[s];
+        fr = (uint32_t)f;
+        if (kStaged) {
+            const int slot = f - f_lo;   // 0 or 1
+            moff = (uint32_t)slot * kMaskSmemWords;
+            roff = (uint32_t)(slot * rmax);
+        } else {
+            const int slot = f - f_lo;
+            if (slot >= 0 && slot < n_staged) {
+                fmask = sm.mask + slot * kMaskSmemWords;
+                frois = sm.rois + (size_t)slot * rmax;
+            } else {
+                fmask = p.masks + (size_t)f * G2W;
+                frois = p.roi_prep + sm.sr0[s];
+            }
+        }
+    };
+    load_sweep();
+    // ring position of tile t_begin + tt: buffer st, its round (fill count)
+    uint32_t tt = 0, round = 0;
+    int st = 0;
+    uint32_t c = 0;
+    if (lane == 0) c = atomicAdd(&sm.kept[2], 1u);
+    c = __shfl_sync(0xFFFFFFFFu, c, 0);
+    while (c < nchunks) {
+        uint32_t cn = 0;   // the warp's next chunk, fetched early
+        if (lane == 0) cn = atomicAdd(&sm.kept[2], 1u);
+        const uint32_t ct = c / (uint32_t)kWarps, sub = c % (uint32_t)kWarps;
+        while (tt < ct) {   // chunks only move forward
+            ++tt;
+            if (++st == nstages) {
+                st = 0;
+                ++round;
+            }
+        }
+        const uint32_t tile = tb + ct;
+        const uint32_t base = tile * (uint32_t)kTile;
+        const uint32_t j0 = sub * 64u + 2u * (uint32_t)lane;
+        const uint32_t i0 = base + j0;   // the lane's first point
+        float2 v0, v1, v2, v3, v4;
+        if (tile < full_tiles) {
+            if (!mbar_wait(&sm.full[st], round & 1u)) {
+                if (lane == 0) set_status(p.hdr, MMBEV_DEV_WAIT_TIMEOUT);
+                return false;
+            }
+            const float2* q2 =
+                reinterpret_cast<const float2*>(sm.stages + (size_t)st * kTile * 5 + 5 * j0);
+            v0 = q2[0]; v1 = q2[1]; v2 = q2[2]; v3 = q2[3]; v4 = q2[4];
+        } else {
+            // the ragged last tile never enters the ring: the lane reads its
+            // points (those below N) from global memory
+            const float* src = p.points + (size_t)i0 * 5;
+            float q[10];
+#pragma unroll
+            for (int k = 0; k < 10; ++k) q[k] = i0 + k / 5 < N ? __ldcs(src + k) : 0.f;
+            v0 = make_float2(q[0], q[1]); v1 = make_float2(q[2], q[3]);
+            v2 = make_float2(q[4], q[5]); v3 = make_float2(q[6], q[7]);
+            v4 = make_float2(q[8], q[9]);
+        }
+        // the chunk is done with the buffer once its reads are complete; the
+        // last of the tile's 32 chunks refills it
+        __threadfence_block();
+        __syncwarp();
+        {
+            uint32_t last = 0;
+            if (lane == 0)  // the counter only grows: a round ends at its kWarps-th arrival
+                last = atomicAdd(&sm.done[st], 1u) == (round + 1u) * kWarps - 1u;
+            last = __shfl_sync(0xFFFFFFFFu, last, 0);
+            if (last) {
+                const int64_t next = (int64_t)tile + nstages;
+                if (next < t_end && next < (int64_t)full_tiles) issue_tile(p, sm, st, next, lane, pol);
+            }
+        }
+        const float px[2] = {v0.x, v2.y}, py[2] = {v0.y, v3.x}, pz[2] = {v1.x, v3.y};
+        const float pi[2] = {v1.y, v4.x}, pd[2] = {v2.x, v4.y};
+        bool valid[2] = {false, false};
+        uint32_t lin[2] = {0u, 0u}, frk[2] = {0u, 0u};
+        int hit[2] = {-1, -1};
+        float x[2], y[2], z[2];
+        int cell[2] = {-1, -1};               // the point's coarse cell (-1: out of range)
+        uint32_t cmo[2] = {0u, 0u}, cro[2] = {0u, 0u};
+        const uint32_t* cm[2] = {nullptr, nullptr};
+        const RoiPrep* cr[2] = {nullptr, nullptr};
+        // a sweep boundary inside the chunk (rare) reloads per point
+        const bool cross = __any_sync(0xFFFFFFFFu, i0 + 1u >= next_off);
+#pragma unroll
+        for (int k = 0; k < 2; ++k) {
+            const uint32_t idx = i0 + (uint32_t)k;
+            if (cross && idx >= next_off && idx < N) {
+                while (s + 1 < S && (uint32_t)sm.soff[s + 1] <= idx) ++s;
+                load_sweep();
+            }
+            compensate(T, px[k], py[k], pz[k], x[k], y[k], z[k]);
+            int cl;
+            if (idx < N && point_cell(p, x[k], y[k], z[k], cl)) cell[k] = cl;
+            if (kStaged) {
+                cmo[k] = moff;
+                cro[k] = roff;
+            } else {
+                cm[k] = fmask;
+                cr[k] = frois;
+            }
+            frk[k] = fr;
+        }
+        // Alg. 1 ROI test in rank order over the union of the warp's
+        // candidates: each step tests one ROI index for all 64 points (a
+        // broadcast read when the warp's points share a frame); a point keeps
+        // its first hit.
+        for (int w = 0; w < p.mask_words; ++w) {
+            uint32_t m[2];
+#pragma unroll
+            for (int k = 0; k < 2; ++k) {
+                m[k] = 0u;
+                if (cell[k] >= 0 && hit[k] < 0) {
+                    const int wi = cell[k] * p.mask_words + w;
+                    m[k] = kStaged ? sm.mask[cmo[k] + wi] : cm[k][wi];
+                }
+            }
+            uint32_t u = __reduce_or_sync(0xFFFFFFFFu, m[0] | m[1]);
+            while (u) {
+                const int b = __ffs(u) - 1;
+                u &= u - 1u;
+#pragma unroll
+                for (int k = 0; k < 2; ++k)
+                    if (((m[k] >> b) & 1u) && hit[k] < 0 &&
+                        roi_hit(kStaged ? sm.rois + cro[k] : cr[k], w * 32 + b, x[k], y[k]))
+                        hit[k] = w * 32 + b;
+            }
+        }
+        // Alg. 1: an in-range point inside no ROI is kept with probability
+        // rho_out (a SplitMix64 draw keyed by its index within the frame)
+        if (p.rho_thr) {
+#pragma unroll
+            for (int k = 0; k < 2; ++k) {
+                if (hit[k] >= 0 || cell[k] < 0) continue;
+                const uint32_t f = frk[k];
+                const int64_t j = (int64_t)(i0 + k) - sm.soff[p.frame_sweep_off[f]];
+                if ((uint32_t)(splitmix64_nth(p.seed, (uint64_t)j + 1ull) >> 40) < p.rho_thr)
+                    hit[k] = p.frame_roi_off[f + 1] - p.frame_roi_off[f];  // rank R_f
+            }
+        }
+#pragma unroll
+        for (int k = 0; k < 2; ++k) valid[k] = hit[k] >= 0 && voxel_lin(p, x[k], y[k], z[k], lin[k]);
+        // compaction in the 32-point regions, input order kept: the record
+        // position of a kept point grows with its index
+        const uint32_t b0 = __ballot_sync(0xFFFFFFFFu, valid[0]);
+        const uint32_t b1 = __ballot_sync(0xFFFFFFFFu, valid[1]);
+        const uint32_t below = lt & half_mask;
+        const uint32_t rank0 = __popc(b0 & below) + __popc(b1 & below);
+        const uint32_t region = tile * (uint32_t)(kTile / kRegion) + sub * 2u + (uint32_t)(lane >> 4);
+        // the block's dense list of kept points (any order): one shared
+        // atomic per warp reserves the warp's entries
+        const uint32_t nk = __popc(b0) + __popc(b1);
+        uint32_t lbase = 0;
+        if (lane == 0 && nk) lbase = atomicAdd(&sm.kept[0], nk);
+        lbase = __shfl_sync(0xFFFFFFFFu, lbase, 0);
+#pragma unroll
+        for (int k = 0; k < 2; ++k) {
+            if (valid[k]) {
+                const uint32_t rk = rank0 + (k ? (uint32_t)valid[0] : 0u);
+                const uint32_t at = region * (uint32_t)kRegion + rk;
+                const uint32_t li = lbase + (k ? __popc(b0) + __popc(b1 & lt) : __popc(b0 & lt));
+                plist[li] = make_uint4(lin[k], frk[k], at, 0u);
+                uint4* rec = p.records + 2 * (size_t)at;
+                rec[0] = make_uint4(__float_as_uint(x[k]), __float_as_uint(y[k]),
+                                    __float_as_uint(z[k]), __float_as_uint(pi[k]));
+                rec[1] = make_uint4(__float_as_uint(pd[k]), (uint32_t)hit[k], 0u, 0u);
+            }
+        }
+        c = __shfl_sync(0xFFFFFFFFu, cn, 0);
+    }
+    return true;
 }
 
 __global__ void __launch_bounds__(kThreads, 1) k_classify(Params p, int rmax, int nstages) {
@@ -181,187 +419,24 @@ __global__ void __launch_bounds__(kThreads, 1) k_classify(Params p, int rmax, in
             mbar_init(&sm.full[s], kChunks);
             sm.done[s] = 0u;
         }
-        sm.kept[0] = sm.kept[1] = 0u;
+        sm.kept[0] = sm.kept[1] = sm.kept[2] = 0u;
         mbar_fence_init();
     }
     __syncthreads();
-    // lanes 0..kChunks-1 of one warp each move one chunk of a tile
-    auto issue = [&](int stage, int64_t tile) {
-        if (lane < kChunks) {
-            const size_t off = (size_t)lane * kChunkBytes;
-            mbar_expect_tx(&sm.full[stage], kChunkBytes);
-            tma_load(reinterpret_cast<unsigned char*>(sm.stages + (size_t)stage * kTile * 5) + off,
-                     reinterpret_cast<const unsigned char*>(p.points + tile * kTile * 5) + off,
-                     kChunkBytes, &sm.full[stage], pol);
-        }
-    };
     if (warp == 0)
         for (int s = 0; s < nstages; ++s) {
             const int64_t tile = t_begin + s;
-            if (tile < t_end && tile < full_tiles) issue(s, tile);
+            if (tile < t_end && tile < full_tiles) issue_tile(p, sm, s, tile, lane, pol);
         }
 
-    // Lane l takes points 2l and 2l+1 of the warp's 64: their ten floats are
-    // five 8-byte shared loads, conflict-free (lane stride 40 bytes). Lanes
-    // 0-15 cover region 2*warp, lanes 16-31 region 2*warp+1.
-    const uint32_t lt = (1u << lane) - 1u;
-    const uint32_t half_mask = lane < 16 ? 0x0000FFFFu : 0xFFFF0000u;
-    uint4* plist = p.plist + t_begin * kTile;   // room for every point of the range
-    // the sweep of this lane's current point and what depends on it
-    int s = find_sweep(sm.soff, S, t_begin * kTile + warp * 64 + 2 * lane);
-    int64_t next_off = 0;      // first index of the next sweep
-    float T[12];
-    uint32_t fr = 0;
-    const uint32_t* fmask = nullptr;
-    const RoiPrep* frois = nullptr;
-    auto load_sweep = [&]() {
-        next_off = sm.soff[s + 1];
-        if (tf_staged) {
-            const float4* t4 = reinterpret_cast<const float4*>(sm.tf + s * 12);
-            const float4 a = t4[0], b = t4[1], c = t4[2];
-            T[0] = a.x; T[1] = a.y; T[2] = a.z; T[3] = a.w;
-            T[4] = b.x; T[5] = b.y; T[6] = b.z; T[7] = b.w;
-            T[8] = c.x; T[9] = c.y; T[10] = c.z; T[11] = c.w;
-        } else {
-#pragma unroll
-            for (int c = 0; c < 12; ++c) T[c] = __ldg(p.sweep_tf + (size_t)s * 16 + c);
-        }
-        const int f = sm.sfr[s];
-        fr = (uint32_t)f;
-        const int slot = f - f_lo;
-        if (slot >= 0 && slot < n_staged) {
-            fmask = sm.mask + slot * kMaskSmemWords;
-            frois = sm.rois + (size_t)slot * rmax;
-        } else {
-            fmask = p.masks + (size_t)f * G2W;
-            frois = p.roi_prep + sm.sr0[s];
-        }
-    };
-    load_sweep();
-    int st = 0;
-    uint32_t parity = 0, round = 0;
-    for (int64_t tile = t_begin; tile < t_end; ++tile) {
-        float* sp = sm.stages + (size_t)st * kTile * 5;
-        const int64_t base = tile * kTile;
-        const int n = (int)((N - base) < kTile ? (N - base) : kTile);
-        if (tile < full_tiles) {
-            if (!mbar_wait(&sm.full[st], parity)) {
-                if (lane == 0) set_status(p.hdr, MMBEV_DEV_WAIT_TIMEOUT);
-                return;
-            }
-        } else {
-            // the ragged last tile: this warp loads its own 64 points
-            const float* src = p.points + base * 5;
-            for (int k = warp * 320 + lane; k < warp * 320 + 320 && k < n * 5; k += 32)
-                sp[k] = __ldcs(src + k);
-            __syncwarp();
-        }
-        const int j0 = warp * 64 + 2 * lane;
-        const float2* q2 = reinterpret_cast<const float2*>(sp + 5 * j0);
-        const float2 v0 = q2[0], v1 = q2[1], v2 = q2[2], v3 = q2[3], v4 = q2[4];
-        // the warp is done with the buffer once its reads are complete; the
-        // last warp of the round refills it
-        __threadfence_block();
-        __syncwarp();
-        {
-            uint32_t last = 0;
-            if (lane == 0)  // the counter only grows: a round ends at its kWarps-th arrival
-                last = atomicAdd(&sm.done[st], 1u) == (round + 1u) * kWarps - 1u;
-            last = __shfl_sync(0xFFFFFFFFu, last, 0);
-            if (last) {
-                const int64_t next = tile + nstages;
-                if (next < t_end && next < full_tiles) issue(st, next);
-            }
-        }
-        const float px[2] = {v0.x, v2.y}, py[2] = {v0.y, v3.x}, pz[2] = {v1.x, v3.y};
-        const float pi[2] = {v1.y, v4.x}, pd[2] = {v2.x, v4.y};
-        bool valid[2] = {false, false};
-        uint32_t lin[2] = {0u, 0u}, frk[2] = {0u, 0u};
-        int hit[2] = {-1, -1};
-        float x[2], y[2], z[2];
-        const uint32_t* cm[2] = {nullptr, nullptr};   // the point's coarse-cell mask words
-        const RoiPrep* cr[2] = {frois, frois};         // its frame's ROIs
-#pragma unroll
-        for (int k = 0; k < 2; ++k) {
-            x[k] = y[k] = z[k] = 0.f;
-            if (j0 + k < n) {
-                const int64_t idx = base + j0 + k;
-                if (idx >= next_off) {
-                    while (s + 1 < S && sm.soff[s + 1] <= idx) ++s;
-                    load_sweep();
-                }
-                compensate(T, px[k], py[k], pz[k], x[k], y[k], z[k]);
-                int cell;
-                if (point_cell(p, x[k], y[k], z[k], cell)) cm[k] = fmask + cell * p.mask_words;
-                cr[k] = frois;
-                frk[k] = fr;
-            }
-        }
-        // Alg. 1 ROI test in rank order over the union of the warp's
-        // candidates: each step tests one ROI index for all 64 points (a
-        // broadcast read when the warp's points share a frame); a point keeps
-        // its first hit.
-        for (int w = 0; w < p.mask_words; ++w) {
-            uint32_t m[2];
-#pragma unroll
-            for (int k = 0; k < 2; ++k) m[k] = (cm[k] && hit[k] < 0) ? cm[k][w] : 0u;
-            uint32_t u = __reduce_or_sync(0xFFFFFFFFu, m[0] | m[1]);
-            while (u) {
-                const int b = __ffs(u) - 1;
-                u &= u - 1u;
-#pragma unroll
-                for (int k = 0; k < 2; ++k)
-                    if (((m[k] >> b) & 1u) && hit[k] < 0 && roi_hit(cr[k], w * 32 + b, x[k], y[k]))
-                        hit[k] = w * 32 + b;
-            }
-        }
-        // Alg. 1: an in-range point inside no ROI is kept with probability
-        // rho_out (a SplitMix64 draw keyed by its index within the frame)
-        if (p.rho_thr) {
-#pragma unroll
-            for (int k = 0; k < 2; ++k) {
-                if (hit[k] >= 0 || !cm[k]) continue;
-                const uint32_t f = frk[k];
-                const int64_t j = base + j0 + k - sm.soff[p.frame_sweep_off[f]];
-                if ((uint32_t)(splitmix64_nth(p.seed, (uint64_t)j + 1ull) >> 40) < p.rho_thr)
-                    hit[k] = p.frame_roi_off[f + 1] - p.frame_roi_off[f];  // rank R_f
-            }
-        }
-#pragma unroll
-        for (int k = 0; k < 2; ++k) valid[k] = hit[k] >= 0 && voxel_lin(p, x[k], y[k], z[k], lin[k]);
-        // compaction in the 32-point regions, input order kept: the record
-        // position of a kept point grows with its index
-        const uint32_t b0 = __ballot_sync(0xFFFFFFFFu, valid[0]);
-        const uint32_t b1 = __ballot_sync(0xFFFFFFFFu, valid[1]);
-        const uint32_t below = lt & half_mask;
-        const uint32_t rank0 = __popc(b0 & below) + __popc(b1 & below);
-        const uint32_t region =
-            (uint32_t)(tile * (kTile / kRegion)) + (uint32_t)(warp * 2) + (lane >> 4);
-        // the block's dense list of kept points (any order): one shared
-        // atomic per warp reserves the warp's entries
-        const uint32_t nk = __popc(b0) + __popc(b1);
-        uint32_t lbase = 0;
-        if (lane == 0 && nk) lbase = atomicAdd(&sm.kept[0], nk);
-        lbase = __shfl_sync(0xFFFFFFFFu, lbase, 0);
-#pragma unroll
-        for (int k = 0; k < 2; ++k) {
-            if (valid[k]) {
-                const uint32_t rk = rank0 + (k ? (uint32_t)valid[0] : 0u);
-                const uint32_t at = region * (uint32_t)kRegion + rk;
-                const uint32_t li = lbase + (k ? __popc(b0) + __popc(b1 & lt) : __popc(b0 & lt));
-                plist[li] = make_uint4(lin[k], frk[k], at, 0u);
-                uint4* rec = p.records + 2 * (size_t)at;
-                rec[0] = make_uint4(__float_as_uint(x[k]), __float_as_uint(y[k]),
-                                    __float_as_uint(z[k]), __float_as_uint(pi[k]));
-                rec[1] = make_uint4(__float_as_uint(pd[k]), (uint32_t)hit[k], 0u, 0u);
-            }
-        }
-        if (++st == nstages) {
-            st = 0;
-            parity ^= 1u;
-            ++round;
-        }
-    }
+    // The frames of the block's range: when the (at most two) staged ones
+    // cover it, every mask and ROI read is a shared-memory read.
+    const int64_t last_pt = (t_end * kTile < N ? t_end * kTile : N) - 1;
+    const int f_hi = p.sweep_frame[find_sweep(p.sweep_off, S, last_pt)];
+    const bool ok = f_hi - f_lo < n_staged
+                        ? classify_range<true>(p, sm, rmax, nstages, t_begin, t_end, f_lo, n_staged)
+                        : classify_range<false>(p, sm, rmax, nstages, t_begin, t_end, f_lo, n_staged);
+    if (!ok) return;
     // the last warp to leave publishes the block's list length
     if (lane == 0) {
         __threadfence_block();
