@@ -504,7 +504,10 @@ class Voxelizer:
         frames go up on a side stream while earlier chunks are voxelized.
         With ``pack_dst`` (a uint8 tensor of ``pack_bytes``, on the device or
         pinned), each chunk's kept rows are packed there as it completes.
-        Device staging is allocated on first use and kept."""
+        Device staging is allocated on first use and kept: two sets, used in
+        turn, so that a call's uploads can run while the previous call still
+        computes (they wait only for the call before that one to have
+        finished reading the set they overwrite)."""
         if pack_dst is not None and (pack_dst.dtype != torch.uint8 or not pack_dst.is_contiguous()
                                      or not (pack_dst.is_cuda or pack_dst.is_pinned())):
             raise ValueError("pack_dst must be a contiguous uint8 device or pinned tensor")
@@ -518,14 +521,23 @@ class Voxelizer:
         dev = self.out.nvox.device
         need = (h_points.shape, h_sweep_tf.shape, h_rois.shape)
         if getattr(self, "_staging_shape", None) != need:
-            self._staging = tuple(torch.empty(sh, dtype=torch.float32, device=dev) for sh in need)
+            self._staging = [tuple(torch.empty(sh, dtype=torch.float32, device=dev) for sh in need)
+                             for _ in range(2)]
+            self._staging_read = [None, None]   # event: the last call using the set is done
+            self._staging_next = 0
             self._staging_shape = need
             self._copy_stream = torch.cuda.Stream(device=dev)
-        d_pts, d_tf, d_rois = self._staging
+        k = self._staging_next
+        self._staging_next = 1 - k
+        d_pts, d_tf, d_rois = self._staging[k]
         st = stream if stream is not None else torch.cuda.current_stream(dev)
-        # the staging buffers are reused across calls: copies of this call
-        # start after the previous work on `st` has read them
-        self._copy_stream.wait_stream(st)
+        # this call's copies overwrite set k: they start once the call that
+        # last read it has finished (on first use, after the earlier work on
+        # `st`)
+        if self._staging_read[k] is None:
+            self._copy_stream.wait_stream(st)
+        else:
+            self._copy_stream.wait_event(self._staging_read[k])
         opts = _ExecOpts(None, int(table_log2_override), float(self.rho_out),
                          int(self.seed) & (2**64 - 1))
         nr = h_rois.shape[0] if h_rois.dim() > 1 else h_rois.numel() // 5
@@ -542,6 +554,9 @@ class Voxelizer:
             _stream(self._copy_stream),
             ctypes.byref(opts))
         _check(rc, "mmbev_voxelize_roi_batched_host")
+        done = torch.cuda.Event()
+        done.record(st)
+        self._staging_read[k] = done
         return self.out
 
     def status(self) -> int:

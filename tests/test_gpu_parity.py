@@ -770,3 +770,44 @@ def test_host_input_call_keeps_an_early_chunks_status(mmbev_lib, cuda_dev):
                 chunk_frames=1)
     torch.cuda.synchronize(cuda_dev)
     assert vx.status() == 0
+
+
+@pytest.mark.gpu
+def test_back_to_back_host_calls_without_a_sync(mmbev_lib, cuda_dev):
+    """Host-input calls issued back to back, with no synchronization between
+    them: a call's uploads may overlap the previous call's work (the binding
+    alternates two staging sets). Every call's packed rows equal those of the
+    device-input call on the same inputs."""
+    import torch
+    ws = [synth.concat_frames([synth.nuscenes_frame(s), synth.nuscenes_frame(s + 1)], f"pair{s}")
+          for s in (11, 21, 31)]
+    w0 = ws[0]
+    rmax = max(int(np.max(np.diff(w.frame_roi_offsets))) for w in ws)
+    mk = lambda: mmbev_lib.Voxelizer(w0.num_points, rmax, w0.max_voxels, w0.num_frames,
+                                     w0.voxel_size, w0.pc_range, w0.max_pts_per_voxel,
+                                     w0.roi_margin, device=cuda_dev)
+    nb = mmbev_lib.pack_bytes(w0.num_frames, w0.max_voxels)
+    ref = mk()
+    want = []
+    for w in ws:
+        pts, tf, rois = to_dev(w, cuda_dev)
+        out = ref(pts, w.sweep_offsets, tf, rois, w.frame_sweep_offsets, w.frame_roi_offsets)
+        buf = torch.zeros(nb, dtype=torch.uint8).pin_memory()
+        mmbev_lib.pack_voxels(out, w0.max_voxels, buf)
+        torch.cuda.synchronize(cuda_dev)
+        want.append(buf)
+    host = [tuple(torch.from_numpy(np.ascontiguousarray(a, np.float32).reshape(sh)).pin_memory()
+                  for a, sh in ((w.points, (-1, 5)), (w.sweep_tf, (-1, 16)), (w.rois, (-1, 5))))
+            for w in ws]
+    vx = mk()
+    got = [torch.full((nb,), 0xCD, dtype=torch.uint8).pin_memory() for _ in ws]
+    for rnd in range(2):
+        for w, (h_pts, h_tf, h_rois), dst in zip(ws, host, got):
+            vx.run_host(h_pts, w.sweep_offsets, h_tf, h_rois, w.frame_sweep_offsets,
+                        w.frame_roi_offsets, chunk_frames=1, pack_dst=dst)
+        torch.cuda.synchronize(cuda_dev)
+        assert vx.status() == 0
+        for i, (g, e) in enumerate(zip(got, want)):
+            total = int(e[4 * w0.num_frames:4 * w0.num_frames + 4].view(torch.int32)[0])
+            used = 4 * (w0.num_frames + 1) + 36 * total
+            assert torch.equal(g[:used], e[:used]), f"round {rnd}, call {i}"
