@@ -231,6 +231,7 @@ void bind_layout(Params* p, const Layout& L, uint8_t* ws) {
     p->coarse_inv[1] = (float)((double)L.coarse / ((double)p->rmax[1] - (double)p->rmin[1]));
     p->bucket_log2 = L.bucket_log2;
     p->buckets_per_frame = L.buckets_per_frame;
+    p->div_bf = udiv_make(L.buckets_per_frame);
     p->num_buckets = L.num_buckets;
 }
 

@@ -147,6 +147,7 @@ struct Params {
     // bucket ordering
     int32_t bucket_log2;
     uint32_t buckets_per_frame;
+    UDiv div_bf;            // division by buckets_per_frame (bucket -> frame)
     uint32_t num_buckets;   // num_frames * buckets_per_frame
     // hash table
     uint8_t* table;

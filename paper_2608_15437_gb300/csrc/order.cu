@@ -164,7 +164,7 @@ __global__ void __launch_bounds__(kThreads) k_frames(Params p) {
         const uint32_t U = min(ld_cg(&p.hdr->num_occ), p.occ_cap);
         const uint32_t gs = gridDim.x * blockDim.x;
         for (uint32_t d = blockIdx.x * blockDim.x + threadIdx.x; d < U; d += gs) {
-            const uint32_t f = p.d_bucket[d] / p.buckets_per_frame;
+            const uint32_t f = udiv(p.div_bf, p.d_bucket[d]);
             if (ld_cg(&p.frame_u[f]) <= (uint32_t)p.max_voxels) continue;
             const int r0 = p.frame_roi_off[f];
             const uint32_t rn = (uint32_t)(p.frame_roi_off[f + 1] - r0);  // background rank
@@ -217,7 +217,7 @@ __global__ void __launch_bounds__(kThreads) k_capped_census(Params p) {
         uint32_t b = 0;
         if (d < U) {
             b = p.d_bucket[d];
-            const FrameInfo fi = p.finfo[b / p.buckets_per_frame];
+            const FrameInfo fi = p.finfo[udiv(p.div_bf, b)];
             if (fi.capped) {
                 const uint32_t h = p.occ[d];
                 const uint32_t r = slot_minrank(p, h);
@@ -316,7 +316,7 @@ __global__ void __launch_bounds__(kThreads) k_scatter(Params p) {
         if (pos == kUnset) continue;
         const uint32_t b = p.d_bucket[d];
         const unsigned long long o = p.boff[b];
-        const uint64_t at = (uint64_t)p.finfo[b / p.buckets_per_frame].ibase + (uint32_t)o +
+        const uint64_t at = (uint64_t)p.finfo[udiv(p.div_bf, b)].ibase + (uint32_t)o +
                             (uint32_t)(o >> 32) + pos;
         if (at < U) p.items[at] = make_uint2(p.occ[d], p.d_lin[d]);
         else set_status(p.hdr, MMBEV_DEV_BOUNDS);
@@ -358,12 +358,11 @@ __global__ void __launch_bounds__(kRankWarps * 32) k_rank(Params p) {
     const uint32_t lbmask = (1u << p.bucket_log2) - 1u;
     const uint32_t U = min(ld_cg(&p.hdr->num_occ), p.occ_cap);
     const uint32_t NE = min(ld_cg(&p.hdr->num_nonempty), p.num_buckets);
-    const uint32_t Bf = p.buckets_per_frame;
     const uint32_t gw = blockIdx.x * kRankWarps + wl;
     const uint32_t nw = gridDim.x * kRankWarps;
     for (uint32_t e = gw; e < NE; e += nw) {
         const uint32_t b = p.nonempty[e];
-        const uint32_t f = b / Bf;
+        const uint32_t f = udiv(p.div_bf, b);
         const FrameInfo fi = p.finfo[f];
         const bool capped = fi.capped != 0;
         const unsigned long long cv = capped ? p.bcnt2[b] : p.bcnt[b];
@@ -375,18 +374,36 @@ __global__ void __launch_bounds__(kRankWarps * 32) k_rank(Params p) {
             if (lane == 0) set_status(p.hdr, MMBEV_DEV_BOUNDS);
             continue;
         }
-        if (!capped && n <= 32) {
-            // a bucket of at most 32 voxels in a frame under the cap (most
-            // buckets): lane i holds item i, and its rank in the bucket is
-            // the number of the bucket's (distinct) linear indices below its
-            // own, counted over the warp with shuffles
-            uint2 it = make_uint2(0u, 0u);
-            if ((uint32_t)lane < n) it = p.items[start + lane];
-            const uint32_t key = (uint32_t)lane < n ? (it.y & lbmask) : 0xFFFFFFFFu;
-            uint32_t r = 0;
-            for (uint32_t j = 0; j < n; ++j) r += __shfl_sync(0xFFFFFFFFu, key, j) < key;
-            if ((uint32_t)lane < n) {
-                const uint32_t vid = a0 + r;
+        if (!capped && n <= 64) {
+            // a bucket of at most 64 voxels in a frame under the cap (95 % of
+            // the buckets of 32 nuScenes-shaped frames): lane i holds items i
+            // and i + 32, and an item's rank in the bucket is the number of
+            // the bucket's (distinct) linear indices below its own, counted
+            // over the warp with shuffles
+            const uint32_t i1 = (uint32_t)lane + 32u;
+            uint2 it0 = make_uint2(0u, 0u), it1 = make_uint2(0u, 0u);
+            if ((uint32_t)lane < n) it0 = p.items[start + lane];
+            if (i1 < n) it1 = p.items[start + i1];
+            const uint32_t k0 = (uint32_t)lane < n ? (it0.y & lbmask) : 0xFFFFFFFFu;
+            const uint32_t k1 = i1 < n ? (it1.y & lbmask) : 0xFFFFFFFFu;
+            uint32_t r0 = 0, r1 = 0;
+            const uint32_t n0 = n < 32u ? n : 32u;
+            for (uint32_t j = 0; j < n0; ++j) {
+                const uint32_t x = __shfl_sync(0xFFFFFFFFu, k0, j);
+                r0 += x < k0;
+                r1 += x < k1;
+            }
+            for (uint32_t j = 32; j < n; ++j) {
+                const uint32_t x = __shfl_sync(0xFFFFFFFFu, k1, j - 32u);
+                r0 += x < k0;
+                r1 += x < k1;
+            }
+#pragma unroll
+            for (int q = 0; q < 2; ++q) {
+                const uint32_t idx = q ? i1 : (uint32_t)lane;
+                if (idx >= n) continue;
+                const uint2 it = q ? it1 : it0;
+                const uint32_t vid = a0 + (q ? r1 : r0);
                 if (vid < fi.nvox) write_rank(p, fi.vbase + vid, f, vid, it.x, it.y);
                 else {
                     set_status(p.hdr, MMBEV_DEV_BOUNDS);

@@ -35,11 +35,12 @@ namespace {
 
 constexpr int kThreads = 1024;
 constexpr int kWarps = kThreads / 32;         // 32
+constexpr int kTileChunks = kTile / 64;       // 64-point chunks per tile (32)
 constexpr int kTfStageMax = 512;              // sweeps whose transforms sit in smem
 constexpr int kMaskSmemWords = 4096;          // one staged frame's coarse mask (16 KB)
 constexpr int kChunks = 8;                    // bulk copies per tile
 constexpr int kChunkBytes = kTileBytes / kChunks;
-static_assert(kTile == kWarps * 2 * kRegion, "a warp covers two regions of a tile");
+static_assert(kTile == kTileChunks * 2 * kRegion, "a chunk covers two regions of a tile");
 
 // ---- TMA / mbarrier helpers (inline PTX)
 __device__ __forceinline__ uint32_t smem_addr(const void* p) {
@@ -178,7 +179,7 @@ __device__ __forceinline__ bool classify_range(const Params& p, const ClsSmem& s
     const uint32_t lt = (1u << lane) - 1u;
     const uint32_t half_mask = lane < 16 ? 0x0000FFFFu : 0xFFFF0000u;
     uint4* plist = p.plist + t_begin * kTile;   // room for every point of the range
-    const uint32_t nchunks = (uint32_t)(t_end - t_begin) * (uint32_t)kWarps;
+    const uint32_t nchunks = (uint32_t)(t_end - t_begin) * (uint32_t)kTileChunks;
     const uint32_t tb = (uint32_t)t_begin;
     // the sweep of this lane's current point and what depends on it (points
     // only move forward: chunks are taken in increasing order)
@@ -228,7 +229,7 @@ __device__ __forceinline__ bool classify_range(const Params& p, const ClsSmem& s
     while (c < nchunks) {
         uint32_t cn = 0;   // the warp's next chunk, fetched early
         if (lane == 0) cn = atomicAdd(&sm.kept[2], 1u);
-        const uint32_t ct = c / (uint32_t)kWarps, sub = c % (uint32_t)kWarps;
+        const uint32_t ct = c / (uint32_t)kTileChunks, sub = c % (uint32_t)kTileChunks;
         while (tt < ct) {   // chunks only move forward
             ++tt;
             if (++st == nstages) {
@@ -266,8 +267,8 @@ __device__ __forceinline__ bool classify_range(const Params& p, const ClsSmem& s
         __syncwarp();
         {
             uint32_t last = 0;
-            if (lane == 0)  // the counter only grows: a round ends at its kWarps-th arrival
-                last = atomicAdd(&sm.done[st], 1u) == (round + 1u) * kWarps - 1u;
+            if (lane == 0)  // the counter only grows: a round ends at its kTileChunks-th arrival
+                last = atomicAdd(&sm.done[st], 1u) == (round + 1u) * kTileChunks - 1u;
             last = __shfl_sync(0xFFFFFFFFu, last, 0);
             if (last) {
                 const int64_t next = (int64_t)tile + nstages;
