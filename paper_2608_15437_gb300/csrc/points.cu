@@ -9,9 +9,10 @@
 // for each other: they take 64-point chunks (32 to a tile) in increasing
 // order from a shared-memory counter, each as soon as it has finished the
 // last, and whichever warp finishes the last chunk of a buffer's tile (a
-// shared-memory counter) refills it with the tile one ring length ahead. A
-// fixed chunk per warp and tile would make every tile wait for its slowest
-// chunk: chunks whose points meet many ROIs cost several times the others.
+// shared-memory counter) refills it with the tile one ring length ahead. With
+// a fixed chunk per warp and tile, warps instead polled the barrier of a tile
+// that one slow chunk held back (chunks whose points meet many ROIs cost
+// several times the others).
 // Per point: Eq. 6 motion compensation, range crop, Alg. 1 inside-ROI test
 // (coarse candidate mask, then the exact rotated-box test in rank order;
 // the first hit is the point's rank; a point inside no ROI is kept with
