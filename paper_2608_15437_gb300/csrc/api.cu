@@ -49,13 +49,17 @@ int mask_words_for(int32_t max_rois_frame) {
     return w < 1 ? 1 : w;
 }
 
-// Coarse candidate grid: at most 4,096 mask words per frame, so a frame's
-// mask fits the classify kernel's 16 KB shared-memory slot.
+// Coarse candidate grid: G x G cells with G the largest even number (at most
+// 64) whose mask of G^2 * mask_words words fits the classify kernel's
+// shared-memory room per staged frame: 8,192 words (32 KB) up to 64 ROIs a
+// frame, 4,096 words beyond, where the staged ROI tables grow. Even G keeps
+// each frame's mask a whole number of 16-byte vectors.
 int coarse_for(int mask_words) {
-    if (mask_words <= 1) return 64;
-    if (mask_words <= 4) return 32;
-    if (mask_words <= 16) return 16;
-    return 8;
+    const int w = mask_words < 1 ? 1 : mask_words;
+    const int room = w <= 2 ? 8192 : 4096;
+    int g = 64;
+    while (g > 8 && g * g * w > room) g -= 2;
+    return g;
 }
 
 constexpr uint32_t kSlotStride = 16;

@@ -38,7 +38,7 @@ constexpr int kThreads = 1024;
 constexpr int kWarps = kThreads / 32;         // 32
 constexpr int kTileChunks = kTile / 64;       // 64-point chunks per tile (32)
 constexpr int kTfStageMax = 512;              // sweeps whose transforms sit in smem
-constexpr int kMaskSmemWords = 4096;          // one staged frame's coarse mask (16 KB)
+constexpr int kMaskSmemWords = 8192;          // largest staged coarse mask of a frame (32 KB)
 constexpr int kChunks = 8;                    // bulk copies per tile
 constexpr int kChunkBytes = kTileBytes / kChunks;
 static_assert(kTile == kTileChunks * 2 * kRegion, "a chunk covers two regions of a tile");
@@ -93,7 +93,7 @@ __device__ __forceinline__ bool mbar_wait(uint64_t* bar, uint32_t parity) {
 
 struct ClsSmem {
     float* stages;    // [nstages][kTile * 5]
-    uint32_t* mask;   // [2][kMaskSmemWords] coarse masks of the staged frames
+    uint32_t* mask;   // [2][coarse^2 * mask_words] coarse masks of the staged frames
     RoiPrep* rois;    // [2][rmax] prepared ROIs of the staged frames
     float* tf;        // [S][12] when staged
     int64_t* soff;    // [S+1]
@@ -106,23 +106,24 @@ struct ClsSmem {
 
 __host__ __device__ inline size_t align16(size_t o) { return (o + 15) & ~(size_t)15; }
 
-__host__ __device__ inline size_t classify_smem_bytes(int S, int rmax, int nstages) {
+// g2w: words of one frame's coarse mask (coarse^2 * mask_words).
+__host__ __device__ inline size_t classify_smem_bytes(int S, int rmax, int nstages, int g2w) {
     const bool tf_staged = S <= kTfStageMax;
-    size_t o = (size_t)nstages * kTileBytes + 2 * kMaskSmemWords * 4 + 2 * (size_t)rmax * 32;
+    size_t o = (size_t)nstages * kTileBytes + 2 * (size_t)g2w * 4 + 2 * (size_t)rmax * 32;
     o += tf_staged ? (size_t)S * 48 : 0;
     o += (size_t)(S + 1) * 8 + (size_t)S * 8;
     o = align16(o);
     return o + (size_t)nstages * 8 + (size_t)nstages * 4 + 16;
 }
 
-__device__ __forceinline__ ClsSmem carve(unsigned char* smem, int S, int rmax, bool tf_staged,
+__device__ __forceinline__ ClsSmem carve(unsigned char* smem, int S, int rmax, int g2w, bool tf_staged,
                                          int nstages) {
     ClsSmem s;
     size_t o = 0;
     s.stages = reinterpret_cast<float*>(smem);
     o += (size_t)nstages * kTileBytes;
     s.mask = reinterpret_cast<uint32_t*>(smem + o);
-    o += 2 * kMaskSmemWords * 4;
+    o += 2 * (size_t)g2w * 4;
     s.rois = reinterpret_cast<RoiPrep*>(smem + o);
     o += 2 * (size_t)rmax * 32;
     s.tf = reinterpret_cast<float*>(smem + o);
@@ -207,12 +208,12 @@ __device__ __forceinline__ bool classify_range(const Params& p, const ClsSmem& s
         fr = (uint32_t)f;
         if (kStaged) {
             const int slot = f - f_lo;   // 0 or 1
-            moff = (uint32_t)slot * kMaskSmemWords;
+            moff = (uint32_t)(slot * G2W);
             roff = (uint32_t)(slot * rmax);
         } else {
             const int slot = f - f_lo;
             if (slot >= 0 && slot < n_staged) {
-                fmask = sm.mask + slot * kMaskSmemWords;
+                fmask = sm.mask + slot * G2W;
                 frois = sm.rois + (size_t)slot * rmax;
             } else {
                 fmask = p.masks + (size_t)f * G2W;
@@ -383,7 +384,8 @@ __global__ void __launch_bounds__(kThreads, 1) k_classify(Params p, int rmax, in
     const int t = threadIdx.x, lane = t & 31, warp = t >> 5;
     const int S = p.num_sweeps;
     const bool tf_staged = S <= kTfStageMax;
-    ClsSmem sm = carve(smem, S, rmax, tf_staged, nstages);
+    const int G2W = p.coarse * p.coarse * p.mask_words;
+    ClsSmem sm = carve(smem, S, rmax, G2W, tf_staged, nstages);
 
     const int64_t N = p.num_points;
     const int64_t num_tiles = (N + kTile - 1) / kTile;
@@ -391,7 +393,6 @@ __global__ void __launch_bounds__(kThreads, 1) k_classify(Params p, int rmax, in
     const int64_t t_begin = (int64_t)blockIdx.x * num_tiles / gridDim.x;
     const int64_t t_end = ((int64_t)blockIdx.x + 1) * num_tiles / gridDim.x;
     if (t_begin >= t_end) return;
-    const int G2W = p.coarse * p.coarse * p.mask_words;
 
     for (int i = t; i <= S; i += kThreads) sm.soff[i] = p.sweep_off[i];
     for (int i = t; i < S; i += kThreads) {
@@ -410,7 +411,7 @@ __global__ void __launch_bounds__(kThreads, 1) k_classify(Params p, int rmax, in
         const int r0 = p.frame_roi_off[f];
         const int rn = min(p.frame_roi_off[f + 1] - r0, rmax);
         const uint32_t* gm = p.masks + (size_t)f * G2W;
-        for (int i = t; i < G2W; i += kThreads) sm.mask[k * kMaskSmemWords + i] = gm[i];
+        for (int i = t; i < G2W; i += kThreads) sm.mask[k * G2W + i] = gm[i];
         for (int i = t; i < rn * 2; i += kThreads)
             reinterpret_cast<float4*>(sm.rois + (size_t)k * rmax)[i] =
                 reinterpret_cast<const float4*>(p.roi_prep + r0)[i];
@@ -482,8 +483,10 @@ cudaError_t launch_classify(const Params& p, int rmax, int num_sms, bool pdl, cu
     if (rmax < 1) rmax = 1;
     constexpr size_t kSmemLimit = 227 * 1024;
     int nstages = 4;
-    while (nstages > 2 && classify_smem_bytes(p.num_sweeps, rmax, nstages) > kSmemLimit) --nstages;
-    const size_t smem = classify_smem_bytes(p.num_sweeps, rmax, nstages);
+    const int g2w = p.coarse * p.coarse * p.mask_words;
+    while (nstages > 2 && classify_smem_bytes(p.num_sweeps, rmax, nstages, g2w) > kSmemLimit)
+        --nstages;
+    const size_t smem = classify_smem_bytes(p.num_sweeps, rmax, nstages, g2w);
     if (smem > kSmemLimit) return cudaErrorInvalidValue;
     static std::atomic<int> configured[64];
     int dev = 0;

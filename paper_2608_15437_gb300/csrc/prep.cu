@@ -145,9 +145,9 @@ __global__ void k_zero(uint4* ptr, size_t n16, uint8_t* tail, size_t ntail) {
 
 }  // namespace
 
-// Largest coarse mask a frame block holds in shared memory: 4,096 words (the
+// Largest coarse mask a frame block holds in shared memory: 8,192 words (the
 // coarse grid shrinks as the ROI count grows).
-constexpr int kPrepSmemMax = 4096 * 4;
+constexpr int kPrepSmemMax = 8192 * 4;
 
 cudaError_t launch_prep(const Params& p, const HostDesc& d, cudaStream_t st) {
     // Raise the dynamic shared memory limit once per device (outside any
