@@ -53,6 +53,21 @@ def test_voxelize_parity(oracle_mod, mmbev_lib, cuda_dev, name):
     assert _table_is_clean(table)
 
 
+@pytest.mark.parametrize("n_rois", [33, 48, 64, 65, 96])
+def test_mask_sizes_between_the_configs(oracle_mod, mmbev_lib, cuda_dev, n_rois):
+    """ROI counts whose candidate masks the configs do not reach: two mask
+    words per cell on the 64 x 64 grid (33-64 ROIs: 32 KB per staged frame,
+    a ring of three tiles) and three words on a 36 x 36 grid (65-96 ROIs),
+    over three frames, so blocks stage two frames."""
+    w = synth.concat_frames([synth.roi_coverage(n_rois, scene_seed=s) for s in (1, 2, 3)],
+                            f"roi{n_rois}x3")
+    got, status, table, _ = run_gpu(mmbev_lib, w, cuda_dev)
+    assert status == 0
+    want = run_oracle(oracle_mod, w)
+    assert assert_frames_equal(got, want, w.name) == 1.0
+    assert _table_is_clean(table)
+
+
 def test_batch32_parity(oracle_mod, mmbev_lib, cuda_dev):
     """The benchmark's workload and launch configuration: 32 frames, 11.1 M
     points, one call."""
