@@ -1,4 +1,4 @@
-// Stages: voxel feature encoder (S5 of the path; Alg. 1 "VoxelFeatureEncoder").
+// Stage 10: voxel feature encoder (S5 of the path; Alg. 1 "VoxelFeatureEncoder").
 //
 // Each kept voxel's slot gives its point count n and the start of its
 // segment in `seg`, which lists the record positions of all n points (in

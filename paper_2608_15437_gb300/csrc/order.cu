@@ -1,4 +1,4 @@
-// Stages 3-8: voxel cap and canonical order (S4 of the path).
+// Stages 5-9: voxel cap and canonical order (S4 of the path).
 //
 // The voxels of a frame must come out in ascending linear index, and when a
 // frame has more than max_voxels voxels only the max_voxels smallest by
@@ -22,14 +22,14 @@
 // voxel's output position is A + min(c, q), where A counts below-voxels and
 // c counts tie-voxels with a smaller lin in the same frame.
 //
-//   frames          (stages 3-4) rank histogram of capped frames, then (the
+//   frames          (stage 5)  rank histogram of capped frames, then (the
 //                              last block) per frame: r*, q, kept count,
 //                              output base, item-segment base
-//   capped census   (stage 5)  per voxel of a capped frame: class, bucket count
-//   scan            (stage 6)  one block per chunk of 1024 buckets of a frame:
+//   capped census   (stage 6)  per voxel of a capped frame: class, bucket count
+//   scan            (stage 7)  one block per chunk of 1024 buckets of a frame:
 //                              exclusive scan of counters
-//   scatter         (stage 7)  voxel ids grouped by bucket
-//   rank            (stage 8)  per non-empty bucket: bitmaps, popcounts, output
+//   scatter         (stage 8)  voxel ids grouped by bucket
+//   rank            (stage 9)  per non-empty bucket: bitmaps, popcounts, output
 //                              position, coordinates
 #include "mmbev_internal.cuh"
 
@@ -48,7 +48,7 @@ __device__ bool block_any_capped(const Params& p) {
     return __syncthreads_or(mine) != 0;
 }
 
-// ---------------------------------------------------------------- stages 3-4
+// ---------------------------------------------------------------- stage 5
 // Per frame: r*, q, kept count, output base, item-segment base, from the
 // minimum-rank histogram of the capped frames (F <= 1024 frames). Run by one
 // block of any multiple of 32 threads.
@@ -181,7 +181,7 @@ __global__ void __launch_bounds__(kThreads) k_frames(Params p) {
     frames_body(p, s_nvox, s_u, s_wsum);
 }
 
-// ---------------------------------------------------------------- stage 5
+// ---------------------------------------------------------------- stage 6
 // Warp-aggregated atomicAdd on cnt[b] for the lanes with `mine` set (1 for a
 // rank-below voxel, 1<<32 for a rank-tie voxel); returns each such lane's
 // position in the bucket (old lo + old hi + the group lanes before it).
@@ -231,8 +231,8 @@ __global__ void __launch_bounds__(kThreads) k_capped_census(Params p) {
     }
 }
 
-// ---------------------------------------------------------------- stage 6
-// One block per frame: boff[b] = sum of the frame's counters before b.
+// ---------------------------------------------------------------- stage 7
+// boff[b] = sum of the frame's counters before b.
 constexpr int kScanThreads = (int)kScanChunk;   // one bucket per thread
 
 // One block per (frame, chunk of kScanChunk buckets): the chunk's base is the
@@ -306,7 +306,7 @@ __global__ void __launch_bounds__(kScanThreads) k_scan(Params p) {
     }
 }
 
-// ---------------------------------------------------------------- stage 7
+// ---------------------------------------------------------------- stage 8
 __global__ void __launch_bounds__(kThreads) k_scatter(Params p) {
     pdl_wait();
     const uint32_t U = min(ld_cg(&p.hdr->num_occ), p.occ_cap);
@@ -323,7 +323,7 @@ __global__ void __launch_bounds__(kThreads) k_scatter(Params p) {
     }
 }
 
-// ---------------------------------------------------------------- stage 8
+// ---------------------------------------------------------------- stage 9
 // Output row `vid` of frame f (call-wide index g) is the voxel in slot h with
 // linear index lin: its slot and coordinates.
 __device__ __forceinline__ void write_rank(const Params& p, uint32_t g, uint32_t f, uint32_t vid,
