@@ -112,9 +112,9 @@ __device__ __forceinline__ void finalize_light(const Params& p, const uint32_t* 
             for (int c = 0; c < 8; ++c) sorted_insert<B>(best, v[c]);
         }
         const int cnt = (int)(n < (uint32_t)K ? n : (uint32_t)K);
-        if (cnt > 0 && best[cnt - 1] >= p.rec_cap) set_status(p.hdr, MMBEV_DEV_BOUNDS);
         // the kept records, all loads of a round in flight, summed in order
-        constexpr int R = B < 6 ? B : 6;
+        // (constant indices into `best` keep it in registers)
+        constexpr int R = B < 3 ? B : 3;
         float acc[5] = {0.f, 0.f, 0.f, 0.f, 0.f};
 #pragma unroll
         for (int j0 = 0; j0 < B; j0 += R) {
@@ -123,7 +123,10 @@ __device__ __forceinline__ void finalize_light(const Params& p, const uint32_t* 
             float dt[R];
 #pragma unroll
             for (int c = 0; c < R; ++c)
-                if (j0 + c < cnt) load_record(p, best[j0 + c], ra[c], dt[c]);
+                if (j0 + c < cnt) {
+                    if (best[j0 + c] >= p.rec_cap) set_status(p.hdr, MMBEV_DEV_BOUNDS);
+                    load_record(p, best[j0 + c], ra[c], dt[c]);
+                }
 #pragma unroll
             for (int c = 0; c < R; ++c)
                 if (j0 + c < cnt) add_record(acc, ra[c], dt[c]);
@@ -286,8 +289,11 @@ __device__ __forceinline__ void finalize_heavy(const Params& p, const uint32_t* 
     }
 }
 
+// Up to K = 12, six blocks fit an SM (40 registers, no spill): the light
+// blocks start beside the heavy ones.
 template <int BL, int BH>
-__global__ void __launch_bounds__(kThreads) k_finalize(Params p, uint32_t heavy_blocks) {
+__global__ void __launch_bounds__(kThreads, (BL <= 12 ? 6 : 1))
+    k_finalize(Params p, uint32_t heavy_blocks) {
     __shared__ uint32_t s_vbase[kMaxFrames + 1];
     __shared__ uint32_t s_cand[kThreads / 32][kMaxK];
     pdl_wait();
@@ -307,8 +313,8 @@ __global__ void __launch_bounds__(kThreads) k_finalize(Params p, uint32_t heavy_
 }  // namespace
 
 cudaError_t launch_finalize(const Params& p, int num_sms, bool pdl, cudaStream_t st) {
-    // two heavy blocks per SM, six light ones: at 64 registers four blocks
-    // fit an SM, so the light blocks start while the heavy ones run
+    // two heavy blocks per SM, six light ones, so the light blocks start
+    // while the heavy ones run
     const uint32_t heavy = (uint32_t)num_sms * 2;
     const dim3 grid(num_sms * 8), block(kThreads);
     if (p.K <= 4) return launch_k(k_finalize<4, 4>, grid, block, 0, st, pdl, p, heavy);
