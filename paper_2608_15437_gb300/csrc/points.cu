@@ -367,10 +367,12 @@ __device__ __forceinline__ bool classify_range(const Params& p, const ClsSmem& s
                 const uint32_t at = region * (uint32_t)kRegion + rk;
                 const uint32_t li = lbase + (k ? __popc(b0) + __popc(b1 & lt) : __popc(b0 & lt));
                 plist[li] = make_uint4(lin[k], frk[k], at, 0u);
+                // records are read again only by the finalize stage: streaming
+                // stores leave L2 to the lists and the hash table in between
                 uint4* rec = p.records + 2 * (size_t)at;
-                rec[0] = make_uint4(__float_as_uint(x[k]), __float_as_uint(y[k]),
-                                    __float_as_uint(z[k]), __float_as_uint(pi[k]));
-                rec[1] = make_uint4(__float_as_uint(pd[k]), (uint32_t)hit[k], 0u, 0u);
+                __stcs(rec, make_uint4(__float_as_uint(x[k]), __float_as_uint(y[k]),
+                                       __float_as_uint(z[k]), __float_as_uint(pi[k])));
+                __stcs(rec + 1, make_uint4(__float_as_uint(pd[k]), (uint32_t)hit[k], 0u, 0u));
             }
         }
         c = __shfl_sync(0xFFFFFFFFu, cn, 0);
