@@ -257,6 +257,12 @@ typedef struct mmbev_exec_opts {
  *               serial).
  * Everything else as mmbev_voxelize_roi_batched_ex; opts->stage_events must
  * be NULL. The workspace status accumulates over the chunks.
+ * Ordering: the call is asynchronous. The host inputs must stay unchanged
+ * until the copies have run. The copies are ordered after earlier work on
+ * copy_stream only, not on `stream`: a caller that reuses the staging
+ * buffers makes copy_stream wait (an event) for the last call that read
+ * them. With two staging sets used in turn, a call's uploads overlap the
+ * previous call's work (the Python binding does this).
  */
 int mmbev_voxelize_roi_batched_host(
     const float *h_points, const int64_t *sweep_offsets, int32_t num_sweeps,
