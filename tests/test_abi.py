@@ -229,3 +229,15 @@ def test_scatter_bev_update_checks_its_arguments(mmbev_lib):
     bad = np.asarray([100, 0, 2], np.int32)
     assert lib.mmbev_scatter_bev_update(None, None, fake, fake, fake, 2, 10, bad.ctypes.data_as(P),
                                         P(0x7f3000000000), need, None) == -1
+
+
+def test_stage_names_follow_the_launch_order(mmbev_lib):
+    # one name per kernel of a call, in launch order; out of range: empty
+    names = mmbev_lib.stage_names()
+    assert names == ["prep", "classify", "insert", "compact", "scatter_points", "frames",
+                     "capped_census", "scan", "scatter", "rank", "finalize"]
+    lib = mmbev_lib.load()
+    assert lib.mmbev_stage_name(mmbev_lib.NUM_STAGES) == b""
+    assert lib.mmbev_stage_name(-1) == b""
+    text = open(HEADER).read()
+    assert re.search(r"#define MMBEV_NUM_STAGES\s+%d\b" % mmbev_lib.NUM_STAGES, text)
