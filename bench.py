@@ -71,7 +71,8 @@ def workload_desc(w):
         "frames_per_gpu": w.num_frames,
         "points_per_gpu": w.num_points,
         "input_mb_per_gpu": round(w.points.nbytes / 1e6, 1),
-        "l2": "inputs (222 MB/step) larger than the 129 MB L2; no flush",
+        "l2": ("inputs (222 MB/step) larger than the 129 MB L2, no flush in the timed region; "
+               "l2_flushed gives the call after a 258 MB buffer write"),
     }
 
 
@@ -141,6 +142,10 @@ class ClockSampler:
         for line in self.proc.stdout:
             self.lines.append(line.strip())
 
+    def mark(self) -> int:
+        """Index of the next sample: brackets a window for ``summary``."""
+        return len(self.lines)
+
     def stop(self):
         if self.proc is None:
             return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["nvidia-smi unavailable"]}
@@ -151,9 +156,15 @@ class ClockSampler:
             self.proc.kill()
         if self.thread:
             self.thread.join(timeout=2)
+        out = self.summary(0, len(self.lines))
+        out["window_s"] = round(time.perf_counter() - self.t0, 3)
+        return out
+
+    def summary(self, i0: int, i1: int):
+        """Median SM clock, max clock and throttle reasons of samples [i0, i1)."""
         sm, smax, reasons = [], [], set()
         names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
-        for ln in self.lines:
+        for ln in self.lines[i0:i1]:
             parts = [x.strip() for x in ln.split(",")]
             if len(parts) < 9:
                 continue
@@ -167,29 +178,72 @@ class ClockSampler:
                     reasons.add(name)
         return {"sm_mhz": float(np.median(sm)) if sm else None,
                 "sm_max_mhz": float(max(smax)) if smax else None,
-                "samples": len(sm), "window_s": round(time.perf_counter() - self.t0, 3),
-                "reasons": sorted(reasons)}
+                "samples": len(sm), "reasons": sorted(reasons)}
+
+
+def cpu_model() -> str:
+    """The host CPU's model name (lscpu, else /proc/cpuinfo)."""
+    try:
+        out = subprocess.run(["lscpu"], capture_output=True, text=True, timeout=10).stdout
+        for ln in out.splitlines():
+            if ln.strip().lower().startswith("model name"):
+                return ln.split(":", 1)[1].strip()
+    except (OSError, subprocess.SubprocessError):
+        pass
+    try:
+        with open("/proc/cpuinfo") as fh:
+            for ln in fh:
+                if ln.lower().startswith(("model name", "cpu model")):
+                    return ln.split(":", 1)[1].strip()
+    except OSError:
+        pass
+    return "unknown"
+
+
+class PinnedToOneCore:
+    """Run the enclosed block on one host core (the last one this process may
+    use), then restore the process's affinity."""
+
+    def __enter__(self):
+        self.saved = None
+        self.core = None
+        if hasattr(os, "sched_getaffinity"):
+            self.saved = os.sched_getaffinity(0)
+            self.core = max(self.saved)
+            os.sched_setaffinity(0, {self.core})
+        return self
+
+    def __exit__(self, *exc):
+        if self.saved is not None:
+            os.sched_setaffinity(0, self.saved)
+        return False
+
+
+def host_desc(pin):
+    return {"nproc": os.cpu_count(),
+            "allowed_cores": (len(pin.saved) if pin.saved is not None else None),
+            "pinned_core": pin.core, "cpu_model": cpu_model()}
 
 
 def cpu_oracle_baseline(w, budget_s: float = 12.0):
-    """The oracle as it stands, single-threaded on a host core, on whole
-    frames of the same batch until about budget_s seconds have run."""
+    """The oracle as it stands, single-threaded and pinned to one host core,
+    on whole frames of the same batch until about budget_s seconds have run."""
     import oracle
     oracle.build()
-    pts = 0
     frames = 0
-    t0 = time.perf_counter()
     f = 0
-    while True:
-        fw = w.frame(f % w.num_frames)
-        oracle.voxelize_roi(fw.points, fw.sweep_offsets, fw.sweep_tf, fw.rois, fw.roi_margin,
-                            fw.voxel_size, fw.pc_range, fw.max_pts_per_voxel, fw.max_voxels)
-        frames += 1
-        f += 1
-        if time.perf_counter() - t0 >= budget_s:
-            break
-    dt = time.perf_counter() - t0
-    return frames, dt
+    with PinnedToOneCore() as pin:
+        t0 = time.perf_counter()
+        while True:
+            fw = w.frame(f % w.num_frames)
+            oracle.voxelize_roi(fw.points, fw.sweep_offsets, fw.sweep_tf, fw.rois, fw.roi_margin,
+                                fw.voxel_size, fw.pc_range, fw.max_pts_per_voxel, fw.max_voxels)
+            frames += 1
+            f += 1
+            if time.perf_counter() - t0 >= budget_s:
+                break
+        dt = time.perf_counter() - t0
+    return frames, dt, host_desc(pin)
 
 
 def run_reference(args):
@@ -209,20 +263,21 @@ def run_reference(args):
     pts_done = 0
     times = []
     f = 0
-    for step in range(args.warmup + args.steps):
-        t0 = time.perf_counter()
-        npts = 0
-        for _ in range(per_step):
-            fw = frames[f % len(frames)]
-            oracle.voxelize_roi(fw.points, fw.sweep_offsets, fw.sweep_tf, fw.rois,
-                                fw.roi_margin, fw.voxel_size, fw.pc_range,
-                                fw.max_pts_per_voxel, fw.max_voxels)
-            npts += in_roi[f % len(frames)]
-            f += 1
-        dt = time.perf_counter() - t0
-        if step >= args.warmup:
-            times.append(dt)
-            pts_done += npts
+    with PinnedToOneCore() as pin:
+        for step in range(args.warmup + args.steps):
+            t0 = time.perf_counter()
+            npts = 0
+            for _ in range(per_step):
+                fw = frames[f % len(frames)]
+                oracle.voxelize_roi(fw.points, fw.sweep_offsets, fw.sweep_tf, fw.rois,
+                                    fw.roi_margin, fw.voxel_size, fw.pc_range,
+                                    fw.max_pts_per_voxel, fw.max_voxels)
+                npts += in_roi[f % len(frames)]
+                f += 1
+            dt = time.perf_counter() - t0
+            if step >= args.warmup:
+                times.append(dt)
+                pts_done += npts
     total = sum(times)
     value = pts_done / total
     line = {
@@ -233,7 +288,8 @@ def run_reference(args):
         "config": workload_desc(w),
         "cpu_baseline": {"kind": "oracle", "value": value, "unit": "points/s", "cores": 1,
                          "sample": f"{per_step} whole frames of the batch per step, "
-                                   "single-threaded C oracle"},
+                                   "single-threaded C oracle pinned to one core",
+                         **host_desc(pin)},
         "e2e": {"value": value, "unit": "points/s", "h2d_bytes_per_step": 0,
                 "d2h_bytes_per_step": 0},
     }
@@ -359,6 +415,37 @@ def run_gpu(args):
     if world > 1:
         dist.barrier()
     ms_total = start.elapsed_time(end)
+    i_timed = sampler.mark()
+    # a sustained window of the same calls, about a second and a half long, so
+    # that the clock samples (every 50 ms) describe the clock the calls ran at
+    n_sus = max(args.steps, int(1500.0 / max(ms_total / args.steps, 1e-3)))
+    i_sus = sampler.mark()
+    start.record(stream)
+    for k in range(n_sus):
+        step()
+    end.record(stream)
+    torch.cuda.synchronize(dev)
+    sus_ms = start.elapsed_time(end)
+    i_sus_end = sampler.mark()
+    sus_clock = sampler.summary(i_sus, i_sus_end)
+    sus_us = 1e3 * sus_ms / n_sus
+    sustained = {"calls": n_sus, "us_per_call": round(sus_us, 2), **sus_clock,
+                 "us_x_mhz": (round(sus_us * sus_clock["sm_mhz"], 1)
+                              if sus_clock.get("sm_mhz") else None)}
+    # each call after a write of a buffer twice the size of L2: nothing the
+    # previous call left in L2 (lists, counters, outputs) survives
+    flush = torch.empty(2 * 129 * 2**20 // 4, dtype=torch.float32, device=dev)
+    n_fl = max(3, min(args.steps, 50))
+    fl_ms = 0.0
+    for k in range(n_fl):
+        flush.fill_(float(k))
+        start.record(stream)
+        step()
+        end.record(stream)
+        torch.cuda.synchronize(dev)
+        fl_ms += start.elapsed_time(end)
+    del flush
+    l2_flushed = {"calls": n_fl, "us_per_call": round(1e3 * fl_ms / n_fl, 2)}
     # timed region 2, the per-kernel breakdown: the same K calls with a CUDA
     # event on the launching stream between consecutive kernels
     for k in range(args.steps):
@@ -404,7 +491,10 @@ def run_gpu(args):
         b1.record(stream)
         torch.cuda.synchronize(dev)
         bev_upd_us = 1e3 * b0.elapsed_time(b1) / args.steps
-    clocks = sampler.stop()
+    clocks_all = sampler.stop()
+    # the clocks of the timed region and the sustained window that follows it
+    clocks = sampler.summary(0, i_sus_end)
+    clocks["window_s"] = clocks_all.get("window_s")
     status = vx.status()
     if status != 0:
         raise RuntimeError(f"device status {status:#x} after the timed steps")
@@ -515,16 +605,22 @@ def run_gpu(args):
                          "frac": achieved / peak, "traffic": profile_traffic(names[dom])},
             "stage_sum_us": round(1e3 * float(stage_ms.sum()), 2),
             "clocks": clocks,
+            "sustained": sustained,
+            "l2_flushed": l2_flushed,
             "e2e": {"value": e2e_value, "unit": "points/s", "h2d_bytes_per_step": h2d_bytes,
                     "d2h_bytes_per_step": d2h_bytes, "steps": e2e_steps},
             "gpu_launches": nstage * args.steps,
         }
-        frames, secs = cpu_oracle_baseline(w)
+        if world == 1 and not args.no_small_configs:
+            # the single-frame configs (L2-resident, latency-bound): warm us
+            # per call, eager and replayed from a CUDA graph
+            line["single_frame_configs"] = small_config_rows(args, dev)
+        frames, secs, host = cpu_oracle_baseline(w)
         pts_per_frame = n_in_roi / w.num_frames
         line["cpu_baseline"] = {
             "kind": "oracle", "value": frames * pts_per_frame / secs, "unit": "points/s",
             "cores": 1, "sample": f"{frames} whole frames of this batch, single-threaded C "
-                                  f"oracle, {secs:.1f} s"}
+                                  f"oracle pinned to one core, {secs:.1f} s", **host}
         print(json.dumps(line), flush=True)
     if world > 1:
         dist.destroy_process_group()
@@ -534,16 +630,14 @@ def run_gpu(args):
 SMALL_CONFIGS = ("tiny", "nuscenes", "ouster", "roi_0", "roi_8", "roi_32", "roi_128", "roi_full")
 
 
-def run_small_configs(args):
+def small_config_rows(args, dev):
     """The single-frame configs (tiny, nuScenes- and Ouster-shaped, the ROI
     coverage sweep): L2-resident, so reported as warm us per call, eager and
-    replayed from a CUDA graph, with no roofline claim. One JSON line."""
+    replayed from a CUDA graph, with no roofline claim."""
     import torch
 
     import paper_2608_15437_gb300 as mmbev
 
-    dev = torch.device("cuda", 0)
-    mmbev.load()
     rows = {}
     for name in SMALL_CONFIGS:
         w = synth.CONFIGS[name]()
@@ -592,7 +686,20 @@ def run_small_configs(args):
         rows[name] = {"points": int(w.num_points), "in_roi_points": n_in, "voxels": nvox,
                       "rois": int(w.rois.reshape(-1, 5).shape[0]), "us_eager": round(eager, 2),
                       "us_graph": round(graph, 2),
+                      "kept_fraction": round(n_in / max(int(w.num_points), 1), 4),
                       "in_roi_points_per_s_graph": round(n_in / (graph * 1e-6), 1)}
+    return rows
+
+
+def run_small_configs(args):
+    """The single-frame configs alone, as one JSON line."""
+    import torch
+
+    import paper_2608_15437_gb300 as mmbev
+
+    dev = torch.device("cuda", 0)
+    mmbev.load()
+    rows = small_config_rows(args, dev)
     print(json.dumps({"metric": "us per single-frame call (warm; eager and CUDA-graph replay)",
                       "unit": "us", "n_gpus": 1, "data": "synthetic",
                       "higher_is_better": False, "configs": rows}))
@@ -626,6 +733,8 @@ def main():
     ap.add_argument("--frames", type=int, default=FRAMES,
                     help="frames per GPU (the headline workload is 32; fewer for small "
                          "profiling cases)")
+    ap.add_argument("--no-small-configs", action="store_true",
+                    help="leave the single-frame configs out of the headline line")
     ap.add_argument("--small-configs", action="store_true",
                     help="instead of the headline: warm us per call of the single-frame "
                          "configs (tiny, nuScenes, Ouster, ROI sweep)")

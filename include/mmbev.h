@@ -103,7 +103,7 @@ typedef enum mmbev_status {
  * Bytes of hash table for calls of up to max_points points (and
  * max_pts_per_voxel points kept per voxel, which must lie in
  * [1, MMBEV_MAX_PTS_PER_VOXEL] but does not change the size). The capacity
- * is the power of two >= 2*max_points slots of 32 bytes (load factor <= 1/2
+ * is the power of two >= 2*max_points slots of 16 bytes (load factor <= 1/2
  * whatever the inputs), each slot holding a voxel key, its minimum ROI rank,
  * its point count and the start of its point list. Returns 0 for invalid
  * arguments.
@@ -197,6 +197,19 @@ int mmbev_classify_points(const float *points, const int64_t *sweep_offsets,
                           const int32_t *frame_roi_offsets, float *out_xyz,
                           int64_t *out_lin, int32_t *out_rank,
                           void *workspace, size_t workspace_bytes, cudaStream_t stream);
+
+/*
+ * The prepared form of ROI boxes that the inside test of Alg. 1 uses (Eq. 1
+ * box with its margin; Sec. IV-F), as the voxelize calls compute it on the
+ * device, for checking against an independent evaluation:
+ *   rois        device, mmbev_roi_t [num_rois].
+ *   roi_margin  r of Eq. 1, >= 0 and finite.
+ *   out         device, float32 [num_rois][6]: cx, cy, c = (float)cos((double)yaw),
+ *               s = (float)sin((double)yaw), hl = 0.5f*l + r, hw = 0.5f*w + r.
+ * Asynchronous on `stream`; one kernel.
+ */
+int mmbev_prep_rois(const mmbev_roi_t *rois, int32_t num_rois, float roi_margin, float *out,
+                    cudaStream_t stream);
 
 /*
  * Copy the device status word of the last call that used `workspace` into
@@ -307,13 +320,16 @@ int mmbev_voxelize_roi_batched_ex(const float *points, const int64_t *sweep_offs
  *   Returns MMBEV_EWORKSPACE, before any launch, when the call needs more
  *   than the array holds: mmbev_table_size(N, K) rounded up to 256 bytes
  *   plus mmbev_workspace_size(N, num_rois, max_voxels, 1, voxel_size, range)
- *   must not exceed MMBEV_NOALLOC_SCRATCH_BYTES (a 400,000-point frame with
- *   K <= 12 fits).
- * The first call on a device looks up the array's device address with that
+ *   must not exceed MMBEV_NOALLOC_SCRATCH_BYTES. K does not enter the sum.
+ *   On the grids of the tiny, nuScenes- and Ouster-shaped workloads, with
+ *   their ROI counts and voxel caps, that allows up to about 575,000 points.
+ * The first call on a device (and the first in each new context of it, as
+ * after cudaDeviceReset) looks up the array's device address with that
  * device current; make that first call before any stream capture. Every
- * call zeroes the table part of the array first, since the array keeps the
- * previous call's contents. All calls on a device share the one array:
- * calls whose executions overlap on the GPU race and must be serialized.
+ * call zeroes the table part of the array first (16 bytes per slot of
+ * mmbev_table_size), since the array keeps the previous call's contents.
+ * All calls on a device share the one array: calls whose executions overlap
+ * on the GPU race and must be serialized.
  */
 #define MMBEV_NOALLOC_SCRATCH_BYTES (96u << 20)
 int mmbev_voxelize_roi_noalloc(const float *points, const int64_t *sweep_offsets,

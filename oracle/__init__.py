@@ -69,6 +69,8 @@ def _load():
         lib.oracle_crit_thresholds.restype = None
         lib.oracle_splitmix64.argtypes = [u64, u64]
         lib.oracle_splitmix64.restype = u64
+        lib.oracle_roi_boxes.argtypes = [P, i32, f32, P]
+        lib.oracle_roi_boxes.restype = None
         _lib = lib
     return _lib
 
@@ -101,6 +103,16 @@ def classify(points, sweep_offsets, sweep_tf, rois, roi_margin, voxel_size, pc_r
     if rc != 0:
         raise ValueError(f"oracle_classify failed with status {rc}")
     return xyz, lin, rank
+
+
+def roi_boxes(rois, roi_margin):
+    """The Eq. 1 box form of each ROI the inside test uses: float32 [R, 4] =
+    (cos(yaw), sin(yaw)) from libm in double rounded to fp32, and the
+    half-extents 0.5*l + r, 0.5*w + r in fp32."""
+    rois = _c(rois, np.float32).reshape(-1, 5)
+    out = np.zeros((rois.shape[0], 4), np.float32)
+    _load().oracle_roi_boxes(_ptr(rois), rois.shape[0], float(roi_margin), _ptr(out))
+    return out
 
 
 def splitmix64(seed, n):

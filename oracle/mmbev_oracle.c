@@ -104,15 +104,30 @@ static void compensate(const float *T, float x, float y, float z,
     a = T[8] * x; b = T[9] * y; a = a + b; c = T[10] * z; a = a + c; *zo = a + T[11];
 }
 
-/* Eq. 1 box, rotated by yaw, half-extents grown by the margin. The point is
- * inside when its coordinates in the box frame lie within the half-extents
- * (boundary included). l runs along the heading, w across it. */
+/* Eq. 1 box, rotated by yaw, half-extents grown by the margin: the heading's
+ * cosine and sine (libm, in double, rounded to fp32) and the two half-extents
+ * (l along the heading, w across it). */
+static void roi_box(const oracle_roi_t *r, float margin, float out[4])
+{
+    out[0] = (float)cos((double)r->yaw);
+    out[1] = (float)sin((double)r->yaw);
+    out[2] = 0.5f * r->l + margin;
+    out[3] = 0.5f * r->w + margin;
+}
+
+/* Exposed for the pins: roi_box of n ROIs, out[n][4] = (c, s, hl, hw). */
+void oracle_roi_boxes(const oracle_roi_t *r, int32_t n, float margin, float *out)
+{
+    for (int32_t i = 0; i < n; ++i) roi_box(&r[i], margin, out + 4 * (size_t)i);
+}
+
+/* The point is inside the box when its coordinates in the box frame lie
+ * within the half-extents (boundary included). */
 static int inside_roi(const oracle_roi_t *r, float margin, float x, float y)
 {
-    float c = (float)cos((double)r->yaw);
-    float s = (float)sin((double)r->yaw);
-    float hl = 0.5f * r->l + margin;
-    float hw = 0.5f * r->w + margin;
+    float box[4];
+    roi_box(r, margin, box);
+    float c = box[0], s = box[1], hl = box[2], hw = box[3];
     float dx = x - r->cx;
     float dy = y - r->cy;
     float p, q, u, v;

@@ -86,6 +86,8 @@ def load():
     lib.mmbev_classify_points.restype = ctypes.c_int
     lib.mmbev_voxelize_roi_noalloc.argtypes = vox + [P, P, P, P, P, P]
     lib.mmbev_voxelize_roi_noalloc.restype = ctypes.c_int
+    lib.mmbev_prep_rois.argtypes = [P, i32, f32, P, P]
+    lib.mmbev_prep_rois.restype = ctypes.c_int
     lib.mmbev_get_status.argtypes = [P, sz, ctypes.POINTER(ctypes.c_uint32), P]
     lib.mmbev_get_status.restype = ctypes.c_int
     lib.mmbev_stage_name.argtypes = [i32]
@@ -326,6 +328,18 @@ def classify_points(points: torch.Tensor, sweep_offsets, sweep_tf: torch.Tensor,
         workspace.numel(), _stream(stream))
     _check(rc, "mmbev_classify_points")
     return xyz[:n], lin[:n], rank[:n]
+
+
+def prep_rois(rois: torch.Tensor, roi_margin: float, stream=None) -> torch.Tensor:
+    """The prepared boxes the inside test uses (``mmbev_prep_rois``): float32
+    [R, 6] = (cx, cy, cos(yaw), sin(yaw), hl, hw) as the device computes them."""
+    lib = load()
+    nr = rois.shape[0] if rois.dim() > 1 else rois.numel() // 5
+    out = torch.empty((max(nr, 1), 6), dtype=torch.float32, device=rois.device)
+    rc = lib.mmbev_prep_rois(_dptr(rois, torch.float32, "rois"), nr, float(roi_margin),
+                             _dptr(out), _stream(stream))
+    _check(rc, "mmbev_prep_rois")
+    return out[:nr]
 
 
 CRIT_FIELDS = ("v_ego", "dt", "a_brake", "d_min", "theta_max_deg", "theta_min_deg", "v_wide",

@@ -594,6 +594,14 @@ int mmbev_classify_points(const float* points, const int64_t* sweep_offsets, int
     return e == cudaSuccess ? MMBEV_OK : MMBEV_ECUDA;
 }
 
+int mmbev_prep_rois(const mmbev_roi_t* rois, int32_t num_rois, float roi_margin, float* out,
+                    cudaStream_t stream) {
+    if (num_rois < 0 || (num_rois > 0 && (!rois || !out))) return MMBEV_EINVAL;
+    if (!std::isfinite(roi_margin) || !(roi_margin >= 0.0f)) return MMBEV_EINVAL;
+    return launch_prep_rois(rois, num_rois, roi_margin, out, stream) == cudaSuccess ? MMBEV_OK
+                                                                                   : MMBEV_ECUDA;
+}
+
 int mmbev_get_status(const void* workspace, size_t workspace_bytes, uint32_t* host_status,
                      cudaStream_t stream) {
     if (!workspace || !host_status || workspace_bytes < sizeof(Header)) return MMBEV_EINVAL;

@@ -235,6 +235,22 @@ __device__ __forceinline__ void compensate(const float* T, float x, float y, flo
                              __fmul_rn(T[10], z)), T[11]);
 }
 
+// Eq. 1 box of one ROI in the form the inside test takes: cos and sin of the
+// yaw evaluated in double and rounded to fp32, half-extents grown by the
+// margin (0.5*l + r along the heading, 0.5*w + r across it), in fp32.
+__device__ __forceinline__ RoiPrep prep_roi(const mmbev_roi_t& in, float margin) {
+    RoiPrep rp;
+    rp.cx = in.cx;
+    rp.cy = in.cy;
+    rp.c = (float)cos((double)in.yaw);
+    rp.s = (float)sin((double)in.yaw);
+    rp.hl = __fadd_rn(__fmul_rn(0.5f, in.l), margin);
+    rp.hw = __fadd_rn(__fmul_rn(0.5f, in.w), margin);
+    rp.pad0 = 0.f;
+    rp.pad1 = 0.f;
+    return rp;
+}
+
 // Alg. 1 inside test against one prepared ROI (boundary inclusive).
 __device__ __forceinline__ bool roi_contains(const RoiPrep& r, float x, float y) {
     const float dx = __fsub_rn(x, r.cx);
@@ -372,6 +388,9 @@ __device__ __forceinline__ uint32_t slot_minrank(const Params& p, uint32_t h) {
 // All launchers enqueue on `st` and return the launch's error code. `pdl`
 // launches the kernel as a programmatic dependent of the preceding one.
 cudaError_t launch_prep(const Params& p, const HostDesc& d, cudaStream_t st);
+// The prepared form (cx, cy, c, s, hl, hw) of n ROIs into out[n][6].
+cudaError_t launch_prep_rois(const mmbev_roi_t* rois, int32_t n, float margin, float* out,
+                             cudaStream_t st);
 cudaError_t launch_classify(const Params& p, int rmax, int num_sms, bool pdl, cudaStream_t st);
 cudaError_t launch_classify_points(const Params& p, cudaStream_t st);
 cudaError_t launch_insert(const Params& p, bool pdl, cudaStream_t st);

@@ -14,8 +14,10 @@
 // contents, so each call first zeroes the part that must start at zero (the
 // hash table). Calls whose executions overlap on the GPU (two streams, or two
 // host threads) race on the array; serialize them.
-#include <atomic>
+#include <cuda.h>   // driver types only: the two entry points below are fetched at run time
+
 #include <cstring>
+#include <mutex>
 
 #include "mmbev_internal.cuh"
 
@@ -25,24 +27,86 @@ namespace {
 static __device__ __align__(256) unsigned char g_noalloc_scratch[MMBEV_NOALLOC_SCRATCH_BYTES];
 
 constexpr int kMaxDevices = 64;
-std::atomic<void*> g_scratch_addr[kMaxDevices];
 
 size_t round256(size_t x) { return (x + 255) / 256 * 256; }
 
-// Device address of g_noalloc_scratch on the current device. In host code
-// the array's name is only a stand-in, so the address is looked up once per
-// device with that device current, on the first call.
+// Driver calls that name the current context, fetched through the runtime so
+// that the library keeps no link-time dependency on the driver library.
+using CtxGetCurrentFn = CUresult (*)(CUcontext*);
+using CtxGetIdFn = CUresult (*)(CUcontext, unsigned long long*);
+
+struct DriverFns {
+    CtxGetCurrentFn get_current = nullptr;
+    CtxGetIdFn get_id = nullptr;
+    bool ok = false;
+};
+
+const DriverFns& driver_fns() {
+    static DriverFns fns = [] {
+        DriverFns f;
+        void* a = nullptr;
+        void* b = nullptr;
+        cudaDriverEntryPointQueryResult qa = cudaDriverEntryPointSymbolNotFound;
+        cudaDriverEntryPointQueryResult qb = cudaDriverEntryPointSymbolNotFound;
+        if (cudaGetDriverEntryPointByVersion("cuCtxGetCurrent", &a, 12000, cudaEnableDefault,
+                                             &qa) == cudaSuccess &&
+            cudaGetDriverEntryPointByVersion("cuCtxGetId", &b, 12000, cudaEnableDefault, &qb) ==
+                cudaSuccess &&
+            qa == cudaDriverEntryPointSuccess && qb == cudaDriverEntryPointSuccess && a && b) {
+            f.get_current = reinterpret_cast<CtxGetCurrentFn>(a);
+            f.get_id = reinterpret_cast<CtxGetIdFn>(b);
+            f.ok = true;
+        }
+        return f;
+    }();
+    return fns;
+}
+
+// Unique id (for the life of the process) of the context current on this
+// thread, or 0 when none is current or the driver cannot say.
+unsigned long long current_context_id() {
+    const DriverFns& f = driver_fns();
+    if (!f.ok) return 0;
+    CUcontext ctx = nullptr;
+    if (f.get_current(&ctx) != CUDA_SUCCESS || ctx == nullptr) return 0;
+    unsigned long long id = 0;
+    if (f.get_id(ctx, &id) != CUDA_SUCCESS) return 0;
+    return id;
+}
+
+struct ScratchCache {
+    unsigned long long ctx_id = 0;   // 0: nothing cached
+    void* addr = nullptr;
+};
+std::mutex g_cache_mu;
+ScratchCache g_cache[kMaxDevices];
+
+// Device address of g_noalloc_scratch in the current device's context. In
+// host code the array's name is only a stand-in, so the address is looked up
+// with cudaGetSymbolAddress, with the device current, and cached per device
+// together with the id of the context it belongs to. The first call on a
+// device does the lookup (and may load the module), so make it before any
+// stream capture. A call in another context of the device, or after
+// cudaDeviceReset has replaced the primary context, sees a different id and
+// looks the address up again instead of using a stale one.
 cudaError_t scratch_address(void** out) {
     int dev = 0;
     cudaError_t e = cudaGetDevice(&dev);
     if (e != cudaSuccess) return e;
     if (dev < 0 || dev >= kMaxDevices) return cudaErrorInvalidDevice;
-    void* p = g_scratch_addr[dev].load(std::memory_order_acquire);
-    if (p == nullptr) {
-        e = cudaGetSymbolAddress(&p, g_noalloc_scratch);
-        if (e != cudaSuccess) return e;
-        g_scratch_addr[dev].store(p, std::memory_order_release);
+    std::lock_guard<std::mutex> lock(g_cache_mu);
+    const unsigned long long id = current_context_id();
+    if (id != 0 && g_cache[dev].ctx_id == id) {
+        *out = g_cache[dev].addr;
+        return cudaSuccess;
     }
+    void* p = nullptr;
+    e = cudaGetSymbolAddress(&p, g_noalloc_scratch);   // makes the primary context current if none is
+    if (e != cudaSuccess) return e;
+    // cache only under a known context id; without one, look up every call
+    const unsigned long long id2 = current_context_id();
+    g_cache[dev].ctx_id = id2;
+    g_cache[dev].addr = id2 != 0 ? p : nullptr;
     *out = p;
     return cudaSuccess;
 }

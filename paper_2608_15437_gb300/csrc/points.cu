@@ -101,7 +101,8 @@ struct ClsSmem {
     int32_t* sr0;     // [S] first ROI of that frame
     uint64_t* full;   // [nstages] tile arrived
     uint32_t* done;   // [nstages] warps finished with the buffer
-    uint32_t* kept;   // [4] kept points of the block, warps finished, next chunk, -
+    uint32_t* issued; // [nstages] fills issued into the buffer
+    uint32_t* kept;   // [4] kept points of the block, -, next chunk, abort flag
 };
 
 __host__ __device__ inline size_t align16(size_t o) { return (o + 15) & ~(size_t)15; }
@@ -113,7 +114,7 @@ __host__ __device__ inline size_t classify_smem_bytes(int S, int rmax, int nstag
     o += tf_staged ? (size_t)S * 48 : 0;
     o += (size_t)(S + 1) * 8 + (size_t)S * 8;
     o = align16(o);
-    return o + (size_t)nstages * 8 + (size_t)nstages * 4 + 16;
+    return o + (size_t)nstages * 8 + (size_t)nstages * 8 + 16;
 }
 
 __device__ __forceinline__ ClsSmem carve(unsigned char* smem, int S, int rmax, int g2w, bool tf_staged,
@@ -139,6 +140,8 @@ __device__ __forceinline__ ClsSmem carve(unsigned char* smem, int S, int rmax, i
     o += (size_t)nstages * 8;
     s.done = reinterpret_cast<uint32_t*>(smem + o);
     o += (size_t)nstages * 4;
+    s.issued = reinterpret_cast<uint32_t*>(smem + o);
+    o += (size_t)nstages * 4;
     s.kept = reinterpret_cast<uint32_t*>(smem + o);
     return s;
 }
@@ -147,6 +150,7 @@ __device__ __forceinline__ ClsSmem carve(unsigned char* smem, int S, int rmax, i
 // buffer `stage`.
 __device__ __forceinline__ void issue_tile(const Params& p, const ClsSmem& sm, int stage,
                                            int64_t tile, int lane, uint64_t pol) {
+    if (lane == 0) sm.issued[stage] += 1u;   // one warp refills a buffer at a time
     if (lane < kChunks) {
         const size_t off = (size_t)lane * kChunkBytes;
         mbar_expect_tx(&sm.full[stage], kChunkBytes);
@@ -229,6 +233,8 @@ __device__ __forceinline__ bool classify_range(const Params& p, const ClsSmem& s
     if (lane == 0) c = atomicAdd(&sm.kept[2], 1u);
     c = __shfl_sync(0xFFFFFFFFu, c, 0);
     while (c < nchunks) {
+        // another warp gave up waiting: stop taking chunks
+        if (*reinterpret_cast<volatile uint32_t*>(&sm.kept[3])) return false;
         uint32_t cn = 0;   // the warp's next chunk, fetched early
         if (lane == 0) cn = atomicAdd(&sm.kept[2], 1u);
         const uint32_t ct = c / (uint32_t)kTileChunks, sub = c % (uint32_t)kTileChunks;
@@ -246,7 +252,10 @@ __device__ __forceinline__ bool classify_range(const Params& p, const ClsSmem& s
         float2 v0, v1, v2, v3, v4;
         if (tile < full_tiles) {
             if (!mbar_wait(&sm.full[st], round & 1u)) {
-                if (lane == 0) set_status(p.hdr, MMBEV_DEV_WAIT_TIMEOUT);
+                if (lane == 0) {
+                    set_status(p.hdr, MMBEV_DEV_WAIT_TIMEOUT);
+                    atomicExch(&sm.kept[3], 1u);
+                }
                 return false;
             }
             const float2* q2 =
@@ -423,8 +432,9 @@ __global__ void __launch_bounds__(kThreads, 1) k_classify(Params p, int rmax, in
         for (int s = 0; s < nstages; ++s) {
             mbar_init(&sm.full[s], kChunks);
             sm.done[s] = 0u;
+            sm.issued[s] = 0u;
         }
-        sm.kept[0] = sm.kept[1] = sm.kept[2] = 0u;
+        sm.kept[0] = sm.kept[1] = sm.kept[2] = sm.kept[3] = 0u;
         mbar_fence_init();
     }
     __syncthreads();
@@ -438,19 +448,28 @@ __global__ void __launch_bounds__(kThreads, 1) k_classify(Params p, int rmax, in
     // cover it, every mask and ROI read is a shared-memory read.
     const int64_t last_pt = (t_end * kTile < N ? t_end * kTile : N) - 1;
     const int f_hi = p.sweep_frame[find_sweep(p.sweep_off, S, last_pt)];
-    const bool ok = f_hi - f_lo < n_staged
-                        ? classify_range<true>(p, sm, rmax, nstages, t_begin, t_end, f_lo, n_staged)
-                        : classify_range<false>(p, sm, rmax, nstages, t_begin, t_end, f_lo, n_staged);
-    if (!ok) return;
-    // the last warp to leave publishes the block's list length
-    if (lane == 0) {
-        __threadfence_block();
-        if (atomicAdd(&sm.kept[1], 1u) == (uint32_t)(kWarps - 1)) {
-            const uint32_t tot = atomicAdd(&sm.kept[0], 0u);
-            p.cls_cnt[blockIdx.x] = tot;
-            if (tot) atomicAdd(&p.hdr->num_rec, tot);
+    if (f_hi - f_lo < n_staged)
+        classify_range<true>(p, sm, rmax, nstages, t_begin, t_end, f_lo, n_staged);
+    else
+        classify_range<false>(p, sm, rmax, nstages, t_begin, t_end, f_lo, n_staged);
+    __syncthreads();
+    if (t != 0) return;
+    if (sm.kept[3]) {
+        // A wait gave up (the status word says so). Before the block exits,
+        // every bulk copy still in flight into its shared memory must land:
+        // a buffer has at most one fill outstanding, the last one issued, so
+        // wait (bounded again) for that fill's phase. The block's list is
+        // published as empty.
+        for (int s = 0; s < nstages; ++s) {
+            const uint32_t k = sm.issued[s];
+            if (k > 0) (void)mbar_wait(&sm.full[s], (k - 1u) & 1u);
         }
+        p.cls_cnt[blockIdx.x] = 0u;
+        return;
     }
+    const uint32_t tot = sm.kept[0];
+    p.cls_cnt[blockIdx.x] = tot;
+    if (tot) atomicAdd(&p.hdr->num_rec, tot);
 }
 
 // One thread per point: the per-point view of S1-S2 for testing.

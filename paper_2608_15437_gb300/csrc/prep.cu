@@ -66,16 +66,7 @@ k_prep(Params p, const __grid_constant__ HostDesc d) {
         // one thread per ROI: cos/sin of the yaw in double, rounded to fp32
         // (the definition), half-extents grown by the margin, cell range
         for (int r = t; r < rn; r += blockDim.x) {
-            const mmbev_roi_t in = p.rois[r0 + r];
-            RoiPrep rp;
-            rp.cx = in.cx;
-            rp.cy = in.cy;
-            rp.c = (float)cos((double)in.yaw);
-            rp.s = (float)sin((double)in.yaw);
-            rp.hl = __fadd_rn(__fmul_rn(0.5f, in.l), p.margin);
-            rp.hw = __fadd_rn(__fmul_rn(0.5f, in.w), p.margin);
-            rp.pad0 = 0.f;
-            rp.pad1 = 0.f;
+            const RoiPrep rp = prep_roi(p.rois[r0 + r], p.margin);
             p.roi_prep[r0 + r] = rp;
             s_rng[r] = roi_cells(p, rp);
         }
@@ -135,6 +126,15 @@ k_prep(Params p, const __grid_constant__ HostDesc d) {
     }
 }
 
+// One thread per ROI: the prepared form the classify pass tests against.
+__global__ void k_prep_rois(const mmbev_roi_t* rois, int32_t n, float margin, float* out) {
+    const int i = blockIdx.x * blockDim.x + threadIdx.x;
+    if (i >= n) return;
+    const RoiPrep rp = prep_roi(rois[i], margin);
+    float* o = out + (size_t)i * 6;
+    o[0] = rp.cx; o[1] = rp.cy; o[2] = rp.c; o[3] = rp.s; o[4] = rp.hl; o[5] = rp.hw;
+}
+
 __global__ void k_zero(uint4* ptr, size_t n16, uint8_t* tail, size_t ntail) {
     const size_t gs = (size_t)gridDim.x * blockDim.x;
     for (size_t i = (size_t)blockIdx.x * blockDim.x + threadIdx.x; i < n16; i += gs)
@@ -164,6 +164,13 @@ cudaError_t launch_prep(const Params& p, const HostDesc& d, cudaStream_t st) {
     const size_t smem = (size_t)p.coarse * p.coarse * p.mask_words * sizeof(uint32_t);
     if (smem > (size_t)kPrepSmemMax) return cudaErrorInvalidValue;
     k_prep<<<p.num_frames + kZeroBlocks, kPrepThreads, smem, st>>>(p, d);
+    return cudaGetLastError();
+}
+
+cudaError_t launch_prep_rois(const mmbev_roi_t* rois, int32_t n, float margin, float* out,
+                             cudaStream_t st) {
+    if (n <= 0) return cudaSuccess;
+    k_prep_rois<<<(unsigned)((n + 255) / 256), 256, 0, st>>>(rois, n, margin, out);
     return cudaGetLastError();
 }
 

@@ -39,6 +39,40 @@ def test_classify_bit_exact(oracle_mod, mmbev_lib, cuda_dev, name):
     assert np.array_equal(rank.cpu().numpy(), erank)
 
 
+def test_roi_prep_trig_matches_libm_on_a_million_yaws(oracle_mod, mmbev_lib, cuda_dev):
+    """The device's fp32 cos/sin of each yaw (CUDA's double cos/sin, rounded)
+    against the oracle's (libm's double cos/sin, rounded), bit for bit: the
+    two agree unless a double result lies within an ulp of an fp32 rounding
+    boundary, which would flip points on an ROI edge (Eq. 1; Alg. 1's inside
+    test). 1,200,000 yaws uniform over eight turns, plus every multiple of
+    pi/4 in that span and its three fp32 neighbours on each side."""
+    import torch
+    rng = np.random.default_rng(11)
+    n = 1_200_000
+    yaws = rng.uniform(-8 * np.pi, 8 * np.pi, n).astype(np.float32)
+    k = (np.arange(-32, 33) * (np.pi / 4)).astype(np.float32)
+    extra = [k]
+    up, dn = k, k
+    for _ in range(3):
+        up = np.nextafter(up, np.float32(np.inf))
+        dn = np.nextafter(dn, np.float32(-np.inf))
+        extra += [up, dn]
+    yaws = np.concatenate([yaws] + extra).astype(np.float32)
+    rois = np.zeros((yaws.size, 5), np.float32)
+    rois[:, 0] = rng.uniform(-50, 50, yaws.size)
+    rois[:, 1] = rng.uniform(-50, 50, yaws.size)
+    rois[:, 2] = rng.uniform(0.5, 6, yaws.size)
+    rois[:, 3] = rng.uniform(0.5, 12, yaws.size)
+    rois[:, 4] = yaws
+    margin = 0.37
+    got = mmbev_lib.prep_rois(torch.from_numpy(rois).to(cuda_dev), margin).cpu().numpy()
+    want = oracle_mod.roi_boxes(rois, margin)
+    assert yaws.size > 1_000_000
+    assert np.array_equal(got[:, 0:2].view(np.uint32), rois[:, 0:2].view(np.uint32))
+    bad = np.nonzero(np.any(got[:, 2:6].view(np.uint32) != want.view(np.uint32), axis=1))[0]
+    assert bad.size == 0, f"{bad.size} of {yaws.size} ROIs differ, e.g. yaw {yaws[bad[:5]]}"
+
+
 # ------------------------------------------------------------------ whole path, full sizes
 
 @pytest.mark.parametrize("name", ["tiny", "nuscenes", "ouster", "roi_0", "roi_8", "roi_32",

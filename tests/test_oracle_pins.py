@@ -248,6 +248,41 @@ def test_margin_grows_both_half_extents(oracle_mod):
     assert rank.tolist() == [0, -1, 0, -1]
 
 
+def _trig_yaws(n_uniform, seed=7):
+    """Yaws over several turns plus the multiples of pi/4 and their fp32
+    neighbours (where cos and sin cross zero or meet each other)."""
+    rng = np.random.default_rng(seed)
+    u = rng.uniform(-8 * np.pi, 8 * np.pi, n_uniform).astype(np.float32)
+    k = (np.arange(-32, 33) * (np.pi / 4)).astype(np.float32)
+    near = [k]
+    for steps in (1, 2, 3):
+        near.append(np.nextafter(k, np.float32(np.inf)))
+        near.append(np.nextafter(k, np.float32(-np.inf)))
+        k = near[-2]
+    return np.concatenate([u] + near).astype(np.float32)
+
+
+def test_roi_box_trig_is_the_rounded_true_value(oracle_mod):
+    # Eq. 1 box: the heading's cosine and sine, evaluated in double and
+    # rounded to fp32. Checked against a 40-digit evaluation (mpmath): the
+    # oracle's value must be the fp32 nearest to the true one, up to the
+    # double-precision step before the rounding.
+    mpmath = pytest.importorskip("mpmath")
+    mpmath.mp.dps = 40
+    yaws = _trig_yaws(20000)
+    rois = np.zeros((yaws.size, 5), np.float32)
+    rois[:, 2], rois[:, 3], rois[:, 4] = 2.0, 4.0, yaws
+    box = oracle_mod.roi_boxes(rois, 0.5)
+    for i, yaw in enumerate(yaws.tolist()):
+        for col, fn in ((0, mpmath.cos), (1, mpmath.sin)):
+            true = fn(mpmath.mpf(yaw))
+            got = float(box[i, col])
+            ulp = float(np.spacing(np.float32(abs(got)))) if got != 0.0 else 2.0 ** -149
+            slack = 0.5 * ulp + 2.0 ** -52 * abs(float(true))
+            assert abs(got - float(true)) <= slack, (yaw, col, got, float(true))
+    assert np.all(box[:, 2] == 2.5) and np.all(box[:, 3] == 1.5)   # 0.5*4 + 0.5, 0.5*2 + 0.5
+
+
 def test_no_rois_keeps_nothing(oracle_mod):
     w = synth.tiny(0)
     _, lin, _ = oracle_mod.classify(w.points, w.sweep_offsets, w.sweep_tf, w.rois[:0], 0.5,
