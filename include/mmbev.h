@@ -8,7 +8,7 @@
  *   S1  per-sweep ego-motion compensation, p' = R p + T          (Sec. IV-D, Eq. 6-7)
  *   S2  range crop and inside-any-ROI test against criticality-ranked,
  *       margin-grown rotated BEV boxes, then the voxel index        (Alg. 1; Eq. 1)
- *   S3  voxel hash insert / dedup                                   (Alg. 1, "Voxelize")
+ *   S3  voxel dedup                                                 (Alg. 1, "Voxelize")
  *   S4  voxel cap and canonical (ascending linear index) order      (Sec. IV-F "hard
  *                                                                    voxelization"; Sec. IV-C)
  *   S5  mean features over the first K points of each voxel         (Alg. 1, "VoxelFeatureEncoder")
@@ -43,22 +43,20 @@
  * synchronizes, never allocates and reads its host arrays only during the
  * call, so it can be captured in a CUDA graph. The caller owns every buffer.
  *
- * Two caller-owned device buffers carry the library's state:
- *   - `table` (size from mmbev_table_size): the open-addressing voxel hash
- *     table. It must be all zero before the first call (mmbev_table_clear)
- *     and every successful call leaves it all zero again. Its capacity is
- *     derived from table_bytes and max_pts_per_voxel alone, so one table can
- *     serve calls of any shape. Calls that share a table must not overlap.
- *   - `workspace` (size from mmbev_workspace_size): scratch with no state
- *     across calls, except the device status word read by mmbev_get_status.
+ * One caller-owned device buffer, the `workspace` (size from
+ * mmbev_workspace_size), is the library's scratch. It carries no state from
+ * one call to the next, except the device status word that
+ * mmbev_get_status reads; any contents are fine on entry. Calls that share
+ * a workspace must not overlap on the GPU.
  *
  * Errors. A status below zero is returned before any launch when a host
  * argument is invalid (MMBEV_EINVAL) or a buffer is too small
  * (MMBEV_EWORKSPACE), and after a failed launch (MMBEV_ECUDA). Conditions
- * only the device can see (hash table full, an internal wait that timed out)
- * set bits in a device status word instead; no kernel traps or spins
- * without bound. mmbev_get_status reads it. After a non-zero device status
- * the outputs are invalid and the table must be cleared again.
+ * only the device can see (an internal wait that timed out, an internal
+ * index out of its bounds) set bits in a device status word instead; no
+ * kernel traps or spins without bound. mmbev_get_status reads it. After a
+ * non-zero device status the outputs are invalid; the next call starts
+ * afresh.
  */
 #ifndef MMBEV_H_
 #define MMBEV_H_
@@ -84,11 +82,11 @@ typedef enum mmbev_status {
     MMBEV_OK = 0,
     MMBEV_EINVAL = -1,      /* invalid host argument; nothing launched */
     MMBEV_ECUDA = -2,       /* a CUDA runtime call or launch failed */
-    MMBEV_EWORKSPACE = -3   /* table or workspace smaller than required */
+    MMBEV_EWORKSPACE = -3   /* workspace or another buffer smaller than required */
 } mmbev_status_t;
 
 /* Device status bits (mmbev_get_status). */
-#define MMBEV_DEV_TABLE_FULL   0x1u  /* a voxel key found no free slot */
+#define MMBEV_DEV_TABLE_FULL   0x1u  /* components: a voxel key found no free slot */
 #define MMBEV_DEV_WAIT_TIMEOUT 0x2u  /* an internal inter-block wait gave up */
 #define MMBEV_DEV_BOUNDS       0x4u  /* an internal index failed its bounds check */
 #define MMBEV_DEV_UNSORTED     0x8u  /* components: a frame's rows do not ascend by linear index */
@@ -100,28 +98,16 @@ typedef enum mmbev_status {
 #define MMBEV_MAX_PTS_PER_VOXEL   64
 
 /*
- * Bytes of hash table for calls of up to max_points points (and
- * max_pts_per_voxel points kept per voxel, which must lie in
- * [1, MMBEV_MAX_PTS_PER_VOXEL] but does not change the size). The capacity
- * is the power of two >= 2*max_points slots of 16 bytes (load factor <= 1/2
- * whatever the inputs), each slot holding a voxel key, its minimum ROI rank,
- * its point count and the start of its point list. Returns 0 for invalid
- * arguments.
- */
-size_t mmbev_table_size(int64_t max_points, int32_t max_pts_per_voxel);
-
-/*
  * Bytes of scratch workspace for a call with up to max_points points,
  * max_rois_per_frame ROIs in any frame, max_voxels kept voxels per frame and
  * num_frames frames on the grid given by voxel_size[3] and range[6] (host
- * arrays). Returns 0 for invalid arguments.
+ * arrays). About 88 bytes per point (records, lists and per-voxel results,
+ * all sized for every point kept) plus 20 bytes per bucket of 2^13
+ * consecutive cells of each frame's grid. Returns 0 for invalid arguments.
  */
 size_t mmbev_workspace_size(int64_t max_points, int32_t max_rois_per_frame,
                             int32_t max_voxels, int32_t num_frames,
                             const float voxel_size[3], const float range[6]);
-
-/* Zero a hash table (device pointer, table_bytes bytes) on `stream`. */
-int mmbev_table_clear(void *table, size_t table_bytes, cudaStream_t stream);
 
 /*
  * One frame (Alg. 1 on the union of n sweeps, Eq. 7).
@@ -152,8 +138,8 @@ int mmbev_voxelize_roi(const float *points, const int64_t *sweep_offsets,
                        const float voxel_size[3], const float range[6],
                        int32_t max_pts_per_voxel, int32_t max_voxels,
                        float *out_feats, int32_t *out_coords, int32_t *out_counts,
-                       int32_t *out_nvox, void *table, size_t table_bytes,
-                       void *workspace, size_t workspace_bytes, cudaStream_t stream);
+                       int32_t *out_nvox, void *workspace, size_t workspace_bytes,
+                       cudaStream_t stream);
 
 /*
  * num_frames independent frames in one call; the result equals num_frames
@@ -177,7 +163,6 @@ int mmbev_voxelize_roi_batched(const float *points, const int64_t *sweep_offsets
                                const int32_t *frame_roi_offsets,
                                float *out_feats, int32_t *out_coords,
                                int32_t *out_counts, int32_t *out_nvox,
-                               void *table, size_t table_bytes,
                                void *workspace, size_t workspace_bytes,
                                cudaStream_t stream);
 
@@ -187,7 +172,7 @@ int mmbev_voxelize_roi_batched(const float *points, const int64_t *sweep_offsets
  *   out_xyz   device, float32 [N][3], compensated coordinates of every point
  *   out_lin   device, int64 [N], frame-local voxel linear index, -1 if dropped
  *   out_rank  device, int32 [N], ROI rank, -1 if dropped
- * Needs only the workspace (no table).
+ * Needs only the workspace.
  */
 int mmbev_classify_points(const float *points, const int64_t *sweep_offsets,
                           int32_t num_sweeps, const float *sweep_tf,
@@ -225,10 +210,11 @@ int mmbev_get_status(const void *workspace, size_t workspace_bytes,
  *                     caller: event k is recorded on `stream` before stage k
  *                     and the last one after the final stage, so the caller
  *                     can time each kernel with cudaEventElapsedTime.
- *   table_log2_override  0, or log2 of the slot count the insert stage uses
- *                     instead of the power of two >= 1.25 x the call's kept
- *                     points (at most table_bytes / 16; a full table sets
- *                     MMBEV_DEV_TABLE_FULL).
+ *   inject_status     0 for use. A test hook: MMBEV_DEV_* bits that the
+ *                     call's first kernel sets in the device status word as
+ *                     a device-side failure would (in the first chunk only,
+ *                     for mmbev_voxelize_roi_batched_host), so that callers
+ *                     can check how a failure is reported without one.
  *   rho_out           keep probability, in [0, 1], of an in-range point inside
  *                     no ROI (Alg. 1; the other entry points use 0). The draw
  *                     for the j-th point of a frame (0-based, within that
@@ -241,10 +227,10 @@ int mmbev_get_status(const void *workspace, size_t workspace_bytes,
  *                     Outside [0, 1] or NaN: MMBEV_EINVAL.
  *   seed              the generator's seed.
  */
-#define MMBEV_NUM_STAGES 11
+#define MMBEV_NUM_STAGES 6
 typedef struct mmbev_exec_opts {
     cudaEvent_t *stage_events;
-    int32_t table_log2_override;
+    uint32_t inject_status;
     float rho_out;
     uint64_t seed;
 } mmbev_exec_opts_t;
@@ -283,8 +269,8 @@ int mmbev_voxelize_roi_batched_host(
     const float voxel_size[3], const float range[6], int32_t max_pts_per_voxel,
     int32_t max_voxels, int32_t num_frames, const int32_t *frame_sweep_offsets,
     const int32_t *frame_roi_offsets, float *d_points, float *d_sweep_tf, mmbev_roi_t *d_rois,
-    float *out_feats, int32_t *out_coords, int32_t *out_counts, int32_t *out_nvox, void *table,
-    size_t table_bytes, void *workspace, size_t workspace_bytes, void *pack_dst,
+    float *out_feats, int32_t *out_coords, int32_t *out_counts, int32_t *out_nvox,
+    void *workspace, size_t workspace_bytes, void *pack_dst,
     size_t pack_bytes, int32_t chunk_frames, cudaStream_t stream, cudaStream_t copy_stream,
     const mmbev_exec_opts_t *opts);
 
@@ -298,7 +284,6 @@ int mmbev_voxelize_roi_batched_ex(const float *points, const int64_t *sweep_offs
                                   const int32_t *frame_roi_offsets,
                                   float *out_feats, int32_t *out_coords,
                                   int32_t *out_counts, int32_t *out_nvox,
-                                  void *table, size_t table_bytes,
                                   void *workspace, size_t workspace_bytes,
                                   cudaStream_t stream, const mmbev_exec_opts_t *opts);
 
@@ -309,27 +294,25 @@ int mmbev_voxelize_roi_batched_ex(const float *points, const int64_t *sweep_offs
  * example a real-time perception process that forbids allocation after
  * start-up (allocation may synchronize the device and has unbounded
  * latency), or a host that owns every device buffer and lends the library
- * only its inputs and outputs. Here the hash table and the workspace come
- * from one file-scope device array of MMBEV_NOALLOC_SCRATCH_BYTES, which
- * every GPU that loads the library keeps until the process exits; the call
- * allocates nothing.
- *   Arguments are those of mmbev_voxelize_roi without the table and
- *   workspace, plus
+ * only its inputs and outputs. Here the workspace is one file-scope
+ * device array of MMBEV_NOALLOC_SCRATCH_BYTES, which every GPU that loads
+ * the library keeps until the process exits; the call allocates nothing.
+ *   Arguments are those of mmbev_voxelize_roi without the workspace, plus
  *   out_status  device, uint32 scalar or NULL: receives the call's device
  *               status word (MMBEV_DEV_* bits, 0 = no device-side error).
  *   Returns MMBEV_EWORKSPACE, before any launch, when the call needs more
- *   than the array holds: mmbev_table_size(N, K) rounded up to 256 bytes
- *   plus mmbev_workspace_size(N, num_rois, max_voxels, 1, voxel_size, range)
- *   must not exceed MMBEV_NOALLOC_SCRATCH_BYTES. K does not enter the sum.
- *   On the grids of the tiny, nuScenes- and Ouster-shaped workloads, with
- *   their ROI counts and voxel caps, that allows up to about 575,000 points.
+ *   than the array holds: mmbev_workspace_size(N, num_rois, max_voxels, 1,
+ *   voxel_size, range) must not exceed MMBEV_NOALLOC_SCRATCH_BYTES; K and
+ *   max_voxels do not enter it. On the grids of the tiny, nuScenes- and
+ *   Ouster-shaped workloads, with their ROI counts, that allows up to about
+ *   1,100,000 points.
  * The first call on a device (and the first in each new context of it, as
  * after cudaDeviceReset) looks up the array's device address with that
- * device current; make that first call before any stream capture. Every
- * call zeroes the table part of the array first (16 bytes per slot of
- * mmbev_table_size), since the array keeps the previous call's contents.
- * All calls on a device share the one array: calls whose executions overlap
- * on the GPU race and must be serialized.
+ * device current; make that first call before any stream capture. The
+ * array keeps the previous call's contents; nothing in it needs to start at
+ * zero, since every call initialises the part it reads. All calls on a
+ * device share the one array: calls whose executions overlap on the GPU
+ * race and must be serialized.
  */
 #define MMBEV_NOALLOC_SCRATCH_BYTES (96u << 20)
 int mmbev_voxelize_roi_noalloc(const float *points, const int64_t *sweep_offsets,

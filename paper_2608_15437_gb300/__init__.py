@@ -21,7 +21,7 @@ import torch
 _PKG = os.path.dirname(os.path.abspath(__file__))
 LIB_PATH = os.path.join(_PKG, "libmmbev.so")
 
-NUM_STAGES = 11
+NUM_STAGES = 6
 DEV_TABLE_FULL = 0x1
 DEV_WAIT_TIMEOUT = 0x2
 DEV_BOUNDS = 0x4
@@ -35,7 +35,7 @@ class MMBEVError(RuntimeError):
 
 
 class _ExecOpts(ctypes.Structure):
-    _fields_ = [("stage_events", ctypes.c_void_p), ("table_log2_override", ctypes.c_int32),
+    _fields_ = [("stage_events", ctypes.c_void_p), ("inject_status", ctypes.c_uint32),
                 ("rho_out", ctypes.c_float), ("seed", ctypes.c_uint64)]
 
 
@@ -49,16 +49,12 @@ def load():
     lib = ctypes.CDLL(LIB_PATH)
     P, i32, i64, f32, sz = (ctypes.c_void_p, ctypes.c_int32, ctypes.c_int64, ctypes.c_float,
                             ctypes.c_size_t)
-    lib.mmbev_table_size.argtypes = [i64, i32]
-    lib.mmbev_table_size.restype = sz
     lib.mmbev_workspace_size.argtypes = [i64, i32, i32, i32, P, P]
     lib.mmbev_workspace_size.restype = sz
-    lib.mmbev_table_clear.argtypes = [P, sz, P]
-    lib.mmbev_table_clear.restype = ctypes.c_int
     vox = [P, P, i32, P, P, i32, f32, P, P, i32, i32]
-    lib.mmbev_voxelize_roi.argtypes = vox + [P, P, P, P, P, sz, P, sz, P]
+    lib.mmbev_voxelize_roi.argtypes = vox + [P, P, P, P, P, sz, P]
     lib.mmbev_voxelize_roi.restype = ctypes.c_int
-    batched = vox + [i32, P, P, P, P, P, P, P, sz, P, sz, P]
+    batched = vox + [i32, P, P, P, P, P, P, P, sz, P]
     lib.mmbev_voxelize_roi_batched.argtypes = batched
     lib.mmbev_voxelize_roi_batched.restype = ctypes.c_int
     lib.mmbev_pack_size.argtypes = [i32, i32]
@@ -78,7 +74,7 @@ def load():
     lib.mmbev_voxelize_roi_batched_ex.argtypes = batched + [ctypes.POINTER(_ExecOpts)]
     lib.mmbev_voxelize_roi_batched_ex.restype = ctypes.c_int
     lib.mmbev_voxelize_roi_batched_host.argtypes = (
-        [P, P, i32, P, P, i32, f32, P, P, i32, i32, i32, P, P, P, P, P, P, P, P, P, P, sz, P, sz,
+        [P, P, i32, P, P, i32, f32, P, P, i32, i32, i32, P, P, P, P, P, P, P, P, P, P, sz,
          P, sz, i32, P, P, ctypes.POINTER(_ExecOpts)])
     lib.mmbev_voxelize_roi_batched_host.restype = ctypes.c_int
     lib.mmbev_classify_points.argtypes = [P, P, i32, P, P, i32, f32, P, P, i32, P, P,
@@ -141,14 +137,6 @@ def _stream(stream):
     return ctypes.c_void_p(s.cuda_stream)
 
 
-def table_size(max_points: int, max_pts_per_voxel: int) -> int:
-    """Bytes of hash table for up to max_points points and K points per voxel."""
-    n = load().mmbev_table_size(int(max_points), int(max_pts_per_voxel))
-    if n == 0:
-        raise ValueError("invalid table size arguments")
-    return int(n)
-
-
 def workspace_size(max_points, max_rois_per_frame, max_voxels, num_frames, voxel_size,
                    pc_range) -> int:
     vs = _host(voxel_size, np.float32)
@@ -158,18 +146,6 @@ def workspace_size(max_points, max_rois_per_frame, max_voxels, num_frames, voxel
     if n == 0:
         raise ValueError("invalid workspace size arguments")
     return int(n)
-
-
-def table_clear(table: torch.Tensor, stream=None):
-    _check(load().mmbev_table_clear(_dptr(table, torch.uint8, "table"), table.numel(),
-                                    _stream(stream)), "mmbev_table_clear")
-
-
-def new_table(max_points: int, max_pts_per_voxel: int, device="cuda") -> torch.Tensor:
-    """An all-zero hash table sized for the given limits."""
-    t = torch.empty(table_size(max_points, max_pts_per_voxel), dtype=torch.uint8, device=device)
-    table_clear(t)
-    return t
 
 
 def new_workspace(max_points, max_rois_per_frame, max_voxels, num_frames, voxel_size, pc_range,
@@ -213,9 +189,9 @@ class Outputs:
 def voxelize_roi_batched(points: torch.Tensor, sweep_offsets, sweep_tf: torch.Tensor,
                          rois: torch.Tensor, roi_margin: float, voxel_size, pc_range,
                          max_pts_per_voxel: int, max_voxels: int, frame_sweep_offsets,
-                         frame_roi_offsets, *, table: torch.Tensor, workspace: torch.Tensor,
+                         frame_roi_offsets, *, workspace: torch.Tensor,
                          out: Outputs | None = None, stream=None, stage_events=None,
-                         table_log2_override: int = 0, rho_out: float = 0.0,
+                         inject_status: int = 0, rho_out: float = 0.0,
                          seed: int = 0) -> Outputs:
     """Voxelize F independent frames in one call (``mmbev_voxelize_roi_batched``).
 
@@ -225,7 +201,8 @@ def voxelize_roi_batched(points: torch.Tensor, sweep_offsets, sweep_tf: torch.Te
     NUM_STAGES + 1 ``torch.cuda.Event(enable_timing=True)`` already recorded
     once, brackets each kernel of the call. ``rho_out`` keeps points inside
     no ROI with that probability (SplitMix64 draws keyed by ``seed`` and the
-    point's index within its frame).
+    point's index within its frame). ``inject_status`` is a test hook: status
+    bits the call reports as if a device-side failure had set them.
     """
     lib = load()
     so = _host(sweep_offsets, np.int64)
@@ -241,13 +218,11 @@ def voxelize_roi_batched(points: torch.Tensor, sweep_offsets, sweep_tf: torch.Te
             rois.shape[0] if rois.dim() > 1 else rois.numel() // 5, float(roi_margin), _hptr(vs),
             _hptr(rg), int(max_pts_per_voxel), int(max_voxels), nf, _hptr(fso), _hptr(fro),
             _dptr(out.feats), _dptr(out.coords), _dptr(out.counts), _dptr(out.nvox),
-            _dptr(table, torch.uint8, "table"), table.numel(),
             _dptr(workspace, torch.uint8, "workspace"), workspace.numel(), _stream(stream)]
-    if stage_events is None and not table_log2_override and not rho_out:
+    if stage_events is None and not inject_status and not rho_out:
         rc = lib.mmbev_voxelize_roi_batched(*args)
     else:
-        opts = _ExecOpts(None, int(table_log2_override), float(rho_out),
-                         int(seed) & (2**64 - 1))
+        opts = _ExecOpts(None, int(inject_status), float(rho_out), int(seed) & (2**64 - 1))
         if stage_events is not None:
             assert len(stage_events) == NUM_STAGES + 1
             arr = (ctypes.c_void_p * len(stage_events))(*[e.cuda_event for e in stage_events])
@@ -259,7 +234,7 @@ def voxelize_roi_batched(points: torch.Tensor, sweep_offsets, sweep_tf: torch.Te
 
 def voxelize_roi(points: torch.Tensor, sweep_offsets, sweep_tf: torch.Tensor, rois: torch.Tensor,
                  roi_margin: float, voxel_size, pc_range, max_pts_per_voxel: int,
-                 max_voxels: int, *, table: torch.Tensor, workspace: torch.Tensor,
+                 max_voxels: int, *, workspace: torch.Tensor,
                  out: Outputs | None = None, stream=None) -> Outputs:
     """One frame (``mmbev_voxelize_roi``); out.nvox holds one entry."""
     lib = load()
@@ -274,7 +249,6 @@ def voxelize_roi(points: torch.Tensor, sweep_offsets, sweep_tf: torch.Tensor, ro
         _dptr(sweep_tf, torch.float32, "sweep_tf"), _dptr(rois, torch.float32, "rois"), nr,
         float(roi_margin), _hptr(vs), _hptr(rg), int(max_pts_per_voxel), int(max_voxels),
         _dptr(out.feats), _dptr(out.coords), _dptr(out.counts), _dptr(out.nvox),
-        _dptr(table, torch.uint8, "table"), table.numel(),
         _dptr(workspace, torch.uint8, "workspace"), workspace.numel(), _stream(stream))
     _check(rc, "mmbev_voxelize_roi")
     return out
@@ -284,7 +258,7 @@ def voxelize_roi_noalloc(points: torch.Tensor, sweep_offsets, sweep_tf: torch.Te
                          rois: torch.Tensor, roi_margin: float, voxel_size, pc_range,
                          max_pts_per_voxel: int, max_voxels: int, *, out: Outputs,
                          status: torch.Tensor | None = None, stream=None) -> Outputs:
-    """One frame without table or workspace (``mmbev_voxelize_roi_noalloc``),
+    """One frame without a workspace (``mmbev_voxelize_roi_noalloc``),
     for callers that cannot allocate device memory: the library's own
     file-scope device array serves as scratch. ``out`` (and ``status``, a
     1-element uint32/int32 device tensor) must be allocated by the caller."""
@@ -482,8 +456,8 @@ def scatter_bev_update(prev: "Outputs | None", out: "Outputs", max_voxels: int, 
 
 
 class Voxelizer:
-    """Owns a table and a workspace sized for one workload shape and runs the
-    batched entry point on device tensors."""
+    """Owns a workspace sized for one workload shape and runs the batched
+    entry point on device tensors."""
 
     def __init__(self, max_points, max_rois_per_frame, max_voxels, num_frames, voxel_size,
                  pc_range, max_pts_per_voxel, roi_margin, device="cuda", rho_out=0.0, seed=0):
@@ -495,7 +469,6 @@ class Voxelizer:
         self.K = int(max_pts_per_voxel)
         self.margin = float(roi_margin)
         self.num_frames = int(num_frames)
-        self.table = new_table(max_points, max_pts_per_voxel, device)
         self.workspace = new_workspace(max_points, max_rois_per_frame, max_voxels, num_frames,
                                        voxel_size, pc_range, device)
         self.out = Outputs.empty(num_frames, self.max_voxels, device)
@@ -504,7 +477,7 @@ class Voxelizer:
                  frame_roi_offsets, stream=None, stage_events=None) -> Outputs:
         return voxelize_roi_batched(points, sweep_offsets, sweep_tf, rois, self.margin,
                                     self.voxel_size, self.pc_range, self.K, self.max_voxels,
-                                    frame_sweep_offsets, frame_roi_offsets, table=self.table,
+                                    frame_sweep_offsets, frame_roi_offsets,
                                     workspace=self.workspace, out=self.out, stream=stream,
                                     stage_events=stage_events, rho_out=self.rho_out,
                                     seed=self.seed)
@@ -512,7 +485,7 @@ class Voxelizer:
     def run_host(self, h_points: torch.Tensor, sweep_offsets, h_sweep_tf: torch.Tensor,
                  h_rois: torch.Tensor, frame_sweep_offsets, frame_roi_offsets,
                  chunk_frames: int = 8, stream=None, pack_dst: torch.Tensor | None = None,
-                 table_log2_override: int = 0) -> Outputs:
+                 inject_status: int = 0) -> Outputs:
         """The batched call on pinned host inputs
         (``mmbev_voxelize_roi_batched_host``): chunks of ``chunk_frames``
         frames go up on a side stream while earlier chunks are voxelized.
@@ -521,7 +494,8 @@ class Voxelizer:
         Device staging is allocated on first use and kept: two sets, used in
         turn, so that a call's uploads can run while the previous call still
         computes (they wait only for the call before that one to have
-        finished reading the set they overwrite)."""
+        finished reading the set they overwrite). ``inject_status`` is the
+        test hook of ``voxelize_roi_batched``, applied to the first chunk."""
         if pack_dst is not None and (pack_dst.dtype != torch.uint8 or not pack_dst.is_contiguous()
                                      or not (pack_dst.is_cuda or pack_dst.is_pinned())):
             raise ValueError("pack_dst must be a contiguous uint8 device or pinned tensor")
@@ -552,7 +526,7 @@ class Voxelizer:
             self._copy_stream.wait_stream(st)
         else:
             self._copy_stream.wait_event(self._staging_read[k])
-        opts = _ExecOpts(None, int(table_log2_override), float(self.rho_out),
+        opts = _ExecOpts(None, int(inject_status), float(self.rho_out),
                          int(self.seed) & (2**64 - 1))
         nr = h_rois.shape[0] if h_rois.dim() > 1 else h_rois.numel() // 5
         rc = lib.mmbev_voxelize_roi_batched_host(
@@ -561,8 +535,7 @@ class Voxelizer:
             self.margin, _hptr(self.voxel_size), _hptr(self.pc_range), self.K, self.max_voxels,
             len(fso) - 1, _hptr(fso), _hptr(fro), _dptr(d_pts), _dptr(d_tf), _dptr(d_rois),
             _dptr(self.out.feats), _dptr(self.out.coords), _dptr(self.out.counts),
-            _dptr(self.out.nvox), _dptr(self.table), self.table.numel(), _dptr(self.workspace),
-            self.workspace.numel(),
+            _dptr(self.out.nvox), _dptr(self.workspace), self.workspace.numel(),
             None if pack_dst is None else ctypes.c_void_p(pack_dst.data_ptr()),
             0 if pack_dst is None else pack_dst.numel(), int(chunk_frames), _stream(st),
             _stream(self._copy_stream),

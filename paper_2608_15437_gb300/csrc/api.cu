@@ -62,17 +62,13 @@ int coarse_for(int mask_words) {
     return g;
 }
 
-constexpr uint32_t kSlotStride = 16;
-
-constexpr uint32_t kMaxInsertBlocks = 2048;
-
 // Byte offsets of every workspace array for one call shape.
 struct Layout {
-    size_t hdr, sweep_off, sweep_frame, fso, fro, roi_prep, masks, hist, frame_u, finfo;
-    size_t records, plist, rs, cls_cnt, seg, newlist, blockcount, bcnt, bcnt2, boff, ctot, nonempty, occ, d_bucket,
-        d_pos, d_lin, items, vid_slot, heavy, huge;
+    size_t hdr, sweep_off, sweep_frame, fso, fro, roi_prep, masks;
+    size_t records, plist, cls_cnt, bcnt, boff, ucnt, large, small, scan_state, items, temps,
+        bcap;
     size_t total;
-    uint32_t num_buckets, buckets_per_frame, num_tiles, scan_chunks;
+    uint32_t num_buckets, buckets_per_frame, num_tiles, scan_tiles;
     int bucket_log2, mask_words, coarse;
 };
 
@@ -86,7 +82,8 @@ Layout make_layout(int64_t max_points, int64_t rois_total, int32_t max_rois_fram
     L.coarse = coarse_for(L.mask_words);
     const size_t F = (size_t)num_frames, R = (size_t)(rois_total > 0 ? rois_total : 1);
     const size_t U = (size_t)(max_points > 0 ? max_points : 1);
-    const size_t B2 = ((size_t)L.num_buckets + 1) / 2 * 2;  // zeroed as 16-byte pairs
+    const size_t B4 = ((size_t)L.num_buckets + 4) / 4 * 4;  // zeroed as 16-byte words
+    L.scan_tiles = (uint32_t)(((size_t)L.num_buckets + kScanTile - 1) / kScanTile);
     L.num_tiles = (uint32_t)((U + kTile - 1) / kTile);
     const size_t TS = (size_t)L.num_tiles * kTile;        // record slots, tile-aligned
     size_t o = 0;
@@ -106,32 +103,20 @@ Layout make_layout(int64_t max_points, int64_t rois_total, int32_t max_rois_fram
         if (c * c * (size_t)w > mask_words_frame) mask_words_frame = c * c * (size_t)w;
     }
     L.masks = take(sizeof(uint32_t) * F * mask_words_frame);
-    L.hist = take(sizeof(uint32_t) * (R + F));
-    L.frame_u = take(sizeof(uint32_t) * F);
-    L.finfo = take(sizeof(FrameInfo) * F);
     L.records = take(32 * TS);
-    L.plist = take(16 * TS);
-    L.rs = take(8 * TS);
+    L.plist = take(16 * TS);      // after the scatter stage: point lists of large buckets
     L.cls_cnt = take(sizeof(uint32_t) * kMaxClsGrid);
-    L.seg = take(sizeof(uint32_t) * U);
-    L.newlist = take(16 * (U + 32 + (size_t)kMaxInsertBlocks * 256));
-    L.blockcount = take(sizeof(uint32_t) * kMaxInsertBlocks);
-    L.bcnt = take(sizeof(unsigned long long) * B2);
-    L.bcnt2 = take(sizeof(unsigned long long) * B2);
-    L.boff = take(sizeof(unsigned long long) * B2);
-    L.scan_chunks = (L.buckets_per_frame + kScanChunk - 1) / kScanChunk;
-    L.ctot = take(sizeof(uint32_t) * F * L.scan_chunks);
-    L.nonempty = take(sizeof(uint32_t) * B2);
-    L.occ = take(sizeof(uint32_t) * U);
-    L.d_bucket = take(sizeof(uint32_t) * U);
-    L.d_pos = take(sizeof(uint32_t) * U);
-    L.d_lin = take(sizeof(uint32_t) * U);
-    L.items = take(sizeof(uint2) * U);
-    L.vid_slot = take(sizeof(uint32_t) * (F * (size_t)(max_voxels > 0 ? max_voxels : 1)));
-    // slots with more than kLightMax (kHugeMin) of the at most U points
-    L.heavy = take(sizeof(uint32_t) * (U / (kLightMax + 1) + 1));
-    L.huge = take(sizeof(uint32_t) * (U / (kHugeMin + 1) + 1));
+    L.bcnt = take(sizeof(uint32_t) * B4);
+    L.boff = take(sizeof(uint32_t) * (B4 + 4));
+    L.ucnt = take(sizeof(uint32_t) * B4);
+    L.large = take(sizeof(uint32_t) * B4);
+    L.small = take(sizeof(uint32_t) * B4);
+    L.scan_state = take(sizeof(unsigned long long) * ((size_t)L.scan_tiles + 2));
+    L.items = take(sizeof(uint2) * TS);
+    L.temps = take(sizeof(VoxTemp) * TS);
+    L.bcap = take(sizeof(uint2) * B4);
     L.total = o;
+    (void)max_voxels;
     return L;
 }
 
@@ -202,33 +187,23 @@ void bind_layout(Params* p, const Layout& L, uint8_t* ws) {
     p->frame_roi_off = reinterpret_cast<int32_t*>(ws + L.fro);
     p->roi_prep = reinterpret_cast<RoiPrep*>(ws + L.roi_prep);
     p->masks = reinterpret_cast<uint32_t*>(ws + L.masks);
-    p->hist = reinterpret_cast<uint32_t*>(ws + L.hist);
-    p->frame_u = reinterpret_cast<uint32_t*>(ws + L.frame_u);
-    p->finfo = reinterpret_cast<FrameInfo*>(ws + L.finfo);
     p->records = reinterpret_cast<uint4*>(ws + L.records);
     p->plist = reinterpret_cast<uint4*>(ws + L.plist);
-    p->rs = reinterpret_cast<uint2*>(ws + L.rs);
+    p->seg2 = reinterpret_cast<uint2*>(ws + L.plist);
     p->cls_cnt = reinterpret_cast<uint32_t*>(ws + L.cls_cnt);
-    p->seg = reinterpret_cast<uint32_t*>(ws + L.seg);
     p->num_regions = (uint32_t)((p->num_points + kTile - 1) / kTile) * (kTile / kRegion);
-    p->newlist = reinterpret_cast<uint4*>(ws + L.newlist);
-    p->blockcount = reinterpret_cast<uint32_t*>(ws + L.blockcount);
-    p->bcnt = reinterpret_cast<unsigned long long*>(ws + L.bcnt);
-    p->bcnt2 = reinterpret_cast<unsigned long long*>(ws + L.bcnt2);
-    p->boff = reinterpret_cast<unsigned long long*>(ws + L.boff);
-    p->ctot = reinterpret_cast<uint32_t*>(ws + L.ctot);
-    p->scan_chunks = L.scan_chunks;
-    p->nonempty = reinterpret_cast<uint32_t*>(ws + L.nonempty);
-    p->occ = reinterpret_cast<uint32_t*>(ws + L.occ);
-    p->d_bucket = reinterpret_cast<uint32_t*>(ws + L.d_bucket);
-    p->d_pos = reinterpret_cast<uint32_t*>(ws + L.d_pos);
-    p->d_lin = reinterpret_cast<uint32_t*>(ws + L.d_lin);
+    p->bcnt = reinterpret_cast<uint32_t*>(ws + L.bcnt);
+    p->boff = reinterpret_cast<uint32_t*>(ws + L.boff);
+    p->ucnt = reinterpret_cast<uint32_t*>(ws + L.ucnt);
+    p->large = reinterpret_cast<uint32_t*>(ws + L.large);
+    p->small = reinterpret_cast<uint32_t*>(ws + L.small);
+    p->scan_state = reinterpret_cast<unsigned long long*>(ws + L.scan_state);
+    p->scan_tiles = L.scan_tiles;
     p->items = reinterpret_cast<uint2*>(ws + L.items);
-    p->vid_slot = reinterpret_cast<uint32_t*>(ws + L.vid_slot);
-    p->heavy = reinterpret_cast<uint32_t*>(ws + L.heavy);
-    p->huge = reinterpret_cast<uint32_t*>(ws + L.huge);
-    p->occ_cap = (uint32_t)(p->num_points > 0 ? p->num_points : 1);
+    p->temps = reinterpret_cast<VoxTemp*>(ws + L.temps);
+    p->bcap = reinterpret_cast<uint2*>(ws + L.bcap);
     p->rec_cap = p->num_regions * (uint32_t)kRegion;
+    p->item_cap = p->rec_cap;
     p->mask_words = L.mask_words;
     p->coarse = L.coarse;
     p->coarse_inv[0] = (float)((double)L.coarse / ((double)p->rmax[0] - (double)p->rmin[0]));
@@ -245,8 +220,7 @@ void bind_layout(Params* p, const Layout& L, uint8_t* ws) {
     } while (0)
 
 const char* const kStageNames[MMBEV_NUM_STAGES] = {
-    "prep", "classify", "insert", "compact", "scatter_points", "frames",
-    "capped_census", "scan", "scatter", "rank", "finalize"};
+    "prep", "classify", "scan", "scatter", "buckets", "output"};
 
 }  // namespace
 
@@ -270,15 +244,6 @@ using namespace mmbev;
 
 extern "C" {
 
-size_t mmbev_table_size(int64_t max_points, int32_t max_pts_per_voxel) {
-    if (max_points < 0 || max_points > 0xFFFFFFFEll) return 0;
-    if (max_pts_per_voxel < 1 || max_pts_per_voxel > kMaxK) return 0;
-    uint64_t h = 1024;
-    while (h < 2ull * (uint64_t)max_points) h <<= 1;
-    if (h > (1ull << 31)) return 0;
-    return (size_t)h * kSlotStride;
-}
-
 size_t mmbev_workspace_size(int64_t max_points, int32_t max_rois_per_frame, int32_t max_voxels,
                             int32_t num_frames, const float voxel_size[3], const float range[6]) {
     Grid g;
@@ -289,12 +254,6 @@ size_t mmbev_workspace_size(int64_t max_points, int32_t max_rois_per_frame, int3
     const Layout L = make_layout(max_points, (int64_t)max_rois_per_frame * num_frames,
                                  max_rois_per_frame, max_voxels, num_frames, g);
     return L.total;
-}
-
-int mmbev_table_clear(void* table, size_t table_bytes, cudaStream_t stream) {
-    if (!table && table_bytes) return MMBEV_EINVAL;
-    if (reinterpret_cast<uintptr_t>(table) & 15u) return MMBEV_EINVAL;
-    return launch_zero(table, table_bytes, stream) == cudaSuccess ? MMBEV_OK : MMBEV_ECUDA;
 }
 
 }  // extern "C"
@@ -309,7 +268,7 @@ int voxelize_batched(const float* points, const int64_t* sweep_offsets, int32_t 
                      int32_t max_pts_per_voxel, int32_t max_voxels, int32_t num_frames,
                      const int32_t* frame_sweep_offsets, const int32_t* frame_roi_offsets,
                      float* out_feats, int32_t* out_coords, int32_t* out_counts,
-                     int32_t* out_nvox, void* table, size_t table_bytes, void* workspace,
+                     int32_t* out_nvox, void* workspace,
                      size_t workspace_bytes, cudaStream_t stream, const mmbev_exec_opts_t* opts,
                      bool keep_status) {
     HostDesc desc;  // ~25 KB; consumed by the prep launch's parameter copy
@@ -321,7 +280,6 @@ int voxelize_batched(const float* points, const int64_t* sweep_offsets, int32_t 
     if (!out_nvox) return MMBEV_EINVAL;
     if (max_voxels > 0 && (!out_feats || !out_coords || !out_counts)) return MMBEV_EINVAL;
     if (!workspace || (reinterpret_cast<uintptr_t>(workspace) & (kAlign - 1))) return MMBEV_EINVAL;
-    if (!table || (reinterpret_cast<uintptr_t>(table) & 15u)) return MMBEV_EINVAL;
     int rc = validate_common(points, sweep_offsets, num_sweeps, sweep_tf, rois, num_rois,
                              roi_margin, voxel_size, range, num_frames, frame_sweep_offsets,
                              frame_roi_offsets, &p, &desc, &g, &rmax);
@@ -336,14 +294,6 @@ int voxelize_batched(const float* points, const int64_t* sweep_offsets, int32_t 
     p.out_coords = out_coords;
     p.out_counts = out_counts;
     p.out_nvox = out_nvox;
-    // Hash table: its capacity is the largest power of two of slots that
-    // fits and must reach 2N; the insert stage then uses the first
-    // pow2(1.25 x kept points) of them, or the override.
-    const uint64_t fit = table_bytes / kSlotStride;
-    uint32_t lg = 0;
-    while (lg < 31 && (2ull << lg) <= fit) ++lg;
-    if ((1ull << lg) > fit) return MMBEV_EWORKSPACE;
-    p.table_log2_fixed = 0;
     p.rho_thr = 0u;
     p.seed = 0ull;
     if (opts) {
@@ -352,31 +302,17 @@ int voxelize_batched(const float* points, const int64_t* sweep_offsets, int32_t 
         // floor(rho * 2^24); rho = 1 keeps every draw
         p.rho_thr = rho >= 1.0f ? (1u << 24) : (uint32_t)std::floor((double)rho * 16777216.0);
         p.seed = opts->seed;
+        p.inject_status = opts->inject_status;
     }
-    if (opts && opts->table_log2_override > 0) {
-        if (opts->table_log2_override > (int32_t)lg) return MMBEV_EWORKSPACE;
-        p.table_log2_fixed = opts->table_log2_override;
-    } else if ((1ull << lg) < 2ull * (uint64_t)p.num_points) {
-        return MMBEV_EWORKSPACE;
-    }
-    p.table = static_cast<uint8_t*>(table);
-    p.table_log2 = lg;
 
     const int sms = num_sms();
     if (sms <= 0) return MMBEV_ECUDA;
     {
-        // classify: one block per SM (at most one per tile); insert: a
-        // persistent grid whose blocks each own a sub-list with room for
-        // every entry their warps can take
+        // classify: one block per SM (at most one per tile)
         const uint64_t tiles = ((uint64_t)p.num_points + kTile - 1) / kTile;
         uint64_t g = tiles < (uint64_t)sms ? tiles : (uint64_t)sms;
         if (g > (uint64_t)kMaxClsGrid) g = kMaxClsGrid;
         p.cls_grid = (uint32_t)g;
-        p.ins_blocks = insert_blocks(sms);
-        if (p.ins_blocks > kMaxInsertBlocks) p.ins_blocks = kMaxInsertBlocks;
-        const uint64_t warps = (uint64_t)p.ins_blocks * 8;
-        const uint64_t batches = ((uint64_t)p.num_points + 31) / 32;
-        p.ins_cap = (uint32_t)(256 * ((batches + warps - 1) / warps));
     }
     cudaEvent_t* ev = opts ? opts->stage_events : nullptr;
     int stage = 0;
@@ -394,23 +330,13 @@ int voxelize_batched(const float* points, const int64_t* sweep_offsets, int32_t 
         if ((e = mark()) != cudaSuccess) break;
         if ((e = launch_classify(p, rmax, sms, pdl, stream)) != cudaSuccess) break;
         if ((e = mark()) != cudaSuccess) break;
-        if ((e = launch_insert(p, pdl, stream)) != cudaSuccess) break;
+        if ((e = launch_bucket_scan(p, pdl, stream)) != cudaSuccess) break;
         if ((e = mark()) != cudaSuccess) break;
-        if ((e = launch_compact(p, pdl, stream)) != cudaSuccess) break;
+        if ((e = launch_bucket_scatter(p, sms, pdl, stream)) != cudaSuccess) break;
         if ((e = mark()) != cudaSuccess) break;
-        if ((e = launch_scatter_points(p, pdl, stream)) != cudaSuccess) break;
+        if ((e = launch_buckets(p, sms, pdl, stream)) != cudaSuccess) break;
         if ((e = mark()) != cudaSuccess) break;
-        if ((e = launch_frames(p, sms, pdl, stream)) != cudaSuccess) break;
-        if ((e = mark()) != cudaSuccess) break;
-        if ((e = launch_capped_census(p, sms, pdl, stream)) != cudaSuccess) break;
-        if ((e = mark()) != cudaSuccess) break;
-        if ((e = launch_scan(p, pdl, stream)) != cudaSuccess) break;
-        if ((e = mark()) != cudaSuccess) break;
-        if ((e = launch_scatter(p, sms, pdl, stream)) != cudaSuccess) break;
-        if ((e = mark()) != cudaSuccess) break;
-        if ((e = launch_rank(p, sms, pdl, stream)) != cudaSuccess) break;
-        if ((e = mark()) != cudaSuccess) break;
-        if ((e = launch_finalize(p, sms, pdl, stream)) != cudaSuccess) break;
+        if ((e = launch_output(p, sms, pdl, stream)) != cudaSuccess) break;
         if ((e = mark()) != cudaSuccess) break;
     } while (0);
     return e == cudaSuccess ? MMBEV_OK : MMBEV_ECUDA;
@@ -428,13 +354,13 @@ int mmbev_voxelize_roi_batched_ex(const float* points, const int64_t* sweep_offs
                                   int32_t num_frames, const int32_t* frame_sweep_offsets,
                                   const int32_t* frame_roi_offsets, float* out_feats,
                                   int32_t* out_coords, int32_t* out_counts, int32_t* out_nvox,
-                                  void* table, size_t table_bytes, void* workspace,
+                                  void* workspace,
                                   size_t workspace_bytes, cudaStream_t stream,
                                   const mmbev_exec_opts_t* opts) {
     return voxelize_batched(points, sweep_offsets, num_sweeps, sweep_tf, rois, num_rois,
                             roi_margin, voxel_size, range, max_pts_per_voxel, max_voxels,
                             num_frames, frame_sweep_offsets, frame_roi_offsets, out_feats,
-                            out_coords, out_counts, out_nvox, table, table_bytes, workspace,
+                            out_coords, out_counts, out_nvox, workspace,
                             workspace_bytes, stream, opts, false);
 }
 
@@ -444,8 +370,8 @@ int mmbev_voxelize_roi_batched_host(
     const float voxel_size[3], const float range[6], int32_t max_pts_per_voxel,
     int32_t max_voxels, int32_t num_frames, const int32_t* frame_sweep_offsets,
     const int32_t* frame_roi_offsets, float* d_points, float* d_sweep_tf, mmbev_roi_t* d_rois,
-    float* out_feats, int32_t* out_coords, int32_t* out_counts, int32_t* out_nvox, void* table,
-    size_t table_bytes, void* workspace, size_t workspace_bytes, void* pack_dst,
+    float* out_feats, int32_t* out_coords, int32_t* out_counts, int32_t* out_nvox,
+    void* workspace, size_t workspace_bytes, void* pack_dst,
     size_t pack_bytes, int32_t chunk_frames, cudaStream_t stream, cudaStream_t copy_stream,
     const mmbev_exec_opts_t* opts) {
     if (num_frames < 1 || num_frames > kMaxFrames || chunk_frames < 1) return MMBEV_EINVAL;
@@ -511,14 +437,20 @@ int mmbev_voxelize_roi_batched_host(
         fro.assign(frame_roi_offsets + f0, frame_roi_offsets + f1 + 1);
         for (int32_t& v : fro) v -= r0;
         const size_t row0 = (size_t)f0 * (size_t)max_voxels;
+        // a test hook's status bits go into the first chunk only
+        mmbev_exec_opts_t copts{};
+        if (opts) {
+            copts = *opts;
+            if (c > 0) copts.inject_status = 0u;
+        }
         rc = voxelize_batched(
             d_points ? d_points + 5 * p0 : nullptr, so.data(), s1 - s0,
             d_sweep_tf ? d_sweep_tf + 16 * (size_t)s0 : nullptr, d_rois ? d_rois + r0 : nullptr,
             r1 - r0, roi_margin, voxel_size, range, max_pts_per_voxel, max_voxels, f1 - f0,
             fso.data(), fro.data(), out_feats ? out_feats + 5 * row0 : nullptr,
             out_coords ? out_coords + 3 * row0 : nullptr,
-            out_counts ? out_counts + row0 : nullptr, out_nvox + f0, table, table_bytes,
-            workspace, workspace_bytes, stream, opts, c > 0);
+            out_counts ? out_counts + row0 : nullptr, out_nvox + f0,
+            workspace, workspace_bytes, stream, opts ? &copts : nullptr, c > 0);
         // the chunk's kept rows into the packed buffer (offsets of frames
         // f0..f1 and their records), while later chunks go up and run
         if (rc == MMBEV_OK && pack_dst &&
@@ -539,13 +471,13 @@ int mmbev_voxelize_roi_batched(const float* points, const int64_t* sweep_offsets
                                const int32_t* frame_sweep_offsets,
                                const int32_t* frame_roi_offsets, float* out_feats,
                                int32_t* out_coords, int32_t* out_counts, int32_t* out_nvox,
-                               void* table, size_t table_bytes, void* workspace,
+                               void* workspace,
                                size_t workspace_bytes, cudaStream_t stream) {
     return mmbev_voxelize_roi_batched_ex(points, sweep_offsets, num_sweeps, sweep_tf, rois,
                                          num_rois, roi_margin, voxel_size, range,
                                          max_pts_per_voxel, max_voxels, num_frames,
                                          frame_sweep_offsets, frame_roi_offsets, out_feats,
-                                         out_coords, out_counts, out_nvox, table, table_bytes,
+                                         out_coords, out_counts, out_nvox,
                                          workspace, workspace_bytes, stream, nullptr);
 }
 
@@ -553,15 +485,15 @@ int mmbev_voxelize_roi(const float* points, const int64_t* sweep_offsets, int32_
                        const float* sweep_tf, const mmbev_roi_t* rois, int32_t num_rois,
                        float roi_margin, const float voxel_size[3], const float range[6],
                        int32_t max_pts_per_voxel, int32_t max_voxels, float* out_feats,
-                       int32_t* out_coords, int32_t* out_counts, int32_t* out_nvox, void* table,
-                       size_t table_bytes, void* workspace, size_t workspace_bytes,
+                       int32_t* out_coords, int32_t* out_counts, int32_t* out_nvox,
+                       void* workspace, size_t workspace_bytes,
                        cudaStream_t stream) {
     const int32_t fso[2] = {0, num_sweeps};
     const int32_t fro[2] = {0, num_rois};
     return mmbev_voxelize_roi_batched_ex(points, sweep_offsets, num_sweeps, sweep_tf, rois,
                                          num_rois, roi_margin, voxel_size, range,
                                          max_pts_per_voxel, max_voxels, 1, fso, fro, out_feats,
-                                         out_coords, out_counts, out_nvox, table, table_bytes,
+                                         out_coords, out_counts, out_nvox,
                                          workspace, workspace_bytes, stream, nullptr);
 }
 

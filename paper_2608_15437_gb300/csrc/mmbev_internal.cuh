@@ -10,24 +10,23 @@
 //               {x', y', z', intensity} {dt, ROI rank, -, -}. Region g holds
 //               points 32g .. 32g+31, so positions increase with the point
 //               index and "first K by position" is "first K by index".
+//   buckets     a frame's linear indices cut into buckets of 2^LB consecutive
+//               cells (LB <= 13); bucket b = frame * Bf + (lin >> LB) over the
+//               whole call, so ascending b is ascending (frame, lin).
+//   bcnt        workspace [B], kept points per bucket, counted by the
+//               classify pass (its atomic also numbers the point's arrival).
 //   plist       workspace, per classify block a dense list (any order) of its
-//               kept points {lin, frame, position}, starting at the block's
-//               first tile * 2048; cls_cnt holds the lengths.
-//   rs          workspace, parallel to plist: {slot, arrival number of the
-//               point in its voxel}, from the insert kernel.
-//   table       caller's hash table of 16-byte slots: { u64 key+1 (0 =
-//               empty), u32 0xFFFFFFFF-minrank (0 = none), u32 count (points
-//               of the voxel) }. Insert uses the first H slots, H the power of
-//               two >= 1.25 x the kept points of the call (at most the
-//               buffer's capacity, >= 2 x the points). Once the voxels are
-//               listed the key's low word holds the voxel's segment offset.
-//   newlist     workspace, per insert block a sub-list of the voxels that
-//               block created {slot, lin, frame}; the compact kernel
-//               concatenates the sub-lists into the occupied-voxel list.
-//   seg         workspace, the record positions of each voxel's points,
-//               voxel after voxel (CSR); a voxel's first K points are its K
-//               smallest positions.
-//   workspace   Header + per-call arrays (see Layout).
+//               kept points {bucket, position, low bits of lin | rank << 16,
+//               arrival}, starting at the block's first tile * 2048; cls_cnt
+//               holds the lengths.
+//   boff        workspace [B + 1], exclusive prefix of bcnt over the call: the
+//               bucket's first item.
+//   items       workspace [M], the kept points grouped by bucket (counting
+//               sort by bucket): {position, low bits of lin | rank << 16}.
+//   temps       workspace [M], per bucket its voxels in ascending lin at
+//               boff[b] + v: {5 mean features, count, minimum rank, low lin}.
+//   ucnt        workspace [B], voxels per bucket.
+//   workspace   Header + per-call arrays (see Layout in api.cu).
 #pragma once
 
 #include <cstdint>
@@ -50,14 +49,17 @@ constexpr int kRegion = 32;
 // Classify blocks (one per SM, at most this many).
 constexpr int kMaxClsGrid = 1000;
 
-// Bucket bitmap ordering: a bucket spans 2^kBucketLog2Max consecutive linear
-// indices of one frame (fewer when the grid is smaller); one warp ranks a
-// bucket with shared-memory bitmaps.
+// Buckets span 2^LB consecutive linear indices of one frame, LB at most this.
 constexpr int kBucketLog2Max = 13;
 
-// The scan of a frame's bucket counters runs in chunks of this many buckets,
-// one block each; the compact kernel counts voxels per chunk as well.
-constexpr uint32_t kScanChunk = 1024;
+// The bucket scan works in tiles of this many buckets (1024 threads x 4).
+constexpr uint32_t kScanTile = 4096;
+
+// Bucket sizes: up to kSmallMax kept points a bucket is one warp's work, else
+// a block's; up to kSegSmem points the block keeps the bucket's point lists
+// in shared memory, beyond that in the global scratch aliased on plist.
+constexpr uint32_t kSmallMax = 64;
+constexpr uint32_t kSegSmem = 2048;
 
 // Bounded waits.
 constexpr uint32_t kSpinLimit = 1u << 22;
@@ -93,30 +95,26 @@ struct __align__(16) RoiPrep {
     float hl, hw, pad0, pad1;
 };
 
-// Per-frame results of the frames stage.
-struct __align__(16) FrameInfo {
-    uint32_t capped;  // more voxels than max_voxels
-    uint32_t rstar;   // rank threshold: ranks < rstar kept, == rstar partly
-    uint32_t q;       // how many rank-rstar voxels are kept (smallest lin first)
-    uint32_t nvox;    // kept voxels
-    uint32_t vbase;   // exclusive prefix of nvox over frames
-    uint32_t ibase;   // exclusive prefix of the frame's voxel count (item segment)
-    uint32_t pad[2];
+// One voxel of a bucket, in ascending lin: the mean features, the count of
+// points kept (min(n, K)), the minimum ROI rank over all its points and the
+// low LB bits of its linear index.
+struct __align__(16) VoxTemp {
+    float f[5];
+    uint32_t count;
+    uint32_t minrank;
+    uint32_t lo;
 };
 
 // Workspace header; zeroed by the prep kernel at the start of every call.
 struct __align__(16) Header {
-    uint32_t status;       // MMBEV_DEV_* bits (first word: read by mmbev_get_status)
-    uint32_t num_occ;      // occupied slots (unique voxels over all frames)
-    uint32_t total_kept;   // kept voxels over all frames
-    uint32_t any_capped;   // some frame has more voxels than max_voxels
-    uint32_t num_rec;      // kept points (records) of the call
-    uint32_t num_nonempty; // non-empty buckets listed by the scan stage
-    uint32_t seg_total;    // point entries reserved in seg
-    uint32_t num_heavy;    // kept voxels with 33 .. 1024 points
-    uint32_t num_huge;     // kept voxels with more than 1024 points
-    uint32_t frames_done;  // blocks of the frames stage that finished their histogram share
-    uint32_t pad[6];
+    uint32_t status;        // MMBEV_DEV_* bits (first word: read by mmbev_get_status)
+    uint32_t num_rec;       // kept points (records) of the call
+    uint32_t scan_ticket;   // scan tiles started, in order
+    uint32_t n_large;       // buckets of more than kSmallMax points (block work)
+    uint32_t n_small;       // buckets of 1 .. kSmallMax points (warp work)
+    uint32_t large_ticket;  // large buckets taken by the bucket stage
+    uint32_t small_ticket;  // small buckets taken
+    uint32_t pad[9];
 };
 
 // Everything a kernel needs; passed by value.
@@ -144,15 +142,13 @@ struct Params {
     uint32_t rho_thr;       // keep a point inside no ROI when its draw's top 24 bits < rho_thr
     uint64_t seed;          // SplitMix64 seed of those draws
     int32_t keep_status = 0;  // prep leaves the status word as it is (later chunks of a call)
-    // bucket ordering
-    int32_t bucket_log2;
-    uint32_t buckets_per_frame;
-    UDiv div_bf;            // division by buckets_per_frame (bucket -> frame)
-    uint32_t num_buckets;   // num_frames * buckets_per_frame
-    // hash table
-    uint8_t* table;
-    uint32_t table_log2;    // the buffer's capacity (log2 slots)
-    int32_t table_log2_fixed;  // > 0: use this many slots instead of sizing by the points
+    uint32_t inject_status = 0;  // test hook: status bits prep sets as a failure would
+    // buckets
+    int32_t bucket_log2;       // LB
+    uint32_t buckets_per_frame;  // Bf
+    UDiv div_bf;               // division by Bf (bucket -> frame)
+    uint32_t num_buckets;      // B = F * Bf
+    uint32_t scan_tiles;       // ceil(B / kScanTile)
     // workspace arrays
     Header* hdr;
     int64_t* sweep_off;     // [S+1]
@@ -161,36 +157,23 @@ struct Params {
     int32_t* frame_roi_off;    // [F+1]
     RoiPrep* roi_prep;      // [R]
     uint32_t* masks;        // [F][coarse^2][mask_words]
-    uint32_t* hist;         // [R + F] voxels per minimum rank 0 .. R_f (capped frames)
-    uint32_t* frame_u;      // [F] unique voxels per frame
-    FrameInfo* finfo;       // [F]
     uint4* records;         // [regions*32][2] kept points' features and rank
-    uint4* plist;           // [tiles*2048] per classify block: kept {lin, frame, position}
-    uint2* rs;              // [tiles*2048] parallel to plist: {slot, arrival}
+    uint4* plist;           // [tiles*2048] per classify block: {bucket, pos, lo|rank<<16, arrival}
+    uint2* seg2;            // [tiles*2048] point lists of buckets over kSegSmem (aliases plist)
     uint32_t* cls_cnt;      // [kMaxClsGrid] list length of each classify block
     uint32_t cls_grid;      // classify blocks of the call
-    uint32_t* seg;          // [N] record positions, voxel by voxel
     uint32_t num_regions;
-    uint4* newlist;         // [ins_blocks * ins_cap] voxels created, per insert block
-    uint32_t* blockcount;   // [ins_blocks] voxels each insert block created
-    uint32_t ins_blocks;    // grid of the insert kernel
-    uint32_t ins_cap;       // room of each insert block's sub-list
-    unsigned long long* bcnt;   // [B] voxels per bucket (every frame, no classes)
-    unsigned long long* bcnt2;  // [B] capped frames: lo = rank-below, hi = rank-tie
-    unsigned long long* boff;   // [B] exclusive offsets within the frame (lo, hi)
-    uint32_t* ctot;         // [F * scan_chunks] voxels per scan chunk (uncapped frames)
-    uint32_t scan_chunks;   // scan chunks per frame
-    uint32_t* occ;          // [occ_cap] slot of each unique voxel
-    uint32_t* d_bucket;     // [occ_cap]
-    uint32_t* d_pos;        // [occ_cap] position inside the bucket
-    uint32_t* d_lin;        // [occ_cap] linear index of each unique voxel
-    uint2* items;           // [occ_cap] (slot, lin) grouped by bucket
-    uint32_t* nonempty;     // [B] non-empty bucket ids
-    uint32_t* vid_slot;     // [F*max_voxels] slot of each kept voxel, output order
-    uint32_t* heavy;        // [F*max_voxels] kept voxels with 33 .. 1024 points
-    uint32_t* huge;         // [F*max_voxels] kept voxels with more than 1024 points
-    uint32_t occ_cap;
     uint32_t rec_cap;       // record positions of the call (regions * 32)
+    uint32_t* bcnt;         // [B] kept points per bucket
+    uint32_t* boff;         // [B + 1] first item of each bucket
+    uint32_t* ucnt;         // [B] voxels per bucket
+    uint32_t* large;        // [B] buckets of more than kSmallMax points
+    uint32_t* small;        // [B] buckets of 1 .. kSmallMax points
+    unsigned long long* scan_state;  // [scan_tiles] look-back words of the bucket scan
+    uint2* items;           // [rec_cap] kept points grouped by bucket
+    VoxTemp* temps;         // [rec_cap] voxels grouped by bucket
+    uint2* bcap;            // [B] capped frames: voxels below / at the threshold rank
+    uint32_t item_cap;      // room of items and temps (rec_cap)
     // outputs
     float* out_feats;
     int32_t* out_coords;
@@ -333,26 +316,6 @@ __device__ __forceinline__ int find_sweep(const int64_t* off, int nsweeps, int64
     return lo;
 }
 
-// Slot addressing (16-byte slots).
-constexpr uint32_t kSlotBytes = 16;
-__device__ __forceinline__ unsigned long long* slot_key(const Params& p, uint32_t h) {
-    return reinterpret_cast<unsigned long long*>(p.table + (size_t)h * kSlotBytes);
-}
-__device__ __forceinline__ uint32_t* slot_rank(const Params& p, uint32_t h) {
-    return reinterpret_cast<uint32_t*>(p.table + (size_t)h * kSlotBytes + 8);
-}
-__device__ __forceinline__ uint32_t* slot_cnt(const Params& p, uint32_t h) {
-    return reinterpret_cast<uint32_t*>(p.table + (size_t)h * kSlotBytes + 12);
-}
-// valid once the voxel list is built: the key is no longer needed
-__device__ __forceinline__ uint32_t* slot_seg(const Params& p, uint32_t h) {
-    return reinterpret_cast<uint32_t*>(p.table + (size_t)h * kSlotBytes);
-}
-
-__device__ __forceinline__ void zero_slot(const Params& p, uint32_t h) {
-    *reinterpret_cast<uint4*>(p.table + (size_t)h * kSlotBytes) = make_uint4(0u, 0u, 0u, 0u);
-}
-
 // The n-th output (n >= 1) of SplitMix64 (Steele, Lea and Flood, OOPSLA
 // 2014) started at state `seed`: the finalizer of seed + n * golden gamma.
 __device__ __forceinline__ uint64_t splitmix64_nth(uint64_t seed, uint64_t n) {
@@ -379,8 +342,12 @@ __device__ __forceinline__ unsigned long long ld_cg(const unsigned long long* a)
     return __ldcg(a);
 }
 
-__device__ __forceinline__ uint32_t slot_minrank(const Params& p, uint32_t h) {
-    return 0xFFFFFFFFu - ld_cg(slot_rank(p, h));
+// Acquire load at GPU scope, issued anew every time (for polling a word that
+// another block publishes).
+__device__ __forceinline__ unsigned long long ld_acquire(const unsigned long long* a) {
+    unsigned long long v;
+    asm volatile("ld.acquire.gpu.global.u64 %0, [%1];" : "=l"(v) : "l"(a) : "memory");
+    return v;
 }
 
 // ---------------------------------------------------------------- launchers
@@ -393,29 +360,16 @@ cudaError_t launch_prep_rois(const mmbev_roi_t* rois, int32_t n, float margin, f
                              cudaStream_t st);
 cudaError_t launch_classify(const Params& p, int rmax, int num_sms, bool pdl, cudaStream_t st);
 cudaError_t launch_classify_points(const Params& p, cudaStream_t st);
-cudaError_t launch_insert(const Params& p, bool pdl, cudaStream_t st);
-cudaError_t launch_insert(const Params& p, bool pdl, cudaStream_t st);
-cudaError_t launch_compact(const Params& p, bool pdl, cudaStream_t st);
-uint32_t insert_blocks(int num_sms);
-cudaError_t launch_scatter_points(const Params& p, bool pdl, cudaStream_t st);
-cudaError_t launch_frames(const Params& p, int num_sms, bool pdl, cudaStream_t st);
-cudaError_t launch_capped_census(const Params& p, int num_sms, bool pdl, cudaStream_t st);
-cudaError_t launch_scan(const Params& p, bool pdl, cudaStream_t st);
-cudaError_t launch_scatter(const Params& p, int num_sms, bool pdl, cudaStream_t st);
-cudaError_t launch_rank(const Params& p, int num_sms, bool pdl, cudaStream_t st);
-cudaError_t launch_finalize(const Params& p, int num_sms, bool pdl, cudaStream_t st);
+cudaError_t launch_bucket_scan(const Params& p, bool pdl, cudaStream_t st);
+cudaError_t launch_bucket_scatter(const Params& p, int num_sms, bool pdl, cudaStream_t st);
+cudaError_t launch_buckets(const Params& p, int num_sms, bool pdl, cudaStream_t st);
+cudaError_t launch_output(const Params& p, int num_sms, bool pdl, cudaStream_t st);
 // Kept rows of frames [f0, f1) of a call's outputs into a packed buffer
 // (mmbev_pack_voxels' layout for F frames).
 cudaError_t launch_pack(const float* feats, const int32_t* coords, const int32_t* counts,
                         const int32_t* nvox, int32_t F, int32_t f0, int32_t f1,
                         int32_t max_voxels, void* dst, cudaStream_t stream);
 int num_sms();   // of the current device, cached
-
-// Voxels with more points than kLightMax are "heavy" (a warp each in the
-// finalize stage), with more than kHugeMin "huge" (a block each); the compact
-// stage lists their slots.
-constexpr uint32_t kLightMax = 32;
-constexpr uint32_t kHugeMin = 1024;
 cudaError_t launch_zero(void* ptr, size_t bytes, cudaStream_t st);
 
 // Launch `kern` with an optional programmatic-stream-serialization attribute.

@@ -6,14 +6,15 @@
 // device and has unbounded latency), a host that hands the library only
 // pre-registered input and output buffers, or code running where the CUDA
 // allocator is owned by another framework. This entry point serves them: the
-// hash table and the scratch workspace live in one file-scope device array of
+// scratch workspace lives in one file-scope device array of
 // MMBEV_NOALLOC_SCRATCH_BYTES, which every GPU that loads this library holds
 // until the process exits. The caller passes only inputs and outputs.
 //
 // The array is shared by every call on a device and keeps the last call's
-// contents, so each call first zeroes the part that must start at zero (the
-// hash table). Calls whose executions overlap on the GPU (two streams, or two
-// host threads) race on the array; serialize them.
+// contents. Nothing in it has to start at zero: the call's first kernel
+// clears the counters the later ones accumulate into. Calls whose
+// executions overlap on the GPU (two streams, or two host threads) race on
+// the array; serialize them.
 #include <cuda.h>   // driver types only: the two entry points below are fetched at run time
 
 #include <cstring>
@@ -23,12 +24,10 @@
 
 namespace {
 
-// Scratch of the no-allocation entry point: the hash table, then the workspace.
+// Scratch of the no-allocation entry point: the workspace of its call.
 static __device__ __align__(256) unsigned char g_noalloc_scratch[MMBEV_NOALLOC_SCRATCH_BYTES];
 
 constexpr int kMaxDevices = 64;
-
-size_t round256(size_t x) { return (x + 255) / 256 * 256; }
 
 // Driver calls that name the current context, fetched through the runtime so
 // that the library keeps no link-time dependency on the driver library.
@@ -125,26 +124,22 @@ extern "C" int mmbev_voxelize_roi_noalloc(const float* points, const int64_t* sw
     if (!sweep_offsets || num_sweeps < 0 || num_sweeps > MMBEV_MAX_SWEEPS) return MMBEV_EINVAL;
     const int64_t n = sweep_offsets[num_sweeps];
     if (n < 0) return MMBEV_EINVAL;
-    const size_t table_bytes = mmbev_table_size(n, max_pts_per_voxel);
     const size_t ws_bytes = mmbev_workspace_size(n, num_rois, max_voxels, 1, voxel_size, range);
-    if (table_bytes == 0 || ws_bytes == 0) return MMBEV_EINVAL;
-    const size_t ws_off = round256(table_bytes);
-    if (ws_off + ws_bytes > (size_t)MMBEV_NOALLOC_SCRATCH_BYTES) return MMBEV_EWORKSPACE;
+    if (ws_bytes == 0) return MMBEV_EINVAL;
+    if (ws_bytes > (size_t)MMBEV_NOALLOC_SCRATCH_BYTES) return MMBEV_EWORKSPACE;
 
     void* base = nullptr;
     if (scratch_address(&base) != cudaSuccess) return MMBEV_ECUDA;
     unsigned char* scratch = static_cast<unsigned char*>(base);
-    // The previous call may have left anything here: zero the table region.
-    if (mmbev::launch_zero(scratch, table_bytes, stream) != cudaSuccess) return MMBEV_ECUDA;
     const int rc = mmbev_voxelize_roi(points, sweep_offsets, num_sweeps, sweep_tf, rois, num_rois,
                                       roi_margin, voxel_size, range, max_pts_per_voxel,
                                       max_voxels, out_feats, out_coords, out_counts, out_nvox,
-                                      scratch, table_bytes, scratch + ws_off, ws_bytes, stream);
+                                      scratch, ws_bytes, stream);
     if (rc != MMBEV_OK) return rc;
     if (out_status) {
         // the device status word is the first word of the workspace
-        if (cudaMemcpyAsync(out_status, scratch + ws_off, sizeof(uint32_t),
-                            cudaMemcpyDeviceToDevice, stream) != cudaSuccess)
+        if (cudaMemcpyAsync(out_status, scratch, sizeof(uint32_t), cudaMemcpyDeviceToDevice,
+                            stream) != cudaSuccess)
             return MMBEV_ECUDA;
     }
     return MMBEV_OK;

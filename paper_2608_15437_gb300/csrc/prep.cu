@@ -96,7 +96,8 @@ k_prep(Params p, const __grid_constant__ HostDesc d) {
     const size_t gt = (size_t)zb * blockDim.x + t;
     const size_t gs = (size_t)nz * blockDim.x;
     if (gt < sizeof(Header) / 4 && !(gt == 0 && p.keep_status))   // word 0: the status
-        reinterpret_cast<uint32_t*>(p.hdr)[gt] = 0u;
+        reinterpret_cast<uint32_t*>(p.hdr)[gt] = gt == 0 ? p.inject_status : 0u;
+    if (gt == 0 && p.keep_status && p.inject_status) set_status(p.hdr, p.inject_status);
     for (size_t i = gt; i <= (size_t)p.num_sweeps; i += gs) p.sweep_off[i] = d.sweep_off[i];
     for (size_t i = gt; i <= (size_t)p.num_frames; i += gs) {
         p.frame_sweep_off[i] = d.frame_sweep_off[i];
@@ -111,17 +112,13 @@ k_prep(Params p, const __grid_constant__ HostDesc d) {
         }
         p.sweep_frame[s] = lo;
     }
-    if (p.hist)
-        for (size_t i = gt; i < (size_t)p.num_rois + p.num_frames; i += gs) p.hist[i] = 0u;
-    if (p.frame_u)
-        for (size_t i = gt; i < (size_t)p.num_frames; i += gs) p.frame_u[i] = 0u;
-    if (p.ctot)
-        for (size_t i = gt; i < (size_t)p.num_frames * p.scan_chunks; i += gs) p.ctot[i] = 0u;
-    if (p.cls_cnt)  // a classify block that gives up leaves its list empty
+    if (p.cls_cnt)
         for (size_t i = gt; i < (size_t)kMaxClsGrid; i += gs) p.cls_cnt[i] = 0u;
+    if (p.scan_state)
+        for (size_t i = gt; i < (size_t)p.scan_tiles; i += gs) p.scan_state[i] = 0ull;
     if (p.bcnt) {
-        uint4* b4 = reinterpret_cast<uint4*>(p.bcnt);  // B u64 counters, B even or padded
-        const size_t n4 = ((size_t)p.num_buckets + 1) / 2;
+        uint4* b4 = reinterpret_cast<uint4*>(p.bcnt);  // B counters, padded to a multiple of 4
+        const size_t n4 = ((size_t)p.num_buckets + 3) / 4;
         for (size_t i = gt; i < n4; i += gs) b4[i] = make_uint4(0u, 0u, 0u, 0u);
     }
 }

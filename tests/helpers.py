@@ -16,31 +16,29 @@ def to_dev(w, dev, rois=None):
     return pts, tf, rois_t
 
 
-def run_gpu(mmbev, w, dev, K=None, maxv=None, table_log2_override=0, table=None, workspace=None,
+def run_gpu(mmbev, w, dev, K=None, maxv=None, inject_status=0, workspace=None,
             stream=None, rho_out=0.0, seed=0):
     """Batched C-ABI call on w; returns (per-frame list of (feats, coords,
-    counts), device status, table, workspace)."""
+    counts), device status, workspace)."""
     import torch
     K = w.max_pts_per_voxel if K is None else K
     maxv = w.max_voxels if maxv is None else maxv
     pts, tf, rois = to_dev(w, dev)
     nf = w.num_frames
     rmax = int(np.max(np.diff(w.frame_roi_offsets))) if nf else 0
-    if table is None:
-        table = mmbev.new_table(max(w.num_points, 1), K, dev)
     if workspace is None:
         workspace = mmbev.new_workspace(max(w.num_points, 1), rmax, maxv, nf, w.voxel_size,
                                         w.pc_range, dev)
     out = mmbev.voxelize_roi_batched(pts, w.sweep_offsets, tf, rois, w.roi_margin, w.voxel_size,
                                      w.pc_range, K, maxv, w.frame_sweep_offsets,
-                                     w.frame_roi_offsets, table=table, workspace=workspace,
-                                     table_log2_override=table_log2_override, stream=stream,
+                                     w.frame_roi_offsets, workspace=workspace,
+                                     inject_status=inject_status, stream=stream,
                                      rho_out=rho_out, seed=seed)
     torch.cuda.synchronize(dev)
     status = mmbev.get_status(workspace)
     nvox = out.nvox.cpu().numpy()
     frames = [out.frame(f, maxv, nvox[f]) for f in range(nf)]
-    return frames, status, table, workspace
+    return frames, status, workspace
 
 
 def run_oracle(oracle, w, K=None, maxv=None, rho_out=0.0, seed=0):

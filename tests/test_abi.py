@@ -24,7 +24,7 @@ def declared_functions():
 def test_header_declares_the_boundary():
     names = declared_functions()
     for required in ("mmbev_voxelize_roi", "mmbev_voxelize_roi_batched", "mmbev_workspace_size",
-                     "mmbev_table_size", "mmbev_classify_points", "mmbev_get_status"):
+                     "mmbev_classify_points", "mmbev_get_status", "mmbev_prep_rois"):
         assert required in names
 
 
@@ -35,14 +35,6 @@ def test_library_exports_every_declared_symbol(mmbev_lib):
 
 
 def test_sizes_are_host_only(mmbev_lib):
-    # capacity: next power of two >= 2N (at least 1024) slots of 16 bytes
-    assert mmbev_lib.table_size(20000, 10) == 65536 * 16
-    assert mmbev_lib.table_size(100, 1) == 1024 * 16
-    assert mmbev_lib.table_size(11110400, 64) == (1 << 25) * 16
-    with pytest.raises(ValueError):
-        mmbev_lib.table_size(100, 0)
-    with pytest.raises(ValueError):
-        mmbev_lib.table_size(100, 65)
     a = mmbev_lib.workspace_size(20000, 4, 16000, 1, TINY_VS, TINY_RG)
     b = mmbev_lib.workspace_size(40000, 4, 16000, 1, TINY_VS, TINY_RG)
     c = mmbev_lib.workspace_size(20000, 4, 16000, 2, TINY_VS, TINY_RG)
@@ -52,8 +44,7 @@ def test_sizes_are_host_only(mmbev_lib):
 
 
 def _call(lib, *, so=(0, 100), fso=None, fro=None, nr=1, K=10, maxv=100, vs=TINY_VS, rg=TINY_RG,
-          margin=0.5, ws_bytes=1 << 30, table_bytes=1 << 30, ws=0x7f0000000000,
-          table=0x7f1000000000):
+          margin=0.5, ws_bytes=1 << 30, ws=0x7f0000000000):
     so = np.asarray(so, np.int64)
     ns = len(so) - 1
     fso = np.asarray([0, ns] if fso is None else fso, np.int32)
@@ -65,14 +56,14 @@ def _call(lib, *, so=(0, 100), fso=None, fro=None, nr=1, K=10, maxv=100, vs=TINY
     return lib.mmbev_voxelize_roi_batched(
         fake, so.ctypes.data_as(P), ns, fake, fake, nr, margin, vs.ctypes.data_as(P),
         rg.ctypes.data_as(P), K, maxv, len(fso) - 1, fso.ctypes.data_as(P), fro.ctypes.data_as(P),
-        fake, fake, fake, fake, P(table), table_bytes, P(ws), ws_bytes, None)
+        fake, fake, fake, fake, P(ws), ws_bytes, None)
 
 
 @pytest.mark.parametrize("kw", [
     dict(K=0), dict(K=65), dict(maxv=-1), dict(so=(1, 100)), dict(so=(0, 50, 40)),
     dict(fso=(0, 2)), dict(fro=(0, 2)), dict(margin=-0.1), dict(margin=float("nan")),
     dict(vs=(0.2, 0.0, 8.0)), dict(rg=(0, 0, 0, 0, 1, 1)), dict(rg=(0, 0, 0, float("inf"), 1, 1)),
-    dict(ws=0x7f0000000010), dict(table=0x7f1000000004), dict(nr=2000, fro=(0, 2000)),
+    dict(ws=0x7f0000000010), dict(nr=2000, fro=(0, 2000)),
     dict(vs=(1e-4, 1e-4, 1e-4)),   # more than 2^32 cells
     dict(so=[0] * 2050),            # too many sweeps
 ])
@@ -83,7 +74,6 @@ def test_invalid_arguments_are_rejected_before_launch(mmbev_lib, kw):
 def test_small_buffers_are_rejected_before_launch(mmbev_lib):
     lib = mmbev_lib.load()
     assert _call(lib, ws_bytes=1024) == -3
-    assert _call(lib, table_bytes=16 * 100) == -3   # fewer than 2N slots
 
 
 @pytest.mark.parametrize("rho", [-0.1, 1.5, float("nan")])
@@ -98,8 +88,7 @@ def test_rho_out_outside_unit_interval_is_rejected(mmbev_lib, rho):
     rc = lib.mmbev_voxelize_roi_batched_ex(
         fake, so.ctypes.data_as(P), 1, fake, fake, 1, 0.5, TINY_VS.ctypes.data_as(P),
         TINY_RG.ctypes.data_as(P), 10, 100, 1, fso.ctypes.data_as(P), fro.ctypes.data_as(P),
-        fake, fake, fake, fake, P(0x7f1000000000), 1 << 30, P(0x7f0000000000), 1 << 30, None,
-        ctypes.byref(opts))
+        fake, fake, fake, fake, P(0x7f0000000000), 1 << 30, None, ctypes.byref(opts))
     assert rc == -1
 
 
@@ -205,8 +194,8 @@ def test_host_input_call_checks_offsets_before_copying(mmbev_lib):
         return lib.mmbev_voxelize_roi_batched_host(
             fake, so.ctypes.data_as(P), nsw, fake, fake, nroi, 0.5, vs.ctypes.data_as(P),
             rg.ctypes.data_as(P), 10, 1000, len(fso) - 1, fso.ctypes.data_as(P),
-            fro.ctypes.data_as(P), fake, fake, fake, fake, fake, fake, fake, fake, 1 << 20, fake,
-            1 << 20, None, 0, chunk, None, None, None)
+            fro.ctypes.data_as(P), fake, fake, fake, fake, fake, fake, fake, fake, 1 << 20,
+            None, 0, chunk, None, None, None)
 
     assert call([0, 1, 2], [0, 1, 3], chunk=0) == -1           # chunk_frames < 1
     assert call([1, 1, 2], [0, 1, 3]) == -1                     # frames must start at sweep 0
@@ -234,8 +223,7 @@ def test_scatter_bev_update_checks_its_arguments(mmbev_lib):
 def test_stage_names_follow_the_launch_order(mmbev_lib):
     # one name per kernel of a call, in launch order; out of range: empty
     names = mmbev_lib.stage_names()
-    assert names == ["prep", "classify", "insert", "compact", "scatter_points", "frames",
-                     "capped_census", "scan", "scatter", "rank", "finalize"]
+    assert names == ["prep", "classify", "scan", "scatter", "buckets", "output"]
     lib = mmbev_lib.load()
     assert lib.mmbev_stage_name(mmbev_lib.NUM_STAGES) == b""
     assert lib.mmbev_stage_name(-1) == b""

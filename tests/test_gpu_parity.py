@@ -79,12 +79,11 @@ def test_roi_prep_trig_matches_libm_on_a_million_yaws(oracle_mod, mmbev_lib, cud
                                   "roi_128", "roi_full"])
 def test_voxelize_parity(oracle_mod, mmbev_lib, cuda_dev, name):
     w = synth.CONFIGS[name]()
-    got, status, table, _ = run_gpu(mmbev_lib, w, cuda_dev)
+    got, status, _ = run_gpu(mmbev_lib, w, cuda_dev)
     assert status == 0
     want = run_oracle(oracle_mod, w)
     exact = assert_frames_equal(got, want, name)
     assert exact == 1.0, f"{name}: {exact:.6f} of feature values bit-exact"
-    assert _table_is_clean(table)
 
 
 @pytest.mark.parametrize("n_rois", [33, 48, 64, 65, 96])
@@ -95,22 +94,20 @@ def test_mask_sizes_between_the_configs(oracle_mod, mmbev_lib, cuda_dev, n_rois)
     over three frames, so blocks stage two frames."""
     w = synth.concat_frames([synth.roi_coverage(n_rois, scene_seed=s) for s in (1, 2, 3)],
                             f"roi{n_rois}x3")
-    got, status, table, _ = run_gpu(mmbev_lib, w, cuda_dev)
+    got, status, _ = run_gpu(mmbev_lib, w, cuda_dev)
     assert status == 0
     want = run_oracle(oracle_mod, w)
     assert assert_frames_equal(got, want, w.name) == 1.0
-    assert _table_is_clean(table)
 
 
 def test_batch32_parity(oracle_mod, mmbev_lib, cuda_dev):
     """The benchmark's workload and launch configuration: 32 frames, 11.1 M
     points, one call."""
     w = synth.streaming_batch(32)
-    got, status, table, _ = run_gpu(mmbev_lib, w, cuda_dev)
+    got, status, _ = run_gpu(mmbev_lib, w, cuda_dev)
     assert status == 0
     want = run_oracle(oracle_mod, w)
     assert assert_frames_equal(got, want, "batch32") == 1.0
-    assert _table_is_clean(table)
 
 
 # ------------------------------------------------------------------ cap path
@@ -118,12 +115,11 @@ def test_batch32_parity(oracle_mod, mmbev_lib, cuda_dev):
 @pytest.mark.parametrize("maxv", [1, 777, 5000, 13000])
 def test_cap_parity(oracle_mod, mmbev_lib, cuda_dev, maxv):
     w = synth.nuscenes_frame(1)
-    got, status, table, _ = run_gpu(mmbev_lib, w, cuda_dev, maxv=maxv)
+    got, status, _ = run_gpu(mmbev_lib, w, cuda_dev, maxv=maxv)
     want = run_oracle(oracle_mod, w, maxv=maxv)
     assert status == 0
     assert got[0][1].shape[0] == maxv
     assert_frames_equal(got, want, f"cap {maxv}")
-    assert _table_is_clean(table)
 
 
 def test_cap_full_coverage_and_mixed_frames(oracle_mod, mmbev_lib, cuda_dev):
@@ -134,19 +130,17 @@ def test_cap_full_coverage_and_mixed_frames(oracle_mod, mmbev_lib, cuda_dev):
         f.max_voxels = 40000
         f.max_pts_per_voxel = 10
     b = synth.concat_frames(frames, "mixed")
-    got, status, table, _ = run_gpu(mmbev_lib, b, cuda_dev)
+    got, status, _ = run_gpu(mmbev_lib, b, cuda_dev)
     want = run_oracle(oracle_mod, b)
     assert status == 0
     assert_frames_equal(got, want, "mixed")
     assert [g[1].shape[0] for g in got][0] == 40000
-    assert _table_is_clean(table)
 
 
 def test_max_voxels_zero(oracle_mod, mmbev_lib, cuda_dev):
     w = synth.tiny(0)
-    got, status, table, _ = run_gpu(mmbev_lib, w, cuda_dev, maxv=0)
+    got, status, _ = run_gpu(mmbev_lib, w, cuda_dev, maxv=0)
     assert status == 0 and got[0][1].shape[0] == 0
-    assert _table_is_clean(table)
 
 
 # ------------------------------------------------------------------ per-voxel cap K
@@ -154,11 +148,10 @@ def test_max_voxels_zero(oracle_mod, mmbev_lib, cuda_dev):
 @pytest.mark.parametrize("K", [1, 3, 12, 20, 33, 64])   # every finalize instantiation
 def test_points_per_voxel(oracle_mod, mmbev_lib, cuda_dev, K):
     w = synth.nuscenes_frame(1)
-    got, status, table, _ = run_gpu(mmbev_lib, w, cuda_dev, K=K)
+    got, status, _ = run_gpu(mmbev_lib, w, cuda_dev, K=K)
     want = run_oracle(oracle_mod, w, K=K)
     assert status == 0
     assert_frames_equal(got, want, f"K={K}")
-    assert _table_is_clean(table)
 
 
 # ------------------------------------------------------------------ edge cases
@@ -181,15 +174,14 @@ FULL = [[0.0, 0.0, 1000.0, 1000.0, 0.0]]
 
 def test_empty_input(oracle_mod, mmbev_lib, cuda_dev):
     w = _custom(np.zeros((0, 5)), [0, 0], [EYE], FULL)
-    got, status, table, _ = run_gpu(mmbev_lib, w, cuda_dev)
+    got, status, _ = run_gpu(mmbev_lib, w, cuda_dev)
     assert status == 0 and got[0][1].shape[0] == 0
 
 
 def test_no_rois(oracle_mod, mmbev_lib, cuda_dev):
     w = synth.tiny(0).with_rois(np.zeros((0, 5), np.float32))
-    got, status, table, _ = run_gpu(mmbev_lib, w, cuda_dev)
+    got, status, _ = run_gpu(mmbev_lib, w, cuda_dev)
     assert status == 0 and got[0][1].shape[0] == 0
-    assert _table_is_clean(table)
 
 
 def test_ragged_tiles_and_empty_sweeps(oracle_mod, mmbev_lib, cuda_dev):
@@ -212,7 +204,7 @@ def test_ragged_tiles_and_empty_sweeps(oracle_mod, mmbev_lib, cuda_dev):
         tfs.append(t.reshape(16))
     rois = [[0, 0, 8, 12, 0.4], [5, 5, 3, 3, 1.0], [-10, 3, 6, 2, 2.0]]
     w = _custom(pts, offs, tfs, rois, vs=(0.1, 0.1, 0.2), K=4, maxv=100000)
-    got, status, table, _ = run_gpu(mmbev_lib, w, cuda_dev)
+    got, status, _ = run_gpu(mmbev_lib, w, cuda_dev)
     assert status == 0
     assert_frames_equal(got, run_oracle(oracle_mod, w), "ragged")
     assert got[0][1].shape[0] > 100
@@ -234,7 +226,7 @@ def test_many_sweeps_per_tile(oracle_mod, mmbev_lib, cuda_dev):
         t[0, 3] = 0.01 * s
         tfs.append(t.reshape(16))
     w = _custom(pts, np.arange(S + 1) * m, tfs, FULL, vs=(0.5, 0.5, 0.5), K=3, maxv=100000)
-    got, status, table, _ = run_gpu(mmbev_lib, w, cuda_dev)
+    got, status, _ = run_gpu(mmbev_lib, w, cuda_dev)
     assert status == 0
     assert_frames_equal(got, run_oracle(oracle_mod, w), "many sweeps")
 
@@ -250,7 +242,7 @@ def test_non_finite_and_boundary_points(oracle_mod, mmbev_lib, cuda_dev):
     pts[:, 3] = np.arange(len(rows)) / 16.0
     rois = [[0.0, 0.0, 2.0, 4.0, 0.0], [51.0, 0.0, 1.0, 1.0, 0.0], [-51.0, 0, 1, 1, 0]]
     w = _custom(pts, [0, len(rows)], [EYE], rois, margin=0.5)
-    got, status, table, _ = run_gpu(mmbev_lib, w, cuda_dev)
+    got, status, _ = run_gpu(mmbev_lib, w, cuda_dev)
     want = run_oracle(oracle_mod, w)
     assert status == 0
     assert_frames_equal(got, want, "boundaries")
@@ -262,7 +254,7 @@ def test_duplicate_points_in_one_voxel(oracle_mod, mmbev_lib, cuda_dev):
     pts = np.tile(np.array([[1.05, 2.05, 0.3, 0.5, 0.0]], np.float32), (n, 1))
     pts[:, 3] = (np.arange(n) % 32) / 32.0
     w = _custom(pts, [0, n], [EYE], FULL, K=10)
-    got, status, table, _ = run_gpu(mmbev_lib, w, cuda_dev)
+    got, status, _ = run_gpu(mmbev_lib, w, cuda_dev)
     assert status == 0
     assert got[0][2].tolist() == [10]
     assert_frames_equal(got, run_oracle(oracle_mod, w), "duplicates")
@@ -283,10 +275,9 @@ def test_tiny_grid_and_many_frames(oracle_mod, mmbev_lib, cuda_dev):
         frames.append(_custom(pts, [0, n], [EYE], rois, margin=0.1, vs=(0.5, 2 / 3, 1.0),
                               rg=(-1, -1, -1, 1, 1, 1), K=2, maxv=5))
     b = synth.concat_frames(frames, "many")
-    got, status, table, _ = run_gpu(mmbev_lib, b, cuda_dev)
+    got, status, _ = run_gpu(mmbev_lib, b, cuda_dev)
     assert status == 0
     assert_frames_equal(got, run_oracle(oracle_mod, b), "many frames")
-    assert _table_is_clean(table)
 
 
 def test_max_rois_per_frame(oracle_mod, mmbev_lib, cuda_dev):
@@ -296,7 +287,7 @@ def test_max_rois_per_frame(oracle_mod, mmbev_lib, cuda_dev):
     rois = np.stack([rng.uniform(-50, 50, r), rng.uniform(-50, 50, r), rng.uniform(0.5, 3, r),
                      rng.uniform(0.5, 6, r), rng.uniform(0, 6.3, r)], 1).astype(np.float32)
     w = synth.tiny(0).with_rois(rois)
-    got, status, table, _ = run_gpu(mmbev_lib, w, cuda_dev)
+    got, status, _ = run_gpu(mmbev_lib, w, cuda_dev)
     assert status == 0
     assert_frames_equal(got, run_oracle(oracle_mod, w), "1024 rois")
     assert got[0][1].shape[0] > 500
@@ -305,22 +296,20 @@ def test_max_rois_per_frame(oracle_mod, mmbev_lib, cuda_dev):
 def test_single_frame_entry_equals_batched(oracle_mod, mmbev_lib, cuda_dev):
     w = synth.nuscenes_frame(5)
     pts, tf, rois = to_dev(w, cuda_dev)
-    table = mmbev_lib.new_table(w.num_points, w.max_pts_per_voxel, cuda_dev)
     ws = mmbev_lib.new_workspace(w.num_points, w.rois.shape[0], w.max_voxels, 1, w.voxel_size,
                                  w.pc_range, cuda_dev)
     out = mmbev_lib.voxelize_roi(pts, w.sweep_offsets, tf, rois, w.roi_margin, w.voxel_size,
-                                 w.pc_range, w.max_pts_per_voxel, w.max_voxels, table=table,
-                                 workspace=ws)
+                                 w.pc_range, w.max_pts_per_voxel, w.max_voxels, workspace=ws)
     got = [out.frame(0, w.max_voxels)]
     assert mmbev_lib.get_status(ws) == 0
     assert_frames_equal(got, run_oracle(oracle_mod, w), "single-frame entry")
 
 
-def test_repeat_calls_are_deterministic_and_leave_table_clean(mmbev_lib, cuda_dev):
+def test_repeat_calls_on_one_workspace_are_deterministic(mmbev_lib, cuda_dev):
+    # the second call finds the first call's leftovers in the workspace
     w = synth.ouster_frame(2)
-    a, s1, table, ws = run_gpu(mmbev_lib, w, cuda_dev)
-    assert _table_is_clean(table)
-    b, s2, _, _ = run_gpu(mmbev_lib, w, cuda_dev, table=table, workspace=ws)
+    a, s1, ws = run_gpu(mmbev_lib, w, cuda_dev)
+    b, s2, _ = run_gpu(mmbev_lib, w, cuda_dev, workspace=ws)
     assert s1 == 0 and s2 == 0
     for (af, ac, an), (bf, bc, bn) in zip(a, b):
         assert np.array_equal(af.view(np.uint32), bf.view(np.uint32))
@@ -332,7 +321,7 @@ def test_non_default_stream(oracle_mod, mmbev_lib, cuda_dev):
     w = synth.tiny(1)
     s = torch.cuda.Stream(cuda_dev)
     with torch.cuda.stream(s):
-        got, status, table, _ = run_gpu(mmbev_lib, w, cuda_dev, stream=s)
+        got, status, _ = run_gpu(mmbev_lib, w, cuda_dev, stream=s)
     assert status == 0
     assert_frames_equal(got, run_oracle(oracle_mod, w), "stream")
 
@@ -341,14 +330,13 @@ def test_graph_capture_replays_the_call(oracle_mod, mmbev_lib, cuda_dev):
     import torch
     w = synth.nuscenes_frame(3)
     pts, tf, rois = to_dev(w, cuda_dev)
-    table = mmbev_lib.new_table(w.num_points, w.max_pts_per_voxel, cuda_dev)
     ws = mmbev_lib.new_workspace(w.num_points, w.rois.shape[0], w.max_voxels, 1, w.voxel_size,
                                  w.pc_range, cuda_dev)
     out = mmbev_lib.Outputs.empty(1, w.max_voxels, cuda_dev)
     # one eager call first, as before any capture
     mmbev_lib.voxelize_roi_batched(pts, w.sweep_offsets, tf, rois, w.roi_margin, w.voxel_size,
                                    w.pc_range, w.max_pts_per_voxel, w.max_voxels,
-                                   w.frame_sweep_offsets, w.frame_roi_offsets, table=table,
+                                   w.frame_sweep_offsets, w.frame_roi_offsets,
                                    workspace=ws, out=out)
     torch.cuda.synchronize()
     out.feats.zero_()
@@ -361,27 +349,28 @@ def test_graph_capture_replays_the_call(oracle_mod, mmbev_lib, cuda_dev):
     with torch.cuda.graph(g, stream=s):
         mmbev_lib.voxelize_roi_batched(pts, w.sweep_offsets, tf, rois, w.roi_margin, w.voxel_size,
                                        w.pc_range, w.max_pts_per_voxel, w.max_voxels,
-                                       w.frame_sweep_offsets, w.frame_roi_offsets, table=table,
+                                       w.frame_sweep_offsets, w.frame_roi_offsets,
                                        workspace=ws, out=out)
     for _ in range(3):
         g.replay()
     torch.cuda.synchronize()
     assert mmbev_lib.get_status(ws) == 0
     assert_frames_equal([out.frame(0, w.max_voxels)], run_oracle(oracle_mod, w), "graph")
-    assert _table_is_clean(table)
 
 
 # ------------------------------------------------------------------ device-side failures
 
-def test_full_table_sets_status_and_returns(mmbev_lib, cuda_dev):
-    # 64 slots for ~14,000 voxels: inserts that find no slot set
-    # MMBEV_DEV_TABLE_FULL; the call still completes and releases every slot.
+def test_reported_status_reaches_the_caller_and_clears(oracle_mod, mmbev_lib, cuda_dev):
+    # A device-side failure is reported through the workspace's status word.
+    # The test hook sets bits there as a failing kernel would (no kernel
+    # fails): they reach mmbev_get_status, the call's results stay valid, and
+    # the next call on the same workspace starts with a clear word.
     w = synth.nuscenes_frame(1)
-    got, status, table, _ = run_gpu(mmbev_lib, w, cuda_dev, table_log2_override=6)
-    assert status & mmbev_lib.DEV_TABLE_FULL
-    assert _table_is_clean(table)
-    # the same table then serves a correct call
-    got2, status2, _, _ = run_gpu(mmbev_lib, synth.tiny(0), cuda_dev, table=table)
+    got, status, ws = run_gpu(mmbev_lib, w, cuda_dev,
+                              inject_status=mmbev_lib.DEV_WAIT_TIMEOUT | mmbev_lib.DEV_BOUNDS)
+    assert status == mmbev_lib.DEV_WAIT_TIMEOUT | mmbev_lib.DEV_BOUNDS
+    assert_frames_equal(got, run_oracle(oracle_mod, w), "hooked call")
+    _, status2, _ = run_gpu(mmbev_lib, synth.tiny(0), cuda_dev, workspace=ws)
     assert status2 == 0
 
 
@@ -389,12 +378,11 @@ def test_workspace_too_small_is_rejected(mmbev_lib, cuda_dev):
     import torch
     w = synth.tiny(0)
     pts, tf, rois = to_dev(w, cuda_dev)
-    table = mmbev_lib.new_table(w.num_points, 10, cuda_dev)
     ws = torch.empty(4096, dtype=torch.uint8, device=cuda_dev)
     with pytest.raises(mmbev_lib.MMBEVError):
         mmbev_lib.voxelize_roi_batched(pts, w.sweep_offsets, tf, rois, 0.5, w.voxel_size,
                                        w.pc_range, 10, 16000, w.frame_sweep_offsets,
-                                       w.frame_roi_offsets, table=table, workspace=ws)
+                                       w.frame_roi_offsets, workspace=ws)
 
 
 # ------------------------------------------------------------------ rho_out (Alg. 1)
@@ -404,11 +392,10 @@ def test_workspace_too_small_is_rejected(mmbev_lib, cuda_dev):
 def test_rho_out_parity(oracle_mod, mmbev_lib, cuda_dev, rho):
     # points inside no ROI kept with probability rho (SplitMix64 draws), rank R_f
     w = synth.nuscenes_frame(1)
-    got, status, table, _ = run_gpu(mmbev_lib, w, cuda_dev, rho_out=rho, seed=7)
+    got, status, _ = run_gpu(mmbev_lib, w, cuda_dev, rho_out=rho, seed=7)
     assert status == 0
     want = run_oracle(oracle_mod, w, rho_out=rho, seed=7)
     assert assert_frames_equal(got, want, f"rho={rho}") == 1.0
-    assert _table_is_clean(table)
 
 
 @pytest.mark.gpu
@@ -417,19 +404,18 @@ def test_rho_out_with_the_cap(oracle_mod, mmbev_lib, cuda_dev):
     # R_f) go first, then the rank-tie split by lin
     w = synth.nuscenes_frame(1)
     for maxv in (9000, 30000):
-        got, status, table, _ = run_gpu(mmbev_lib, w, cuda_dev, maxv=maxv, rho_out=1.0, seed=3)
+        got, status, _ = run_gpu(mmbev_lib, w, cuda_dev, maxv=maxv, rho_out=1.0, seed=3)
         assert status == 0
         want = run_oracle(oracle_mod, w, maxv=maxv, rho_out=1.0, seed=3)
         assert len(want[0][1]) == maxv
         assert assert_frames_equal(got, want, f"rho cap {maxv}") == 1.0
-        assert _table_is_clean(table)
 
 
 @pytest.mark.gpu
 def test_rho_out_batched_frames(oracle_mod, mmbev_lib, cuda_dev):
     # draws use frame-local indices: a batch equals its frames
     w = synth.concat_frames([synth.nuscenes_frame(s) for s in (1, 2, 3)], "three")
-    got, status, _, _ = run_gpu(mmbev_lib, w, cuda_dev, rho_out=0.3, seed=12345)
+    got, status, _ = run_gpu(mmbev_lib, w, cuda_dev, rho_out=0.3, seed=12345)
     assert status == 0
     want = run_oracle(oracle_mod, w, rho_out=0.3, seed=12345)
     assert assert_frames_equal(got, want, "rho batch") == 1.0
@@ -438,8 +424,8 @@ def test_rho_out_batched_frames(oracle_mod, mmbev_lib, cuda_dev):
 @pytest.mark.gpu
 def test_rho_out_seed_changes_the_draws(mmbev_lib, cuda_dev):
     w = synth.nuscenes_frame(1).with_rois(np.zeros((0, 5), np.float32))
-    a, _, _, _ = run_gpu(mmbev_lib, w, cuda_dev, rho_out=0.5, seed=1)
-    b, _, _, _ = run_gpu(mmbev_lib, w, cuda_dev, rho_out=0.5, seed=2)
+    a, _, _ = run_gpu(mmbev_lib, w, cuda_dev, rho_out=0.5, seed=1)
+    b, _, _ = run_gpu(mmbev_lib, w, cuda_dev, rho_out=0.5, seed=2)
     assert not np.array_equal(a[0][1], b[0][1])
 
 
@@ -455,7 +441,7 @@ def test_scatter_bev_parity(oracle_mod, mmbev_lib, cuda_dev, name):
         base = synth.nuscenes_frame(1)
         w = synth.concat_frames([base, synth.nuscenes_frame(2)], "two")
         w.voxel_size = np.array([0.075, 0.075, 8.0], np.float32)
-    got, status, _, _ = run_gpu(mmbev_lib, w, cuda_dev)
+    got, status, _ = run_gpu(mmbev_lib, w, cuda_dev)
     assert status == 0
     want = run_oracle(oracle_mod, w)
     assert_frames_equal(got, want, name)
@@ -799,8 +785,8 @@ def test_scatter_bev_update_equals_a_fresh_scatter(oracle_mod, mmbev_lib, cuda_d
 @pytest.mark.gpu
 def test_host_input_call_keeps_an_early_chunks_status(mmbev_lib, cuda_dev):
     """The workspace status accumulates over the chunks of a host-input call:
-    a table overflow in the first chunk is still reported after a later chunk
-    that fits."""
+    a status bit set in the first chunk (the test hook, standing in for a
+    device-side failure there) is still reported after the later chunks."""
     import torch
     w = synth.concat_frames([synth.nuscenes_frame(1), synth.tiny(2)], "big_then_small")
     rmax = int(np.max(np.diff(w.frame_roi_offsets)))
@@ -809,11 +795,10 @@ def test_host_input_call_keeps_an_early_chunks_status(mmbev_lib, cuda_dev):
     h_pts = torch.from_numpy(np.ascontiguousarray(w.points)).pin_memory()
     h_tf = torch.from_numpy(np.ascontiguousarray(w.sweep_tf)).pin_memory()
     h_rois = torch.from_numpy(np.ascontiguousarray(w.rois, np.float32).reshape(-1, 5)).pin_memory()
-    # 1024 slots: too few for the first frame's voxels, enough for the second's
     vx.run_host(h_pts, w.sweep_offsets, h_tf, h_rois, w.frame_sweep_offsets, w.frame_roi_offsets,
-                chunk_frames=1, table_log2_override=10)
+                chunk_frames=1, inject_status=mmbev_lib.DEV_BOUNDS)
     torch.cuda.synchronize(cuda_dev)
-    assert vx.status() & mmbev_lib.DEV_TABLE_FULL   # from the first chunk
+    assert vx.status() == mmbev_lib.DEV_BOUNDS   # set in the first chunk only
     # the next call starts clean: the first chunk resets the status
     vx.run_host(h_pts, w.sweep_offsets, h_tf, h_rois, w.frame_sweep_offsets, w.frame_roi_offsets,
                 chunk_frames=1)

@@ -2,8 +2,8 @@
 
 mmbev_voxelize_roi_noalloc serves callers that cannot allocate device memory
 (for example a real-time process that forbids cudaMalloc after start-up, or a
-host that lends the library only its input and output buffers): its table
-and workspace are the library's own file-scope device array. Two calls in a
+host that lends the library only its input and output buffers): its
+workspace is the library's own file-scope device array. Two calls in a
 row, on frames of different shapes, must give what mmbev_voxelize_roi gives
 with caller-owned buffers, so the second call also shows that the shared
 array's leftovers from the first do not leak into it. This file is collected
@@ -21,12 +21,10 @@ pytestmark = pytest.mark.gpu
 
 def _with_workspace(mmbev, w, dev):
     pts, tf, rois = to_dev(w, dev)
-    table = mmbev.new_table(w.num_points, w.max_pts_per_voxel, dev)
     ws = mmbev.new_workspace(w.num_points, w.rois.shape[0], w.max_voxels, 1, w.voxel_size,
                              w.pc_range, dev)
     out = mmbev.voxelize_roi(pts, w.sweep_offsets, tf, rois, w.roi_margin, w.voxel_size,
-                             w.pc_range, w.max_pts_per_voxel, w.max_voxels, table=table,
-                             workspace=ws)
+                             w.pc_range, w.max_pts_per_voxel, w.max_voxels, workspace=ws)
     torch.cuda.synchronize(dev)
     assert mmbev.get_status(ws) == 0
     return [out.frame(0, w.max_voxels)]
@@ -56,9 +54,8 @@ def test_no_alloc_matches_workspace_entry_on_two_calls(mmbev_lib, cuda_dev):
 
 def test_no_alloc_rejects_calls_beyond_its_array(mmbev_lib, cuda_dev):
     w = synth.concat_frames([synth.nuscenes_frame(s) for s in range(1, 6)], "five")
-    need = (mmbev_lib.table_size(w.num_points, 10) +
-            mmbev_lib.workspace_size(w.num_points, w.rois.shape[0], 1000, 1, w.voxel_size,
-                                     w.pc_range))
+    need = mmbev_lib.workspace_size(w.num_points, w.rois.shape[0], 1000, 1, w.voxel_size,
+                                    w.pc_range)
     assert need > 96 * 2**20           # more than the array holds
     pts, tf, rois = to_dev(w, cuda_dev)
     out = mmbev_lib.Outputs.empty(1, 1000, cuda_dev)
