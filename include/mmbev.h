@@ -227,7 +227,7 @@ int mmbev_get_status(const void *workspace, size_t workspace_bytes,
  *                     Outside [0, 1] or NaN: MMBEV_EINVAL.
  *   seed              the generator's seed.
  */
-#define MMBEV_NUM_STAGES 6
+#define MMBEV_NUM_STAGES 7
 typedef struct mmbev_exec_opts {
     cudaEvent_t *stage_events;
     uint32_t inject_status;

@@ -21,7 +21,7 @@ import torch
 _PKG = os.path.dirname(os.path.abspath(__file__))
 LIB_PATH = os.path.join(_PKG, "libmmbev.so")
 
-NUM_STAGES = 6
+NUM_STAGES = 7
 DEV_TABLE_FULL = 0x1
 DEV_WAIT_TIMEOUT = 0x2
 DEV_BOUNDS = 0x4

@@ -65,10 +65,13 @@ int coarse_for(int mask_words) {
 // Byte offsets of every workspace array for one call shape.
 struct Layout {
     size_t hdr, sweep_off, sweep_frame, fso, fro, roi_prep, masks;
-    size_t records, plist, cls_cnt, bcnt, boff, ucnt, large, small, scan_state, items, temps,
-        bcap;
+    size_t records, plist, cls_cnt, bcnt, boff, ucnt, jobs, sjobs, hjobs, hj0, hbits, pnv, mtasks,
+        scan_state,
+        items, vdesc,
+        vitems, ssum, ftot, bcap;
     size_t total;
-    uint32_t num_buckets, buckets_per_frame, num_tiles, scan_tiles;
+    uint32_t num_buckets, buckets_per_frame, num_tiles, scan_tiles, out_slices, job_cap, part_cap,
+        huge_cap, mtask_cap;
     int bucket_log2, mask_words, coarse;
 };
 
@@ -109,11 +112,27 @@ Layout make_layout(int64_t max_points, int64_t rois_total, int32_t max_rois_fram
     L.bcnt = take(sizeof(uint32_t) * B4);
     L.boff = take(sizeof(uint32_t) * (B4 + 4));
     L.ucnt = take(sizeof(uint32_t) * B4);
-    L.large = take(sizeof(uint32_t) * B4);
-    L.small = take(sizeof(uint32_t) * B4);
+    // block jobs: at most one a bucket; parts of split buckets: at most two
+    // per kPart kept points
+    L.huge_cap = (uint32_t)(TS / kPart + 1);
+    L.job_cap = (uint32_t)(B4 + 2);
+    L.part_cap = (uint32_t)(2 * (TS / kPart) + 2);
+    L.jobs = take(sizeof(uint4) * L.job_cap);
+    L.sjobs = take(sizeof(uint4) * B4);
+    L.hjobs = take(sizeof(uint4) * L.part_cap);
+    L.hj0 = take(sizeof(uint32_t) * L.huge_cap);
+    L.hbits = take(sizeof(uint32_t) * ((size_t)1 << kBucketLog2Max) / 32 * L.huge_cap);
+    L.pnv = take(sizeof(uint32_t) * L.part_cap);
+    // merge tasks: one per kMergeItems points of a split bucket, rounded up
+    L.mtask_cap = (uint32_t)(L.huge_cap + TS / kMergeItems + 1);
+    L.mtasks = take(sizeof(uint2) * L.mtask_cap);
     L.scan_state = take(sizeof(unsigned long long) * ((size_t)L.scan_tiles + 2));
     L.items = take(sizeof(uint2) * TS);
-    L.temps = take(sizeof(VoxTemp) * TS);
+    L.vdesc = take(sizeof(uint4) * TS);
+    L.vitems = take(sizeof(uint32_t) * TS);
+    L.out_slices = output_slices(L.buckets_per_frame);
+    L.ssum = take(sizeof(uint32_t) * F * L.out_slices);
+    L.ftot = take(sizeof(uint32_t) * F);
     L.bcap = take(sizeof(uint2) * B4);
     L.total = o;
     (void)max_voxels;
@@ -189,18 +208,31 @@ void bind_layout(Params* p, const Layout& L, uint8_t* ws) {
     p->masks = reinterpret_cast<uint32_t*>(ws + L.masks);
     p->records = reinterpret_cast<uint4*>(ws + L.records);
     p->plist = reinterpret_cast<uint4*>(ws + L.plist);
-    p->seg2 = reinterpret_cast<uint2*>(ws + L.plist);
+    p->pdesc = reinterpret_cast<uint4*>(ws + L.plist);
     p->cls_cnt = reinterpret_cast<uint32_t*>(ws + L.cls_cnt);
     p->num_regions = (uint32_t)((p->num_points + kTile - 1) / kTile) * (kTile / kRegion);
     p->bcnt = reinterpret_cast<uint32_t*>(ws + L.bcnt);
     p->boff = reinterpret_cast<uint32_t*>(ws + L.boff);
     p->ucnt = reinterpret_cast<uint32_t*>(ws + L.ucnt);
-    p->large = reinterpret_cast<uint32_t*>(ws + L.large);
-    p->small = reinterpret_cast<uint32_t*>(ws + L.small);
+    p->jobs = reinterpret_cast<uint4*>(ws + L.jobs);
+    p->sjobs = reinterpret_cast<uint4*>(ws + L.sjobs);
+    p->job_cap = L.job_cap;
+    p->hjobs = reinterpret_cast<uint4*>(ws + L.hjobs);
+    p->part_cap = L.part_cap;
+    p->hj0 = reinterpret_cast<uint32_t*>(ws + L.hj0);
+    p->hbits = reinterpret_cast<uint32_t*>(ws + L.hbits);
+    p->huge_cap = L.huge_cap;
+    p->pnv = reinterpret_cast<uint32_t*>(ws + L.pnv);
+    p->mtasks = reinterpret_cast<uint2*>(ws + L.mtasks);
+    p->mtask_cap = L.mtask_cap;
     p->scan_state = reinterpret_cast<unsigned long long*>(ws + L.scan_state);
     p->scan_tiles = L.scan_tiles;
     p->items = reinterpret_cast<uint2*>(ws + L.items);
-    p->temps = reinterpret_cast<VoxTemp*>(ws + L.temps);
+    p->vdesc = reinterpret_cast<uint4*>(ws + L.vdesc);
+    p->vitems = reinterpret_cast<uint32_t*>(ws + L.vitems);
+    p->ssum = reinterpret_cast<uint32_t*>(ws + L.ssum);
+    p->ftot = reinterpret_cast<uint32_t*>(ws + L.ftot);
+    p->out_slices = L.out_slices;
     p->bcap = reinterpret_cast<uint2*>(ws + L.bcap);
     p->rec_cap = p->num_regions * (uint32_t)kRegion;
     p->item_cap = p->rec_cap;
@@ -220,7 +252,7 @@ void bind_layout(Params* p, const Layout& L, uint8_t* ws) {
     } while (0)
 
 const char* const kStageNames[MMBEV_NUM_STAGES] = {
-    "prep", "classify", "scan", "scatter", "buckets", "output"};
+    "prep", "classify", "scan", "scatter", "buckets", "merge", "output"};
 
 }  // namespace
 
@@ -335,6 +367,8 @@ int voxelize_batched(const float* points, const int64_t* sweep_offsets, int32_t 
         if ((e = launch_bucket_scatter(p, sms, pdl, stream)) != cudaSuccess) break;
         if ((e = mark()) != cudaSuccess) break;
         if ((e = launch_buckets(p, sms, pdl, stream)) != cudaSuccess) break;
+        if ((e = mark()) != cudaSuccess) break;
+        if ((e = launch_merge(p, sms, pdl, stream)) != cudaSuccess) break;
         if ((e = mark()) != cudaSuccess) break;
         if ((e = launch_output(p, sms, pdl, stream)) != cudaSuccess) break;
         if ((e = mark()) != cudaSuccess) break;

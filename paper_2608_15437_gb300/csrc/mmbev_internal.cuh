@@ -23,9 +23,13 @@
 //               bucket's first item.
 //   items       workspace [M], the kept points grouped by bucket (counting
 //               sort by bucket): {position, low bits of lin | rank << 16}.
-//   temps       workspace [M], per bucket its voxels in ascending lin at
-//               boff[b] + v: {5 mean features, count, minimum rank, low lin}.
-//   ucnt        workspace [B], voxels per bucket.
+//   vdesc       workspace [M], per bucket its voxels in ascending lin at
+//               boff[b] + v: {first vitem, point count, low lin bits,
+//               minimum rank}.
+//   vitems      workspace [M], each voxel's kept record positions (its K
+//               smallest), ascending, at the voxel's first vitem.
+//   ucnt        workspace [B], voxels per bucket; ssum [F][slices] voxels
+//               per slice of 512 buckets of a frame.
 //   workspace   Header + per-call arrays (see Layout in api.cu).
 #pragma once
 
@@ -55,11 +59,13 @@ constexpr int kBucketLog2Max = 13;
 // The bucket scan works in tiles of this many buckets (1024 threads x 4).
 constexpr uint32_t kScanTile = 4096;
 
-// Bucket sizes: up to kSmallMax kept points a bucket is one warp's work, else
-// a block's; up to kSegSmem points the block keeps the bucket's point lists
-// in shared memory, beyond that in the global scratch aliased on plist.
-constexpr uint32_t kSmallMax = 64;
-constexpr uint32_t kSegSmem = 2048;
+// Bucket sizes: up to kWarpJobMax kept points a bucket is one warp's work,
+// up to kPart one block's; a larger bucket is split into parts of kPart
+// points (a block each) whose voxel lists the merge stage combines, one
+// merge task per kMergeItems points (each a range of the low lin bits).
+constexpr uint32_t kWarpJobMax = 256;
+constexpr uint32_t kPart = 2048;
+constexpr uint32_t kMergeItems = 8192;
 
 // Bounded waits.
 constexpr uint32_t kSpinLimit = 1u << 22;
@@ -95,26 +101,19 @@ struct __align__(16) RoiPrep {
     float hl, hw, pad0, pad1;
 };
 
-// One voxel of a bucket, in ascending lin: the mean features, the count of
-// points kept (min(n, K)), the minimum ROI rank over all its points and the
-// low LB bits of its linear index.
-struct __align__(16) VoxTemp {
-    float f[5];
-    uint32_t count;
-    uint32_t minrank;
-    uint32_t lo;
-};
-
 // Workspace header; zeroed by the prep kernel at the start of every call.
 struct __align__(16) Header {
     uint32_t status;        // MMBEV_DEV_* bits (first word: read by mmbev_get_status)
     uint32_t num_rec;       // kept points (records) of the call
     uint32_t scan_ticket;   // scan tiles started, in order
-    uint32_t n_large;       // buckets of more than kSmallMax points (block work)
-    uint32_t n_small;       // buckets of 1 .. kSmallMax points (warp work)
-    uint32_t large_ticket;  // large buckets taken by the bucket stage
-    uint32_t small_ticket;  // small buckets taken
-    uint32_t pad[9];
+    uint32_t n_large;       // block jobs: buckets of kWarpJobMax+1 .. kPart points
+    uint32_t n_small;       // warp jobs: buckets of 1 .. kWarpJobMax points
+    uint32_t large_ticket;  // parts, then block jobs, taken by the bucket stage
+    uint32_t n_huge;        // buckets split in parts
+    uint32_t n_parts;       // parts of the split buckets
+    uint32_t n_mtasks;      // merge tasks: ranges of low lin bits of split buckets
+    uint32_t small_ticket;  // warp jobs taken by the bucket stage
+    uint32_t pad[6];
 };
 
 // Everything a kernel needs; passed by value.
@@ -158,8 +157,8 @@ struct Params {
     RoiPrep* roi_prep;      // [R]
     uint32_t* masks;        // [F][coarse^2][mask_words]
     uint4* records;         // [regions*32][2] kept points' features and rank
-    uint4* plist;           // [tiles*2048] per classify block: {bucket, pos, lo|rank<<16, arrival}
-    uint2* seg2;            // [tiles*2048] point lists of buckets over kSegSmem (aliases plist)
+    uint4* plist;           // [tiles*2048] per classify block: {bucket, pos, lo|rank<<16, -}
+    uint4* pdesc;           // [tiles*2048] voxel lists of the parts of split buckets (aliases plist)
     uint32_t* cls_cnt;      // [kMaxClsGrid] list length of each classify block
     uint32_t cls_grid;      // classify blocks of the call
     uint32_t num_regions;
@@ -167,13 +166,26 @@ struct Params {
     uint32_t* bcnt;         // [B] kept points per bucket
     uint32_t* boff;         // [B + 1] first item of each bucket
     uint32_t* ucnt;         // [B] voxels per bucket
-    uint32_t* large;        // [B] buckets of more than kSmallMax points
-    uint32_t* small;        // [B] buckets of 1 .. kSmallMax points
+    uint4* jobs;            // [job_cap] block jobs {bucket, first item, points, ~0}
+    uint4* sjobs;           // [B] warp jobs {bucket, first item, points, -}
+    uint32_t job_cap;
+    uint4* hjobs;           // [part_cap] parts {bucket, first item, points, split index}
+    uint32_t part_cap;
+    uint32_t* hj0;          // [huge_cap] first part of each split bucket
+    uint32_t* hbits;        // [huge_cap][2^kBucketLog2Max / 32] union occupancy of each split bucket
+    uint32_t huge_cap;
+    uint32_t* pnv;          // [part_cap] voxels of each part
+    uint2* mtasks;          // [mtask_cap] merge tasks {split index, range | ranges << 16}
+    uint32_t mtask_cap;
     unsigned long long* scan_state;  // [scan_tiles] look-back words of the bucket scan
     uint2* items;           // [rec_cap] kept points grouped by bucket
-    VoxTemp* temps;         // [rec_cap] voxels grouped by bucket
+    uint4* vdesc;           // [rec_cap] voxel descriptors grouped by bucket
+    uint32_t* vitems;       // [rec_cap] kept positions of each voxel
+    uint32_t* ssum;         // [F * out_slices] voxels per frame slice
+    uint32_t* ftot;         // [F] voxels per frame
+    uint32_t out_slices;    // slices of 512 buckets per frame
     uint2* bcap;            // [B] capped frames: voxels below / at the threshold rank
-    uint32_t item_cap;      // room of items and temps (rec_cap)
+    uint32_t item_cap;      // room of items, vdesc and vitems (rec_cap)
     // outputs
     float* out_feats;
     int32_t* out_coords;
@@ -363,7 +375,9 @@ cudaError_t launch_classify_points(const Params& p, cudaStream_t st);
 cudaError_t launch_bucket_scan(const Params& p, bool pdl, cudaStream_t st);
 cudaError_t launch_bucket_scatter(const Params& p, int num_sms, bool pdl, cudaStream_t st);
 cudaError_t launch_buckets(const Params& p, int num_sms, bool pdl, cudaStream_t st);
+cudaError_t launch_merge(const Params& p, int num_sms, bool pdl, cudaStream_t st);
 cudaError_t launch_output(const Params& p, int num_sms, bool pdl, cudaStream_t st);
+uint32_t output_slices(uint32_t buckets_per_frame);   // slices of a frame for the output stage
 // Kept rows of frames [f0, f1) of a call's outputs into a packed buffer
 // (mmbev_pack_voxels' layout for F frames).
 cudaError_t launch_pack(const float* feats, const int32_t* coords, const int32_t* counts,

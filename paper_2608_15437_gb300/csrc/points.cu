@@ -23,10 +23,10 @@
 // region's kept points) gets a 32-byte record with the compensated features
 // and the ROI rank, so later stages never touch the raw points again. The
 // point is counted into its bucket of 2^LB consecutive linear indices of its
-// frame (one global atomic, whose old value numbers the point's arrival in
-// the bucket), and the block appends {bucket, position, low lin bits | rank,
-// arrival} to its own dense list (order immaterial), from which the scatter
-// stage sorts the kept points by bucket.
+// frame (one global add per group of the warp's points in a bucket), and the
+// block appends {bucket, position, low lin bits | rank} to its own dense list
+// (order immaterial), from which the scatter stage sorts the kept points by
+// bucket.
 //
 // The classify-only entry point (per-point outputs for testing S1-S2) uses a
 // plain one-thread-per-point kernel built from the same device functions.
@@ -375,20 +375,23 @@ __device__ __forceinline__ bool classify_range(const Params& p, const ClsSmem& s
         const uint32_t lo_mask = (1u << p.bucket_log2) - 1u;
 #pragma unroll
         for (int k = 0; k < 2; ++k) {
+            // the point's bucket, counted once per group of the warp's points
+            // that share it (no return value: the add does not stall the warp)
+            const uint32_t bk =
+                valid[k] ? frk[k] * p.buckets_per_frame + (lin[k] >> p.bucket_log2) : kUnset;
+            const uint32_t grp = __match_any_sync(0xFFFFFFFFu, bk);
+            if (valid[k] && lane == __ffs(grp) - 1) atomicAdd(&p.bcnt[bk], (uint32_t)__popc(grp));
             if (valid[k]) {
                 const uint32_t rk = rank0 + (k ? (uint32_t)valid[0] : 0u);
                 const uint32_t at = region * (uint32_t)kRegion + rk;
                 const uint32_t li = lbase + (k ? __popc(b0) + __popc(b1 & lt) : __popc(b0 & lt));
-                // the point's bucket: its count and the point's arrival in it
-                const uint32_t bk = frk[k] * p.buckets_per_frame + (lin[k] >> p.bucket_log2);
-                const uint32_t arr = atomicAdd(&p.bcnt[bk], 1u);
                 // records are read again only by the bucket stage: streaming
                 // stores leave L2 to the lists and counters in between
                 uint4* rec = p.records + 2 * (size_t)at;
                 __stcs(rec, make_uint4(__float_as_uint(x[k]), __float_as_uint(y[k]),
                                        __float_as_uint(z[k]), __float_as_uint(pi[k])));
                 __stcs(rec + 1, make_uint4(__float_as_uint(pd[k]), (uint32_t)hit[k], 0u, 0u));
-                plist[li] = make_uint4(bk, at, (lin[k] & lo_mask) | ((uint32_t)hit[k] << 16), arr);
+                plist[li] = make_uint4(bk, at, (lin[k] & lo_mask) | ((uint32_t)hit[k] << 16), 0u);
             }
         }
         c = __shfl_sync(0xFFFFFFFFu, cn, 0);

@@ -116,6 +116,10 @@ k_prep(Params p, const __grid_constant__ HostDesc d) {
         for (size_t i = gt; i < (size_t)kMaxClsGrid; i += gs) p.cls_cnt[i] = 0u;
     if (p.scan_state)
         for (size_t i = gt; i < (size_t)p.scan_tiles; i += gs) p.scan_state[i] = 0ull;
+    if (p.ssum)
+        for (size_t i = gt; i < (size_t)p.num_frames * p.out_slices; i += gs) p.ssum[i] = 0u;
+    if (p.ftot)
+        for (size_t i = gt; i < (size_t)p.num_frames; i += gs) p.ftot[i] = 0u;
     if (p.bcnt) {
         uint4* b4 = reinterpret_cast<uint4*>(p.bcnt);  // B counters, padded to a multiple of 4
         const size_t n4 = ((size_t)p.num_buckets + 3) / 4;
