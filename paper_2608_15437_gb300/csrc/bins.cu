@@ -105,6 +105,39 @@ __device__ __forceinline__ void sorted_insert(uint32_t (&b)[B], uint32_t v) {
     }
 }
 
+// Ascending order of a[0..B) (unused entries ~0u, which end last): an
+// odd-even transposition network for small B, a bitonic network for the
+// larger (power-of-two) ones.
+template <int B>
+__device__ __forceinline__ void sort_small(uint32_t (&a)[B]) {
+    if constexpr (B <= 16) {
+#pragma unroll
+        for (int r = 0; r < B; ++r)
+#pragma unroll
+            for (int j = r & 1; j + 1 < B; j += 2) {
+                const uint32_t lo = min(a[j], a[j + 1]), hi = max(a[j], a[j + 1]);
+                a[j] = lo;
+                a[j + 1] = hi;
+            }
+    } else {
+        static_assert((B & (B - 1)) == 0, "bitonic network: a power of two");
+#pragma unroll
+        for (int k = 2; k <= B; k <<= 1)
+#pragma unroll
+            for (int j = k >> 1; j > 0; j >>= 1)
+#pragma unroll
+                for (int i = 0; i < B; ++i) {
+                    const int l = i ^ j;
+                    if (l > i) {
+                        const uint32_t lo = min(a[i], a[l]), hi = max(a[i], a[l]);
+                        const bool up = (i & k) == 0;
+                        a[i] = up ? lo : hi;
+                        a[l] = up ? hi : lo;
+                    }
+                }
+    }
+}
+
 // Voxel of low lin bits `lo` in a bucket: its rank among the bucket's
 // distinct low bits, from the occupancy bitmap and its word prefixes.
 __device__ __forceinline__ uint32_t voxel_of(const uint32_t* bm, const uint32_t* wpre, uint32_t lo) {
@@ -136,33 +169,37 @@ struct KeptOut {
     uint32_t at;
 };
 
-// One voxel by one thread: entries seg[st, st+cnt) {position, lo | rank <<
-// 16} (any order; cnt <= B, or only the B smallest positions are kept). Its
-// K smallest positions go out in ascending order, its descriptor to *desc.
-template <int B>
-__device__ __forceinline__ void select_by_thread(const Params& p, const uint2* seg, uint32_t st,
-                                                 uint32_t cnt, const KeptOut& ko, uint4* desc) {
-    uint32_t best[B];
-#pragma unroll
-    for (int j = 0; j < B; ++j) best[j] = kUnset;
-    uint32_t mr = kUnset;
-    const uint32_t lo = seg[st].y & 0xFFFFu;
-    for (uint32_t i0 = 0; i0 < cnt; i0 += 4) {   // four entries in flight
-        uint2 e[4];
-#pragma unroll
-        for (int c = 0; c < 4; ++c)
-            e[c] = i0 + c < cnt ? seg[st + i0 + c] : make_uint2(kUnset, kUnset);
-#pragma unroll
-        for (int c = 0; c < 4; ++c) {
-            sorted_insert<B>(best, e[c].x);
-            mr = min(mr, e[c].y >> 16);
-        }
+// Voxels of at most 32 points, a thread per point (entry i of a job's
+// voxel-sorted entries). A voxel of at most K points keeps all its points:
+// each goes to the voxel's kept list at its place in the voxel's run, in no
+// particular order (the output stage sorts a voxel's kept positions before
+// summing). In a denser one a point's rank by position among the voxel's
+// points is where it goes, if below K. The voxel's first entry also writes
+// the descriptor (count, low bits, minimum rank). Denser voxels are selected
+// by a warp or by the block.
+template <typename KO>
+__device__ __forceinline__ void select_small(const Params& p, const uint2* seg, uint32_t i,
+                                             const uint32_t* bm, const uint32_t* wpre,
+                                             const uint32_t* vc, const KO& kept_out,
+                                             uint4* desc) {
+    const uint2 me = seg[i];
+    const uint32_t lo = me.y & 0xFFFFu;
+    const uint32_t v = voxel_of(bm, wpre, lo);
+    const uint32_t st = v ? vc[v - 1] : 0u, cnt = vc[v] - st;
+    if (cnt > 32u) return;
+    const uint32_t K = (uint32_t)p.K;
+    uint32_t r = i - st;
+    if (cnt > K) {
+        r = 0;
+        for (uint32_t j = st; j < st + cnt; ++j) r += seg[j].x < me.x ? 1u : 0u;
     }
-    const uint32_t kept = min(cnt, (uint32_t)p.K);
-#pragma unroll
-    for (int j = 0; j < B; ++j)
-        if ((uint32_t)j < kept) ko.out[j * ko.stride] = best[j];
-    *desc = make_uint4(ko.at, cnt, lo, mr);
+    const KeptOut ko = kept_out(st);
+    if (r < K) ko.out[r * ko.stride] = me.x;
+    if (i == st) {
+        uint32_t mr = kUnset;
+        for (uint32_t j = st; j < st + cnt; ++j) mr = min(mr, seg[j].y >> 16);
+        desc[v] = make_uint4(ko.at, cnt, lo, mr);
+    }
 }
 
 // One voxel by a whole warp (any count): each lane keeps the B smallest
@@ -687,19 +724,18 @@ __device__ void bucket_by_block(const Params& p, const uint4& job, uint32_t jidx
     };
     for (uint32_t v = t; v < nv; v += kBT) {
         const uint32_t st = v ? vc[v - 1] : 0u, cnt = vc[v] - st;
-        if (cnt <= 32) {
-            select_by_thread<BL>(p, seg, st, cnt, kept_out(st), desc + v);
-        } else if (cnt > kWarpMax) {
+        if (cnt > kWarpMax) {
             const uint32_t k = atomicAdd(&s_huge[kHugeList], 1u);
             if (k < kHugeList) s_huge[k] = v;
         }
     }
+    for (uint32_t i = t; i < n; i += kBT) select_small(p, seg, i, bm, wpre, vc, kept_out, desc);
     __syncthreads();
     const uint32_t nh = s_huge[kHugeList];
     for (uint32_t v = warp; v < nv; v += kBT / 32) {
         const uint32_t st = v ? vc[v - 1] : 0u, cnt = vc[v] - st;
         // heavy voxels, and huge ones beyond the list's room
-        if (cnt > 32 && (cnt <= kWarpMax || nh > kHugeList))
+        if (cnt > 32u && (cnt <= kWarpMax || nh > kHugeList))
             select_by_warp<BH>(p, seg, st, cnt, kept_out(st), desc + v);
     }
     if (nh <= kHugeList) {
@@ -849,14 +885,11 @@ __device__ void bucket_by_warp(const Params& p, const uint4& job, unsigned char*
     }
     __syncwarp();
     uint4* desc = p.vdesc + s;
-    for (uint32_t vv = lane; vv < nv; vv += 32) {
-        const uint32_t st = vv ? vc[vv - 1] : 0u, cnt = vc[vv] - st;
-        if (cnt <= 32)
-            select_by_thread<BL>(p, seg, st, cnt, KeptOut{p.vitems + s + st, 1u, s + st}, desc + vv);
-    }
+    auto kept_out = [&](uint32_t st) { return KeptOut{p.vitems + s + st, 1u, s + st}; };
+    for (uint32_t i = lane; i < n; i += 32) select_small(p, seg, i, bm, wpre, vc, kept_out, desc);
     for (uint32_t vv = 0; vv < nv; ++vv) {   // warp-uniform
         const uint32_t st = vv ? vc[vv - 1] : 0u, cnt = vc[vv] - st;
-        if (cnt > 32)
+        if (cnt > 32u)
             select_by_warp<BH>(p, seg, st, cnt, KeptOut{p.vitems + s + st, 1u, s + st}, desc + vv);
     }
     if (lane == 0) publish_bucket(p, b, nv);
@@ -1061,7 +1094,7 @@ __global__ void __launch_bounds__(merge_threads<B>(), 1) k_merge(Params p) {
                 __syncthreads();   // s_ppre of the next group
             }
         };
-        // the kept positions of entry d that are candidates (ascending), eight
+        // the kept positions of entry d (its candidates, in any order), eight
         // loads in flight: g(j, position); stops early when g returns false
         auto for_candidates = [&](const uint4& d, auto&& g) {
             const uint32_t kq = min(d.y, K);
@@ -1139,7 +1172,10 @@ __global__ void __launch_bounds__(merge_threads<B>(), 1) k_merge(Params p) {
                 __syncthreads();
                 for_entries([&](const uint4& d, uint32_t v) {
                     if (v != w0) return;
-                    for_candidates(d, [&](uint32_t, uint32_t c) { return kmin_insert(cand, K, c); });
+                    for_candidates(d, [&](uint32_t, uint32_t c) {
+                        kmin_insert(cand, K, c);
+                        return true;
+                    });
                 });
                 const uint32_t kept = min(vcount[w0], K);
                 for (uint32_t j = t; j < kept; j += MT) p.vitems[s + kof[w0] + j] = cand[j];
@@ -1257,7 +1293,8 @@ __device__ __forceinline__ void finalize_voxel(const Params& p, uint32_t f, uint
     }
     uint32_t pos[B];
 #pragma unroll
-    for (int j = 0; j < B; ++j) pos[j] = (uint32_t)j < kept ? p.vitems[d.x + j] : 0u;
+    for (int j = 0; j < B; ++j) pos[j] = (uint32_t)j < kept ? p.vitems[d.x + j] : kUnset;
+    sort_small<B>(pos);   // kept positions come in any order; the sum goes by index
     constexpr int R = B < 4 ? B : 4;   // record loads in flight
     float acc[5] = {0.f, 0.f, 0.f, 0.f, 0.f};
 #pragma unroll
