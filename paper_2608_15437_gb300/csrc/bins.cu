@@ -138,6 +138,12 @@ __device__ __forceinline__ void sort_small(uint32_t (&a)[B]) {
     }
 }
 
+// Low lin bits of an item's second word, masked to the bucket's size: an
+// index into a bucket bitmap whatever the word holds.
+__device__ __forceinline__ uint32_t item_lo(const Params& p, uint32_t y) {
+    return y & ((1u << p.bucket_log2) - 1u);
+}
+
 // Voxel of low lin bits `lo` in a bucket: its rank among the bucket's
 // distinct low bits, from the occupancy bitmap and its word prefixes.
 __device__ __forceinline__ uint32_t voxel_of(const uint32_t* bm, const uint32_t* wpre, uint32_t lo) {
@@ -183,7 +189,7 @@ __device__ __forceinline__ void select_small(const Params& p, const uint2* seg, 
                                              const uint32_t* vc, const KO& kept_out,
                                              uint4* desc) {
     const uint2 me = seg[i];
-    const uint32_t lo = me.y & 0xFFFFu;
+    const uint32_t lo = item_lo(p, me.y);
     const uint32_t v = voxel_of(bm, wpre, lo);
     const uint32_t st = v ? vc[v - 1] : 0u, cnt = vc[v] - st;
     if (cnt > 32u) return;
@@ -227,7 +233,7 @@ __device__ __forceinline__ void select_by_warp(const Params& p, const uint2* seg
         }
     }
     mr = __reduce_min_sync(kFull, mr);
-    const uint32_t lo = seg[st].y & 0xFFFFu;
+    const uint32_t lo = item_lo(p, seg[st].y);
     const uint32_t kept = min(cnt, (uint32_t)p.K);
     for (uint32_t j = 0; j < kept; ++j) {
         const uint32_t m = __reduce_min_sync(kFull, best[0]);
@@ -304,7 +310,7 @@ __device__ __forceinline__ void select_by_block(const Params& p, const uint2* se
                 best[B - 1] = kUnset;
             }
         }
-        if (lane == 0) *desc = make_uint4(ko.at, cnt, seg[st].y & 0xFFFFu, s_mr);
+        if (lane == 0) *desc = make_uint4(ko.at, cnt, item_lo(p, seg[st].y), s_mr);
     }
     __syncthreads();
 }
@@ -348,24 +354,6 @@ static_assert(kScanTile == kScanThreads * 4, "four buckets a thread");
 constexpr unsigned long long kAggFlag = 1ull << 32;    // tile total published
 constexpr unsigned long long kIncFlag = 2ull << 32;    // tile inclusive prefix published
 
-// Append the job `d` of each lane with `take` to list `dst` of length counter
-// `cnt` with one atomic per warp.
-__device__ __forceinline__ void warp_append(bool take, const uint4& d, uint32_t* cnt, uint4* dst,
-                                            uint32_t cap, Header* hdr) {
-    const int lane = threadIdx.x & 31;
-    const uint32_t m = __ballot_sync(kFull, take);
-    if (!m) return;
-    const int leader = __ffs(m) - 1;
-    uint32_t base = 0;
-    if (lane == leader) base = atomicAdd(cnt, (uint32_t)__popc(m));
-    base = __shfl_sync(kFull, base, leader);
-    if (take) {
-        const uint32_t at = base + __popc(m & ((1u << lane) - 1u));
-        if (at < cap) dst[at] = d;
-        else set_status(hdr, MMBEV_DEV_BOUNDS);
-    }
-}
-
 // Stage 2. The tile's inclusive prefix comes from its predecessors by
 // decoupled look-back, done by warp 0 over 32 predecessors at a time: each
 // lane waits (bounded) until its predecessor has published at least its
@@ -376,7 +364,7 @@ __device__ __forceinline__ void warp_append(bool take, const uint4& d, uint32_t*
 // last part to finish merges.
 __global__ void __launch_bounds__(kScanThreads) k_bucket_scan(Params p) {
     __shared__ uint32_t s_warp[kScanThreads / 32];
-    __shared__ uint32_t s_tile, s_base;
+    __shared__ uint32_t s_tile, s_base, s_jbase[2];
     pdl_wait();
     const int t = threadIdx.x, lane = t & 31;
     // tiles are numbered in the order their blocks start, so a tile only
@@ -434,6 +422,23 @@ __global__ void __launch_bounds__(kScanThreads) k_bucket_scan(Params p) {
         if (lane == 0) s_base = base;
     }
     __syncthreads();
+    // the tile's warp jobs and block jobs: one reservation a list for the
+    // whole tile (counts packed small | large << 16; a tile has 4,096 buckets)
+    uint32_t jc = 0;
+#pragma unroll
+    for (int k = 0; k < 4; ++k) {
+        const bool ok = b0 + k < B;
+        jc += ok && c[k] > 0u && c[k] <= kWarpJobMax ? 1u : 0u;
+        jc += ok && c[k] > kWarpJobMax && c[k] <= kPart ? 1u << 16 : 0u;
+    }
+    uint32_t jtot = 0;
+    uint32_t jex = block_exclusive_scan(jc, s_warp, &jtot);
+    if (t == 0) {
+        s_jbase[0] = jtot & 0xFFFFu ? atomicAdd(&p.hdr->n_small, jtot & 0xFFFFu) : 0u;
+        s_jbase[1] = jtot >> 16 ? atomicAdd(&p.hdr->n_large, jtot >> 16) : 0u;
+    }
+    __syncthreads();
+    uint32_t js = s_jbase[0] + (jex & 0xFFFFu), jl = s_jbase[1] + (jex >> 16);
     uint32_t run = s_base + excl;
 #pragma unroll
     for (int k = 0; k < 4; ++k) {
@@ -444,10 +449,16 @@ __global__ void __launch_bounds__(kScanThreads) k_bucket_scan(Params p) {
             if (b == B - 1u) p.boff[B] = run + c[k];
         }
         const uint4 d = make_uint4(b, run, c[k], kUnset);
-        warp_append(b < B && c[k] > kWarpJobMax && c[k] <= kPart, d, &p.hdr->n_large, p.jobs,
-                    p.job_cap, p.hdr);
-        warp_append(b < B && c[k] > 0u && c[k] <= kWarpJobMax, d, &p.hdr->n_small, p.sjobs, B,
-                    p.hdr);
+        if (b < B && c[k] > 0u && c[k] <= kWarpJobMax) {
+            if (js < B) p.sjobs[js] = d;
+            else set_status(p.hdr, MMBEV_DEV_BOUNDS);
+            ++js;
+        }
+        if (b < B && c[k] > kWarpJobMax && c[k] <= kPart) {
+            if (jl < p.job_cap) p.jobs[jl] = d;
+            else set_status(p.hdr, MMBEV_DEV_BOUNDS);
+            ++jl;
+        }
         if (b < B && c[k] > kPart) {   // parts of a bucket too large for one block
             const uint32_t P = (c[k] + kPart - 1) / kPart;
             const uint32_t h = atomicAdd(&p.hdr->n_huge, 1u);
@@ -479,10 +490,13 @@ __global__ void __launch_bounds__(kScanThreads) k_bucket_scan(Params p) {
 
 constexpr int kThreads = 256;
 
-// Prefix sums of the classify blocks' list lengths (off[0..G]) and the
-// first plist entry of each list (list l starts at tile t_begin(l) * 2048).
+// Prefix sums of the classify blocks' list lengths (off[0..G]) and of their
+// units of kUnit entries (uoff[0..G]), and the first plist entry of each list
+// (list l starts at tile t_begin(l) * 2048).
+constexpr uint32_t kUnit = 256;   // entries a warp takes at once (8 per lane)
 struct Lists {
     uint32_t off[kMaxClsGrid + 1];
+    uint32_t uoff[kMaxClsGrid + 1];
     uint32_t start[kMaxClsGrid];
 };
 
@@ -504,65 +518,78 @@ __device__ __forceinline__ uint32_t lists_scan(const Params& p, Lists& L, uint32
         }
         sum += c[k];
     }
-    uint32_t total = 0;
+    uint32_t usum = 0;
+#pragma unroll
+    for (int k = 0; k < 4; ++k) usum += (c[k] + kUnit - 1) / kUnit;
+    uint32_t total = 0, utotal = 0;
     uint32_t run = block_exclusive_scan(sum, s_warp, &total);
+    uint32_t urun = block_exclusive_scan(usum, s_warp, &utotal);
 #pragma unroll
     for (int k = 0; k < 4; ++k) {
         const uint32_t l = (uint32_t)threadIdx.x * 4 + k;
-        if (l <= G) L.off[l] = run;
+        if (l <= G) {
+            L.off[l] = run;
+            L.uoff[l] = urun;
+        }
         run += c[k];
+        urun += (c[k] + kUnit - 1) / kUnit;
     }
     __syncthreads();
-    return L.off[G];
+    return L.uoff[G];
 }
 
-// plist index of the i-th entry of the concatenated lists.
-__device__ __forceinline__ size_t list_entry(const Params& p, const Lists& L, uint32_t i) {
-    uint32_t lo = 0, hi = p.cls_grid;  // L.off[lo] <= i < L.off[hi]
-    while (hi - lo > 1) {
-        const uint32_t mid = (lo + hi) >> 1;
-        if (L.off[mid] <= i) lo = mid; else hi = mid;
-    }
-    return (size_t)L.start[lo] + (i - L.off[lo]);
-}
-
-// Each warp takes U batches of 32 consecutive entries. Entries of one bucket
-// in a batch (neighbours in a classify block's list often share one) take
-// their places with one atomic on the bucket's cursor (ucnt, zero after the
-// scan stage; it ends at the bucket's count).
+// Each warp takes units of kUnit consecutive entries of one classify block's
+// list (eight groups of 32). The entries of one bucket in a group take their
+// places with one atomic on the bucket's cursor (ucnt, zero after the scan
+// stage; it ends at the bucket's count).
 __global__ void __launch_bounds__(kThreads) k_bucket_scatter(Params p) {
     __shared__ Lists L;
     __shared__ uint32_t s_warp[kThreads / 32];
     pdl_wait();
-    const uint32_t M = lists_scan(p, L, s_warp);
+    const uint32_t NU = lists_scan(p, L, s_warp);
+    const uint32_t G = p.cls_grid;
     const int lane = threadIdx.x & 31;
     const uint32_t lt = (1u << lane) - 1u;
     const uint32_t gw = (blockIdx.x * blockDim.x + threadIdx.x) >> 5;
     const uint32_t nw = (gridDim.x * blockDim.x) >> 5;
-    constexpr int U = 4;
-    for (uint32_t base = gw * 32u * U; base < M; base += nw * 32u * U) {   // warp-uniform
+    constexpr int U = kUnit / 32;
+    for (uint32_t unit = gw; unit < NU; unit += nw) {   // warp-uniform
+        uint32_t l = 0, hi = G;   // its list: uoff[l] <= unit < uoff[l + 1]
+        while (hi - l > 1) {
+            const uint32_t mid = (l + hi) >> 1;
+            if (L.uoff[mid] <= unit) l = mid; else hi = mid;
+        }
+        const uint32_t k0 = (unit - L.uoff[l]) * kUnit, cnt = L.off[l + 1] - L.off[l];
+        const uint4* src = p.plist + L.start[l];
         uint4 e[U];
 #pragma unroll
         for (int u = 0; u < U; ++u) {
-            const uint32_t i = base + (uint32_t)u * 32u + (uint32_t)lane;
-            e[u] = i < M ? __ldcs(p.plist + list_entry(p, L, i)) : make_uint4(kUnset, 0u, 0u, 0u);
+            const uint32_t j = k0 + (uint32_t)u * 32u + (uint32_t)lane;
+            e[u] = j < cnt ? __ldcs(src + j) : make_uint4(kUnset, 0u, 0u, 0u);
             if (e[u].x >= p.num_buckets) e[u].x = kUnset;
         }
-        uint32_t old[U], rk[U];
+        // The entries of one bucket in a group of 32 take their arrival
+        // numbers with one atomic by the group's first lane. Every number and
+        // bucket offset is requested before any is used, so that their
+        // latencies overlap.
+        uint32_t bo[U], grp[U], old[U];
+#pragma unroll
+        for (int u = 0; u < U; ++u) bo[u] = e[u].x != kUnset ? __ldg(p.boff + e[u].x) : 0u;
+#pragma unroll
+        for (int u = 0; u < U; ++u) grp[u] = __match_any_sync(kFull, e[u].x);
 #pragma unroll
         for (int u = 0; u < U; ++u) {
-            const uint32_t grp = __match_any_sync(kFull, e[u].x);
-            const int leader = __ffs(grp) - 1;
             old[u] = 0u;
-            if (e[u].x != kUnset && lane == leader)
-                old[u] = atomicAdd(&p.ucnt[e[u].x], (uint32_t)__popc(grp));
-            rk[u] = __popc(grp & lt);
-            old[u] = __shfl_sync(kFull, old[u], leader);
+            if (e[u].x != kUnset && lane == __ffs(grp[u]) - 1)
+                old[u] = atomicAdd(&p.ucnt[e[u].x], (uint32_t)__popc(grp[u]));
         }
+#pragma unroll
+        for (int u = 0; u < U; ++u)
+            old[u] = __shfl_sync(kFull, old[u], __ffs(grp[u]) - 1) + __popc(grp[u] & lt);
 #pragma unroll
         for (int u = 0; u < U; ++u) {
             if (e[u].x == kUnset) continue;
-            const uint32_t at = __ldg(p.boff + e[u].x) + old[u] + rk[u];
+            const uint32_t at = bo[u] + old[u];
             if (at < p.item_cap) p.items[at] = make_uint2(e[u].y, e[u].z);
             else set_status(p.hdr, MMBEV_DEV_BOUNDS);
         }
@@ -629,7 +656,7 @@ __device__ void bucket_by_block(const Params& p, const uint4& job, uint32_t jidx
         }
 #pragma unroll
         for (uint32_t c = 0; c < kIl; ++c) {
-            const uint32_t lo = e[c].x != kUnset ? e[c].y & 0xFFFFu : kUnset;
+            const uint32_t lo = e[c].x != kUnset ? item_lo(p, e[c].y) : kUnset;
             const uint32_t grp = __match_any_sync(kFull, lo);
             if (lo != kUnset && lane == __ffs(grp) - 1) atomicOr(&bm[lo >> 5], 1u << (lo & 31));
         }
@@ -665,7 +692,7 @@ __device__ void bucket_by_block(const Params& p, const uint4& job, uint32_t jidx
         }
 #pragma unroll
         for (uint32_t c = 0; c < kIl; ++c) {
-            const uint32_t v = e[c].x != kUnset ? voxel_of(bm, wpre, e[c].y & 0xFFFFu) : kUnset;
+            const uint32_t v = e[c].x != kUnset ? voxel_of(bm, wpre, item_lo(p, e[c].y)) : kUnset;
             const uint32_t grp = __match_any_sync(kFull, v);
             if (v != kUnset && lane == __ffs(grp) - 1) atomicAdd(&vc[v], (uint32_t)__popc(grp));
         }
@@ -699,7 +726,7 @@ __device__ void bucket_by_block(const Params& p, const uint4& job, uint32_t jidx
         }
 #pragma unroll
         for (uint32_t c = 0; c < kIl; ++c) {
-            const uint32_t v = e[c].x != kUnset ? voxel_of(bm, wpre, e[c].y & 0xFFFFu) : kUnset;
+            const uint32_t v = e[c].x != kUnset ? voxel_of(bm, wpre, item_lo(p, e[c].y)) : kUnset;
             const uint32_t grp = __match_any_sync(kFull, v);
             const int leader = __ffs(grp) - 1;
             uint32_t base = 0;
@@ -769,7 +796,7 @@ __device__ void bucket_tiny(const Params& p, const uint4& job) {
     }
     const bool act = (uint32_t)lane < n;
     const uint2 e = act ? p.items[s + lane] : make_uint2(kUnset, kUnset);
-    const uint32_t lo = act ? (e.y & 0xFFFFu) : kUnset;
+    const uint32_t lo = act ? item_lo(p, e.y) : kUnset;
     const uint32_t rk = e.y >> 16;
     const uint32_t grp = __match_any_sync(kFull, lo);
     const uint32_t K = (uint32_t)p.K;
@@ -830,7 +857,7 @@ __device__ void bucket_by_warp(const Params& p, const uint4& job, unsigned char*
     __syncwarp();
 #pragma unroll
     for (uint32_t c = 0; c < kPer; ++c)
-        if (e[c].x != kUnset) atomicOr(&bm[(e[c].y & 0xFFFFu) >> 5], 1u << (e[c].y & 31));
+        if (e[c].x != kUnset) atomicOr(&bm[item_lo(p, e[c].y) >> 5], 1u << (e[c].y & 31));
     __syncwarp();
     uint32_t pc = 0;
     for (uint32_t k = 0; k < wpl; ++k) {
@@ -852,7 +879,7 @@ __device__ void bucket_by_warp(const Params& p, const uint4& job, unsigned char*
     uint32_t v[kPer];
 #pragma unroll
     for (uint32_t c = 0; c < kPer; ++c) {
-        v[c] = e[c].x != kUnset ? voxel_of(bm, wpre, e[c].y & 0xFFFFu) : kUnset;
+        v[c] = e[c].x != kUnset ? voxel_of(bm, wpre, item_lo(p, e[c].y)) : kUnset;
         const uint32_t grp = __match_any_sync(kFull, v[c]);
         if (v[c] != kUnset && lane == __ffs(grp) - 1) atomicAdd(&vc[v[c]], (uint32_t)__popc(grp));
     }
@@ -1178,7 +1205,11 @@ __global__ void __launch_bounds__(merge_threads<B>(), 1) k_merge(Params p) {
                     });
                 });
                 const uint32_t kept = min(vcount[w0], K);
-                for (uint32_t j = t; j < kept; j += MT) p.vitems[s + kof[w0] + j] = cand[j];
+                if (kof[w0] + kept <= n) {
+                    for (uint32_t j = t; j < kept; j += MT) p.vitems[s + kof[w0] + j] = cand[j];
+                } else if (t == 0) {
+                    set_status(p.hdr, MMBEV_DEV_BOUNDS);
+                }
                 if (t == 0) {
                     put_desc(w0);
                     vcc[w0] = next;   // as if gathered
@@ -1206,7 +1237,8 @@ __global__ void __launch_bounds__(merge_threads<B>(), 1) k_merge(Params p) {
 #pragma unroll
                     for (int j = 0; j < TB; ++j) best[j] = kUnset;
                     for (uint32_t i = st; i < en; ++i) sorted_insert<TB>(best, cand[i]);
-                    const uint32_t kept = min(vcount[v], K);
+                    const uint32_t kept = kof[v] + min(vcount[v], K) <= n ? min(vcount[v], K) : 0u;
+                    if (kept < min(vcount[v], K)) set_status(p.hdr, MMBEV_DEV_BOUNDS);
 #pragma unroll
                     for (int j = 0; j < TB; ++j)
                         if ((uint32_t)j < kept) p.vitems[s + kof[v] + j] = best[j];
@@ -1220,7 +1252,8 @@ __global__ void __launch_bounds__(merge_threads<B>(), 1) k_merge(Params p) {
 #pragma unroll
                     for (int j = 0; j < B; ++j) best[j] = kUnset;
                     for (uint32_t i = st + lane; i < en; i += 32) sorted_insert<B>(best, cand[i]);
-                    const uint32_t kept = min(vcount[v], K);
+                    const uint32_t kept = kof[v] + min(vcount[v], K) <= n ? min(vcount[v], K) : 0u;
+                    if (lane == 0 && kept < min(vcount[v], K)) set_status(p.hdr, MMBEV_DEV_BOUNDS);
                     for (uint32_t j = 0; j < kept; ++j) {
                         const uint32_t m = __reduce_min_sync(kFull, best[0]);
                         if (best[0] == m) {   // positions are distinct: one lane owns m
