@@ -1010,6 +1010,7 @@ __global__ void __launch_bounds__(kBT, (BH <= 12 ? 8 : 2)) k_buckets(Params p) {
 // for the kept offsets, and gathers and selects only its own.
 constexpr uint32_t kMergeGroup = 1024;            // parts whose entry prefix is held at once
 constexpr size_t kMergeSmem = 200 * 1024;         // dynamic shared memory of a merge block
+constexpr uint32_t kStash = 2048;                 // entries a task keeps for its gather
 
 template <int B>
 __host__ __device__ constexpr int merge_threads() { return B <= 12 ? 1024 : B <= 32 ? 512 : 256; }
@@ -1021,7 +1022,7 @@ __global__ void __launch_bounds__(merge_threads<B>(), 1) k_merge(Params p) {
     extern __shared__ __align__(16) uint32_t msm[];
     __shared__ uint32_t s_warp[MT / 32];
     __shared__ uint32_t s_ppre[kMergeGroup + 1];
-    __shared__ uint32_t s_x;
+    __shared__ uint32_t s_x, s_nst;
     pdl_wait();
     const int t = threadIdx.x, lane = t & 31, warp = t >> 5;
     const uint32_t nh = min(p.hdr->n_huge, p.huge_cap);
@@ -1064,8 +1065,11 @@ __global__ void __launch_bounds__(merge_threads<B>(), 1) k_merge(Params p) {
         uint32_t* vmr = vcount + nv;     // minimum rank
         uint32_t* vcc = vmr + nv;        // candidates, then their offsets, then cursors
         uint32_t* kof = vcc + nv;        // kept offsets
-        uint32_t* cand = kof + nv;
-        const uint32_t cap = (uint32_t)(kMergeSmem / 4) - 2u * kBmWords - 4u * nv;
+        const uint32_t sto = (2u * kBmWords + 4u * nv + 3u) & ~3u;   // the stash, 16-byte aligned
+        uint4* stash = reinterpret_cast<uint4*>(msm + sto);          // the task's own entries
+        uint32_t* cand = msm + sto + 4u * kStash;
+        const uint32_t cap = (uint32_t)(kMergeSmem / 4) - sto - 4u * kStash;
+        if (t == 0) s_nst = 0u;
         for (uint32_t v = t; v < nv; v += MT) {
             vcount[v] = 0u;
             vmr[v] = kUnset;
@@ -1098,7 +1102,7 @@ __global__ void __launch_bounds__(merge_threads<B>(), 1) k_merge(Params p) {
             for (uint32_t g0 = 0; g0 < P; g0 += kMergeGroup) {   // block-uniform
                 const uint32_t g1 = min(P, g0 + kMergeGroup), ng = g1 - g0;
                 const uint32_t ne = group_prefix(g0, g1);
-                constexpr int U = 2;
+                constexpr int U = 4;
                 for (uint32_t i0 = t; i0 < ne; i0 += MT * U) {
                     uint4 d[U];
 #pragma unroll
@@ -1141,12 +1145,30 @@ __global__ void __launch_bounds__(merge_threads<B>(), 1) k_merge(Params p) {
                 if (!go) break;
             }
         };
-        // 2. counts, minimum ranks, candidates per voxel
+        // 2. counts, minimum ranks, candidates per voxel; the task's own
+        // entries kept aside for the gather (up to kStash of them)
         for_entries([&](const uint4& d, uint32_t v) {
             atomicAdd(&vcount[v], d.y);
             atomicMin(&vmr[v], d.w);
             atomicAdd(&vcc[v], min(d.y, K));
+            if (v >= v_lo && v < v_hi) {
+                const uint32_t k = atomicAdd(&s_nst, 1u);
+                if (k < kStash) stash[k] = d;
+            }
         });
+        const uint32_t nst = s_nst;
+        // the task's entries: from the stash when they all fit, else read again
+        auto for_task_entries = [&](auto&& f) {
+            if (nst <= kStash) {
+                for (uint32_t i = t; i < nst; i += MT) {
+                    const uint4 d = stash[i];
+                    f(d, voxel_of(bm, wpre, d.z & lomask));
+                }
+                __syncthreads();
+            } else {
+                for_entries(f);
+            }
+        };
         // 3. candidate offsets into vcc, kept offsets into kof (runs of
         // consecutive voxels a thread)
         uint32_t C = 0;
@@ -1197,7 +1219,7 @@ __global__ void __launch_bounds__(merge_threads<B>(), 1) k_merge(Params p) {
                 // one voxel with more candidates than the buffer: K slots
                 for (uint32_t j = t; j < K; j += MT) cand[j] = kUnset;
                 __syncthreads();
-                for_entries([&](const uint4& d, uint32_t v) {
+                for_task_entries([&](const uint4& d, uint32_t v) {
                     if (v != w0) return;
                     for_candidates(d, [&](uint32_t, uint32_t c) {
                         kmin_insert(cand, K, c);
@@ -1216,7 +1238,7 @@ __global__ void __launch_bounds__(merge_threads<B>(), 1) k_merge(Params p) {
                 }
                 w1 = w0 + 1;
             } else {
-                for_entries([&](const uint4& d, uint32_t v) {
+                for_task_entries([&](const uint4& d, uint32_t v) {
                     if (v < w0 || v >= w1) return;
                     const uint32_t at = atomicAdd(&vcc[v], min(d.y, K)) - base;
                     for_candidates(d, [&](uint32_t j, uint32_t c) {
