@@ -226,6 +226,12 @@ int mmbev_get_status(const void *workspace, size_t workspace_bytes,
  *                     voxel cap drops background-only voxels first.
  *                     Outside [0, 1] or NaN: MMBEV_EINVAL.
  *   seed              the generator's seed.
+ *   merge_buffer_words 0 for use. A test hook: when non-zero, the stage that
+ *                     merges buckets split in parts uses at most this many
+ *                     32-bit words of shared memory for its candidates (but
+ *                     at least K) and keeps at most a quarter as many entries
+ *                     aside, so that its windowed and overflow paths run on
+ *                     small inputs. Results do not change.
  */
 #define MMBEV_NUM_STAGES 7
 typedef struct mmbev_exec_opts {
@@ -233,6 +239,7 @@ typedef struct mmbev_exec_opts {
     uint32_t inject_status;
     float rho_out;
     uint64_t seed;
+    uint32_t merge_buffer_words;
 } mmbev_exec_opts_t;
 
 /*

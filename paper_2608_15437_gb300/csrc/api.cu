@@ -335,6 +335,7 @@ int voxelize_batched(const float* points, const int64_t* sweep_offsets, int32_t 
         p.rho_thr = rho >= 1.0f ? (1u << 24) : (uint32_t)std::floor((double)rho * 16777216.0);
         p.seed = opts->seed;
         p.inject_status = opts->inject_status;
+        p.merge_limit = opts->merge_buffer_words;
     }
 
     const int sms = num_sms();

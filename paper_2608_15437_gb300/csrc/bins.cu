@@ -1068,7 +1068,12 @@ __global__ void __launch_bounds__(merge_threads<B>(), 1) k_merge(Params p) {
         const uint32_t sto = (2u * kBmWords + 4u * nv + 3u) & ~3u;   // the stash, 16-byte aligned
         uint4* stash = reinterpret_cast<uint4*>(msm + sto);          // the task's own entries
         uint32_t* cand = msm + sto + 4u * kStash;
-        const uint32_t cap = (uint32_t)(kMergeSmem / 4) - sto - 4u * kStash;
+        uint32_t cap = (uint32_t)(kMergeSmem / 4) - sto - 4u * kStash;
+        uint32_t stash_cap = kStash;
+        if (p.merge_limit) {   // test hook: a smaller buffer and stash
+            cap = max(K, min(cap, p.merge_limit));
+            stash_cap = min(kStash, p.merge_limit / 4u);
+        }
         if (t == 0) s_nst = 0u;
         for (uint32_t v = t; v < nv; v += MT) {
             vcount[v] = 0u;
@@ -1153,13 +1158,13 @@ __global__ void __launch_bounds__(merge_threads<B>(), 1) k_merge(Params p) {
             atomicAdd(&vcc[v], min(d.y, K));
             if (v >= v_lo && v < v_hi) {
                 const uint32_t k = atomicAdd(&s_nst, 1u);
-                if (k < kStash) stash[k] = d;
+                if (k < stash_cap) stash[k] = d;
             }
         });
         const uint32_t nst = s_nst;
         // the task's entries: from the stash when they all fit, else read again
         auto for_task_entries = [&](auto&& f) {
-            if (nst <= kStash) {
+            if (nst <= stash_cap) {
                 for (uint32_t i = t; i < nst; i += MT) {
                     const uint4 d = stash[i];
                     f(d, voxel_of(bm, wpre, d.z & lomask));

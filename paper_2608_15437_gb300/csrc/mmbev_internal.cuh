@@ -142,6 +142,7 @@ struct Params {
     uint64_t seed;          // SplitMix64 seed of those draws
     int32_t keep_status = 0;  // prep leaves the status word as it is (later chunks of a call)
     uint32_t inject_status = 0;  // test hook: status bits prep sets as a failure would
+    uint32_t merge_limit = 0;    // test hook: the merge's buffer words (0: all it has)
     // buckets
     int32_t bucket_log2;       // LB
     uint32_t buckets_per_frame;  // Bf

@@ -369,8 +369,12 @@ __device__ __forceinline__ bool classify_range(const Params& p, const ClsSmem& s
         // the block's dense list of kept points (any order): one shared
         // atomic per warp reserves the warp's entries
         const uint32_t nk = __popc(b0) + __popc(b1);
+        if (nk == 0u) {   // warp-uniform: nothing kept in the chunk
+            c = __shfl_sync(0xFFFFFFFFu, cn, 0);
+            continue;
+        }
         uint32_t lbase = 0;
-        if (lane == 0 && nk) lbase = atomicAdd(&sm.kept[0], nk);
+        if (lane == 0) lbase = atomicAdd(&sm.kept[0], nk);
         lbase = __shfl_sync(0xFFFFFFFFu, lbase, 0);
         const uint32_t lo_mask = (1u << p.bucket_log2) - 1u;
 #pragma unroll
