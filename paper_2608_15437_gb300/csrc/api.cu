@@ -117,7 +117,7 @@ Layout make_layout(int64_t max_points, int64_t rois_total, int32_t max_rois_fram
     L.huge_cap = (uint32_t)(TS / kPart + 1);
     L.job_cap = (uint32_t)(B4 + 2);
     L.part_cap = (uint32_t)(2 * (TS / kPart) + 2);
-    L.jobs = take(sizeof(uint4) * L.job_cap);
+    L.jobs = take(sizeof(uint4) * 3 * (size_t)L.job_cap);
     L.sjobs = take(sizeof(uint4) * B4);
     L.hjobs = take(sizeof(uint4) * L.part_cap);
     L.hj0 = take(sizeof(uint32_t) * L.huge_cap);

@@ -354,6 +354,13 @@ static_assert(kScanTile == kScanThreads * 4, "four buckets a thread");
 constexpr unsigned long long kAggFlag = 1ull << 32;    // tile total published
 constexpr unsigned long long kIncFlag = 2ull << 32;    // tile inclusive prefix published
 
+// Size class of a block job (a bucket of kWarpJobMax+1 .. kPart points):
+// 0 for 1,025-2,048 points, 1 for 513-1,024, 2 for 257-512; 3 otherwise.
+__device__ __forceinline__ uint32_t block_job_class(uint32_t c) {
+    if (c <= kWarpJobMax || c > kPart) return 3u;
+    return c > kPart / 2 ? 0u : c > kPart / 4 ? 1u : 2u;
+}
+
 // Stage 2. The tile's inclusive prefix comes from its predecessors by
 // decoupled look-back, done by warp 0 over 32 predecessors at a time: each
 // lane waits (bounded) until its predecessor has published at least its
@@ -364,7 +371,7 @@ constexpr unsigned long long kIncFlag = 2ull << 32;    // tile inclusive prefix 
 // last part to finish merges.
 __global__ void __launch_bounds__(kScanThreads) k_bucket_scan(Params p) {
     __shared__ uint32_t s_warp[kScanThreads / 32];
-    __shared__ uint32_t s_tile, s_base, s_jbase[2];
+    __shared__ uint32_t s_tile, s_base, s_jbase[4];
     pdl_wait();
     const int t = threadIdx.x, lane = t & 31;
     // tiles are numbered in the order their blocks start, so a tile only
@@ -422,23 +429,33 @@ __global__ void __launch_bounds__(kScanThreads) k_bucket_scan(Params p) {
         if (lane == 0) s_base = base;
     }
     __syncthreads();
-    // the tile's warp jobs and block jobs: one reservation a list for the
-    // whole tile (counts packed small | large << 16; a tile has 4,096 buckets)
-    uint32_t jc = 0;
+    // the tile's warp jobs and block jobs (three size classes, so that the
+    // bucket stage takes the largest first): one reservation a list for the
+    // whole tile (counts packed two to a word; a tile has 4,096 buckets)
+    uint32_t jc0 = 0, jc1 = 0;
 #pragma unroll
     for (int k = 0; k < 4; ++k) {
         const bool ok = b0 + k < B;
-        jc += ok && c[k] > 0u && c[k] <= kWarpJobMax ? 1u : 0u;
-        jc += ok && c[k] > kWarpJobMax && c[k] <= kPart ? 1u << 16 : 0u;
+        const uint32_t cls = block_job_class(c[k]);
+        jc0 += ok && c[k] > 0u && c[k] <= kWarpJobMax ? 1u : 0u;
+        jc0 += ok && cls == 0u ? 1u << 16 : 0u;
+        jc1 += ok && cls == 1u ? 1u : 0u;
+        jc1 += ok && cls == 2u ? 1u << 16 : 0u;
     }
-    uint32_t jtot = 0;
-    uint32_t jex = block_exclusive_scan(jc, s_warp, &jtot);
+    uint32_t jt0 = 0, jt1 = 0;
+    const uint32_t je0 = block_exclusive_scan(jc0, s_warp, &jt0);
+    const uint32_t je1 = block_exclusive_scan(jc1, s_warp, &jt1);
     if (t == 0) {
-        s_jbase[0] = jtot & 0xFFFFu ? atomicAdd(&p.hdr->n_small, jtot & 0xFFFFu) : 0u;
-        s_jbase[1] = jtot >> 16 ? atomicAdd(&p.hdr->n_large, jtot >> 16) : 0u;
+        const uint32_t ns0 = jt0 & 0xFFFFu, nl0 = jt0 >> 16, nl1 = jt1 & 0xFFFFu, nl2 = jt1 >> 16;
+        s_jbase[0] = ns0 ? atomicAdd(&p.hdr->n_small, ns0) : 0u;
+        s_jbase[1] = nl0 ? atomicAdd(&p.hdr->n_large[0], nl0) : 0u;
+        s_jbase[2] = nl1 ? atomicAdd(&p.hdr->n_large[1], nl1) : 0u;
+        s_jbase[3] = nl2 ? atomicAdd(&p.hdr->n_large[2], nl2) : 0u;
     }
     __syncthreads();
-    uint32_t js = s_jbase[0] + (jex & 0xFFFFu), jl = s_jbase[1] + (jex >> 16);
+    uint32_t js = s_jbase[0] + (je0 & 0xFFFFu);
+    uint32_t jl0 = s_jbase[1] + (je0 >> 16), jl1 = s_jbase[2] + (je1 & 0xFFFFu),
+             jl2 = s_jbase[3] + (je1 >> 16);
     uint32_t run = s_base + excl;
 #pragma unroll
     for (int k = 0; k < 4; ++k) {
@@ -454,10 +471,11 @@ __global__ void __launch_bounds__(kScanThreads) k_bucket_scan(Params p) {
             else set_status(p.hdr, MMBEV_DEV_BOUNDS);
             ++js;
         }
-        if (b < B && c[k] > kWarpJobMax && c[k] <= kPart) {
-            if (jl < p.job_cap) p.jobs[jl] = d;
+        const uint32_t cls = block_job_class(c[k]);
+        if (b < B && cls < 3u) {
+            const uint32_t at = cls == 0u ? jl0++ : cls == 1u ? jl1++ : jl2++;
+            if (at < p.job_cap) p.jobs[(size_t)cls * p.job_cap + at] = d;
             else set_status(p.hdr, MMBEV_DEV_BOUNDS);
-            ++jl;
         }
         if (b < B && c[k] > kPart) {   // parts of a bucket too large for one block
             const uint32_t P = (c[k] + kPart - 1) / kPart;
@@ -936,14 +954,24 @@ __global__ void __launch_bounds__(kBT, (BH <= 12 ? 8 : 2)) k_buckets(Params p) {
     __shared__ uint32_t s_jidx;
     pdl_wait();
     const int t = threadIdx.x, warp = t >> 5;
-    // tickets [0, np) are the parts (first, so that the merges of the split
-    // buckets start early), [np, np + nl) the block jobs
+    // tickets: the parts first (so that the merges of the split buckets can
+    // start early), then the block jobs, largest class first (the longest
+    // jobs do not come last)
     const uint32_t np = min(p.hdr->n_parts, p.part_cap);
-    const uint32_t nl = min(p.hdr->n_large, p.job_cap);
+    uint32_t nl[3];
+#pragma unroll
+    for (int q = 0; q < 3; ++q) nl[q] = min(p.hdr->n_large[q], p.job_cap);
     const uint32_t ns = min(p.hdr->n_small, p.num_buckets);
     const uint4 none = make_uint4(kUnset, 0u, 0u, 0u);
     auto job_at = [&](uint32_t k) -> uint4 {
-        return k < np ? p.hjobs[k] : k - np < nl ? p.jobs[k - np] : none;
+        if (k < np) return p.hjobs[k];
+        k -= np;
+#pragma unroll
+        for (int q = 0; q < 3; ++q) {
+            if (k < nl[q]) return p.jobs[(size_t)q * p.job_cap + k];
+            k -= nl[q];
+        }
+        return none;
     };
     uint4 d = none;
     uint32_t jcur = 0, jnext = 0;

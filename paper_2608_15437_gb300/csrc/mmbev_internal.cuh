@@ -106,14 +106,14 @@ struct __align__(16) Header {
     uint32_t status;        // MMBEV_DEV_* bits (first word: read by mmbev_get_status)
     uint32_t num_rec;       // kept points (records) of the call
     uint32_t scan_ticket;   // scan tiles started, in order
-    uint32_t n_large;       // block jobs: buckets of kWarpJobMax+1 .. kPart points
+    uint32_t n_large[3];    // block jobs of 1,025-2,048, 513-1,024 and 257-512 points
     uint32_t n_small;       // warp jobs: buckets of 1 .. kWarpJobMax points
-    uint32_t large_ticket;  // parts, then block jobs, taken by the bucket stage
+    uint32_t large_ticket;  // parts, then block jobs (largest class first), taken by the bucket stage
     uint32_t n_huge;        // buckets split in parts
     uint32_t n_parts;       // parts of the split buckets
     uint32_t n_mtasks;      // merge tasks: ranges of low lin bits of split buckets
     uint32_t small_ticket;  // warp jobs taken by the bucket stage
-    uint32_t pad[6];
+    uint32_t pad[4];
 };
 
 // Everything a kernel needs; passed by value.
@@ -167,7 +167,7 @@ struct Params {
     uint32_t* bcnt;         // [B] kept points per bucket
     uint32_t* boff;         // [B + 1] first item of each bucket
     uint32_t* ucnt;         // [B] voxels per bucket
-    uint4* jobs;            // [job_cap] block jobs {bucket, first item, points, ~0}
+    uint4* jobs;            // [3][job_cap] block jobs by size class {bucket, first item, points, ~0}
     uint4* sjobs;           // [B] warp jobs {bucket, first item, points, -}
     uint32_t job_cap;
     uint4* hjobs;           // [part_cap] parts {bucket, first item, points, split index}
