@@ -251,6 +251,10 @@ __device__ __forceinline__ void select_by_warp(const Params& p, const uint2* seg
 // most kHugeList a bucket; beyond that by warps).
 constexpr uint32_t kWarpMax = 1024;
 constexpr uint32_t kHugeList = 32;
+// Voxels of 33 .. kWarpMax points a block job lists for its warps: a job of
+// at most kPart points has at most kPart / 33 of them.
+constexpr uint32_t kDenseList = 64;
+static_assert(kPart / 33 < kDenseList, "a block job's dense voxels fit the list");
 
 // One voxel by the whole block (every thread calls it): each thread keeps
 // the B smallest positions of every blockDim-th entry, each warp reduces its
@@ -760,7 +764,11 @@ __device__ void bucket_by_block(const Params& p, const uint4& job, uint32_t jidx
     // bucket's go to vdesc and vitems; a part's to the part lists (pdesc, and
     // the .x words of its own items, all read by now).
     __shared__ uint32_t s_huge[kHugeList + 1];   // voxels of more than kWarpMax points
-    if (t == 0) s_huge[kHugeList] = 0u;
+    __shared__ uint32_t s_dense[kDenseList + 1];  // voxels of 33 .. kWarpMax points
+    if (t == 0) {
+        s_huge[kHugeList] = 0u;
+        s_dense[kDenseList] = 0u;
+    }
     __syncthreads();
     uint4* desc = (part ? p.pdesc : p.vdesc) + s;
     auto kept_out = [&](uint32_t st) -> KeptOut {
@@ -772,17 +780,25 @@ __device__ void bucket_by_block(const Params& p, const uint4& job, uint32_t jidx
         if (cnt > kWarpMax) {
             const uint32_t k = atomicAdd(&s_huge[kHugeList], 1u);
             if (k < kHugeList) s_huge[k] = v;
+        } else if (cnt > 32u) {
+            const uint32_t k = atomicAdd(&s_dense[kDenseList], 1u);
+            if (k < kDenseList) s_dense[k] = v;
         }
     }
     for (uint32_t i = t; i < n; i += kBT) select_small(p, seg, i, bm, wpre, vc, kept_out, desc);
     __syncthreads();
     const uint32_t nh = s_huge[kHugeList];
-    for (uint32_t v = warp; v < nv; v += kBT / 32) {
+    const uint32_t nd = min(s_dense[kDenseList], kDenseList);   // never more: see kDenseList
+    for (uint32_t k = warp; k < nd; k += kBT / 32) {
+        const uint32_t v = s_dense[k];
         const uint32_t st = v ? vc[v - 1] : 0u, cnt = vc[v] - st;
-        // heavy voxels, and huge ones beyond the list's room
-        if (cnt > 32u && (cnt <= kWarpMax || nh > kHugeList))
-            select_by_warp<BH>(p, seg, st, cnt, kept_out(st), desc + v);
+        select_by_warp<BH>(p, seg, st, cnt, kept_out(st), desc + v);
     }
+    if (nh > kHugeList)   // huge voxels beyond the list's room, by warps
+        for (uint32_t v = warp; v < nv; v += kBT / 32) {
+            const uint32_t st = v ? vc[v - 1] : 0u, cnt = vc[v] - st;
+            if (cnt > kWarpMax) select_by_warp<BH>(p, seg, st, cnt, kept_out(st), desc + v);
+        }
     if (nh <= kHugeList) {
         for (uint32_t k = 0; k < nh; ++k) {   // block-uniform
             const uint32_t v = s_huge[k];
@@ -932,10 +948,17 @@ __device__ void bucket_by_warp(const Params& p, const uint4& job, unsigned char*
     uint4* desc = p.vdesc + s;
     auto kept_out = [&](uint32_t st) { return KeptOut{p.vitems + s + st, 1u, s + st}; };
     for (uint32_t i = lane; i < n; i += 32) select_small(p, seg, i, bm, wpre, vc, kept_out, desc);
-    for (uint32_t vv = 0; vv < nv; ++vv) {   // warp-uniform
-        const uint32_t st = vv ? vc[vv - 1] : 0u, cnt = vc[vv] - st;
-        if (cnt > 32u)
+    for (uint32_t v0 = 0; v0 < nv; v0 += 32) {   // warp-uniform: voxels of more than 32 points
+        bool dense = false;
+        if (v0 + (uint32_t)lane < nv) {
+            const uint32_t vv = v0 + (uint32_t)lane;
+            dense = vc[vv] - (vv ? vc[vv - 1] : 0u) > 32u;
+        }
+        for (uint32_t m = __ballot_sync(kFull, dense); m; m &= m - 1u) {
+            const uint32_t vv = v0 + (uint32_t)(__ffs(m) - 1);
+            const uint32_t st = vv ? vc[vv - 1] : 0u, cnt = vc[vv] - st;
             select_by_warp<BH>(p, seg, st, cnt, KeptOut{p.vitems + s + st, 1u, s + st}, desc + vv);
+        }
     }
     if (lane == 0) publish_bucket(p, b, nv);
     __syncwarp();
