@@ -1577,7 +1577,7 @@ constexpr uint32_t kMaxSlices = (1u << (32 - kBucketLog2Max)) >> kSliceLog2;   /
 // a scan of the bucket counts of the slices it touches; then each thread
 // finalizes one row.
 template <int B>
-__global__ void __launch_bounds__(kOutThreads) k_output(Params p) {
+__global__ void __launch_bounds__(kOutThreads, (B <= 12 ? 4 : 2)) k_output(Params p) {
     __shared__ uint32_t s_warp[kOutThreads / 32];
     __shared__ uint32_t s_cpre[kMaxFrames + 1];   // chunks before each frame
     __shared__ uint32_t s_spre[kMaxSlices + 1];   // voxels before each slice of a frame
