@@ -110,27 +110,41 @@ def test_batch32_parity(oracle_mod, mmbev_lib, cuda_dev):
     assert assert_frames_equal(got, want, "batch32") == 1.0
 
 
-@pytest.mark.parametrize("words", [16, 200, 3000])
-def test_merge_windows_and_overflow(oracle_mod, mmbev_lib, cuda_dev, words):
-    """Buckets split in parts (more than 2,048 kept points among 2^13
-    consecutive linear indices of one frame), merged with a small buffer:
-    windows of voxels, voxels whose candidates overflow the buffer (merged in
-    K slots) and tasks whose entries overflow their stash (read again) all
-    take their fallback paths, and the results stay those of the oracle."""
-    w = synth.streaming_batch(4)
-    big = 0
-    for f in range(w.num_frames):
-        fr = w.frame(f)
-        _, lin, _ = oracle_mod.classify(fr.points, fr.sweep_offsets, fr.sweep_tf, fr.rois,
-                                        fr.roi_margin, fr.voxel_size, fr.pc_range)
-        kept = lin[lin >= 0]
-        if kept.size:
-            big = max(big, int(np.bincount(kept >> 13).max()))
-    assert big > 2048   # the workload has split buckets
-    want = run_oracle(oracle_mod, w)
-    got, status, _ = run_gpu(mmbev_lib, w, cuda_dev, merge_buffer_words=words)
+_SPLIT = {}
+
+
+def _split_workload(oracle_mod):
+    """Four batch frames, checked (oracle side, once) to have buckets split
+    in parts: more than 2,048 kept points among 2^13 consecutive linear
+    indices of one frame."""
+    if "w" not in _SPLIT:
+        w = synth.streaming_batch(4)
+        big = 0
+        for f in range(w.num_frames):
+            fr = w.frame(f)
+            _, lin, _ = oracle_mod.classify(fr.points, fr.sweep_offsets, fr.sweep_tf, fr.rois,
+                                            fr.roi_margin, fr.voxel_size, fr.pc_range)
+            kept = lin[lin >= 0]
+            if kept.size:
+                big = max(big, int(np.bincount(kept >> 13).max()))
+        _SPLIT["w"], _SPLIT["big"] = w, big
+    assert _SPLIT["big"] > 2048
+    return _SPLIT["w"]
+
+
+@pytest.mark.parametrize("K,words", [(10, 16), (10, 200), (10, 3000), (20, 0), (33, 0),
+                                     (33, 200), (64, 0), (64, 64)])
+def test_merge_windows_and_overflow(oracle_mod, mmbev_lib, cuda_dev, K, words):
+    """Buckets split in parts merged at every K instantiation, with the
+    merge's full buffer (words = 0) or a small one: windows of voxels, voxels
+    whose candidates overflow the buffer (merged in K slots) and tasks whose
+    entries overflow their stash (read again) all take their fallback paths,
+    and the results stay those of the oracle."""
+    w = _split_workload(oracle_mod)
+    want = run_oracle(oracle_mod, w, K=K)
+    got, status, _ = run_gpu(mmbev_lib, w, cuda_dev, K=K, merge_buffer_words=words)
     assert status == 0
-    assert assert_frames_equal(got, want, f"merge buffer {words}") == 1.0
+    assert assert_frames_equal(got, want, f"K={K}, merge buffer {words}") == 1.0
 
 
 # ------------------------------------------------------------------ cap path
