@@ -515,7 +515,7 @@ constexpr int kThreads = 256;
 // Prefix sums of the classify blocks' list lengths (off[0..G]) and of their
 // units of kUnit entries (uoff[0..G]), and the first plist entry of each list
 // (list l starts at tile t_begin(l) * 2048).
-constexpr uint32_t kUnit = 256;   // entries a warp takes at once (8 per lane)
+constexpr uint32_t kUnit = 128;   // entries a warp takes at once (4 per lane)
 struct Lists {
     uint32_t off[kMaxClsGrid + 1];
     uint32_t uoff[kMaxClsGrid + 1];
@@ -561,10 +561,11 @@ __device__ __forceinline__ uint32_t lists_scan(const Params& p, Lists& L, uint32
 }
 
 // Each warp takes units of kUnit consecutive entries of one classify block's
-// list (eight groups of 32). The entries of one bucket in a group take their
+// list (four groups of 32); eight blocks an SM, for twice the loads and
+// atomics in flight that 32 registers a thread allow. The entries of one bucket in a group take their
 // places with one atomic on the bucket's cursor (ucnt, zero after the scan
 // stage; it ends at the bucket's count).
-__global__ void __launch_bounds__(kThreads) k_bucket_scatter(Params p) {
+__global__ void __launch_bounds__(kThreads, 8) k_bucket_scatter(Params p) {
     __shared__ Lists L;
     __shared__ uint32_t s_warp[kThreads / 32];
     pdl_wait();
@@ -1681,7 +1682,7 @@ cudaError_t launch_bucket_scan(const Params& p, bool pdl, cudaStream_t st) {
 }
 
 cudaError_t launch_bucket_scatter(const Params& p, int num_sms, bool pdl, cudaStream_t st) {
-    return launch_k(k_bucket_scatter, dim3(num_sms * 4), dim3(kThreads), 0, st, pdl, p);
+    return launch_k(k_bucket_scatter, dim3(num_sms * 8), dim3(kThreads), 0, st, pdl, p);
 }
 
 template <int BL, int BH>
