@@ -1407,7 +1407,7 @@ __device__ __forceinline__ void finalize_voxel(const Params& p, uint32_t f, uint
 #pragma unroll
     for (int j = 0; j < B; ++j) pos[j] = (uint32_t)j < kept ? p.vitems[d.x + j] : kUnset;
     sort_small<B>(pos);   // kept positions come in any order; the sum goes by index
-    constexpr int R = B < 4 ? B : 4;   // record loads in flight
+    constexpr int R = B < 2 ? B : 2;   // record loads in flight (more warps beat more loads a warp)
     float acc[5] = {0.f, 0.f, 0.f, 0.f, 0.f};
 #pragma unroll
     for (int j0 = 0; j0 < B; j0 += R) {
@@ -1578,7 +1578,7 @@ constexpr uint32_t kMaxSlices = (1u << (32 - kBucketLog2Max)) >> kSliceLog2;   /
 // a scan of the bucket counts of the slices it touches; then each thread
 // finalizes one row.
 template <int B>
-__global__ void __launch_bounds__(kOutThreads, (B <= 12 ? 4 : 2)) k_output(Params p) {
+__global__ void __launch_bounds__(kOutThreads, (B <= 12 ? 6 : 2)) k_output(Params p) {
     __shared__ uint32_t s_warp[kOutThreads / 32];
     __shared__ uint32_t s_cpre[kMaxFrames + 1];   // chunks before each frame
     __shared__ uint32_t s_spre[kMaxSlices + 1];   // voxels before each slice of a frame
@@ -1716,7 +1716,7 @@ cudaError_t launch_merge(const Params& p, int num_sms, bool pdl, cudaStream_t st
 }
 
 cudaError_t launch_output(const Params& p, int num_sms, bool pdl, cudaStream_t st) {
-    const dim3 grid(num_sms * 4), block(kOutThreads);
+    const dim3 grid(num_sms * (p.K <= 12 ? 6 : 2)), block(kOutThreads);
     if (p.K <= 4) return launch_k(k_output<4>, grid, block, 0, st, pdl, p);
     if (p.K <= 12) return launch_k(k_output<12>, grid, block, 0, st, pdl, p);
     if (p.K <= 32) return launch_k(k_output<32>, grid, block, 0, st, pdl, p);
