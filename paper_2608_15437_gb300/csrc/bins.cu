@@ -370,9 +370,9 @@ __device__ __forceinline__ uint32_t block_job_class(uint32_t c) {
 // lane waits (bounded) until its predecessor has published at least its
 // total, and the nearest one that has published its inclusive prefix ends
 // the walk. Then every non-empty bucket becomes jobs of the bucket stage: a
-// small one (at most kWarpJobMax points) a warp job, a larger one a block job,
-// and one of more than kPart points kPart-point parts whose voxel lists the
-// last part to finish merges.
+// small one (at most kWarpJobMax points) a warp job, a larger one a block job
+// (in one of three size classes), and one of more than kPart points
+// kPart-point parts, with the merge tasks that combine their voxel lists.
 __global__ void __launch_bounds__(kScanThreads) k_bucket_scan(Params p) {
     __shared__ uint32_t s_warp[kScanThreads / 32];
     __shared__ uint32_t s_tile, s_base, s_jbase[4];
@@ -637,7 +637,7 @@ constexpr uint32_t kIl = 4;   // items a thread keeps in registers: jobs up to 5
 // bucket, or part of a bucket split in parts (then job.w is the split
 // bucket's index). job = {bucket, first item, points, split index or ~0};
 // jidx its place in the job list.
-template <int BL, int BH>
+template <int BH>
 __device__ void bucket_by_block(const Params& p, const uint4& job, uint32_t jidx,
                                 unsigned char* smem, uint32_t* s_warp) {
     const int t = threadIdx.x, warp = t >> 5;
@@ -866,7 +866,7 @@ __device__ void bucket_tiny(const Params& p, const uint4& job) {
 // A warp job (at most kWarpJobMax points): one bucket by one warp, in its
 // own piece of shared memory; a lane keeps up to eight of its items in
 // registers. job = {bucket, first item, points, -}.
-template <int BL, int BH>
+template <int BH>
 __device__ void bucket_by_warp(const Params& p, const uint4& job, unsigned char* piece) {
     constexpr uint32_t kPer = kWarpJobMax / 32;   // 8
     const int lane = threadIdx.x & 31;
@@ -970,7 +970,7 @@ __device__ void bucket_by_warp(const Params& p, const uint4& job, unsigned char*
 // the current job is worked on, so no thread waits on them. Then each warp
 // takes warp jobs from a second counter the same way, so that warps whose
 // block was busy longest take the fewest.
-template <int BL, int BH>
+template <int BH>
 __global__ void __launch_bounds__(kBT, (BH <= 12 ? 8 : 2)) k_buckets(Params p) {
     extern __shared__ __align__(16) unsigned char smem[];
     __shared__ uint32_t s_warp[kBT / 32];
@@ -1019,7 +1019,7 @@ __global__ void __launch_bounds__(kBT, (BH <= 12 ? 8 : 2)) k_buckets(Params p) {
             jcur = jnext;
             jnext = atomicAdd(&p.hdr->large_ticket, 1u);
         }
-        bucket_by_block<BL, BH>(p, job, jidx, smem, s_warp);
+        bucket_by_block<BH>(p, job, jidx, smem, s_warp);
     }
     // Then the warp jobs, by ticket: the next job's descriptor and the ticket
     // after it are requested before the current job and used after it.
@@ -1038,7 +1038,7 @@ __global__ void __launch_bounds__(kBT, (BH <= 12 ? 8 : 2)) k_buckets(Params p) {
         uint32_t knn = 0;
         if (lane == 0 && kn < ns) knn = atomicAdd(&p.hdr->small_ticket, 1u);
         if (sj.z <= 32u) bucket_tiny(p, sj);
-        else bucket_by_warp<BL, BH>(p, sj, piece);
+        else bucket_by_warp<BH>(p, sj, piece);
         sj = next;
         k = kn;
         kn = k < ns ? __shfl_sync(kFull, knn, 0) : ns;
@@ -1685,27 +1685,27 @@ cudaError_t launch_bucket_scatter(const Params& p, int num_sms, bool pdl, cudaSt
     return launch_k(k_bucket_scatter, dim3(num_sms * 8), dim3(kThreads), 0, st, pdl, p);
 }
 
-template <int BL, int BH>
+template <int BH>
 cudaError_t launch_buckets_t(const Params& p, int num_sms, bool pdl, cudaStream_t st) {
     static std::atomic<int> configured[64];
     int dev = 0;
     cudaError_t e = cudaGetDevice(&dev);
     if (e != cudaSuccess) return e;
     if (dev < 0 || dev >= 64 || !configured[dev].load(std::memory_order_acquire)) {
-        e = cudaFuncSetAttribute(k_buckets<BL, BH>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+        e = cudaFuncSetAttribute(k_buckets<BH>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                  (int)kBlockSmem);
         if (e != cudaSuccess) return e;
         if (dev >= 0 && dev < 64) configured[dev].store(1, std::memory_order_release);
     }
     const int per_sm = BH <= 12 ? 8 : 2;
-    return launch_k(k_buckets<BL, BH>, dim3(num_sms * per_sm), dim3(kBT), kBlockSmem, st, pdl, p);
+    return launch_k(k_buckets<BH>, dim3(num_sms * per_sm), dim3(kBT), kBlockSmem, st, pdl, p);
 }
 
 cudaError_t launch_buckets(const Params& p, int num_sms, bool pdl, cudaStream_t st) {
-    if (p.K <= 4) return launch_buckets_t<4, 4>(p, num_sms, pdl, st);
-    if (p.K <= 12) return launch_buckets_t<12, 12>(p, num_sms, pdl, st);
-    if (p.K <= 32) return launch_buckets_t<32, 32>(p, num_sms, pdl, st);
-    return launch_buckets_t<32, kMaxK>(p, num_sms, pdl, st);
+    if (p.K <= 4) return launch_buckets_t<4>(p, num_sms, pdl, st);
+    if (p.K <= 12) return launch_buckets_t<12>(p, num_sms, pdl, st);
+    if (p.K <= 32) return launch_buckets_t<32>(p, num_sms, pdl, st);
+    return launch_buckets_t<kMaxK>(p, num_sms, pdl, st);
 }
 
 cudaError_t launch_merge(const Params& p, int num_sms, bool pdl, cudaStream_t st) {
