@@ -101,9 +101,9 @@ typedef enum mmbev_status {
  * Bytes of scratch workspace for a call with up to max_points points,
  * max_rois_per_frame ROIs in any frame, max_voxels kept voxels per frame and
  * num_frames frames on the grid given by voxel_size[3] and range[6] (host
- * arrays). About 88 bytes per point (records, lists and per-voxel results,
- * all sized for every point kept) plus 20 bytes per bucket of 2^13
- * consecutive cells of each frame's grid. Returns 0 for invalid arguments.
+ * arrays). About 66 bytes per point (records, sort keys and positions and
+ * per-voxel results, all sized for every point kept) plus about 34 KB per
+ * frame. Returns 0 for invalid arguments.
  */
 size_t mmbev_workspace_size(int64_t max_points, int32_t max_rois_per_frame,
                             int32_t max_voxels, int32_t num_frames,
@@ -226,20 +226,15 @@ int mmbev_get_status(const void *workspace, size_t workspace_bytes,
  *                     voxel cap drops background-only voxels first.
  *                     Outside [0, 1] or NaN: MMBEV_EINVAL.
  *   seed              the generator's seed.
- *   merge_buffer_words 0 for use. A test hook: when non-zero, the stage that
- *                     merges buckets split in parts uses at most this many
- *                     32-bit words of shared memory for its candidates (but
- *                     at least K) and keeps at most a quarter as many entries
- *                     aside, so that its windowed and overflow paths run on
- *                     small inputs. Results do not change.
+ * The stages, in launch order (mmbev_stage_name): prep, classify, compact,
+ * sort (one launch per 8-bit digit of the sort key), runs, emit.
  */
-#define MMBEV_NUM_STAGES 7
+#define MMBEV_NUM_STAGES 6
 typedef struct mmbev_exec_opts {
     cudaEvent_t *stage_events;
     uint32_t inject_status;
     float rho_out;
     uint64_t seed;
-    uint32_t merge_buffer_words;
 } mmbev_exec_opts_t;
 
 /*
@@ -312,7 +307,7 @@ int mmbev_voxelize_roi_batched_ex(const float *points, const int64_t *sweep_offs
  *   voxel_size, range) must not exceed MMBEV_NOALLOC_SCRATCH_BYTES; K and
  *   max_voxels do not enter it. On the grids of the tiny, nuScenes- and
  *   Ouster-shaped workloads, with their ROI counts, that allows up to about
- *   1,100,000 points.
+ *   1,500,000 points.
  * The first call on a device (and the first in each new context of it, as
  * after cudaDeviceReset) looks up the array's device address with that
  * device current; make that first call before any stream capture. The

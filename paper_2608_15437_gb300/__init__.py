@@ -21,7 +21,7 @@ import torch
 _PKG = os.path.dirname(os.path.abspath(__file__))
 LIB_PATH = os.path.join(_PKG, "libmmbev.so")
 
-NUM_STAGES = 7
+NUM_STAGES = 6
 DEV_TABLE_FULL = 0x1
 DEV_WAIT_TIMEOUT = 0x2
 DEV_BOUNDS = 0x4
@@ -36,8 +36,7 @@ class MMBEVError(RuntimeError):
 
 class _ExecOpts(ctypes.Structure):
     _fields_ = [("stage_events", ctypes.c_void_p), ("inject_status", ctypes.c_uint32),
-                ("rho_out", ctypes.c_float), ("seed", ctypes.c_uint64),
-                ("merge_buffer_words", ctypes.c_uint32)]
+                ("rho_out", ctypes.c_float), ("seed", ctypes.c_uint64)]
 
 
 def load():
@@ -193,7 +192,7 @@ def voxelize_roi_batched(points: torch.Tensor, sweep_offsets, sweep_tf: torch.Te
                          frame_roi_offsets, *, workspace: torch.Tensor,
                          out: Outputs | None = None, stream=None, stage_events=None,
                          inject_status: int = 0, rho_out: float = 0.0,
-                         seed: int = 0, merge_buffer_words: int = 0) -> Outputs:
+                         seed: int = 0) -> Outputs:
     """Voxelize F independent frames in one call (``mmbev_voxelize_roi_batched``).
 
     points [N,5] float32, sweep_tf [S,16] float32 and rois [R,5] float32 live
@@ -204,8 +203,6 @@ def voxelize_roi_batched(points: torch.Tensor, sweep_offsets, sweep_tf: torch.Te
     no ROI with that probability (SplitMix64 draws keyed by ``seed`` and the
     point's index within its frame). ``inject_status`` is a test hook: status
     bits the call reports as if a device-side failure had set them.
-    ``merge_buffer_words`` is another: a smaller buffer for the merge stage, so
-    that its windowed and overflow paths run (the results do not change).
     """
     lib = load()
     so = _host(sweep_offsets, np.int64)
@@ -222,11 +219,10 @@ def voxelize_roi_batched(points: torch.Tensor, sweep_offsets, sweep_tf: torch.Te
             _hptr(rg), int(max_pts_per_voxel), int(max_voxels), nf, _hptr(fso), _hptr(fro),
             _dptr(out.feats), _dptr(out.coords), _dptr(out.counts), _dptr(out.nvox),
             _dptr(workspace, torch.uint8, "workspace"), workspace.numel(), _stream(stream)]
-    if stage_events is None and not inject_status and not rho_out and not merge_buffer_words:
+    if stage_events is None and not inject_status and not rho_out:
         rc = lib.mmbev_voxelize_roi_batched(*args)
     else:
-        opts = _ExecOpts(None, int(inject_status), float(rho_out), int(seed) & (2**64 - 1),
-                         int(merge_buffer_words))
+        opts = _ExecOpts(None, int(inject_status), float(rho_out), int(seed) & (2**64 - 1))
         if stage_events is not None:
             assert len(stage_events) == NUM_STAGES + 1
             arr = (ctypes.c_void_p * len(stage_events))(*[e.cuda_event for e in stage_events])
@@ -531,7 +527,7 @@ class Voxelizer:
         else:
             self._copy_stream.wait_event(self._staging_read[k])
         opts = _ExecOpts(None, int(inject_status), float(self.rho_out),
-                         int(self.seed) & (2**64 - 1), 0)
+                         int(self.seed) & (2**64 - 1))
         nr = h_rois.shape[0] if h_rois.dim() > 1 else h_rois.numel() // 5
         rc = lib.mmbev_voxelize_roi_batched_host(
             ctypes.c_void_p(h_points.data_ptr()), _hptr(so), len(so) - 1,

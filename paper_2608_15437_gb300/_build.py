@@ -18,7 +18,7 @@ CSRC = os.path.join(PKG, "csrc")
 INCLUDE = os.path.join(ROOT, "include")
 BUILD = os.path.join(PKG, "_build")
 LIB = os.path.join(PKG, "libmmbev.so")
-SOURCES = ["prep.cu", "points.cu", "bins.cu", "api.cu", "bev.cu", "rois.cu", "components.cu", "pack.cu",
+SOURCES = ["prep.cu", "points.cu", "sort.cu", "api.cu", "bev.cu", "rois.cu", "components.cu", "pack.cu",
            "noalloc.cu"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 FLAGS = ["-O3", "-std=c++17", "-lineinfo", "-Xcompiler", "-fPIC", "-Xcompiler", "-O2",

@@ -38,12 +38,6 @@ bool make_grid(const float* vs, const float* range, Grid* g) {
     return true;
 }
 
-int bucket_log2_for(uint64_t cells) {
-    int lb = 5;
-    while (lb < kBucketLog2Max && (1ull << lb) < cells) ++lb;
-    return lb;
-}
-
 int mask_words_for(int32_t max_rois_frame) {
     const int w = (max_rois_frame + 31) / 32;
     return w < 1 ? 1 : w;
@@ -65,30 +59,28 @@ int coarse_for(int mask_words) {
 // Byte offsets of every workspace array for one call shape.
 struct Layout {
     size_t hdr, sweep_off, sweep_frame, fso, fro, roi_prep, masks;
-    size_t records, plist, cls_cnt, bcnt, boff, ucnt, jobs, sjobs, hjobs, hj0, hbits, pnv, mtasks,
-        scan_state,
-        items, vdesc,
-        vitems, ssum, ftot, bcap;
+    size_t records, ckey, key_a, val_a, rcnt, cls_cnt, fcnt, ftot, hist, sort_state,
+        run_state, vdesc;
     size_t total;
-    uint32_t num_buckets, buckets_per_frame, num_tiles, scan_tiles, out_slices, job_cap, part_cap,
-        huge_cap, mtask_cap;
-    int bucket_log2, mask_words, coarse;
+    uint32_t num_tiles, sort_tiles_cap, run_tiles_cap;
+    int mask_words, coarse;
 };
 
 Layout make_layout(int64_t max_points, int64_t rois_total, int32_t max_rois_frame,
                    int32_t max_voxels, int32_t num_frames, const Grid& g) {
     Layout L{};
-    L.bucket_log2 = bucket_log2_for(g.cells);
-    L.buckets_per_frame = (uint32_t)((g.cells + (1ull << L.bucket_log2) - 1) >> L.bucket_log2);
-    L.num_buckets = L.buckets_per_frame * (uint32_t)num_frames;
+    (void)g;
     L.mask_words = mask_words_for(max_rois_frame);
     L.coarse = coarse_for(L.mask_words);
     const size_t F = (size_t)num_frames, R = (size_t)(rois_total > 0 ? rois_total : 1);
     const size_t U = (size_t)(max_points > 0 ? max_points : 1);
-    const size_t B4 = ((size_t)L.num_buckets + 4) / 4 * 4;  // zeroed as 16-byte words
-    L.scan_tiles = (uint32_t)(((size_t)L.num_buckets + kScanTile - 1) / kScanTile);
     L.num_tiles = (uint32_t)((U + kTile - 1) / kTile);
     const size_t TS = (size_t)L.num_tiles * kTile;        // record slots, tile-aligned
+    const size_t regions = TS / kRegion;
+    // a frame's items are tiled from its own first item: at most one more
+    // tile a frame than the call's items fill
+    L.sort_tiles_cap = (uint32_t)((TS + kSortTile - 1) / kSortTile + F);
+    L.run_tiles_cap = (uint32_t)((TS + kRunTile - 1) / kRunTile + F);
     size_t o = 0;
     auto take = [&](size_t bytes) { const size_t at = o; o = align_up(o + bytes, kAlign); return at; };
     L.hdr = take(sizeof(Header));
@@ -107,33 +99,17 @@ Layout make_layout(int64_t max_points, int64_t rois_total, int32_t max_rois_fram
     }
     L.masks = take(sizeof(uint32_t) * F * mask_words_frame);
     L.records = take(32 * TS);
-    L.plist = take(16 * TS);      // after the scatter stage: point lists of large buckets
+    L.ckey = take(sizeof(unsigned long long) * TS);   // then sort buffer B: lins, positions
+    L.key_a = take(sizeof(uint32_t) * TS);
+    L.val_a = take(sizeof(uint32_t) * TS);
+    L.rcnt = take(regions);
     L.cls_cnt = take(sizeof(uint32_t) * kMaxClsGrid);
-    L.bcnt = take(sizeof(uint32_t) * B4);
-    L.boff = take(sizeof(uint32_t) * (B4 + 4));
-    L.ucnt = take(sizeof(uint32_t) * B4);
-    // block jobs: at most one a bucket; parts of split buckets: at most two
-    // per kPart kept points
-    L.huge_cap = (uint32_t)(TS / kPart + 1);
-    L.job_cap = (uint32_t)(B4 + 2);
-    L.part_cap = (uint32_t)(2 * (TS / kPart) + 2);
-    L.jobs = take(sizeof(uint4) * 3 * (size_t)L.job_cap);
-    L.sjobs = take(sizeof(uint4) * B4);
-    L.hjobs = take(sizeof(uint4) * L.part_cap);
-    L.hj0 = take(sizeof(uint32_t) * L.huge_cap);
-    L.hbits = take(sizeof(uint32_t) * ((size_t)1 << kBucketLog2Max) / 32 * L.huge_cap);
-    L.pnv = take(sizeof(uint32_t) * L.part_cap);
-    // merge tasks: one per kMergeItems points of a split bucket, rounded up
-    L.mtask_cap = (uint32_t)(L.huge_cap + TS / kMergeItems + 1);
-    L.mtasks = take(sizeof(uint2) * L.mtask_cap);
-    L.scan_state = take(sizeof(unsigned long long) * ((size_t)L.scan_tiles + 2));
-    L.items = take(sizeof(uint2) * TS);
-    L.vdesc = take(sizeof(uint4) * TS);
-    L.vitems = take(sizeof(uint32_t) * TS);
-    L.out_slices = output_slices(L.buckets_per_frame);
-    L.ssum = take(sizeof(uint32_t) * F * L.out_slices);
+    L.fcnt = take(sizeof(uint32_t) * F);
     L.ftot = take(sizeof(uint32_t) * F);
-    L.bcap = take(sizeof(uint2) * B4);
+    L.hist = take(sizeof(uint32_t) * F * kMaxPasses * kDigits);
+    L.sort_state = take(sizeof(unsigned long long) * 2 * (size_t)L.sort_tiles_cap * kDigits);
+    L.run_state = take(sizeof(unsigned long long) * ((size_t)L.run_tiles_cap + 1));
+    L.vdesc = take(sizeof(uint4) * TS);
     L.total = o;
     (void)max_voxels;
     return L;
@@ -192,6 +168,13 @@ int validate_common(const float* points, const int64_t* sweep_offsets, int32_t n
         p->dims[a] = g->dims[a];
     }
     p->cells = (uint32_t)g->cells;
+    {
+        // 9-bit digits of the largest lin
+        const uint64_t maxlin = g->cells - 1ull;
+        int bits = 0;
+        while (bits < 64 && (maxlin >> bits) != 0ull) ++bits;
+        p->sort_passes = (bits + kDigitBits - 1) / kDigitBits;
+    }
     p->div_nx = udiv_make(g->dims[0]);
     p->div_ny = udiv_make(g->dims[1]);
     *max_rois_frame = rmax;
@@ -207,43 +190,32 @@ void bind_layout(Params* p, const Layout& L, uint8_t* ws) {
     p->roi_prep = reinterpret_cast<RoiPrep*>(ws + L.roi_prep);
     p->masks = reinterpret_cast<uint32_t*>(ws + L.masks);
     p->records = reinterpret_cast<uint4*>(ws + L.records);
-    p->plist = reinterpret_cast<uint4*>(ws + L.plist);
-    p->pdesc = reinterpret_cast<uint4*>(ws + L.plist);
     p->cls_cnt = reinterpret_cast<uint32_t*>(ws + L.cls_cnt);
     p->num_regions = (uint32_t)((p->num_points + kTile - 1) / kTile) * (kTile / kRegion);
-    p->bcnt = reinterpret_cast<uint32_t*>(ws + L.bcnt);
-    p->boff = reinterpret_cast<uint32_t*>(ws + L.boff);
-    p->ucnt = reinterpret_cast<uint32_t*>(ws + L.ucnt);
-    p->jobs = reinterpret_cast<uint4*>(ws + L.jobs);
-    p->sjobs = reinterpret_cast<uint4*>(ws + L.sjobs);
-    p->job_cap = L.job_cap;
-    p->hjobs = reinterpret_cast<uint4*>(ws + L.hjobs);
-    p->part_cap = L.part_cap;
-    p->hj0 = reinterpret_cast<uint32_t*>(ws + L.hj0);
-    p->hbits = reinterpret_cast<uint32_t*>(ws + L.hbits);
-    p->huge_cap = L.huge_cap;
-    p->pnv = reinterpret_cast<uint32_t*>(ws + L.pnv);
-    p->mtasks = reinterpret_cast<uint2*>(ws + L.mtasks);
-    p->mtask_cap = L.mtask_cap;
-    p->scan_state = reinterpret_cast<unsigned long long*>(ws + L.scan_state);
-    p->scan_tiles = L.scan_tiles;
-    p->items = reinterpret_cast<uint2*>(ws + L.items);
-    p->vdesc = reinterpret_cast<uint4*>(ws + L.vdesc);
-    p->vitems = reinterpret_cast<uint32_t*>(ws + L.vitems);
-    p->ssum = reinterpret_cast<uint32_t*>(ws + L.ssum);
-    p->ftot = reinterpret_cast<uint32_t*>(ws + L.ftot);
-    p->out_slices = L.out_slices;
-    p->bcap = reinterpret_cast<uint2*>(ws + L.bcap);
     p->rec_cap = p->num_regions * (uint32_t)kRegion;
-    p->item_cap = p->rec_cap;
+    p->rcnt = ws + L.rcnt;
+    p->ckey = reinterpret_cast<unsigned long long*>(ws + L.ckey);
+    p->key_b = reinterpret_cast<uint32_t*>(ws + L.ckey);
+    p->val_b = p->key_b + (size_t)p->rec_cap;
+    p->key_a = reinterpret_cast<uint32_t*>(ws + L.key_a);
+    p->val_a = reinterpret_cast<uint32_t*>(ws + L.val_a);
+    // pass k moves A to B for even k, B to A for odd k
+    const bool in_b = (p->sort_passes & 1) != 0;
+    p->skey = in_b ? p->key_b : p->key_a;
+    p->sval = in_b ? p->val_b : p->val_a;
+    p->fcnt = reinterpret_cast<uint32_t*>(ws + L.fcnt);
+    p->ftot = reinterpret_cast<uint32_t*>(ws + L.ftot);
+    p->hist = reinterpret_cast<uint32_t*>(ws + L.hist);
+    p->sort_state = reinterpret_cast<unsigned long long*>(ws + L.sort_state);
+    p->run_state = reinterpret_cast<unsigned long long*>(ws + L.run_state);
+    // room for the look-back words of the radix passes and of the numbering
+    p->sort_tiles_cap = L.sort_tiles_cap;
+    p->run_tiles_cap = L.run_tiles_cap;
+    p->vdesc = reinterpret_cast<uint4*>(ws + L.vdesc);
     p->mask_words = L.mask_words;
     p->coarse = L.coarse;
     p->coarse_inv[0] = (float)((double)L.coarse / ((double)p->rmax[0] - (double)p->rmin[0]));
     p->coarse_inv[1] = (float)((double)L.coarse / ((double)p->rmax[1] - (double)p->rmin[1]));
-    p->bucket_log2 = L.bucket_log2;
-    p->buckets_per_frame = L.buckets_per_frame;
-    p->div_bf = udiv_make(L.buckets_per_frame);
-    p->num_buckets = L.num_buckets;
 }
 
 #define MMBEV_TRY(expr)                                   \
@@ -252,7 +224,7 @@ void bind_layout(Params* p, const Layout& L, uint8_t* ws) {
     } while (0)
 
 const char* const kStageNames[MMBEV_NUM_STAGES] = {
-    "prep", "classify", "scan", "scatter", "buckets", "merge", "output"};
+    "prep", "classify", "compact", "sort", "runs", "emit"};
 
 }  // namespace
 
@@ -335,7 +307,6 @@ int voxelize_batched(const float* points, const int64_t* sweep_offsets, int32_t 
         p.rho_thr = rho >= 1.0f ? (1u << 24) : (uint32_t)std::floor((double)rho * 16777216.0);
         p.seed = opts->seed;
         p.inject_status = opts->inject_status;
-        p.merge_limit = opts->merge_buffer_words;
     }
 
     const int sms = num_sms();
@@ -363,15 +334,13 @@ int voxelize_batched(const float* points, const int64_t* sweep_offsets, int32_t 
         if ((e = mark()) != cudaSuccess) break;
         if ((e = launch_classify(p, rmax, sms, pdl, stream)) != cudaSuccess) break;
         if ((e = mark()) != cudaSuccess) break;
-        if ((e = launch_bucket_scan(p, pdl, stream)) != cudaSuccess) break;
+        if ((e = launch_compact(p, sms, pdl, stream)) != cudaSuccess) break;
         if ((e = mark()) != cudaSuccess) break;
-        if ((e = launch_bucket_scatter(p, sms, pdl, stream)) != cudaSuccess) break;
+        if ((e = launch_sort(p, sms, pdl, stream)) != cudaSuccess) break;
         if ((e = mark()) != cudaSuccess) break;
-        if ((e = launch_buckets(p, sms, pdl, stream)) != cudaSuccess) break;
+        if ((e = launch_runs(p, sms, pdl, stream)) != cudaSuccess) break;
         if ((e = mark()) != cudaSuccess) break;
-        if ((e = launch_merge(p, sms, pdl, stream)) != cudaSuccess) break;
-        if ((e = mark()) != cudaSuccess) break;
-        if ((e = launch_output(p, sms, pdl, stream)) != cudaSuccess) break;
+        if ((e = launch_emit(p, sms, pdl, stream)) != cudaSuccess) break;
         if ((e = mark()) != cudaSuccess) break;
     } while (0);
     return e == cudaSuccess ? MMBEV_OK : MMBEV_ECUDA;

@@ -10,26 +10,20 @@
 //               {x', y', z', intensity} {dt, ROI rank, -, -}. Region g holds
 //               points 32g .. 32g+31, so positions increase with the point
 //               index and "first K by position" is "first K by index".
-//   buckets     a frame's linear indices cut into buckets of 2^LB consecutive
-//               cells (LB <= 13); bucket b = frame * Bf + (lin >> LB) over the
-//               whole call, so ascending b is ascending (frame, lin).
-//   bcnt        workspace [B], kept points per bucket, counted by the
-//               classify pass (its atomic also numbers the point's arrival).
-//   plist       workspace, per classify block a dense list (any order) of its
-//               kept points {bucket, position, low bits of lin | rank << 16,
-//               arrival}, starting at the block's first tile * 2048; cls_cnt
-//               holds the lengths.
-//   boff        workspace [B + 1], exclusive prefix of bcnt over the call: the
-//               bucket's first item.
-//   items       workspace [M], the kept points grouped by bucket (counting
-//               sort by bucket): {position, low bits of lin | rank << 16}.
-//   vdesc       workspace [M], per bucket its voxels in ascending lin at
-//               boff[b] + v: {first vitem, point count, low lin bits,
-//               minimum rank}.
-//   vitems      workspace [M], each voxel's kept record positions (its K
-//               smallest), ascending, at the voxel's first vitem.
-//   ucnt        workspace [B], voxels per bucket; ssum [F][slices] voxels
-//               per slice of 512 buckets of a frame.
+//   rcnt, ckey  workspace, per region its kept points (one byte), and per
+//               record position the kept point's frame and lin
+//               (frame << 32 | lin), both written by classify.
+//   keys/vals   workspace, two buffers of M lins and M record positions: the
+//               kept points in position order (the compaction stage), so
+//               frame by frame, then after each 9-bit LSD radix pass, done
+//               within each frame, sorted by one more digit. Every pass is
+//               stable, so the last leaves each voxel's points together, in
+//               ascending lin, in ascending position. Frame f's items start
+//               at the sum of the kept counts fcnt of the frames before it.
+//   vdesc       workspace, voxel v of frame f at (frame f's first item) + v,
+//               voxels in ascending lin: {first item, end item, lin,
+//               minimum ROI rank}, the items being the voxel's run.
+//   ftot        workspace [F], voxels of each frame.
 //   workspace   Header + per-call arrays (see Layout in api.cu).
 #pragma once
 
@@ -53,19 +47,16 @@ constexpr int kRegion = 32;
 // Classify blocks (one per SM, at most this many).
 constexpr int kMaxClsGrid = 1000;
 
-// Buckets span 2^LB consecutive linear indices of one frame, LB at most this.
-constexpr int kBucketLog2Max = 13;
+// The kept points are sorted by lin within each frame with 9-bit digits:
+// at most four passes for grids of up to 2^32 cells.
+constexpr int kDigitBits = 9;
+constexpr int kDigits = 1 << kDigitBits;
+constexpr int kMaxPasses = 4;
+constexpr uint32_t kNoLin = 0xFFFFFFFFu;   // above every lin (cells < 2^32)
 
-// The bucket scan works in tiles of this many buckets (1024 threads x 4).
-constexpr uint32_t kScanTile = 4096;
-
-// Bucket sizes: up to kWarpJobMax kept points a bucket is one warp's work,
-// up to kPart one block's; a larger bucket is split into parts of kPart
-// points (a block each) whose voxel lists the merge stage combines, one
-// merge task per kMergeItems points (each a range of the low lin bits).
-constexpr uint32_t kWarpJobMax = 256;
-constexpr uint32_t kPart = 2048;
-constexpr uint32_t kMergeItems = 8192;
+// Tiles of the radix passes and of the voxel numbering (within one frame).
+constexpr uint32_t kSortTile = 4096;
+constexpr uint32_t kRunTile = 2048;
 
 // Bounded waits.
 constexpr uint32_t kSpinLimit = 1u << 22;
@@ -105,15 +96,9 @@ struct __align__(16) RoiPrep {
 struct __align__(16) Header {
     uint32_t status;        // MMBEV_DEV_* bits (first word: read by mmbev_get_status)
     uint32_t num_rec;       // kept points (records) of the call
-    uint32_t scan_ticket;   // scan tiles started, in order
-    uint32_t n_large[3];    // block jobs of 1,025-2,048, 513-1,024 and 257-512 points
-    uint32_t n_small;       // warp jobs: buckets of 1 .. kWarpJobMax points
-    uint32_t large_ticket;  // parts, then block jobs (largest class first), taken by the bucket stage
-    uint32_t n_huge;        // buckets split in parts
-    uint32_t n_parts;       // parts of the split buckets
-    uint32_t n_mtasks;      // merge tasks: ranges of low lin bits of split buckets
-    uint32_t small_ticket;  // warp jobs taken by the bucket stage
-    uint32_t pad[4];
+    uint32_t run_ticket;    // voxel numbering tiles started, in order
+    uint32_t sort_ticket[kMaxPasses];   // radix pass tiles started, in order
+    uint32_t pad[3];
 };
 
 // Everything a kernel needs; passed by value.
@@ -142,13 +127,8 @@ struct Params {
     uint64_t seed;          // SplitMix64 seed of those draws
     int32_t keep_status = 0;  // prep leaves the status word as it is (later chunks of a call)
     uint32_t inject_status = 0;  // test hook: status bits prep sets as a failure would
-    uint32_t merge_limit = 0;    // test hook: the merge's buffer words (0: all it has)
-    // buckets
-    int32_t bucket_log2;       // LB
-    uint32_t buckets_per_frame;  // Bf
-    UDiv div_bf;               // division by Bf (bucket -> frame)
-    uint32_t num_buckets;      // B = F * Bf
-    uint32_t scan_tiles;       // ceil(B / kScanTile)
+    // the sort of the kept points
+    int32_t sort_passes;       // 9-bit digits of the largest lin
     // workspace arrays
     Header* hdr;
     int64_t* sweep_off;     // [S+1]
@@ -158,35 +138,26 @@ struct Params {
     RoiPrep* roi_prep;      // [R]
     uint32_t* masks;        // [F][coarse^2][mask_words]
     uint4* records;         // [regions*32][2] kept points' features and rank
-    uint4* plist;           // [tiles*2048] per classify block: {bucket, pos, lo|rank<<16, -}
-    uint4* pdesc;           // [tiles*2048] voxel lists of the parts of split buckets (aliases plist)
-    uint32_t* cls_cnt;      // [kMaxClsGrid] list length of each classify block
+    uint32_t* cls_cnt;      // [kMaxClsGrid] kept points of each classify block
     uint32_t cls_grid;      // classify blocks of the call
     uint32_t num_regions;
     uint32_t rec_cap;       // record positions of the call (regions * 32)
-    uint32_t* bcnt;         // [B] kept points per bucket
-    uint32_t* boff;         // [B + 1] first item of each bucket
-    uint32_t* ucnt;         // [B] voxels per bucket
-    uint4* jobs;            // [3][job_cap] block jobs by size class {bucket, first item, points, ~0}
-    uint4* sjobs;           // [B] warp jobs {bucket, first item, points, -}
-    uint32_t job_cap;
-    uint4* hjobs;           // [part_cap] parts {bucket, first item, points, split index}
-    uint32_t part_cap;
-    uint32_t* hj0;          // [huge_cap] first part of each split bucket
-    uint32_t* hbits;        // [huge_cap][2^kBucketLog2Max / 32] union occupancy of each split bucket
-    uint32_t huge_cap;
-    uint32_t* pnv;          // [part_cap] voxels of each part
-    uint2* mtasks;          // [mtask_cap] merge tasks {split index, range | ranges << 16}
-    uint32_t mtask_cap;
-    unsigned long long* scan_state;  // [scan_tiles] look-back words of the bucket scan
-    uint2* items;           // [rec_cap] kept points grouped by bucket
-    uint4* vdesc;           // [rec_cap] voxel descriptors grouped by bucket
-    uint32_t* vitems;       // [rec_cap] kept positions of each voxel
-    uint32_t* ssum;         // [F * out_slices] voxels per frame slice
-    uint32_t* ftot;         // [F] voxels per frame
-    uint32_t out_slices;    // slices of 512 buckets per frame
-    uint2* bcap;            // [B] capped frames: voxels below / at the threshold rank
-    uint32_t item_cap;      // room of items, vdesc and vitems (rec_cap)
+    uint8_t* rcnt;          // [regions] kept points of each region
+    unsigned long long* ckey;   // [rec_cap] frame << 32 | lin of the kept point at each position
+    uint32_t* key_a;        // [rec_cap] lins, buffer A (the compaction writes it)
+    uint32_t* val_a;        // [rec_cap] record positions, buffer A
+    uint32_t* key_b;        // [rec_cap] buffer B (with val_b, aliases ckey)
+    uint32_t* val_b;
+    const uint32_t* skey;   // the sorted buffer (A or B by the pass count)
+    const uint32_t* sval;
+    uint32_t* fcnt;         // [F] kept points of each frame
+    uint32_t* ftot;         // [F] voxels of each frame
+    uint32_t* hist;         // [F][kMaxPasses][kDigits] digit histograms of each frame's lins
+    unsigned long long* sort_state;   // [2][sort_tiles_cap][kDigits] look-back words of the passes
+    unsigned long long* run_state;    // [run_tiles_cap] look-back words of the voxel numbering
+    uint32_t sort_tiles_cap;  // tiles of a pass, at most (one more a frame for the ragged ends)
+    uint32_t run_tiles_cap;
+    uint4* vdesc;           // [rec_cap] per voxel: {first item, end item, lin, minimum rank}
     // outputs
     float* out_feats;
     int32_t* out_coords;
@@ -373,12 +344,12 @@ cudaError_t launch_prep_rois(const mmbev_roi_t* rois, int32_t n, float margin, f
                              cudaStream_t st);
 cudaError_t launch_classify(const Params& p, int rmax, int num_sms, bool pdl, cudaStream_t st);
 cudaError_t launch_classify_points(const Params& p, cudaStream_t st);
-cudaError_t launch_bucket_scan(const Params& p, bool pdl, cudaStream_t st);
-cudaError_t launch_bucket_scatter(const Params& p, int num_sms, bool pdl, cudaStream_t st);
-cudaError_t launch_buckets(const Params& p, int num_sms, bool pdl, cudaStream_t st);
-cudaError_t launch_merge(const Params& p, int num_sms, bool pdl, cudaStream_t st);
-cudaError_t launch_output(const Params& p, int num_sms, bool pdl, cudaStream_t st);
-uint32_t output_slices(uint32_t buckets_per_frame);   // slices of a frame for the output stage
+// The stages after classify (csrc/sort.cu): compaction and digit histograms,
+// the radix passes, voxel numbering, output rows.
+cudaError_t launch_compact(const Params& p, int num_sms, bool pdl, cudaStream_t st);
+cudaError_t launch_sort(const Params& p, int num_sms, bool pdl, cudaStream_t st);
+cudaError_t launch_runs(const Params& p, int num_sms, bool pdl, cudaStream_t st);
+cudaError_t launch_emit(const Params& p, int num_sms, bool pdl, cudaStream_t st);
 // Kept rows of frames [f0, f1) of a call's outputs into a packed buffer
 // (mmbev_pack_voxels' layout for F frames).
 cudaError_t launch_pack(const float* feats, const int32_t* coords, const int32_t* counts,

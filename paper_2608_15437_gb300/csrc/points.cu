@@ -21,12 +21,10 @@
 // sit in shared memory. Kept points are compacted per 32-point region with
 // warp ballots, in input order: position (region)*32 + (rank among the
 // region's kept points) gets a 32-byte record with the compensated features
-// and the ROI rank, so later stages never touch the raw points again. The
-// point is counted into its bucket of 2^LB consecutive linear indices of its
-// frame (one global add per group of the warp's points in a bucket), and the
-// block appends {bucket, position, low lin bits | rank} to its own dense list
-// (order immaterial), from which the scatter stage sorts the kept points by
-// bucket.
+// and the ROI rank, so later stages never touch the raw points again, and the
+// point's frame and lin (frame << 32 | lin). Every region's kept count goes to a
+// byte array, from which the compaction stage gathers the keys in position
+// order.
 //
 // The classify-only entry point (per-point outputs for testing S1-S2) uses a
 // plain one-thread-per-point kernel built from the same device functions.
@@ -38,7 +36,6 @@ namespace mmbev {
 namespace {
 
 constexpr int kThreads = 1024;
-constexpr int kWarps = kThreads / 32;         // 32
 constexpr int kTileChunks = kTile / 64;       // 64-point chunks per tile (32)
 constexpr int kTfStageMax = 512;              // sweeps whose transforms sit in smem
 constexpr int kMaskSmemWords = 8192;          // largest staged coarse mask of a frame (32 KB)
@@ -72,6 +69,14 @@ __device__ __forceinline__ bool mbar_try_wait(uint64_t* bar, uint32_t parity) {
         : "r"(smem_addr(bar)), "r"(parity)
         : "memory");
     return ok != 0;
+}
+__device__ __forceinline__ uint64_t evict_last_policy() {
+    uint64_t pol;
+    asm volatile("createpolicy.fractional.L2::evict_last.b64 %0, 1.0;" : "=l"(pol));
+    return pol;
+}
+__device__ __forceinline__ void st_u64_hint(unsigned long long* a, unsigned long long v, uint64_t pol) {
+    asm volatile("st.global.L2::cache_hint.u64 [%0], %1, %2;" ::"l"(a), "l"(v), "l"(pol) : "memory");
 }
 __device__ __forceinline__ uint64_t evict_first_policy() {
     uint64_t pol;
@@ -187,7 +192,6 @@ __device__ __forceinline__ bool classify_range(const Params& p, const ClsSmem& s
     const uint64_t pol = evict_first_policy();
     const uint32_t lt = (1u << lane) - 1u;
     const uint32_t half_mask = lane < 16 ? 0x0000FFFFu : 0xFFFF0000u;
-    uint4* plist = p.plist + t_begin * kTile;   // room for every point of the range
     const uint32_t nchunks = (uint32_t)(t_end - t_begin) * (uint32_t)kTileChunks;
     const uint32_t tb = (uint32_t)t_begin;
     // the sweep of this lane's current point and what depends on it (points
@@ -254,7 +258,27 @@ __device__ __forceinline__ bool classify_range(const Params& p, const ClsSmem& s
         const uint32_t i0 = base + j0;   // the lane's first point
         float2 v0, v1, v2, v3, v4;
         if (tile < full_tiles) {
-            if (!mbar_wait(&sm.full[st], round & 1u)) {
+            // A phase-parity wait only tells the phase it waits for from the
+            // one before it. Chunks are handed out up to two per warp (64
+            // chunks, two tiles) ahead of their buffers, and nothing orders
+            // the arrival of tiles in flight: when later tiles land and are
+            // done first, a warp can hold a chunk of a buffer's next round
+            // before the current round's tile has landed, and would see the
+            // previous round's phase as its own (with a ring of two buffers
+            // that takes no reordering at all). So it first waits (bounded)
+            // until every chunk of the buffer's previous round has released
+            // it; the previous phase has completed by then.
+            bool ok = true;
+            if (round > 0u) {
+                uint32_t spins = 0;
+                while (*reinterpret_cast<volatile uint32_t*>(&sm.done[st]) <
+                       round * (uint32_t)kTileChunks)
+                    if (++spins >= kSpinLimit) {
+                        ok = false;
+                        break;
+                    }
+            }
+            if (!ok || !mbar_wait(&sm.full[st], round & 1u)) {
                 if (lane == 0) {
                     set_status(p.hdr, MMBEV_DEV_WAIT_TIMEOUT);
                     atomicExch(&sm.kept[3], 1u);
@@ -366,36 +390,31 @@ __device__ __forceinline__ bool classify_range(const Params& p, const ClsSmem& s
         const uint32_t below = lt & half_mask;
         const uint32_t rank0 = __popc(b0 & below) + __popc(b1 & below);
         const uint32_t region = tile * (uint32_t)(kTile / kRegion) + sub * 2u + (uint32_t)(lane >> 4);
-        // the block's dense list of kept points (any order): one shared
-        // atomic per warp reserves the warp's entries
+        // every region's kept count, so the compaction stage can find the
+        // kept points' keys in position order
+        if ((lane & 15) == 0)
+            p.rcnt[region] = (uint8_t)(__popc(b0 & half_mask) + __popc(b1 & half_mask));
         const uint32_t nk = __popc(b0) + __popc(b1);
         if (nk == 0u) {   // warp-uniform: nothing kept in the chunk
             c = __shfl_sync(0xFFFFFFFFu, cn, 0);
             continue;
         }
-        uint32_t lbase = 0;
-        if (lane == 0) lbase = atomicAdd(&sm.kept[0], nk);
-        lbase = __shfl_sync(0xFFFFFFFFu, lbase, 0);
-        const uint32_t lo_mask = (1u << p.bucket_log2) - 1u;
+        if (lane == 0) atomicAdd(&sm.kept[0], nk);
 #pragma unroll
         for (int k = 0; k < 2; ++k) {
-            // the point's bucket, counted once per group of the warp's points
-            // that share it (no return value: the add does not stall the warp)
-            const uint32_t bk =
-                valid[k] ? frk[k] * p.buckets_per_frame + (lin[k] >> p.bucket_log2) : kUnset;
-            const uint32_t grp = __match_any_sync(0xFFFFFFFFu, bk);
-            if (valid[k] && lane == __ffs(grp) - 1) atomicAdd(&p.bcnt[bk], (uint32_t)__popc(grp));
             if (valid[k]) {
                 const uint32_t rk = rank0 + (k ? (uint32_t)valid[0] : 0u);
                 const uint32_t at = region * (uint32_t)kRegion + rk;
-                const uint32_t li = lbase + (k ? __popc(b0) + __popc(b1 & lt) : __popc(b0 & lt));
-                // records are read again only by the bucket stage: streaming
-                // stores leave L2 to the lists and counters in between
+                // records are read again only by the output stage: streaming
+                // stores leave L2 to the keys in between
                 uint4* rec = p.records + 2 * (size_t)at;
                 __stcs(rec, make_uint4(__float_as_uint(x[k]), __float_as_uint(y[k]),
                                        __float_as_uint(z[k]), __float_as_uint(pi[k])));
                 __stcs(rec + 1, make_uint4(__float_as_uint(pd[k]), (uint32_t)hit[k], 0u, 0u));
-                plist[li] = make_uint4(bk, at, (lin[k] & lo_mask) | ((uint32_t)hit[k] << 16), 0u);
+                // the sort key: the frame, the voxel's lin; kept in L2 past
+                // the input stream for the compaction stage that reads it next
+                st_u64_hint(p.ckey + at, (unsigned long long)frk[k] << 32 | lin[k],
+                            evict_last_policy());
             }
         }
         c = __shfl_sync(0xFFFFFFFFu, cn, 0);

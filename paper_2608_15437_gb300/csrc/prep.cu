@@ -6,7 +6,7 @@
 // whose margin-grown box may touch the cell. The mask is conservative (the
 // exact per-point test of Alg. 1 follows), so it only prunes work. The other
 // blocks copy the host offsets into the workspace and zero the per-call
-// counters.
+// counters and the digit histograms.
 #include <atomic>
 #include <cmath>
 
@@ -114,17 +114,13 @@ k_prep(Params p, const __grid_constant__ HostDesc d) {
     }
     if (p.cls_cnt)
         for (size_t i = gt; i < (size_t)kMaxClsGrid; i += gs) p.cls_cnt[i] = 0u;
-    if (p.scan_state)
-        for (size_t i = gt; i < (size_t)p.scan_tiles; i += gs) p.scan_state[i] = 0ull;
-    if (p.ssum)
-        for (size_t i = gt; i < (size_t)p.num_frames * p.out_slices; i += gs) p.ssum[i] = 0u;
+    // the per-frame counts and digit histograms start at zero
+    if (p.hist)
+        for (size_t i = gt; i < (size_t)p.num_frames * kMaxPasses * kDigits; i += gs) p.hist[i] = 0u;
+    if (p.fcnt)
+        for (size_t i = gt; i < (size_t)p.num_frames; i += gs) p.fcnt[i] = 0u;
     if (p.ftot)
         for (size_t i = gt; i < (size_t)p.num_frames; i += gs) p.ftot[i] = 0u;
-    if (p.bcnt) {
-        uint4* b4 = reinterpret_cast<uint4*>(p.bcnt);  // B counters, padded to a multiple of 4
-        const size_t n4 = ((size_t)p.num_buckets + 3) / 4;
-        for (size_t i = gt; i < n4; i += gs) b4[i] = make_uint4(0u, 0u, 0u, 0u);
-    }
 }
 
 // One thread per ROI: the prepared form the classify pass tests against.

@@ -17,7 +17,7 @@ def to_dev(w, dev, rois=None):
 
 
 def run_gpu(mmbev, w, dev, K=None, maxv=None, inject_status=0, workspace=None,
-            stream=None, rho_out=0.0, seed=0, merge_buffer_words=0):
+            stream=None, rho_out=0.0, seed=0):
     """Batched C-ABI call on w; returns (per-frame list of (feats, coords,
     counts), device status, workspace)."""
     import torch
@@ -33,8 +33,7 @@ def run_gpu(mmbev, w, dev, K=None, maxv=None, inject_status=0, workspace=None,
                                      w.pc_range, K, maxv, w.frame_sweep_offsets,
                                      w.frame_roi_offsets, workspace=workspace,
                                      inject_status=inject_status, stream=stream,
-                                     rho_out=rho_out, seed=seed,
-                                     merge_buffer_words=merge_buffer_words)
+                                     rho_out=rho_out, seed=seed)
     torch.cuda.synchronize(dev)
     status = mmbev.get_status(workspace)
     nvox = out.nvox.cpu().numpy()

@@ -223,7 +223,7 @@ def test_scatter_bev_update_checks_its_arguments(mmbev_lib):
 def test_stage_names_follow_the_launch_order(mmbev_lib):
     # one name per kernel of a call, in launch order; out of range: empty
     names = mmbev_lib.stage_names()
-    assert names == ["prep", "classify", "scan", "scatter", "buckets", "merge", "output"]
+    assert names == ["prep", "classify", "compact", "sort", "runs", "emit"]
     lib = mmbev_lib.load()
     assert lib.mmbev_stage_name(mmbev_lib.NUM_STAGES) == b""
     assert lib.mmbev_stage_name(-1) == b""

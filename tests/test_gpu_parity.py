@@ -110,14 +110,14 @@ def test_batch32_parity(oracle_mod, mmbev_lib, cuda_dev):
     assert assert_frames_equal(got, want, "batch32") == 1.0
 
 
-_SPLIT = {}
+_DENSE = {}
 
 
-def _split_workload(oracle_mod):
-    """Four batch frames, checked (oracle side, once) to have buckets split
-    in parts: more than 2,048 kept points among 2^13 consecutive linear
-    indices of one frame."""
-    if "w" not in _SPLIT:
+def _dense_workload(oracle_mod):
+    """Four batch frames, checked (oracle side, once) to hold a voxel of more
+    than 4,096 kept points: its run in the sorted keys spans more than one
+    tile of a radix pass (4,096 items) and of the voxel numbering (2,048)."""
+    if "w" not in _DENSE:
         w = synth.streaming_batch(4)
         big = 0
         for f in range(w.num_frames):
@@ -126,25 +126,22 @@ def _split_workload(oracle_mod):
                                             fr.roi_margin, fr.voxel_size, fr.pc_range)
             kept = lin[lin >= 0]
             if kept.size:
-                big = max(big, int(np.bincount(kept >> 13).max()))
-        _SPLIT["w"], _SPLIT["big"] = w, big
-    assert _SPLIT["big"] > 2048
-    return _SPLIT["w"]
+                big = max(big, int(np.unique(kept, return_counts=True)[1].max()))
+        _DENSE["w"], _DENSE["big"] = w, big
+    assert _DENSE["big"] > 4096
+    return _DENSE["w"]
 
 
-@pytest.mark.parametrize("K,words", [(10, 16), (10, 200), (10, 3000), (20, 0), (33, 0),
-                                     (33, 200), (64, 0), (64, 64)])
-def test_merge_windows_and_overflow(oracle_mod, mmbev_lib, cuda_dev, K, words):
-    """Buckets split in parts merged at every K instantiation, with the
-    merge's full buffer (words = 0) or a small one: windows of voxels, voxels
-    whose candidates overflow the buffer (merged in K slots) and tasks whose
-    entries overflow their stash (read again) all take their fallback paths,
-    and the results stay those of the oracle."""
-    w = _split_workload(oracle_mod)
+@pytest.mark.parametrize("K", [1, 10, 33, 64])
+def test_dense_voxels_across_tiles(oracle_mod, mmbev_lib, cuda_dev, K):
+    """Runs of thousands of points (one voxel) across radix and numbering
+    tiles keep their first K points by index, at every output instantiation
+    that the K values select."""
+    w = _dense_workload(oracle_mod)
     want = run_oracle(oracle_mod, w, K=K)
-    got, status, _ = run_gpu(mmbev_lib, w, cuda_dev, K=K, merge_buffer_words=words)
+    got, status, _ = run_gpu(mmbev_lib, w, cuda_dev, K=K)
     assert status == 0
-    assert assert_frames_equal(got, want, f"K={K}, merge buffer {words}") == 1.0
+    assert assert_frames_equal(got, want, f"dense voxels, K={K}") == 1.0
 
 
 # ------------------------------------------------------------------ cap path
