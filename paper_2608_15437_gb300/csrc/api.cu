@@ -59,7 +59,7 @@ int coarse_for(int mask_words) {
 // Byte offsets of every workspace array for one call shape.
 struct Layout {
     size_t hdr, sweep_off, sweep_frame, fso, fro, roi_prep, masks;
-    size_t records, ckey, key_a, val_a, rcnt, cls_cnt, fcnt, ftot, hist, sort_state,
+    size_t records, ckey, key_a, val_a, rcnt, cls_cnt, cls_flo, fcnt, ftot, hist, sort_state,
         run_state, vdesc;
     size_t total;
     uint32_t num_tiles, sort_tiles_cap, run_tiles_cap;
@@ -104,6 +104,7 @@ Layout make_layout(int64_t max_points, int64_t rois_total, int32_t max_rois_fram
     L.val_a = take(sizeof(uint32_t) * TS);
     L.rcnt = take(regions);
     L.cls_cnt = take(sizeof(uint32_t) * kMaxClsGrid);
+    L.cls_flo = take(sizeof(uint32_t) * kMaxClsGrid);
     L.fcnt = take(sizeof(uint32_t) * F);
     L.ftot = take(sizeof(uint32_t) * F);
     L.hist = take(sizeof(uint32_t) * F * kMaxPasses * kDigits);
@@ -191,6 +192,7 @@ void bind_layout(Params* p, const Layout& L, uint8_t* ws) {
     p->masks = reinterpret_cast<uint32_t*>(ws + L.masks);
     p->records = reinterpret_cast<uint4*>(ws + L.records);
     p->cls_cnt = reinterpret_cast<uint32_t*>(ws + L.cls_cnt);
+    p->cls_flo = reinterpret_cast<uint32_t*>(ws + L.cls_flo);
     p->num_regions = (uint32_t)((p->num_points + kTile - 1) / kTile) * (kTile / kRegion);
     p->rec_cap = p->num_regions * (uint32_t)kRegion;
     p->rcnt = ws + L.rcnt;

@@ -139,6 +139,7 @@ struct Params {
     uint32_t* masks;        // [F][coarse^2][mask_words]
     uint4* records;         // [regions*32][2] kept points' features and rank
     uint32_t* cls_cnt;      // [kMaxClsGrid] kept points of each classify block
+    uint32_t* cls_flo;      // [kMaxClsGrid] frame of each classify block's first point
     uint32_t cls_grid;      // classify blocks of the call
     uint32_t num_regions;
     uint32_t rec_cap;       // record positions of the call (regions * 32)

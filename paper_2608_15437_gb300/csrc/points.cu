@@ -498,10 +498,12 @@ __global__ void __launch_bounds__(kThreads, 1) k_classify(Params p, int rmax, in
             if (k > 0) (void)mbar_wait(&sm.full[s], (k - 1u) & 1u);
         }
         p.cls_cnt[blockIdx.x] = 0u;
+        p.cls_flo[blockIdx.x] = (uint32_t)f_lo;
         return;
     }
     const uint32_t tot = sm.kept[0];
     p.cls_cnt[blockIdx.x] = tot;
+    p.cls_flo[blockIdx.x] = (uint32_t)f_lo;
     if (tot) atomicAdd(&p.hdr->num_rec, tot);
 }
 

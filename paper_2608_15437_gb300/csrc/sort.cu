@@ -182,27 +182,33 @@ __device__ __forceinline__ uint32_t tile_frame(const uint32_t* s_tpre, uint32_t 
 
 constexpr int kCT = 1024;                      // threads of a compaction block
 constexpr int kCW = kCT / 32;
-constexpr int kCU = 4;                         // entries a lane moves at once
-constexpr uint32_t kCRound = 4 * kCT;          // regions a round (four a thread)
+constexpr uint32_t kCRound = 2 * kCT;          // regions a round (two a thread)
+constexpr int kCU = 4;                         // entries a thread moves at once
+// dynamic shared memory: a round's entry -> region table (two bytes an
+// entry), its regions' first entries, the range's first two frames' digit
+// histograms
+constexpr size_t kCTabBytes = (size_t)kCRound * kRegion * 2;
+constexpr size_t kCSmem = kCTabBytes + (size_t)kCRound * 4 + 2 * (size_t)kMaxPasses * kDigits * 4;
 
 // A block per classify block: it takes the same range of point tiles, whose
 // kept points are the ones after those of the classify blocks before it
 // (their kept counts), so no block waits for another. In rounds of kCRound
-// regions, a thread holds four consecutive regions' kept counts and a block
-// scan gives each region its first dense index; the round's kept points are
-// then split evenly over the warps, kCU * 32 at a time a warp (the region of
-// entry e by a binary search over the threads' prefixes in shared memory, all
-// loads issued before any is used), moving lin and position into buffer A. The range's kept counts
-// and digit histograms go to shared memory for its first two frames (the
-// range's points hold at most two frames unless frames are small; other
-// frames' counts go straight to global memory), then to the frames' totals.
+// regions, a thread holds two regions' kept counts; a block scan gives each
+// region its first entry, and a table in shared memory the region of every
+// entry of the round. Thread t then moves entries t, t + kCT, ... (lin and
+// position, into buffer A at the range's first index + the entry), counting
+// each into its frame's kept count and digit histograms (shared memory for
+// the range's first two frames, which are all its frames unless frames are
+// small; others straight to global memory), added to the frames' totals at
+// the end.
 __global__ void __launch_bounds__(kCT) k_compact(Params p) {
+    extern __shared__ __align__(16) unsigned char c_smem[];
+    uint16_t* s_tab = reinterpret_cast<uint16_t*>(c_smem);
+    uint32_t* s_rpre = reinterpret_cast<uint32_t*>(c_smem + kCTabBytes);
+    uint32_t* s_h = s_rpre + kCRound;   // [2][kMaxPasses * kDigits]
     __shared__ uint32_t s_warp[kCW];
-    __shared__ uint32_t s_h[2][kMaxPasses * kDigits];
     __shared__ uint32_t s_fc[2];
     __shared__ uint32_t s_base;
-    __shared__ uint32_t s_tp[kCT];   // per thread of a round: first entry of its four regions
-    __shared__ uint32_t s_tc[kCT];   // their kept counts, a byte each
     pdl_wait();
     const int t = threadIdx.x, lane = t & 31;
     const uint32_t M = p.hdr->num_rec;
@@ -217,7 +223,7 @@ __global__ void __launch_bounds__(kCT) k_compact(Params p) {
         const size_t rt = min((size_t)(M + kRunTile - 1) / kRunTile + F, (size_t)p.run_tiles_cap);
         for (size_t i = gt; i < rt; i += gs) p.run_state[i] = 0ull;
     }
-    for (int i = t; i < 2 * kMaxPasses * kDigits; i += kCT) (&s_h[0][0])[i] = 0u;
+    for (int i = t; i < 2 * kMaxPasses * kDigits; i += kCT) s_h[i] = 0u;
     if (t < 2) s_fc[t] = 0u;
     {
         // kept points of the classify blocks before this one
@@ -226,65 +232,49 @@ __global__ void __launch_bounds__(kCT) k_compact(Params p) {
         (void)block_exclusive_scan(x, s_warp, &tot);
         if (t == 0) s_base = tot;
     }
-    // the classify block's range of point tiles, split as the classify kernel splits it
+    // the classify block's range of point tiles, split as the classify kernel
+    // splits it, and the frame of its first point
     const uint64_t num_tiles = ((uint64_t)p.num_points + kTile - 1) / kTile;
     const uint64_t t0 = (uint64_t)blockIdx.x * num_tiles / gridDim.x;
     const uint64_t t1 = ((uint64_t)blockIdx.x + 1) * num_tiles / gridDim.x;
     const uint32_t r0 = (uint32_t)t0 * (kTile / kRegion), r1 = (uint32_t)t1 * (kTile / kRegion);
-    const uint32_t f_lo =
-        t0 < t1 ? (uint32_t)p.sweep_frame[find_sweep(p.sweep_off, p.num_sweeps, (int64_t)t0 * kTile)] : 0u;
+    const uint32_t f_lo = p.cls_flo[blockIdx.x];
     __syncthreads();
     uint32_t carry = s_base;
     for (uint32_t rb = r0; rb < r1; rb += kCRound) {   // block-uniform
-        const uint32_t ra = rb + 4u * (uint32_t)t;
-        uint32_t c[4] = {0u, 0u, 0u, 0u};
-        if (ra < r1) {   // r0 and r1 are multiples of 64: four counts in one word
-            const uint32_t w4 = reinterpret_cast<const uint32_t*>(p.rcnt)[ra >> 2];
-#pragma unroll
-            for (int k = 0; k < 4; ++k) c[k] = min((w4 >> (8 * k)) & 0xFFu, (uint32_t)kRegion);
+        const uint32_t ra = rb + 2u * (uint32_t)t;
+        uint32_t c0 = 0u, c1 = 0u;
+        if (ra < r1) {   // r0 and r1 are even: two counts in one 16-bit word
+            const uint32_t w2 = reinterpret_cast<const uint16_t*>(p.rcnt)[ra >> 1];
+            c0 = min(w2 & 0xFFu, (uint32_t)kRegion);
+            c1 = min(w2 >> 8, (uint32_t)kRegion);
         }
-        const uint32_t sum = c[0] + c[1] + c[2] + c[3];
         uint32_t tot = 0;
-        const uint32_t excl = block_exclusive_scan(sum, s_warp, &tot);
-        // the round's entries, split evenly over the warps (kept points
-        // crowd into few regions); entry e belongs to the thread with the
-        // largest prefix <= e, then to one of its four regions
-        s_tp[t] = excl;
-        s_tc[t] = c[0] | c[1] << 8 | c[2] << 16 | c[3] << 24;
+        const uint32_t excl = block_exclusive_scan(c0 + c1, s_warp, &tot);
+        s_rpre[2 * t] = excl;
+        s_rpre[2 * t + 1] = excl + c0;
+        for (uint32_t j = 0; j < c0; ++j) s_tab[excl + j] = (uint16_t)(2 * t);
+        for (uint32_t j = 0; j < c1; ++j) s_tab[excl + c0 + j] = (uint16_t)(2 * t + 1);
         __syncthreads();
-        const uint32_t warp = (uint32_t)t >> 5;
-        const uint32_t w0 = (uint32_t)((uint64_t)tot * warp / kCW);
-        const uint32_t w1 = (uint32_t)((uint64_t)tot * (warp + 1u) / kCW);
-        for (uint32_t e0 = w0; e0 < w1; e0 += 32u * kCU) {
+        for (uint32_t e0 = 0; e0 < tot; e0 += kCU * kCT) {   // block-uniform
+            // kCU entries a thread, their loads issued before any is used
             uint32_t pos[kCU];
             unsigned long long key[kCU];
 #pragma unroll
             for (int u = 0; u < kCU; ++u) {
-                const uint32_t e = e0 + 32u * u + (uint32_t)lane;
-                uint32_t th = 0;
-#pragma unroll
-                for (uint32_t st = kCT / 2; st > 0; st >>= 1)
-                    if (s_tp[th + st] <= e) th += st;
-                const uint32_t w4 = s_tc[th];
-                uint32_t off = e - s_tp[th], k = 0;
-#pragma unroll
-                for (int q = 0; q < 3; ++q) {
-                    const uint32_t cq = (w4 >> (8 * q)) & 0xFFu;
-                    if (k == (uint32_t)q && off >= cq) {
-                        off -= cq;
-                        ++k;
-                    }
-                }
-                pos[u] = e < w1 ? (rb + 4u * th + k) * (uint32_t)kRegion + off : kUnset;
-                key[u] = pos[u] < p.rec_cap ? p.ckey[pos[u]] : ~0ull;
+                const uint32_t e = e0 + (uint32_t)u * kCT + (uint32_t)t;
+                const uint32_t r = e < tot ? s_tab[e] : 0u;
+                pos[u] = (rb + r) * (uint32_t)kRegion + (e - s_rpre[r]);
+                key[u] = e < tot && pos[u] < p.rec_cap ? p.ckey[pos[u]] : ~0ull;
             }
 #pragma unroll
             for (int u = 0; u < kCU; ++u) {
-                const uint32_t e = e0 + 32u * u + (uint32_t)lane;
+                const uint32_t e = e0 + (uint32_t)u * kCT + (uint32_t)t;
+                const bool in = e < tot;
                 const uint32_t f = (uint32_t)(key[u] >> 32), lin = (uint32_t)key[u];
                 const uint32_t d = carry + e;
-                const bool ok = e < w1 && pos[u] < p.rec_cap && f < F && d < p.rec_cap;
-                if (e < w1 && !ok) set_status(p.hdr, MMBEV_DEV_BOUNDS);
+                const bool ok = in && pos[u] < p.rec_cap && f < F && d < p.rec_cap;
+                if (in && !ok) set_status(p.hdr, MMBEV_DEV_BOUNDS);
                 if (ok) {
                     p.key_a[d] = lin;
                     p.val_a[d] = pos[u];
@@ -301,21 +291,21 @@ __global__ void __launch_bounds__(kCT) k_compact(Params p) {
                 if (ok) {
                     for (int q = 0; q < P; ++q) {
                         const uint32_t dg = (lin >> (kDigitBits * q)) & (kDigits - 1u);
-                        if (slot <= 1u) atomicAdd(&s_h[slot][q * kDigits + dg], 1u);
+                        if (slot <= 1u) atomicAdd(&s_h[slot * kMaxPasses * kDigits + q * kDigits + dg], 1u);
                         else atomicAdd(&p.hist[((size_t)f * kMaxPasses + q) * kDigits + dg], 1u);
                     }
                 }
             }
         }
-        __syncthreads();   // s_tp and s_tc are rewritten by the next round
         carry += tot;
+        __syncthreads();   // the table is rewritten by the next round
     }
-    __syncthreads();
     for (uint32_t slot = 0; slot < 2u; ++slot) {
         const uint32_t f = f_lo + slot;
         if (f >= F) break;
+        const uint32_t* h = s_h + slot * kMaxPasses * kDigits;
         for (int i = t; i < P * kDigits; i += kCT)
-            if (s_h[slot][i]) atomicAdd(&p.hist[(size_t)f * kMaxPasses * kDigits + i], s_h[slot][i]);
+            if (h[i]) atomicAdd(&p.hist[(size_t)f * kMaxPasses * kDigits + i], h[i]);
         if (t == 0 && s_fc[slot]) atomicAdd(&p.fcnt[f], s_fc[slot]);
     }
 }
@@ -731,7 +721,16 @@ __global__ void __launch_bounds__(kOutThreads, (B <= 12 ? 6 : 2)) k_emit(Params 
 
 cudaError_t launch_compact(const Params& p, int num_sms, bool pdl, cudaStream_t st) {
     (void)num_sms;   // a block per classify block
-    return launch_k(k_compact, dim3(p.cls_grid > 0 ? p.cls_grid : 1u), dim3(kCT), 0, st, pdl, p);
+    static std::atomic<int> configured[64];
+    int dev = 0;
+    cudaError_t e = cudaGetDevice(&dev);
+    if (e != cudaSuccess) return e;
+    if (dev < 0 || dev >= 64 || !configured[dev].load(std::memory_order_acquire)) {
+        e = cudaFuncSetAttribute(k_compact, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kCSmem);
+        if (e != cudaSuccess) return e;
+        if (dev >= 0 && dev < 64) configured[dev].store(1, std::memory_order_release);
+    }
+    return launch_k(k_compact, dim3(p.cls_grid > 0 ? p.cls_grid : 1u), dim3(kCT), kCSmem, st, pdl, p);
 }
 
 cudaError_t launch_sort(const Params& p, int num_sms, bool pdl, cudaStream_t st) {
