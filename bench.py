@@ -76,6 +76,13 @@ def workload_desc(w):
     }
 
 
+def sort_passes(dims) -> int:
+    """Launches of the sort stage for a grid: one per 9-bit digit of the
+    largest linear index."""
+    maxlin = int(dims[0]) * int(dims[1]) * int(dims[2]) - 1
+    return (maxlin.bit_length() + 8) // 9
+
+
 def read_peaks():
     path = os.path.join(ROOT, "MEASURED_PEAKS.json")
     if os.path.exists(path):
@@ -609,7 +616,8 @@ def run_gpu(args):
             "l2_flushed": l2_flushed,
             "e2e": {"value": e2e_value, "unit": "points/s", "h2d_bytes_per_step": h2d_bytes,
                     "d2h_bytes_per_step": d2h_bytes, "steps": e2e_steps},
-            "gpu_launches": nstage * args.steps,
+            # one launch a stage, but one a 9-bit digit of the lins for the sort
+            "gpu_launches": (nstage - 1 + sort_passes(dims)) * args.steps,
         }
         if world == 1 and not args.no_small_configs:
             # the single-frame configs (L2-resident, latency-bound): warm us
