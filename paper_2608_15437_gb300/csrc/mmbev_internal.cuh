@@ -327,6 +327,16 @@ __device__ __forceinline__ unsigned long long ld_cg(const unsigned long long* a)
     return __ldcg(a);
 }
 
+// Relaxed load at GPU scope, issued anew every time: for look-back words,
+// which carry their flag and value in one word written by one atomic
+// exchange, so that nothing else needs ordering after them. Unlike acquire
+// loads, several can be in flight at once.
+__device__ __forceinline__ unsigned long long ld_relaxed(const unsigned long long* a) {
+    unsigned long long v;
+    asm volatile("ld.relaxed.gpu.global.u64 %0, [%1];" : "=l"(v) : "l"(a) : "memory");
+    return v;
+}
+
 // Acquire load at GPU scope, issued anew every time (for polling a word that
 // another block publishes).
 __device__ __forceinline__ unsigned long long ld_acquire(const unsigned long long* a) {

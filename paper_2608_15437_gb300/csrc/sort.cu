@@ -76,12 +76,12 @@ __device__ __forceinline__ uint32_t block_exclusive_scan(uint32_t v, uint32_t* s
     return wbase + inc - v;
 }
 
-// Bounded wait for a published look-back word; after the first few polls
-// the thread backs off, so that many waiting threads do not crowd L2.
-// False when the wait gave up.
+// Bounded wait for a published look-back word (relaxed loads: the word is
+// its own payload); after the first few polls the thread backs off, so that
+// many waiting threads do not crowd L2. False when the wait gave up.
 __device__ __forceinline__ bool poll_word(const unsigned long long* a, unsigned long long& w) {
     for (uint32_t i = 0; i < kSpinLimit; ++i) {
-        w = ld_acquire(a);
+        w = ld_relaxed(a);
         if (w & kFlags) return true;
         if (i >= 8) __nanosleep(64);
     }
@@ -412,7 +412,7 @@ k_sort_pass(Params p, int pass, const uint32_t* __restrict__ kin, const uint32_t
                     unsigned long long w[4];
 #pragma unroll
                     for (int i = 0; i < 4; ++i)
-                        w[i] = q >= first + (uint32_t)i ? ld_acquire(st + (size_t)(q - i) * kDigits + t)
+                        w[i] = q >= first + (uint32_t)i ? ld_relaxed(st + (size_t)(q - i) * kDigits + t)
                                                         : kInc;
 #pragma unroll
                     for (int i = 0; i < 4; ++i) {
