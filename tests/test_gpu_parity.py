@@ -295,7 +295,11 @@ def test_duplicate_points_in_one_voxel(oracle_mod, mmbev_lib, cuda_dev):
 
 
 def test_tiny_grid_and_many_frames(oracle_mod, mmbev_lib, cuda_dev):
-    # 4 x 3 x 2 = 24 cells (< one 32-cell bucket); 150 frames with 0..3 ROIs
+    # 4 x 3 x 2 = 24 cells (lins of five bits: one radix pass); 150 frames
+    # of up to 60 points with 0..3 ROIs, so a compaction block's range holds
+    # many frames (their counts and histograms go past the two it keeps in
+    # shared memory), every frame is one sort tile, and max_voxels = 5 caps
+    # most of them
     rng = np.random.default_rng(23)
     frames = []
     for f in range(150):
