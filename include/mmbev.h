@@ -227,7 +227,9 @@ int mmbev_get_status(const void *workspace, size_t workspace_bytes,
  *                     Outside [0, 1] or NaN: MMBEV_EINVAL.
  *   seed              the generator's seed.
  * The stages, in launch order (mmbev_stage_name): prep, classify, compact,
- * sort (one launch per 8-bit digit of the sort key), runs, emit.
+ * sort (one launch per 9-bit digit of the largest linear index: three on a
+ * 1440 x 1440 x 40 grid), runs, emit. An event pair brackets each stage,
+ * so the sort's launches are timed together.
  */
 #define MMBEV_NUM_STAGES 6
 typedef struct mmbev_exec_opts {
