@@ -12,7 +12,9 @@
 //
 // The array is shared by every call on a device and keeps the last call's
 // contents. Nothing in it has to start at zero: the call's first kernel
-// clears the counters the later ones accumulate into. Calls whose
+// clears the counters and histograms the later ones accumulate into, and
+// each look-back chain's words are cleared by a kernel that runs before the
+// one that uses them. Calls whose
 // executions overlap on the GPU (two streams, or two host threads) race on
 // the array; serialize them.
 #include <cuda.h>   // driver types only: the two entry points below are fetched at run time
