@@ -144,6 +144,20 @@ def test_dense_voxels_across_tiles(oracle_mod, mmbev_lib, cuda_dev, K):
     assert assert_frames_equal(got, want, f"dense voxels, K={K}") == 1.0
 
 
+@pytest.mark.parametrize("vs", [(0.05, 0.05, 0.2), (0.03, 0.03, 0.1)])
+def test_lins_of_four_digits(oracle_mod, mmbev_lib, cuda_dev, vs):
+    """Grids of more than 2^27 cells over the nuScenes-shaped range
+    (2,160 x 2,160 x 40 and 3,600 x 3,600 x 80): lins of 28 and 30 bits take
+    four 9-bit radix passes, the last on the top digit, and the sorted items
+    end in the first of the two buffers again."""
+    w = synth.nuscenes_frame()
+    w.voxel_size = np.array(vs, np.float32)
+    got, status, _ = run_gpu(mmbev_lib, w, cuda_dev)
+    assert status == 0
+    want = run_oracle(oracle_mod, w)
+    assert assert_frames_equal(got, want, f"voxel size {vs}") == 1.0
+
+
 # ------------------------------------------------------------------ cap path
 
 @pytest.mark.parametrize("maxv", [1, 777, 5000, 13000])
