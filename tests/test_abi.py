@@ -43,6 +43,21 @@ def test_sizes_are_host_only(mmbev_lib):
         mmbev_lib.workspace_size(20000, 4, 16000, 1, TINY_VS, [0, 0, 0, -1, 1, 1])
 
 
+
+def test_workspace_size_follows_the_documented_rule(mmbev_lib):
+    # about 66 bytes a point plus about 34 KB a frame; max_voxels does not
+    # enter; the no-alloc array then holds about 1.5 M points of one frame
+    vs = np.array([0.075, 0.075, 0.2], np.float32)
+    rg = np.array([-54, -54, -5, 54, 54, 3], np.float32)
+    ws = lambda n, mv=120000, F=1: mmbev_lib.workspace_size(n, 30, mv, F, vs, rg)
+    per_point = (ws(2_000_000) - ws(1_000_000)) / 1_000_000
+    assert 65.5 <= per_point <= 66.5
+    assert 32_000 <= ws(1000, F=2) - ws(1000) <= 35_000
+    assert ws(1_000_000, 1) == ws(1_000_000, 200_000)
+    m = re.search(r"#define MMBEV_NOALLOC_SCRATCH_BYTES \((\d+)u << (\d+)\)", open(HEADER).read())
+    cap = int(m.group(1)) << int(m.group(2))
+    assert ws(1_450_000) <= cap < ws(1_600_000)
+
 def _call(lib, *, so=(0, 100), fso=None, fro=None, nr=1, K=10, maxv=100, vs=TINY_VS, rg=TINY_RG,
           margin=0.5, ws_bytes=1 << 30, ws=0x7f0000000000):
     so = np.asarray(so, np.int64)
