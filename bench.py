@@ -1,7 +1,7 @@
 """Benchmark: ROI-aware multi-sweep LiDAR voxelization on GB300.
 
 One step = one call of the whole path (motion compensation, ROI test, voxel
-hash, cap and canonical order, mean features) over a 32-frame streaming batch
+grouping, cap and canonical order, mean features) over a 32-frame streaming batch
 of nuScenes-shaped frames (11,110,400 points, 222 MB of fp32 input), inputs
 resident in HBM. The metric is in-ROI points (points passing the range and
 ROI tests, counted before the caps) per second, over the whole job.

@@ -5,7 +5,7 @@ Python binding of ``libmmbev.so``, the C-ABI library declared in
 from PyTorch tensors (``data_ptr``), host offsets from numpy arrays, and the
 stream from ``torch.cuda.current_stream()``. Every step of the path
 (motion compensation, Eq. 6-7; inside-ROI test, Alg. 1 with the boxes of
-Eq. 1; voxel hash and dedup; cap and canonical order; mean features) runs in
+Eq. 1; grouping by voxel; cap and canonical order; mean features) runs in
 the library's CUDA kernels. There is no CPU fallback: if the library is
 missing, ``load()`` raises.
 """

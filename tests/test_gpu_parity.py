@@ -193,7 +193,7 @@ def test_max_voxels_zero(oracle_mod, mmbev_lib, cuda_dev):
 
 # ------------------------------------------------------------------ per-voxel cap K
 
-@pytest.mark.parametrize("K", [1, 3, 12, 20, 33, 64])   # every finalize instantiation
+@pytest.mark.parametrize("K", [1, 3, 12, 20, 33, 64])   # every k_emit instantiation
 def test_points_per_voxel(oracle_mod, mmbev_lib, cuda_dev, K):
     w = synth.nuscenes_frame(1)
     got, status, _ = run_gpu(mmbev_lib, w, cuda_dev, K=K)
