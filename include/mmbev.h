@@ -96,6 +96,9 @@ typedef enum mmbev_status {
 #define MMBEV_MAX_FRAMES          1024
 #define MMBEV_MAX_ROIS_PER_FRAME  1024
 #define MMBEV_MAX_PTS_PER_VOXEL   64
+/* 2^32 - 2,048 points: the record slots, a whole number of 2,048-point
+ * tiles, keep 32-bit positions. */
+#define MMBEV_MAX_POINTS          4294965248LL
 
 /*
  * Bytes of scratch workspace for a call with up to max_points points,
@@ -103,7 +106,8 @@ typedef enum mmbev_status {
  * num_frames frames on the grid given by voxel_size[3] and range[6] (host
  * arrays). About 66 bytes per point (records, sort keys and positions and
  * per-voxel results, all sized for every point kept) plus about 34 KB per
- * frame. Returns 0 for invalid arguments.
+ * frame. Returns 0 for invalid arguments (max_points above MMBEV_MAX_POINTS
+ * among them).
  */
 size_t mmbev_workspace_size(int64_t max_points, int32_t max_rois_per_frame,
                             int32_t max_voxels, int32_t num_frames,
@@ -112,7 +116,7 @@ size_t mmbev_workspace_size(int64_t max_points, int32_t max_rois_per_frame,
 /*
  * One frame (Alg. 1 on the union of n sweeps, Eq. 7).
  *   points         device, float32 [N][5] (x, y, z, intensity, dt), 16-byte
- *                  aligned; N = sweep_offsets[num_sweeps].
+ *                  aligned; N = sweep_offsets[num_sweeps] <= MMBEV_MAX_POINTS.
  *   sweep_offsets  host, int64 [num_sweeps+1], sweep_offsets[0] = 0,
  *                  nondecreasing; sweep s owns points [off[s], off[s+1]).
  *   num_sweeps     0 <= num_sweeps <= MMBEV_MAX_SWEEPS.

@@ -133,7 +133,7 @@ int validate_common(const float* points, const int64_t* sweep_offsets, int32_t n
     for (int s = 0; s < num_sweeps; ++s)
         if (sweep_offsets[s + 1] < sweep_offsets[s]) return MMBEV_EINVAL;
     const int64_t n = sweep_offsets[num_sweeps];
-    if (n < 0 || n > 0xFFFFFFFEll) return MMBEV_EINVAL;
+    if (n < 0 || n > kMaxPoints) return MMBEV_EINVAL;
     if (fso[0] != 0 || fso[num_frames] != num_sweeps) return MMBEV_EINVAL;
     if (fro[0] != 0 || fro[num_frames] != num_rois) return MMBEV_EINVAL;
     int32_t rmax = 0;
@@ -253,7 +253,7 @@ extern "C" {
 size_t mmbev_workspace_size(int64_t max_points, int32_t max_rois_per_frame, int32_t max_voxels,
                             int32_t num_frames, const float voxel_size[3], const float range[6]) {
     Grid g;
-    if (max_points < 0 || max_rois_per_frame < 0 || max_rois_per_frame > kMaxRoisPerFrame ||
+    if (max_points < 0 || max_points > kMaxPoints || max_rois_per_frame < 0 || max_rois_per_frame > kMaxRoisPerFrame ||
         max_voxels < 0 || num_frames < 1 || num_frames > kMaxFrames)
         return 0;
     if (!make_grid(voxel_size, range, &g)) return 0;

@@ -43,6 +43,9 @@ constexpr int kMaxK = MMBEV_MAX_PTS_PER_VOXEL;
 constexpr int kTile = 2048;
 constexpr int kTileBytes = kTile * 5 * 4;
 constexpr int kRegion = 32;
+// Points of one call: whole tiles of record slots stay below 2^32.
+constexpr int64_t kMaxPoints = MMBEV_MAX_POINTS;
+static_assert(kMaxPoints % kTile == 0 && kMaxPoints + kTile == (int64_t{1} << 32), "point limit");
 
 // Classify blocks (one per SM, at most this many).
 constexpr int kMaxClsGrid = 1000;

@@ -91,6 +91,25 @@ def test_small_buffers_are_rejected_before_launch(mmbev_lib):
     assert _call(lib, ws_bytes=1024) == -3
 
 
+def _max_points():
+    m = re.search(r"#define MMBEV_MAX_POINTS\s+(\d+)LL", open(HEADER).read())
+    return int(m.group(1))
+
+
+def test_point_limit_keeps_record_slots_below_2_32(mmbev_lib):
+    # whole 2,048-point tiles of record slots below 2^32: the largest call
+    # passes validation (and needs far more than the 1 GB workspace given);
+    # one point more is invalid, and so is its workspace size
+    lim = _max_points()
+    assert lim % 2048 == 0 and lim + 2048 == 1 << 32
+    lib = mmbev_lib.load()
+    assert _call(lib, so=(0, lim)) == -3
+    assert _call(lib, so=(0, lim + 1)) == -1
+    assert mmbev_lib.workspace_size(lim, 4, 16000, 1, TINY_VS, TINY_RG) > 66 * lim
+    with pytest.raises(ValueError):
+        mmbev_lib.workspace_size(lim + 1, 4, 16000, 1, TINY_VS, TINY_RG)
+
+
 @pytest.mark.parametrize("rho", [-0.1, 1.5, float("nan")])
 def test_rho_out_outside_unit_interval_is_rejected(mmbev_lib, rho):
     lib = mmbev_lib.load()
