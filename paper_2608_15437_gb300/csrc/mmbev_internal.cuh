@@ -320,6 +320,7 @@ __device__ __forceinline__ uint64_t mix64(uint64_t z) {
     return z ^ (z >> 31);
 }
 
+// Home bucket of a hash key in a power-of-two table (mask = buckets - 1).
 __device__ __forceinline__ uint32_t slot_home(uint32_t mask, unsigned long long key1) {
     return (uint32_t)mix64(key1) & mask;
 }
