@@ -332,6 +332,29 @@ def test_tiny_grid_and_many_frames(oracle_mod, mmbev_lib, cuda_dev):
     assert_frames_equal(got, run_oracle(oracle_mod, b), "many frames")
 
 
+@pytest.mark.parametrize("K", [1, 64])
+def test_grid_of_one_cell(oracle_mod, mmbev_lib, cuda_dev, K):
+    # a 1 x 1 x 1 grid: every lin is 0, so no radix pass runs and the
+    # compacted items, in input order, are already one run a frame; three
+    # frames of 9,000 points span several sort and numbering tiles each
+    rng = np.random.default_rng(25)
+    frames = []
+    for f in range(3):
+        n = 9000
+        pts = np.zeros((n, 5), np.float32)
+        pts[:, :3] = rng.uniform(-0.99, 0.99, (n, 3))
+        pts[:, 3] = rng.uniform(0, 1, n)
+        pts[:, 4] = 0.05 * f
+        frames.append(_custom(pts, [0, n], [EYE], FULL, vs=(2.0, 2.0, 2.0),
+                              rg=(-1, -1, -1, 1, 1, 1), K=K))
+    b = synth.concat_frames(frames, "one cell")
+    got, status, _ = run_gpu(mmbev_lib, b, cuda_dev)
+    assert status == 0
+    want = run_oracle(oracle_mod, b)
+    assert [w[2].tolist() for w in want] == [[K]] * 3
+    assert assert_frames_equal(got, want, "one cell") == 1.0
+
+
 def test_max_rois_per_frame(oracle_mod, mmbev_lib, cuda_dev):
     # 1024 ROIs in a frame: 32 mask words per coarse cell
     rng = np.random.default_rng(24)
