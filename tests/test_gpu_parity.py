@@ -355,6 +355,39 @@ def test_grid_of_one_cell(oracle_mod, mmbev_lib, cuda_dev, K):
     assert assert_frames_equal(got, want, "one cell") == 1.0
 
 
+def _max_frames_and_sweeps():
+    # MMBEV_MAX_FRAMES frames of two sweeps each (MMBEV_MAX_SWEEPS sweeps),
+    # the second sweep moved by a small turn and shift; up to 120 points a
+    # sweep within 3 m, 0-4 rotated ROIs, K = 3 and max_voxels = 40
+    rng = np.random.default_rng(26)
+    frames = []
+    for f in range(1024):
+        n0, n1 = (int(x) for x in rng.integers(0, 121, 2))
+        pts = np.zeros((n0 + n1, 5), np.float32)
+        pts[:, :2] = rng.uniform(-3, 3, (n0 + n1, 2))
+        pts[:, 2] = rng.uniform(-2, 2, n0 + n1)
+        pts[:, 3] = rng.uniform(0, 1, n0 + n1)
+        pts[n0:, 4] = 0.05
+        a = rng.uniform(-0.05, 0.05)
+        t1 = np.eye(4, dtype=np.float32)
+        t1[:2, :2] = [[np.cos(a), -np.sin(a)], [np.sin(a), np.cos(a)]]
+        t1[:2, 3] = rng.uniform(-0.5, 0.5, 2)
+        r = int(rng.integers(0, 5))
+        rois = np.stack([rng.uniform(-3, 3, r), rng.uniform(-3, 3, r), rng.uniform(0.5, 3, r),
+                         rng.uniform(0.5, 3, r), rng.uniform(0, 6.3, r)], 1) if r else np.zeros((0, 5))
+        frames.append(_custom(pts, [0, n0, n0 + n1], [EYE, t1.reshape(16)], rois, margin=0.2,
+                              K=3, maxv=40))
+    return synth.concat_frames(frames, "max frames")
+
+
+def test_max_frames_and_sweeps(oracle_mod, mmbev_lib, cuda_dev):
+    b = _max_frames_and_sweeps()
+    assert b.num_frames == 1024 and len(b.sweep_offsets) == 2049
+    got, status, _ = run_gpu(mmbev_lib, b, cuda_dev)
+    assert status == 0
+    assert assert_frames_equal(got, run_oracle(oracle_mod, b), "max frames") == 1.0
+
+
 def test_max_rois_per_frame(oracle_mod, mmbev_lib, cuda_dev):
     # 1024 ROIs in a frame: 32 mask words per coarse cell
     rng = np.random.default_rng(24)
